@@ -1,0 +1,73 @@
+"""Layer-dropout masks M^{l,t} and kept-sequence lists.
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__.py``).
+
+Follows Eq. (layer_dropout_train): M^{l,t} in {0,1}^B with entries drawn
+Bernoulli(1 - p^{l,t}); the Tensor Granularity subsection: per-sequence (one
+independent draw per sequence b) or per-batch (one draw per layer and step,
+shared by every b); and the "more efficient implementation" paragraph of the
+Preliminary section: the layer runs only on {b_i : M[b_i] = 1}.
+
+Reading of the draw (the paper names no generator):
+  u = word 0 of Philox4x32-10 with key (seed mod 2^32, seed >> 32) and
+      counter (b', l, t mod 2^32, t >> 32), where b' = b per sequence and
+      b' = 0 per batch (so a per-batch mask is the per-sequence draw of
+      sequence 0, broadcast);
+  the layer is dropped for that sequence iff u < thr_l, thr_l = floor(p 2^32).
+Kept lists are in ascending b.
+"""
+
+import numpy as np
+
+from .philox import philox4x32_10, philox4x32_10_np
+
+PER_SEQUENCE, PER_BATCH = "per_sequence", "per_batch"
+
+
+def mask_word(seed, step, layer, b):
+    """The 32-bit uniform word for (seed, step, layer, sequence)."""
+    seed = int(seed)
+    step = int(step)
+    key = (seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
+    ctr = (b, layer, step & 0xFFFFFFFF, (step >> 32) & 0xFFFFFFFF)
+    return philox4x32_10(ctr, key)[0]
+
+
+def draw_masks(seed, step, thresholds, B, granularity=PER_SEQUENCE):
+    """mask[l][b] in {0,1} (1 = keep) for every layer l (uint8, shape [L, B])."""
+    L = len(thresholds)
+    mask = np.zeros((L, B), dtype=np.uint8)
+    for layer in range(L):
+        for b in range(B):
+            bb = b if granularity == PER_SEQUENCE else 0
+            u = mask_word(seed, step, layer, bb)
+            mask[layer, b] = 0 if u < thresholds[layer] else 1
+    return mask
+
+
+def kept_lists(mask):
+    """kept_idx[l] = ascending b with mask[l][b] = 1; kept_cnt[l] = its length.
+
+    Returned as (int32 [L, B] padded with -1, int32 [L])."""
+    L, B = mask.shape
+    idx = np.full((L, B), -1, dtype=np.int32)
+    cnt = np.zeros(L, dtype=np.int32)
+    for layer in range(L):
+        kept = [b for b in range(B) if mask[layer, b] == 1]
+        cnt[layer] = len(kept)
+        idx[layer, : len(kept)] = kept
+    return idx, cnt
+
+
+def words_np(seed, step, layer, b):
+    """Vectorised ``mask_word`` over numpy arrays of (step, layer, b)."""
+    seed = int(seed)
+    step = np.asarray(step, dtype=np.uint64)
+    z = np.zeros(np.broadcast(step, layer, b).shape, dtype=np.uint64)
+    c0 = np.asarray(b, dtype=np.uint64) + z
+    c1 = np.asarray(layer, dtype=np.uint64) + z
+    c2 = (step & np.uint64(0xFFFFFFFF)) + z
+    c3 = (step >> np.uint64(32)) + z
+    k0 = np.uint64(seed & 0xFFFFFFFF) + z
+    k1 = np.uint64((seed >> 32) & 0xFFFFFFFF) + z
+    return philox4x32_10_np(c0, c1, c2, c3, k0, k1)[0]

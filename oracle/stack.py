@@ -1,0 +1,280 @@
+"""Forward and backward of a pre-norm decoder stack under layer dropout.
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__.py``).
+
+Follows Eq. (transformer_layer_dropout_train) with one mask per layer for
+both sub-blocks (layer granularity, Model Granularity subsection):
+
+    Z^l      = X^l + r M^l f_attn(X^l)
+    X^{l+1}  = Z^l + r M^l f_ffn(Z^l)
+
+and the per-sequence case form of the Preliminary section: a dropped
+sequence keeps X^{l+1}[b] = X^l[b]; a kept one gets the residual update with
+r = alpha / (1 - p^{l,t}) (Dropout Scale paragraph and the parameterization
+table's residual rows).  Only kept sequences are evaluated, as in the
+"efficient implementation" paragraph.
+
+The paper leaves the block internals open (its footnote to the transformer
+form); the block here is the one the workloads name: RMSNorm (eps inside the
+square root, gain gamma), rotary position embedding on q and k, causal
+grouped-query attention with scale 1/sqrt(Dh), SwiGLU feed-forward
+h = silu(g) * u, no biases.  Weights use the [out, in] layout: w_qkv rows are
+[Q heads; K heads; V heads], w_gu rows are [gate; up].  Query head h reads
+key/value head floor(h * Hkv / H).  RoPE rotates the pairs (i, i + Dh/2) by
+angle pos * theta^(-2i/Dh) at in-sequence position pos; theta = 0 disables it.
+
+The backward is derived by hand from these definitions (chain rule, no
+autograd).  Everything is float64, one sequence at a time.
+"""
+
+import math
+
+import numpy as np
+
+
+# --------------------------------------------------------------------------
+# building blocks
+# --------------------------------------------------------------------------
+
+def rmsnorm(x, gamma, eps):
+    """RMSNorm of each row: x / sqrt(mean(x^2) + eps) * gamma.
+
+    Returns (output, normalised rows without gamma, reciprocal rms)."""
+    r = 1.0 / np.sqrt(np.mean(x * x, axis=-1) + eps)
+    xn = x * r[:, None]
+    return xn * gamma, xn, r
+
+
+def rmsnorm_backward(dy, xn, r, gamma):
+    """Gradients of rmsnorm w.r.t. its input rows and gamma.
+
+    With xn = x r and r = (mean(x^2) + eps)^(-1/2):
+      d xn = dy * gamma
+      dx   = r * (d xn - xn * mean(d xn * xn))
+      dgamma = sum over rows of dy * xn."""
+    dxn = dy * gamma
+    dx = r[:, None] * (dxn - xn * np.mean(dxn * xn, axis=-1, keepdims=True))
+    dgamma = np.sum(dy * xn, axis=0)
+    return dx, dgamma
+
+
+def rope_tables(S, Dh, theta):
+    """cos, sin of pos * theta^(-2i/Dh), shape [S, Dh/2]."""
+    half = Dh // 2
+    i = np.arange(half, dtype=np.float64)
+    inv_freq = theta ** (-(2.0 * i) / Dh)
+    ang = np.arange(S, dtype=np.float64)[:, None] * inv_freq[None, :]
+    return np.cos(ang), np.sin(ang)
+
+
+def rope(t, cos, sin):
+    """Rotate pairs (i, i+Dh/2) of every head vector; t is [S, heads, Dh]."""
+    half = t.shape[-1] // 2
+    a, b = t[..., :half], t[..., half:]
+    c, s = cos[:, None, :], sin[:, None, :]
+    return np.concatenate([a * c - b * s, b * c + a * s], axis=-1)
+
+
+def rope_backward(dt, cos, sin):
+    """Transpose of ``rope`` (rotation by the opposite angle)."""
+    half = dt.shape[-1] // 2
+    a, b = dt[..., :half], dt[..., half:]
+    c, s = cos[:, None, :], sin[:, None, :]
+    return np.concatenate([a * c + b * s, b * c - a * s], axis=-1)
+
+
+def kv_head(h, H, Hkv):
+    return (h * Hkv) // H
+
+
+def attention_probs(qh, kh):
+    """Causal softmax(q k^T / sqrt(Dh)) for one head: [S, S]."""
+    S, Dh = qh.shape
+    sc = (qh @ kh.T) / math.sqrt(Dh)
+    causal = np.tril(np.ones((S, S), dtype=bool))
+    sc = np.where(causal, sc, -np.inf)
+    sc = sc - np.max(sc, axis=1, keepdims=True)
+    e = np.exp(sc)
+    return e / np.sum(e, axis=1, keepdims=True)
+
+
+def attention(q, k, v):
+    """Causal grouped-query attention. q [S,H,Dh], k/v [S,Hkv,Dh] -> [S,H,Dh]."""
+    S, H, Dh = q.shape
+    Hkv = k.shape[1]
+    o = np.zeros_like(q)
+    for h in range(H):
+        j = kv_head(h, H, Hkv)
+        P = attention_probs(q[:, h, :], k[:, j, :])
+        o[:, h, :] = P @ v[:, j, :]
+    return o
+
+
+def attention_backward(do, q, k, v):
+    """Gradients of ``attention`` w.r.t. q, k, v given d(out) = do.
+
+    Per head, with P the probabilities and c = 1/sqrt(Dh):
+      dv += P^T do;  dP = do v^T;  dS = P * (dP - rowsum(dP * P));
+      dq = c dS k;   dk += c dS^T q
+    (key/value gradients summed over the query heads that share them)."""
+    S, H, Dh = q.shape
+    Hkv = k.shape[1]
+    c = 1.0 / math.sqrt(Dh)
+    dq = np.zeros_like(q)
+    dk = np.zeros_like(k)
+    dv = np.zeros_like(v)
+    for h in range(H):
+        j = kv_head(h, H, Hkv)
+        P = attention_probs(q[:, h, :], k[:, j, :])
+        doh = do[:, h, :]
+        dv[:, j, :] += P.T @ doh
+        dP = doh @ v[:, j, :].T
+        dS = P * (dP - np.sum(dP * P, axis=1, keepdims=True))
+        dq[:, h, :] = c * (dS @ k[:, j, :])
+        dk[:, j, :] += c * (dS.T @ q[:, h, :])
+    return dq, dk, dv
+
+
+def sigmoid(x):
+    with np.errstate(over="ignore"):
+        return 1.0 / (1.0 + np.exp(-x))
+
+
+# --------------------------------------------------------------------------
+# one layer, one sequence
+# --------------------------------------------------------------------------
+
+def _split_qkv(qkv, cfg):
+    S = qkv.shape[0]
+    H, Hkv, Dh = cfg["H"], cfg["Hkv"], cfg["Dh"]
+    q = qkv[:, : H * Dh].reshape(S, H, Dh)
+    k = qkv[:, H * Dh : (H + Hkv) * Dh].reshape(S, Hkv, Dh)
+    v = qkv[:, (H + Hkv) * Dh :].reshape(S, Hkv, Dh)
+    return q, k, v
+
+
+def layer_forward(x, W, cfg, s, rope_cs):
+    """Kept sequence x [S, d] -> X^{l+1}[b] and the values the backward needs."""
+    S = x.shape[0]
+    F = cfg["F"]
+    eps = cfg["eps"]
+    xh, xn, r1 = rmsnorm(x, W["g1"], eps)
+    q, k, v = _split_qkv(xh @ W["w_qkv"].T, cfg)
+    if rope_cs is not None:
+        cos, sin = rope_cs
+        q = rope(q, cos[:S], sin[:S])
+        k = rope(k, cos[:S], sin[:S])
+    o = attention(q, k, v).reshape(S, -1)
+    z = x + s * (o @ W["w_o"].T)
+    zh, zn, r2 = rmsnorm(z, W["g2"], eps)
+    gu = zh @ W["w_gu"].T
+    g, u = gu[:, :F], gu[:, F:]
+    h = g * sigmoid(g) * u
+    out = z + s * (h @ W["w_d"].T)
+    cache = dict(xh=xh, xn=xn, r1=r1, q=q, k=k, v=v, o=o, zh=zh, zn=zn, r2=r2, g=g, u=u, h=h)
+    return out, cache
+
+
+def layer_backward(dout, W, cfg, s, cache, G, rope_cs):
+    """d X^{l+1}[b] -> d X^l[b] for a kept sequence; adds into the layer's
+    weight gradients G."""
+    S = dout.shape[0]
+    H, Hkv, Dh = cfg["H"], cfg["Hkv"], cfg["Dh"]
+    c = cache
+    # FFN branch: out = z + s * (h w_d^T), h = silu(g) u.
+    dy = s * dout
+    G["w_d"] += dy.T @ c["h"]
+    dh = dy @ W["w_d"]
+    sg = sigmoid(c["g"])
+    dg = dh * c["u"] * sg * (1.0 + c["g"] * (1.0 - sg))
+    du = dh * c["g"] * sg
+    dgu = np.concatenate([dg, du], axis=1)
+    G["w_gu"] += dgu.T @ c["zh"]
+    dzh = dgu @ W["w_gu"]
+    dz_norm, dg2 = rmsnorm_backward(dzh, c["zn"], c["r2"], W["g2"])
+    G["g2"] += dg2
+    dz = dout + dz_norm
+    # attention branch: z = x + s * (o w_o^T).
+    da = s * dz
+    G["w_o"] += da.T @ c["o"]
+    do = (da @ W["w_o"]).reshape(S, H, Dh)
+    dq, dk, dv = attention_backward(do, c["q"], c["k"], c["v"])
+    if rope_cs is not None:
+        cos, sin = rope_cs
+        dq = rope_backward(dq, cos[:S], sin[:S])
+        dk = rope_backward(dk, cos[:S], sin[:S])
+    dqkv = np.concatenate([dq.reshape(S, -1), dk.reshape(S, -1), dv.reshape(S, -1)], axis=1)
+    G["w_qkv"] += dqkv.T @ c["xh"]
+    dxh = dqkv @ W["w_qkv"]
+    dx_norm, dg1 = rmsnorm_backward(dxh, c["xn"], c["r1"], W["g1"])
+    G["g1"] += dg1
+    return dz + dx_norm
+
+
+# --------------------------------------------------------------------------
+# the stack
+# --------------------------------------------------------------------------
+
+WEIGHT_NAMES = ("w_qkv", "w_o", "w_gu", "w_d", "g1", "g2")
+
+
+def _layer(layers, l):
+    """Weights of layer l as float64 arrays (``layers`` is a list or a callable)."""
+    W = layers(l) if callable(layers) else layers[l]
+    return {n: np.asarray(W[n], dtype=np.float64) for n in WEIGHT_NAMES}
+
+
+def _rope_cs(cfg, S):
+    theta = cfg.get("rope_theta", 0.0)
+    if not theta:
+        return None
+    return rope_tables(S, cfg["Dh"], theta)
+
+
+def stack_forward(x, layers, cfg, masks, scales):
+    """x [B, S, d] -> (X^L, caches).  masks [L, B] (1 = keep), scales [L]."""
+    X = np.array(x, dtype=np.float64, copy=True)
+    B, S, _ = X.shape
+    L = masks.shape[0]
+    rope_cs = _rope_cs(cfg, S)
+    caches = [[None] * B for _ in range(L)]
+    for l in range(L):
+        if not masks[l].any():
+            continue
+        W = _layer(layers, l)
+        for b in range(B):
+            if masks[l, b]:
+                X[b], caches[l][b] = layer_forward(X[b], W, cfg, scales[l], rope_cs)
+    return X, caches
+
+
+def stack_backward(dy, layers, cfg, masks, scales, caches):
+    """d X^L -> (d X^0, per-layer weight gradients).
+
+    Dropped sequences pass their gradient through unchanged; a layer's weight
+    gradients sum over its kept sequences only (zero if none is kept)."""
+    dX = np.array(dy, dtype=np.float64, copy=True)
+    B, S, _ = dX.shape
+    L = masks.shape[0]
+    rope_cs = _rope_cs(cfg, S)
+    grads = [None] * L
+    for l in reversed(range(L)):
+        W = _layer(layers, l) if masks[l].any() else None
+        G = {n: np.zeros(shape_of(cfg, n)) for n in WEIGHT_NAMES}
+        for b in range(B):
+            if masks[l, b]:
+                dX[b] = layer_backward(dX[b], W, cfg, scales[l], caches[l][b], G, rope_cs)
+        grads[l] = G
+    return dX, grads
+
+
+def shape_of(cfg, name):
+    d, H, Hkv, Dh, F = cfg["d"], cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"]
+    return {
+        "w_qkv": ((H + 2 * Hkv) * Dh, d),
+        "w_o": (d, H * Dh),
+        "w_gu": (2 * F, d),
+        "w_d": (d, F),
+        "g1": (d,),
+        "g2": (d,),
+    }[name]

@@ -1,0 +1,81 @@
+"""An independent dense decoder layer in PyTorch (float64, CPU), used only to
+pin the oracle.
+
+It is written with library routines that the oracle does not use:
+``torch.nn.functional.rms_norm``, ``scaled_dot_product_attention`` with a
+causal mask, complex multiplication for the rotary embedding, ``F.silu``, and
+autograd for every gradient.  A mistake in the oracle's hand-written forward
+or hand-derived backward (a dropped term, a sign, a transposed operand, a
+wrong key/value head) shows up as a mismatch with this module.
+"""
+
+import torch
+import torch.nn.functional as F
+
+
+def _rope_complex(t, theta):
+    """t [S, heads, Dh]; pairs (i, i + Dh/2) rotated as complex numbers."""
+    S, nh, Dh = t.shape
+    half = Dh // 2
+    freqs = 1.0 / (theta ** (torch.arange(0, Dh, 2, dtype=torch.float64) / Dh))
+    ang = torch.outer(torch.arange(S, dtype=torch.float64), freqs)
+    rot = torch.polar(torch.ones_like(ang), ang)[:, None, :]
+    c = torch.complex(t[..., :half], t[..., half:]) * rot
+    return torch.cat([c.real, c.imag], dim=-1)
+
+
+def dense_layer(x, W, cfg):
+    """f for one sequence x [S, d] at rate 0 and scale 1: returns (attn, ffn)
+    callables so that masks and scales can be composed outside."""
+    H, Hkv, Dh, Fh = cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"]
+    eps, theta = cfg["eps"], cfg.get("rope_theta", 0.0)
+    S = x.shape[0]
+
+    def f_attn(xx):
+        xh = F.rms_norm(xx, (xx.shape[-1],), weight=W["g1"], eps=eps)
+        qkv = xh @ W["w_qkv"].T
+        q = qkv[:, : H * Dh].view(S, H, Dh)
+        k = qkv[:, H * Dh : (H + Hkv) * Dh].view(S, Hkv, Dh)
+        v = qkv[:, (H + Hkv) * Dh :].view(S, Hkv, Dh)
+        if theta:
+            q, k = _rope_complex(q, theta), _rope_complex(k, theta)
+        rep = H // Hkv
+        k = k.repeat_interleave(rep, dim=1)
+        v = v.repeat_interleave(rep, dim=1)
+        o = F.scaled_dot_product_attention(
+            q.transpose(0, 1)[None], k.transpose(0, 1)[None], v.transpose(0, 1)[None], is_causal=True
+        )[0].transpose(0, 1).reshape(S, H * Dh)
+        return o @ W["w_o"].T
+
+    def f_ffn(zz):
+        zh = F.rms_norm(zz, (zz.shape[-1],), weight=W["g2"], eps=eps)
+        gu = zh @ W["w_gu"].T
+        return (F.silu(gu[:, :Fh]) * gu[:, Fh:]) @ W["w_d"].T
+
+    return f_attn, f_ffn
+
+
+def masked_stack(x, layers, cfg, masks, scales):
+    """Stack with per-sequence masks, composed from dense layers:
+    a kept sequence gets z = x + s f_attn(x), x' = z + s f_ffn(z); a dropped
+    one is left as it is."""
+    B = x.shape[0]
+    outs = []
+    for b in range(B):
+        xb = x[b]
+        for l in range(masks.shape[0]):
+            if masks[l, b]:
+                f_attn, f_ffn = dense_layer(xb, layers[l], cfg)
+                s = float(scales[l])
+                zb = xb + s * f_attn(xb)
+                xb = zb + s * f_ffn(zb)
+        outs.append(xb)
+    return torch.stack(outs)
+
+
+def to_torch_layers(layers, requires_grad=False):
+    out = []
+    for W in layers:
+        out.append({n: torch.tensor(W[n], dtype=torch.float64, requires_grad=requires_grad)
+                    for n in ("w_qkv", "w_o", "w_gu", "w_d", "g1", "g2")})
+    return out
