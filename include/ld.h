@@ -1,0 +1,194 @@
+/*
+ * ld.h -- C ABI of the layer-dropout decoder-stack library (sm_103a).
+ *
+ * The library runs the forward and backward pass of a pre-norm decoder stack
+ * under layer dropout (stochastic depth), as defined in "Don't Drop Dropout"
+ * (arXiv 2609.05275):
+ *
+ *   Eq. (layer_dropout_train), per-sequence case form (Preliminary section):
+ *     H^{l+1}[b] = H^l[b]                      with probability p^{l,t}
+ *     H^{l+1}[b] = H^l[b] + r f^l(H^l[b])      with probability 1 - p^{l,t}
+ *   Eq. (transformer_layer_dropout_train), one mask for both sub-blocks
+ *   (layer granularity, Model Granularity subsection):
+ *     Z^l = X^l + r M^l f_attn(X^l),   X^{l+1} = Z^l + r M^l f_ffn(Z^l)
+ *   r = alpha / (1 - p) (Dropout Scale paragraph; parameterization table).
+ *
+ * and, as the Preliminary section's "more efficient implementation" asks, it
+ * evaluates f only on the kept sequences: dropped sequences are neither read
+ * nor written, in the forward or in the backward.
+ *
+ * Block: RMSNorm -> fused QKV projection -> RoPE -> causal grouped-query
+ * attention -> output projection -> scaled residual; RMSNorm -> SwiGLU
+ * gate/up -> down projection -> scaled residual.  No biases, no final norm.
+ *
+ * Conventions for every entry point
+ *   - Device pointers are plain CUDA device addresses owned by the caller;
+ *     the library never frees them and keeps none beyond the call, except
+ *     that ld_get_masks / ld_sync read the workspace and stream of the last
+ *     ld_forward / ld_draw_masks on the handle.
+ *   - Matrices are row-major; weights use the [out, in] layout.  The element
+ *     type is bf16 (uint16 storage) unless ld_config.fp32_debug is set, in
+ *     which case every activation, weight and gain is float32.  Weight and
+ *     gain gradients are always float32.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All device
+ *     work is enqueued on it; no entry point synchronises the host except
+ *     ld_get_masks and ld_sync.
+ *   - Errors: argument and shape errors are returned synchronously and
+ *     enqueue nothing.  A device-side error (a bounded wait that expired) is
+ *     recorded in the workspace status word and returned by ld_sync.  No
+ *     entry point aborts or throws.
+ *   - A handle is not thread-safe; use one per host thread.
+ */
+#ifndef LD_H
+#define LD_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  LD_OK = 0,
+  LD_ERR_ARG = 1,      /* null/misaligned pointer, rate outside [0,1], NaN   */
+  LD_ERR_SHAPE = 2,    /* unsupported shape (see ld_create)                  */
+  LD_ERR_STATE = 3,    /* call out of order (backward without its forward)   */
+  LD_ERR_CUDA = 4,     /* a CUDA runtime call failed                         */
+  LD_ERR_TIMEOUT = 5,  /* a device-side bounded wait expired                 */
+  LD_ERR_OOM = 6,      /* host allocation failed                             */
+  LD_ERR_UNSUPPORTED = 7 /* device is not sm_103 / build lacks the kernel    */
+} ld_status;
+
+/* Tensor granularity (Tensor Granularity subsection): one Bernoulli draw per
+ * sequence, or one per layer and step shared by the whole batch. */
+typedef enum { LD_PER_SEQUENCE = 0, LD_PER_BATCH = 1 } ld_granularity;
+
+/* Layer distributions (Dropout Distribution section):
+ *   UNIFORM  p^l = p_max
+ *   ILD      p^l = l/(L-1) * p_max   (p^0 = 0; a one-layer stack gets 0)
+ *   ALD      p^l = p_max * 1[l odd]  (l counted from 0)
+ *   EXPLICIT p^l = p_explicit[l]                                          */
+typedef enum { LD_DIST_UNIFORM = 0, LD_DIST_ILD = 1, LD_DIST_ALD = 2, LD_DIST_EXPLICIT = 3 } ld_dist;
+
+/* Time schedules (Dropout Schedule section), factor applied to p^l:
+ *   CONST 1;  ITS t/(T-1);  DTS 1 - t/(T-1);
+ *   RAMP  s0 + (s1-s0) * clamp((t-t0)/(t1-t0), 0, 1)   (warm-up ramp; not
+ *         in the paper).  The product is clamped to [0, 1].              */
+typedef enum { LD_TIME_CONST = 0, LD_TIME_ITS = 1, LD_TIME_DTS = 2, LD_TIME_RAMP = 3 } ld_time;
+
+typedef struct {
+  int L;            /* layers                                             */
+  int d;            /* model width; multiple of 64                        */
+  int H, Hkv, Dh;   /* query heads, key/value heads (H % Hkv == 0), head
+                       size in {32, 64, 128}; H*Dh multiple of 64          */
+  int F;            /* SwiGLU hidden size; multiple of 64                 */
+  int B, S;         /* sequences per batch (<= 4096), sequence length
+                       (multiple of 64, <= 16384)                         */
+  float eps;        /* RMSNorm epsilon, inside the square root            */
+  float rope_theta; /* RoPE base; 0 disables the rotary embedding         */
+  float alpha;      /* residual multiplier m_L^{-1}; the branch scale is
+                       alpha / (1 - p)                                    */
+  int granularity;  /* ld_granularity                                     */
+  int fp32_debug;   /* 1: float32 storage and SIMT float32 kernels        */
+} ld_config;
+
+typedef struct {
+  int dist;                  /* ld_dist                                   */
+  float p_max;               /* in [0, 1]                                 */
+  const float* p_explicit;   /* host, [L], used by LD_DIST_EXPLICIT; copied */
+  int time;                  /* ld_time                                   */
+  long long T;               /* total steps for ITS / DTS (>= 2)          */
+  long long ramp_t0, ramp_t1;/* RAMP window (t1 > t0)                     */
+  float ramp_s0, ramp_s1;    /* RAMP factors at t0 and t1                 */
+  unsigned long long seed;   /* Philox key                                */
+} ld_schedule;
+
+/* Weights of one layer (device pointers, bf16 or float32):
+ *   w_qkv [(H+2Hkv)*Dh, d]  rows: Q heads, then K heads, then V heads
+ *   w_o   [d, H*Dh]
+ *   w_gu  [2F, d]           rows: gate (F), then up (F)
+ *   w_d   [d, F]
+ *   g1, g2 [d]              RMSNorm gains before attention / FFN          */
+typedef struct { const void *w_qkv, *w_o, *w_gu, *w_d, *g1, *g2; } ld_layer_w;
+
+/* Gradients of one layer (device float32, same shapes; overwritten). */
+typedef struct { float *w_qkv, *w_o, *w_gu, *w_d, *g1, *g2; } ld_layer_g;
+
+/* Validate `cfg` and create a handle.  Allocates host memory only (no CUDA
+ * call), so it can run without a GPU.  LD_ERR_SHAPE for an unsupported
+ * shape, LD_ERR_ARG for null pointers or a non-finite eps/alpha. */
+ld_status ld_create(const ld_config* cfg, void** handle);
+
+/* Bytes of device workspace ld_forward/ld_backward need: the mask tables,
+ * the rotary table and, per layer, the activations saved for the backward,
+ * sized for the worst case (every sequence kept), plus backward scratch.
+ * The caller allocates it (256-byte aligned) and owns it. */
+ld_status ld_workspace_size(void* handle, size_t* bytes);
+
+/* Set the drop-rate schedule (host only; the rates of step t are formed at
+ * ld_forward / ld_draw_masks time).  LD_ERR_ARG if p_max or an explicit
+ * rate is outside [0,1] or NaN, T < 2 for ITS/DTS, or t1 <= t0 for RAMP. */
+ld_status ld_set_schedule(void* handle, const ld_schedule* sched);
+
+/* Host-side view of step t: p[l] = p^{l,t} (double), thr[l] =
+ * floor(p * 2^32) (the mask drops sequence b iff its Philox word u < thr),
+ * scale[l] = alpha / (1 - p) (0 when p = 1).  Any output may be NULL. */
+ld_status ld_get_rates(void* handle, long long step, double* p, unsigned long long* thr, float* scale);
+
+/* Draw the masks of step t into the workspace (the first kernel of
+ * ld_forward, alone).  Philox4x32-10 (Salmon et al., SC'11): key = (seed
+ * low 32 bits, seed high 32 bits), counter = (b', l, t low, t high) with
+ * b' = b per sequence and b' = 0 per batch; word 0 is u.  Kept lists are
+ * ascending in b. */
+ld_status ld_draw_masks(void* handle, long long step, void* workspace, void* stream);
+
+/* Forward of step t, in place on x [B*S, d] (sequence b = rows b*S..b*S+S-1).
+ * W points to L host structs of device pointers.  Rows of dropped sequences
+ * are not touched.  Saves what the backward needs in `workspace`. */
+ld_status ld_forward(void* handle, long long step, const ld_layer_w* W, void* x, void* workspace,
+                     void* stream);
+
+/* Backward of the last ld_forward on this handle and workspace (same W).
+ * dx [B*S, d] holds dY on entry and dX on return (in place); rows of a
+ * sequence dropped at layer l pass through that layer unchanged.  G points
+ * to L host structs of device float32 pointers, overwritten with the weight
+ * and gain gradients (zero for a layer that kept no sequence).
+ * LD_ERR_STATE without a preceding ld_forward on the same workspace. */
+ld_status ld_backward(void* handle, const ld_layer_w* W, void* dx, ld_layer_g* G, void* workspace,
+                      void* stream);
+
+/* Copy the masks of the last ld_forward / ld_draw_masks to host memory:
+ * mask [L*B] (1 = keep), kept_idx [L*B] (ascending, -1 padded), kept_cnt
+ * [L].  Synchronises that call's stream.  Any output may be NULL. */
+ld_status ld_get_masks(void* handle, unsigned char* mask, int* kept_idx, int* kept_cnt);
+
+/* Synchronise the stream of the last call and return the device status word
+ * (LD_OK or LD_ERR_TIMEOUT), clearing it. */
+ld_status ld_sync(void* handle);
+
+/* Release the handle (host memory only). */
+ld_status ld_destroy(void* handle);
+
+/* Static description of a status code. */
+const char* ld_status_str(ld_status status);
+
+/* Dense contraction used by every projection of the block (the linear maps
+ * inside f_attn and f_ffn), exposed for testing and reuse:
+ *   D[m, n] = alpha * sum_k A(m, k) * B(n, k),   m < M, n < N, k < K
+ * A(m,k) = A[m*lda + k] (a_mn_major = 0) or A[k*lda + m] (a_mn_major = 1);
+ * B(n,k) = B[n*ldb + k] (b_mn_major = 0) or B[k*ldb + n] (b_mn_major = 1).
+ * A and B are bf16; D is bf16 (d_f32 = 0) or float32 (d_f32 = 1) with row
+ * stride ldd.  Runs on the tcgen05 tensor cores with TMA-staged operands.
+ * Requirements: M, N, K multiples of 64 (M, N >= 64); lda, ldb, ldd
+ * multiples of 8 elements; pointers 16-byte aligned.  Async on `stream`;
+ * a device-side timeout sets the status word of `status_ws` (an int on the
+ * device, may be NULL). */
+ld_status ld_gemm_bf16(int M, int N, int K, const void* A, int lda, int a_mn_major, const void* B,
+                       int ldb, int b_mn_major, void* D, int ldd, int d_f32, float alpha,
+                       int* status_ws, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LD_H */

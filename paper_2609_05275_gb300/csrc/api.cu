@@ -1,0 +1,623 @@
+// C ABI of the library (include/ld.h): handle, schedule, workspace layout
+// and the per-layer launch sequence of the forward and backward passes.
+//
+// Forward of layer l (kept rows only, compact order, M = kept_cnt[l] * S):
+//   xh  = RMSNorm_1(x[kept])                         (gather; copy of x saved)
+//   qkv = xh W_qkv^T ; RoPE on the q and k heads
+//   o   = causal GQA attention(q, k, v)
+//   x[kept] += r * (o W_o^T)                         (= Z^l, saved compact)
+//   zh  = RMSNorm_2(Z^l[kept]) ; gu = zh W_gu^T ; h = silu(g) * u
+//   x[kept] += r * (h W_d^T)                         (= X^{l+1})
+// with r = alpha / (1 - p^{l,t}) (Eq. transformer_layer_dropout_train and the
+// Dropout Scale paragraph).  Rows of dropped sequences are never touched.
+// The backward walks the layers in reverse and mirrors this; the gradient
+// of a dropped row passes through unchanged (it is the identity there).
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "ld_internal.cuh"
+
+using namespace ldk;
+
+namespace {
+
+size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
+
+struct Layout {
+  size_t status, mask, kidx, kcnt, rcos, rsin;
+  size_t layer0, per_layer;
+  size_t xin, xh, qkv, o, lse, z, zh, gu, h, rstd1, rstd2;  // offsets inside a layer block
+  size_t dy, dh, dgu, dzh, dz, dO, dqkv, dxh, Dvec, dqacc, part;
+  size_t total;
+};
+
+struct Handle {
+  ld_config cfg;
+  bool have_sched = false;
+  ld_schedule sched;
+  std::vector<float> p_expl;
+  Layout lay;
+  size_t esz = 2;
+  int max_rows = 0, nqkv = 0, part_blocks = 0;
+  void* last_ws = nullptr;
+  cudaStream_t last_stream = nullptr;
+  bool have_masks = false;
+  bool fwd_valid = false;
+  void* fwd_ws = nullptr;
+  std::vector<float> fwd_scale;
+};
+
+Handle* H(void* h) { return static_cast<Handle*>(h); }
+
+bool finite(float v) { return std::isfinite(v); }
+
+// ------------------------------------------------------------------ schedule
+// p^l_dist (Dropout Distribution section), widened from float exactly.
+double dist_rate(const Handle* h, int l) {
+  const int L = h->cfg.L;
+  const double pm = (double)h->sched.p_max;
+  switch (h->sched.dist) {
+    case LD_DIST_UNIFORM: return pm;
+    case LD_DIST_ILD: return L == 1 ? 0.0 : (pm * (double)l) / (double)(L - 1);
+    case LD_DIST_ALD: return (l % 2 == 1) ? pm : 0.0;
+    default: return (double)h->p_expl[l];
+  }
+}
+
+// time factor (Dropout Schedule section; RAMP is a warm-up ramp).
+double time_factor(const Handle* h, long long t) {
+  const ld_schedule& s = h->sched;
+  switch (s.time) {
+    case LD_TIME_ITS: return (double)t / (double)(s.T - 1);
+    case LD_TIME_DTS: return 1.0 - (double)t / (double)(s.T - 1);
+    case LD_TIME_RAMP: {
+      double f = (double)(t - s.ramp_t0) / (double)(s.ramp_t1 - s.ramp_t0);
+      f = f < 0.0 ? 0.0 : (f > 1.0 ? 1.0 : f);
+      const double s0 = (double)s.ramp_s0, s1 = (double)s.ramp_s1;
+      return s0 + (s1 - s0) * f;
+    }
+    default: return 1.0;
+  }
+}
+
+void step_rates(const Handle* h, long long t, double* p, unsigned long long* thr, float* scale) {
+  for (int l = 0; l < h->cfg.L; ++l) {
+    double v = dist_rate(h, l) * time_factor(h, t);
+    v = v < 0.0 ? 0.0 : (v > 1.0 ? 1.0 : v);
+    if (p) p[l] = v;
+    if (thr) thr[l] = (unsigned long long)std::floor(v * 4294967296.0);
+    if (scale) scale[l] = v >= 1.0 ? 0.0f : (float)((double)h->cfg.alpha / (1.0 - v));
+  }
+}
+
+// ------------------------------------------------------------------ layout
+void make_layout(Handle* h) {
+  const ld_config& c = h->cfg;
+  const size_t R = (size_t)c.B * c.S, e = h->esz;
+  Layout& y = h->lay;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes);
+    return at;
+  };
+  y.status = take(64);
+  y.mask = take((size_t)c.L * c.B);
+  y.kidx = take((size_t)c.L * c.B * 4);
+  y.kcnt = take((size_t)c.L * 4);
+  y.rcos = take((size_t)c.S * (c.Dh / 2) * 4);
+  y.rsin = take((size_t)c.S * (c.Dh / 2) * 4);
+  // per-layer saved activations
+  size_t lo = 0;
+  auto ltake = [&](size_t bytes) {
+    const size_t at = lo;
+    lo = align_up(lo + bytes);
+    return at;
+  };
+  y.xin = ltake(R * c.d * e);
+  y.xh = ltake(R * c.d * e);
+  y.qkv = ltake(R * h->nqkv * e);
+  y.o = ltake(R * c.H * c.Dh * e);
+  y.lse = ltake((size_t)c.H * R * 4);
+  y.z = ltake(R * c.d * e);
+  y.zh = ltake(R * c.d * e);
+  y.gu = ltake(R * 2 * c.F * e);
+  y.h = ltake(R * c.F * e);
+  y.rstd1 = ltake(R * 4);
+  y.rstd2 = ltake(R * 4);
+  y.per_layer = lo;
+  y.layer0 = off;
+  off = align_up(off + (size_t)c.L * lo);
+  // backward scratch (shared by all layers)
+  y.dy = take(R * c.d * e);
+  y.dh = take(R * c.F * e);
+  y.dgu = take(R * 2 * c.F * e);
+  y.dzh = take(R * c.d * e);
+  y.dz = take(R * c.d * e);
+  y.dO = take(R * c.H * c.Dh * e);
+  y.dqkv = take(R * h->nqkv * e);
+  y.dxh = take(R * c.d * e);
+  y.Dvec = take((size_t)c.H * R * 4);
+  y.dqacc = take(R * c.H * c.Dh * 4);
+  y.part = take((size_t)h->part_blocks * c.d * 4);
+  y.total = off;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
+
+#define LD_CHECK(expr)                      \
+  do {                                      \
+    if ((expr) != cudaSuccess) return LD_ERR_CUDA; \
+  } while (0)
+
+ld_status check_device() {
+  static int ok = -1;
+  if (ok < 0) {
+    int dev = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LD_ERR_CUDA;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    ok = (major == 10 && minor == 3) ? 1 : 0;
+  }
+  return ok ? LD_OK : LD_ERR_UNSUPPORTED;
+}
+
+ld_status check_weights(const Handle* h, const ld_layer_w* W) {
+  if (!W) return LD_ERR_ARG;
+  for (int l = 0; l < h->cfg.L; ++l) {
+    const void* ps[6] = {W[l].w_qkv, W[l].w_o, W[l].w_gu, W[l].w_d, W[l].g1, W[l].g2};
+    for (const void* p : ps)
+      if (!p || !aligned16(p)) return LD_ERR_ARG;
+  }
+  return LD_OK;
+}
+
+GemmArgs gemm_base() {
+  GemmArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.alpha = 1.0f;
+  return a;
+}
+
+// Forward/data-gradient product on the kept rows of layer l:
+// D[M x N] = alpha * A[M x K] B(n, k), M = kept_cnt * S (device-side).
+GemmArgs rows_gemm(const Handle* h, const int* cnt, int N, int K, const void* A, int lda, const void* B, int ldb,
+                   int b_mn) {
+  GemmArgs a = gemm_base();
+  a.M_cnt = cnt;
+  a.M_mul = h->cfg.S;
+  a.M_cap = h->max_rows;
+  a.N = N;
+  a.K = K;
+  a.A = A;
+  a.lda = lda;
+  a.a_mn = 0;
+  a.B = B;
+  a.ldb = ldb;
+  a.b_mn = b_mn;
+  return a;
+}
+
+// Weight-gradient product: dW[M x N] = sum over the kept rows m of
+// X1[m, i] X2[m, j]; the contraction extent is kept_cnt * S (device-side).
+GemmArgs wgrad_gemm(const Handle* h, const int* cnt, int M, int N, const void* X1, int ld1, const void* X2, int ld2,
+                    float* out) {
+  GemmArgs a = gemm_base();
+  a.M = M;
+  a.N = N;
+  a.K_cnt = cnt;
+  a.K_mul = h->cfg.S;
+  a.K_cap = h->max_rows;
+  a.A = X1;
+  a.lda = ld1;
+  a.a_mn = 1;
+  a.B = X2;
+  a.ldb = ld2;
+  a.b_mn = 1;
+  a.epi = EPI_STORE_F32;
+  a.D = out;
+  a.ldd = N;
+  return a;
+}
+
+template <typename T>
+cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
+template <>
+cudaError_t gemm<bf16>(const GemmArgs& a, cudaStream_t st) {
+  return gemm_tc(a, st);
+}
+template <>
+cudaError_t gemm<float>(const GemmArgs& a, cudaStream_t st) {
+  return gemm_simt(a, st);
+}
+
+template <typename T>
+cudaError_t attn_fwd(const Handle* h, const T* qkv, T* o, float* lse, const int* cnt, cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  return launch_attn_fwd_simt<T>(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, h->max_rows, st);
+}
+
+template <typename T>
+cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const T* dO, const float* lse, float* Dvec,
+                     T* dqkv, const int* cnt, cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  cudaError_t e = launch_attn_rowdot<T>(dO, o, c.H * c.Dh, c.H, c.Dh, cnt, c.S, h->max_rows, Dvec, st);
+  if (e != cudaSuccess) return e;
+  return launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, cnt, c.S, c.H, c.Hkv, c.Dh,
+                                 h->max_rows, st);
+}
+
+template <typename T>
+ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv, void* ws, cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  const Layout& y = h->lay;
+  T* x = static_cast<T*>(xv);
+  int* status = at<int>(ws, y.status);
+  unsigned char* mask = at<unsigned char>(ws, y.mask);
+  int* kidx = at<int>(ws, y.kidx);
+  int* kcnt = at<int>(ws, y.kcnt);
+  float* rcos = at<float>(ws, y.rcos);
+  float* rsin = at<float>(ws, y.rsin);
+  (void)status;
+
+  MaskParams P;  // 2 KB kernel parameter, filled on the host
+  P.seed = h->sched.seed;
+  P.step = step;
+  P.L = c.L;
+  P.B = c.B;
+  P.granularity = c.granularity;
+  std::vector<float> scale(c.L);
+  step_rates(h, step, nullptr, P.thr, scale.data());
+  LD_CHECK(launch_mask_compact(P, mask, kidx, kcnt, st));
+  if (c.rope_theta != 0.0f) LD_CHECK(launch_rope_table(rcos, rsin, c.S, c.Dh, (double)c.rope_theta, st));
+
+  const int HD = c.H * c.Dh;
+  for (int l = 0; l < c.L; ++l) {
+    const int* cnt = kcnt + l;
+    const int* ki = kidx + (size_t)l * c.B;
+    char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
+    T* xin = reinterpret_cast<T*>(lb + y.xin);
+    T* xh = reinterpret_cast<T*>(lb + y.xh);
+    T* qkv = reinterpret_cast<T*>(lb + y.qkv);
+    T* o = reinterpret_cast<T*>(lb + y.o);
+    float* lse = reinterpret_cast<float*>(lb + y.lse);
+    T* z = reinterpret_cast<T*>(lb + y.z);
+    T* zh = reinterpret_cast<T*>(lb + y.zh);
+    T* gu = reinterpret_cast<T*>(lb + y.gu);
+    T* hh = reinterpret_cast<T*>(lb + y.h);
+    float* rstd1 = reinterpret_cast<float*>(lb + y.rstd1);
+    float* rstd2 = reinterpret_cast<float*>(lb + y.rstd2);
+    const T* g1 = static_cast<const T*>(W[l].g1);
+    const T* g2 = static_cast<const T*>(W[l].g2);
+    const float s = scale[l];
+
+    LD_CHECK(launch_rmsnorm_fwd<T>(x, 1, ki, cnt, c.S, c.d, h->max_rows, g1, c.eps, xin, xh, rstd1, st));
+    GemmArgs a = rows_gemm(h, cnt, h->nqkv, c.d, xh, c.d, W[l].w_qkv, c.d, 0);
+    a.epi = EPI_STORE;
+    a.D = qkv;
+    a.ldd = h->nqkv;
+    LD_CHECK(gemm<T>(a, st));
+    if (c.rope_theta != 0.0f)
+      LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 0, st));
+    LD_CHECK(attn_fwd<T>(h, qkv, o, lse, cnt, st));
+    a = rows_gemm(h, cnt, c.d, HD, o, HD, W[l].w_o, HD, 0);
+    a.epi = EPI_RESID;
+    a.alpha = s;
+    a.x = x;
+    a.ldx = c.d;
+    a.kept_idx = ki;
+    a.S = c.S;
+    a.save = z;
+    a.ld_save = c.d;
+    LD_CHECK(gemm<T>(a, st));
+    LD_CHECK(launch_rmsnorm_fwd<T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, nullptr, zh, rstd2, st));
+    a = rows_gemm(h, cnt, 2 * c.F, c.d, zh, c.d, W[l].w_gu, c.d, 0);
+    a.epi = EPI_STORE;
+    a.D = gu;
+    a.ldd = 2 * c.F;
+    LD_CHECK(gemm<T>(a, st));
+    LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cnt, c.S, c.F, h->max_rows, st));
+    a = rows_gemm(h, cnt, c.d, c.F, hh, c.F, W[l].w_d, c.F, 0);
+    a.epi = EPI_RESID;
+    a.alpha = s;
+    a.x = x;
+    a.ldx = c.d;
+    a.kept_idx = ki;
+    a.S = c.S;
+    a.save = nullptr;
+    LD_CHECK(gemm<T>(a, st));
+  }
+  h->fwd_scale = scale;
+  return LD_OK;
+}
+
+template <typename T>
+ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G, void* ws, cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  const Layout& y = h->lay;
+  T* dx = static_cast<T*>(dxv);
+  int* kidx = at<int>(ws, y.kidx);
+  int* kcnt = at<int>(ws, y.kcnt);
+  float* rcos = at<float>(ws, y.rcos);
+  float* rsin = at<float>(ws, y.rsin);
+  T* dy = at<T>(ws, y.dy);
+  T* dh = at<T>(ws, y.dh);
+  T* dgu = at<T>(ws, y.dgu);
+  T* dzh = at<T>(ws, y.dzh);
+  T* dz = at<T>(ws, y.dz);
+  T* dO = at<T>(ws, y.dO);
+  T* dqkv = at<T>(ws, y.dqkv);
+  T* dxh = at<T>(ws, y.dxh);
+  float* Dvec = at<float>(ws, y.Dvec);
+  float* part = at<float>(ws, y.part);
+  const int HD = c.H * c.Dh;
+
+  for (int l = c.L - 1; l >= 0; --l) {
+    const int* cnt = kcnt + l;
+    const int* ki = kidx + (size_t)l * c.B;
+    char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
+    T* xin = reinterpret_cast<T*>(lb + y.xin);
+    T* xh = reinterpret_cast<T*>(lb + y.xh);
+    T* qkv = reinterpret_cast<T*>(lb + y.qkv);
+    T* o = reinterpret_cast<T*>(lb + y.o);
+    float* lse = reinterpret_cast<float*>(lb + y.lse);
+    T* z = reinterpret_cast<T*>(lb + y.z);
+    T* zh = reinterpret_cast<T*>(lb + y.zh);
+    T* gu = reinterpret_cast<T*>(lb + y.gu);
+    T* hh = reinterpret_cast<T*>(lb + y.h);
+    float* rstd1 = reinterpret_cast<float*>(lb + y.rstd1);
+    float* rstd2 = reinterpret_cast<float*>(lb + y.rstd2);
+    const T* g1 = static_cast<const T*>(W[l].g1);
+    const T* g2 = static_cast<const T*>(W[l].g2);
+    const float s = h->fwd_scale[l];
+
+    // FFN branch: dy = r * dX^{l+1} on the kept rows.
+    LD_CHECK(launch_gather_scale<T>(dx, ki, cnt, c.S, c.d, h->max_rows, s, dy, st));
+    GemmArgs a = rows_gemm(h, cnt, c.F, c.d, dy, c.d, W[l].w_d, c.F, 1);  // dh = dy W_d
+    a.epi = EPI_STORE;
+    a.D = dh;
+    a.ldd = c.F;
+    LD_CHECK(gemm<T>(a, st));
+    LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cnt, c.S, c.F, h->max_rows, st));
+    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st));  // dW_d = dy^T h
+    a = rows_gemm(h, cnt, c.d, 2 * c.F, dgu, 2 * c.F, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
+    a.epi = EPI_STORE;
+    a.D = dzh;
+    a.ldd = c.d;
+    LD_CHECK(gemm<T>(a, st));
+    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, 2 * c.F, c.d, dgu, 2 * c.F, zh, c.d, G[l].w_gu), st));
+    // dZ = dX^{l+1} + RMSNorm_2 backward; dz = r * dZ for the attention branch
+    LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, ki, cnt, c.S, c.d, h->max_rows, s, dz, part,
+                                   h->part_blocks, st));
+    LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g2, st));
+    // attention branch
+    a = rows_gemm(h, cnt, HD, c.d, dz, c.d, W[l].w_o, HD, 1);  // dO = dz W_o
+    a.epi = EPI_STORE;
+    a.D = dO;
+    a.ldd = HD;
+    LD_CHECK(gemm<T>(a, st));
+    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, HD, dz, c.d, o, HD, G[l].w_o), st));  // dW_o = dz^T o
+    LD_CHECK(attn_bwd<T>(h, ws, qkv, o, dO, lse, Dvec, dqkv, cnt, st));
+    if (c.rope_theta != 0.0f)
+      LD_CHECK(launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1, st));
+    a = rows_gemm(h, cnt, c.d, h->nqkv, dqkv, h->nqkv, W[l].w_qkv, c.d, 1);  // dxh = dqkv W_qkv
+    a.epi = EPI_STORE;
+    a.D = dxh;
+    a.ldd = c.d;
+    LD_CHECK(gemm<T>(a, st));
+    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, h->nqkv, c.d, dqkv, h->nqkv, xh, c.d, G[l].w_qkv), st));
+    // dX^l = dZ + RMSNorm_1 backward
+    LD_CHECK(launch_rmsnorm_bwd<T>(dxh, xin, rstd1, g1, dx, ki, cnt, c.S, c.d, h->max_rows, 1.0f, (T*)nullptr,
+                                   part, h->part_blocks, st));
+    LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g1, st));
+  }
+  return LD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ld_status_str(ld_status s) {
+  switch (s) {
+    case LD_OK: return "ok";
+    case LD_ERR_ARG: return "invalid argument";
+    case LD_ERR_SHAPE: return "unsupported shape";
+    case LD_ERR_STATE: return "call out of order";
+    case LD_ERR_CUDA: return "CUDA error";
+    case LD_ERR_TIMEOUT: return "device-side wait timed out";
+    case LD_ERR_OOM: return "out of host memory";
+    case LD_ERR_UNSUPPORTED: return "unsupported device or build";
+  }
+  return "unknown status";
+}
+
+ld_status ld_create(const ld_config* cfg, void** handle) {
+  if (!cfg || !handle) return LD_ERR_ARG;
+  *handle = nullptr;
+  const ld_config& c = *cfg;
+  if (!finite(c.eps) || !finite(c.alpha) || !finite(c.rope_theta) || c.eps < 0.0f || c.rope_theta < 0.0f)
+    return LD_ERR_ARG;
+  if (c.L < 1 || c.L > LD_MAX_L || c.B < 1 || c.B > LD_MAX_B || c.S < 64 || c.S > 16384 || c.S % 64) return LD_ERR_SHAPE;
+  if (c.d < 64 || c.d % 64 || c.F < 64 || c.F % 64 || c.d > 16384) return LD_ERR_SHAPE;
+  if (c.Dh != 32 && c.Dh != 64 && c.Dh != 128) return LD_ERR_SHAPE;
+  if (c.H < 1 || c.Hkv < 1 || c.H % c.Hkv || (c.H * c.Dh) % 64) return LD_ERR_SHAPE;
+  if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH) return LD_ERR_ARG;
+  if ((long long)c.B * c.S > (1ll << 30)) return LD_ERR_SHAPE;
+  Handle* h = new (std::nothrow) Handle();
+  if (!h) return LD_ERR_OOM;
+  h->cfg = c;
+  h->esz = c.fp32_debug ? 4 : 2;
+  h->max_rows = c.B * c.S;
+  h->nqkv = (c.H + 2 * c.Hkv) * c.Dh;
+  // number of partial-sum blocks of the gain gradient (a launch constant)
+  h->part_blocks = (h->max_rows + 7) / 8;
+  if (h->part_blocks > 2 * 160) h->part_blocks = 2 * 160;
+  make_layout(h);
+  *handle = h;
+  return LD_OK;
+}
+
+ld_status ld_workspace_size(void* handle, size_t* bytes) {
+  if (!handle || !bytes) return LD_ERR_ARG;
+  *bytes = H(handle)->lay.total;
+  return LD_OK;
+}
+
+ld_status ld_set_schedule(void* handle, const ld_schedule* s) {
+  if (!handle || !s) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  if (s->dist < LD_DIST_UNIFORM || s->dist > LD_DIST_EXPLICIT) return LD_ERR_ARG;
+  if (s->time < LD_TIME_CONST || s->time > LD_TIME_RAMP) return LD_ERR_ARG;
+  if (!(s->p_max >= 0.0f && s->p_max <= 1.0f)) return LD_ERR_ARG;
+  if ((s->time == LD_TIME_ITS || s->time == LD_TIME_DTS) && s->T < 2) return LD_ERR_ARG;
+  if (s->time == LD_TIME_RAMP && (s->ramp_t1 <= s->ramp_t0 || !finite(s->ramp_s0) || !finite(s->ramp_s1)))
+    return LD_ERR_ARG;
+  std::vector<float> pe;
+  if (s->dist == LD_DIST_EXPLICIT) {
+    if (!s->p_explicit) return LD_ERR_ARG;
+    pe.assign(s->p_explicit, s->p_explicit + h->cfg.L);
+    for (float v : pe)
+      if (!(v >= 0.0f && v <= 1.0f)) return LD_ERR_ARG;
+  }
+  h->sched = *s;
+  h->sched.p_explicit = nullptr;
+  h->p_expl.swap(pe);
+  h->have_sched = true;
+  return LD_OK;
+}
+
+ld_status ld_get_rates(void* handle, long long step, double* p, unsigned long long* thr, float* scale) {
+  if (!handle) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  if (!h->have_sched) return LD_ERR_STATE;
+  step_rates(h, step, p, thr, scale);
+  return LD_OK;
+}
+
+ld_status ld_draw_masks(void* handle, long long step, void* ws, void* stream) {
+  if (!handle || !ws || !aligned16(ws)) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  if (!h->have_sched) return LD_ERR_STATE;
+  const Layout& y = h->lay;
+  MaskParams P;
+  P.seed = h->sched.seed;
+  P.step = step;
+  P.L = h->cfg.L;
+  P.B = h->cfg.B;
+  P.granularity = h->cfg.granularity;
+  step_rates(h, step, nullptr, P.thr, nullptr);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  LD_CHECK(launch_mask_compact(P, at<unsigned char>(ws, y.mask), at<int>(ws, y.kidx), at<int>(ws, y.kcnt), st));
+  h->last_ws = ws;
+  h->last_stream = st;
+  h->have_masks = true;
+  return LD_OK;
+}
+
+ld_status ld_forward(void* handle, long long step, const ld_layer_w* W, void* x, void* ws, void* stream) {
+  if (!handle || !x || !ws || !aligned16(x) || !aligned16(ws)) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  if (!h->have_sched) return LD_ERR_STATE;
+  ld_status r = check_weights(h, W);
+  if (r != LD_OK) return r;
+  if (!h->cfg.fp32_debug && (r = check_device()) != LD_OK) return r;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  h->fwd_valid = false;
+  r = h->cfg.fp32_debug ? forward_impl<float>(h, step, W, x, ws, st) : forward_impl<bf16>(h, step, W, x, ws, st);
+  h->last_ws = ws;
+  h->last_stream = st;
+  h->have_masks = true;
+  if (r == LD_OK) {
+    h->fwd_valid = true;
+    h->fwd_ws = ws;
+  }
+  return r;
+}
+
+ld_status ld_backward(void* handle, const ld_layer_w* W, void* dx, ld_layer_g* G, void* ws, void* stream) {
+  if (!handle || !dx || !ws || !G || !aligned16(dx)) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  ld_status r = check_weights(h, W);
+  if (r != LD_OK) return r;
+  for (int l = 0; l < h->cfg.L; ++l) {
+    float* ps[6] = {G[l].w_qkv, G[l].w_o, G[l].w_gu, G[l].w_d, G[l].g1, G[l].g2};
+    for (float* p : ps)
+      if (!p || !aligned16(p)) return LD_ERR_ARG;
+  }
+  if (!h->fwd_valid || h->fwd_ws != ws) return LD_ERR_STATE;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  r = h->cfg.fp32_debug ? backward_impl<float>(h, W, dx, G, ws, st) : backward_impl<bf16>(h, W, dx, G, ws, st);
+  h->last_ws = ws;
+  h->last_stream = st;
+  return r;
+}
+
+ld_status ld_get_masks(void* handle, unsigned char* mask, int* kept_idx, int* kept_cnt) {
+  if (!handle) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  if (!h->have_masks) return LD_ERR_STATE;
+  const Layout& y = h->lay;
+  const size_t LB = (size_t)h->cfg.L * h->cfg.B;
+  LD_CHECK(cudaStreamSynchronize(h->last_stream));
+  if (mask) LD_CHECK(cudaMemcpy(mask, at<unsigned char>(h->last_ws, y.mask), LB, cudaMemcpyDeviceToHost));
+  if (kept_idx) LD_CHECK(cudaMemcpy(kept_idx, at<int>(h->last_ws, y.kidx), LB * 4, cudaMemcpyDeviceToHost));
+  if (kept_cnt) LD_CHECK(cudaMemcpy(kept_cnt, at<int>(h->last_ws, y.kcnt), (size_t)h->cfg.L * 4, cudaMemcpyDeviceToHost));
+  return LD_OK;
+}
+
+ld_status ld_sync(void* handle) {
+  if (!handle) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  if (!h->last_ws) return LD_OK;
+  LD_CHECK(cudaStreamSynchronize(h->last_stream));
+  LD_CHECK(cudaGetLastError());
+  int st = 0;
+  int* sw = at<int>(h->last_ws, h->lay.status);
+  LD_CHECK(cudaMemcpy(&st, sw, sizeof(int), cudaMemcpyDeviceToHost));
+  if (st) LD_CHECK(cudaMemset(sw, 0, sizeof(int)));
+  return st ? (ld_status)st : LD_OK;
+}
+
+ld_status ld_destroy(void* handle) {
+  if (!handle) return LD_ERR_ARG;
+  delete H(handle);
+  return LD_OK;
+}
+
+ld_status ld_gemm_bf16(int M, int N, int K, const void* A, int lda, int a_mn, const void* B, int ldb, int b_mn, void* D,
+                       int ldd, int d_f32, float alpha, int* status_ws, void* stream) {
+  if (!A || !B || !D || !aligned16(A) || !aligned16(B) || !aligned16(D)) return LD_ERR_ARG;
+  if (M < 64 || N < 64 || K < 0 || M % 64 || N % 64 || K % 64) return LD_ERR_SHAPE;
+  if (lda % 8 || ldb % 8 || ldd % 8) return LD_ERR_SHAPE;
+  if (lda < (a_mn ? M : K) || ldb < (b_mn ? N : K) || ldd < N) return LD_ERR_SHAPE;
+  ld_status r = check_device();
+  if (r != LD_OK) return r;
+  GemmArgs a = gemm_base();
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  a.A = A;
+  a.lda = lda;
+  a.a_mn = a_mn ? 1 : 0;
+  a.B = B;
+  a.ldb = ldb;
+  a.b_mn = b_mn ? 1 : 0;
+  a.epi = d_f32 ? EPI_STORE_F32 : EPI_STORE;
+  a.D = D;
+  a.ldd = ldd;
+  a.alpha = alpha;
+  a.status = status_ws;
+  LD_CHECK(gemm_tc(a, static_cast<cudaStream_t>(stream)));
+  return LD_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,159 @@
+// Internal declarations shared by the translation units of the library.
+// Not part of the C ABI (include/ld.h is).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/ld.h"
+
+#define LD_MAX_L 256
+#define LD_MAX_B 4096
+
+namespace ldk {
+
+// Element storage: bf16 on the tensor-core path, float on the debug path.
+typedef __nv_bfloat16 bf16;
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+// Device status word: 0 = ok, LD_ERR_TIMEOUT when a bounded wait expired.
+__device__ __forceinline__ void set_status(int* status, int code) {
+  if (status) atomicCAS(status, 0, code);
+}
+
+// Nanosecond wall clock of the GPU (for bounded waits).
+__device__ __forceinline__ uint64_t gtimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Every spin-wait in the library gives up after this long and reports
+// LD_ERR_TIMEOUT through the status word.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+// Row of the residual stream for compact row m of layer l: sequence
+// kept_idx[m / S], position m % S.
+__device__ __forceinline__ long long src_row(const int* kept_idx, int S, long long m) {
+  return (long long)kept_idx[m / S] * S + (m % S);
+}
+
+// ------------------------------------------------------------------------
+// launchers (host side); each returns cudaGetLastError()
+// ------------------------------------------------------------------------
+
+struct MaskParams {
+  unsigned long long seed;
+  long long step;
+  int L, B, granularity;
+  unsigned long long thr[LD_MAX_L];
+};
+cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* kept_idx, int* kept_cnt,
+                                cudaStream_t st);
+
+cudaError_t launch_rope_table(float* cos_t, float* sin_t, int S, int Dh, double theta, cudaStream_t st);
+
+// RMSNorm forward over the rows of layer l (M = *cnt * S rows).  When
+// `gather` is set the source row of compact row m is src_row(kept_idx, S, m),
+// else m.  Writes the normalised rows (out), the reciprocal rms (rstd) and,
+// if copy != null, a compact copy of the source rows.
+template <typename T>
+cudaError_t launch_rmsnorm_fwd(const T* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
+                               int max_rows, const T* gamma, float eps, T* copy, T* out, float* rstd,
+                               cudaStream_t st);
+
+// RMSNorm backward + residual: for compact row m with source row r,
+//   dx[r] += rstd (dyn*g - xn * mean(dyn*g*xn)),  xn = xs[m] * rstd[m]
+// then, if next != null, next[m] = scale * dx[r] (compact, for the next
+// branch).  Partial gain gradients go to part[blockIdx][d]; the number of
+// blocks is returned in *nblocks (a launch constant).
+template <typename T>
+cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, T* dx,
+                               const int* kept_idx, const int* cnt, int S, int d, int max_rows, float scale,
+                               T* next, float* part, int nblocks, cudaStream_t st);
+int rmsnorm_bwd_blocks(int max_rows);
+cudaError_t launch_colsum(const float* part, int nrows, int d, float* out, cudaStream_t st);
+
+template <typename T>
+cudaError_t launch_gather_scale(const T* dx, const int* kept_idx, const int* cnt, int S, int d, int max_rows,
+                                float scale, T* out, cudaStream_t st);
+
+template <typename T>
+cudaError_t launch_rope_apply(T* qkv, int ld, int nheads, int Dh, const float* cos_t, const float* sin_t,
+                              const int* cnt, int S, int max_rows, int inverse, cudaStream_t st);
+
+template <typename T>
+cudaError_t launch_swiglu_fwd(const T* gu, T* h, const int* cnt, int S, int F, int max_rows, cudaStream_t st);
+
+template <typename T>
+cudaError_t launch_swiglu_bwd(const T* dh, const T* gu, T* dgu, const int* cnt, int S, int F, int max_rows,
+                              cudaStream_t st);
+
+template <typename T>
+cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, const int* cnt, int S, int max_rows,
+                               float* Dvec, cudaStream_t st);
+
+// Reference (SIMT) attention, used by the float32 debug path.
+template <typename T>
+cudaError_t launch_attn_fwd_simt(const T* qkv, int ldqkv, T* o, int ldo, float* lse, const int* cnt, int S, int H,
+                                 int Hkv, int Dh, int max_rows, cudaStream_t st);
+template <typename T>
+cudaError_t launch_attn_bwd_simt(const T* qkv, int ldqkv, const T* dO, int ldo, const float* lse, const float* Dvec,
+                                 T* dqkv, const int* cnt, int S, int H, int Hkv, int Dh, int max_rows,
+                                 cudaStream_t st);
+
+// Tensor-core (mma.sync) flash attention for bf16.
+cudaError_t launch_attn_fwd_mma(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S,
+                                int H, int Hkv, int Dh, int max_seqs, cudaStream_t st);
+cudaError_t launch_attn_bwd_mma(const bf16* qkv, int ldqkv, const bf16* o, const bf16* dO, int ldo,
+                                const float* lse, const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt,
+                                int S, int H, int Hkv, int Dh, int max_seqs, cudaStream_t st);
+cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const int* cnt, int S,
+                             int max_rows, cudaStream_t st);
+
+// ------------------------------------------------------------------------
+// GEMM: D(m,n) = alpha * sum_k A(m,k) B(n,k) with a fused epilogue.
+// ------------------------------------------------------------------------
+enum EpiMode { EPI_STORE = 0, EPI_STORE_F32 = 1, EPI_RESID = 2 };
+
+struct GemmArgs {
+  // problem size; a non-null *_cnt makes the extent device-side: (*cnt) * mul
+  int M;
+  const int* M_cnt;
+  int M_mul;
+  int N;
+  int K;
+  const int* K_cnt;
+  int K_mul;
+  int M_cap, K_cap;  // worst-case extents (tensor maps, grid)
+  // operands: A(m,k) = A[m*lda+k] (a_mn=0) or A[k*lda+m] (a_mn=1); same for B(n,k)
+  const void* A;
+  int lda, a_mn;
+  const void* B;
+  int ldb, b_mn;
+  // epilogue
+  int epi;
+  void* D;
+  int ldd;
+  float alpha;
+  // EPI_RESID: x[r] = x[r] + alpha*acc for r = src_row(kept_idx, S, m); save[m] = new x[r]
+  void* x;
+  int ldx;
+  const int* kept_idx;
+  int S;
+  void* save;
+  int ld_save;
+  int* status;
+};
+
+cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st);    // bf16 operands, tcgen05
+cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);  // float operands, SIMT
+int device_sm_count();
+
+}  // namespace ldk

@@ -1,0 +1,86 @@
+// Layer-dropout masks and kept-sequence lists, all layers in one launch.
+//
+// Eq. (layer_dropout_train): M^{l,t} in {0,1}^B ~ Bernoulli(1 - p^{l,t});
+// Tensor Granularity subsection: one draw per sequence, or one per layer
+// and step for the whole batch; Preliminary section: the layer then runs on
+// {b : M[b] = 1} only, which this kernel lists in ascending b.
+//
+// Draw: u = word 0 of Philox4x32-10 (Salmon et al., SC'11) with key
+// (seed lo, seed hi) and counter (b', l, t lo, t hi), b' = b per sequence
+// and 0 per batch.  Sequence b drops layer l iff u < thr_l = floor(p 2^32).
+#include "ld_internal.cuh"
+
+namespace ldk {
+
+// Philox4x32-10 round function and key schedule, from the SC'11 paper:
+// multipliers 0xD2511F53 / 0xCD9E8D57, Weyl increments 0x9E3779B9 /
+// 0xBB67AE85, ten rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k.x += 0x9E3779B9u;
+      k.y += 0xBB67AE85u;
+    }
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+  }
+  return c;
+}
+
+__global__ void mask_compact_kernel(const MaskParams P, unsigned char* __restrict__ mask,
+                                    int* __restrict__ kept_idx, int* __restrict__ kept_cnt) {
+  __shared__ int warp_off[32];
+  __shared__ int base;
+  const int l = blockIdx.x;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const unsigned long long thr = P.thr[l];
+  const uint2 key = make_uint2((uint32_t)P.seed, (uint32_t)(P.seed >> 32));
+  const uint32_t t_lo = (uint32_t)(unsigned long long)P.step, t_hi = (uint32_t)((unsigned long long)P.step >> 32);
+  if (threadIdx.x == 0) base = 0;
+  __syncthreads();
+  for (int b0 = 0; b0 < P.B; b0 += blockDim.x) {
+    const int b = b0 + threadIdx.x;
+    int keep = 0;
+    if (b < P.B) {
+      const uint32_t bb = P.granularity == LD_PER_BATCH ? 0u : (uint32_t)b;
+      const uint32_t u = philox4x32_10(make_uint4(bb, (uint32_t)l, t_lo, t_hi), key).x;
+      keep = (unsigned long long)u >= thr;
+      mask[(size_t)l * P.B + b] = (unsigned char)keep;
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) warp_off[w] = __popc(bal);
+    __syncthreads();
+    if (w == 0) {
+      // exclusive scan of the per-warp counts
+      int v = lane < nw ? warp_off[lane] : 0;
+      int incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      if (lane < nw) warp_off[lane] = incl - v;
+      if (lane == 31) warp_off[31] = incl;  // chunk total (nw <= 31 slots used above)
+    }
+    __syncthreads();
+    if (keep) kept_idx[(size_t)l * P.B + base + warp_off[w] + __popc(bal & ((1u << lane) - 1u))] = b;
+    __syncthreads();
+    if (threadIdx.x == 0) base += warp_off[31];
+    __syncthreads();
+  }
+  for (int i = base + threadIdx.x; i < P.B; i += blockDim.x) kept_idx[(size_t)l * P.B + i] = -1;
+  if (threadIdx.x == 0) kept_cnt[l] = base;
+}
+
+cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* kept_idx, int* kept_cnt,
+                                cudaStream_t st) {
+  // at most 31 warps so that slot 31 of warp_off can hold the chunk total
+  int threads = ((P.B + 31) / 32) * 32;
+  if (threads > 992) threads = 992;
+  mask_compact_kernel<<<P.L, threads, 0, st>>>(P, mask, kept_idx, kept_cnt);
+  return cudaGetLastError();
+}
+
+}  // namespace ldk

@@ -1,0 +1,369 @@
+// Row-wise kernels of the layer (HBM-bound): RMSNorm forward with the
+// kept-row gather, RMSNorm backward with the in-place residual gradient,
+// the scaled gather of the upstream gradient, RoPE, SwiGLU and small
+// reductions.  All of them read the kept count of their layer from device
+// memory and walk compact rows m < kept_cnt * S with a grid-stride loop, so
+// no launch depends on a host-side copy of the masks.
+#include "ld_internal.cuh"
+
+namespace ldk {
+
+// 8 consecutive elements <-> 8 floats (16 bytes of bf16, 32 bytes of float).
+__device__ __forceinline__ void ld8(const bf16* p, float* v) {
+  const uint4 r = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 f = __bfloat1622float2(h[j]);
+    v[2 * j] = f.x;
+    v[2 * j + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void ld8(const float* p, float* v) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0];
+  const float4 b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void st8(bf16* p, const float* v) {
+  uint4 r;
+  __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&r);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) h[j] = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+  *reinterpret_cast<uint4*>(p) = r;
+}
+__device__ __forceinline__ void st8(float* p, const float* v) {
+  reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+// Round to the storage type and back (the value that st8 would store).
+__device__ __forceinline__ float rnd(float v, const bf16*) { return __bfloat162float(__float2bfloat16_rn(v)); }
+__device__ __forceinline__ float rnd(float v, const float*) { return v; }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+static int grid_for(long long work_items, int per_block, int cap) {
+  long long g = (work_items + per_block - 1) / per_block;
+  if (g < 1) g = 1;
+  if (g > cap) g = cap;
+  return (int)g;
+}
+static int g_sms = 0;
+int device_sm_count() {
+  if (!g_sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (g_sms <= 0) g_sms = 148;
+  }
+  return g_sms;
+}
+
+// ---------------------------------------------------------------- RMSNorm fwd
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const T* __restrict__ src, int gather,
+                                                          const int* __restrict__ kept_idx,
+                                                          const int* __restrict__ cnt, int S, int d,
+                                                          const T* __restrict__ gamma, float eps,
+                                                          T* __restrict__ copy, T* __restrict__ out,
+                                                          float* __restrict__ rstd) {
+  const long long M = (long long)(*cnt) * S;
+  const int lane = threadIdx.x & 31;
+  const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
+  for (long long m = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); m < M; m += nwarps) {
+    const long long r = gather ? src_row(kept_idx, S, m) : m;
+    const T* xr = src + r * d;
+    float ss = 0.f;
+    for (int i = lane * 8; i < d; i += 256) {
+      float v[8];
+      ld8(xr + i, v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) ss += v[j] * v[j];
+      if (copy) st8(copy + m * d + i, v);
+    }
+    ss = warp_sum(ss);
+    const float rs = 1.0f / sqrtf(ss / (float)d + eps);
+    if (lane == 0) rstd[m] = rs;
+    for (int i = lane * 8; i < d; i += 256) {
+      float v[8], g[8], o[8];
+      ld8(xr + i, v);
+      ld8(gamma + i, g);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o[j] = (v[j] * rs) * g[j];
+      st8(out + m * d + i, o);
+    }
+  }
+}
+
+template <typename T>
+cudaError_t launch_rmsnorm_fwd(const T* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
+                               int max_rows, const T* gamma, float eps, T* copy, T* out, float* rstd,
+                               cudaStream_t st) {
+  const int grid = grid_for(max_rows, 8, device_sm_count() * 16);
+  rmsnorm_fwd_kernel<T><<<grid, 256, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy, out, rstd);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- RMSNorm bwd
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const T* __restrict__ dyn, const T* __restrict__ xs,
+                                                          const float* __restrict__ rstd,
+                                                          const T* __restrict__ gamma, T* __restrict__ dx,
+                                                          const int* __restrict__ kept_idx,
+                                                          const int* __restrict__ cnt, int S, int d, float scale,
+                                                          T* __restrict__ next, float* __restrict__ part) {
+  extern __shared__ float sg[];  // partial gain gradient of this block, [d]
+  for (int i = threadIdx.x; i < d; i += blockDim.x) sg[i] = 0.f;
+  __syncthreads();
+  const long long M = (long long)(*cnt) * S;
+  const int lane = threadIdx.x & 31;
+  const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
+  for (long long m = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); m < M; m += nwarps) {
+    const long long r = src_row(kept_idx, S, m);
+    const float rs = rstd[m];
+    float dot = 0.f;
+    for (int i = lane * 8; i < d; i += 256) {
+      float dy[8], xv[8], g[8];
+      ld8(dyn + m * d + i, dy);
+      ld8(xs + m * d + i, xv);
+      ld8(gamma + i, g);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float xn = xv[j] * rs;
+        dot += dy[j] * g[j] * xn;
+        atomicAdd(&sg[i + j], dy[j] * xn);
+      }
+    }
+    dot = warp_sum(dot) / (float)d;
+    for (int i = lane * 8; i < d; i += 256) {
+      float dy[8], xv[8], g[8], cur[8], nx[8];
+      ld8(dyn + m * d + i, dy);
+      ld8(xs + m * d + i, xv);
+      ld8(gamma + i, g);
+      ld8(dx + r * d + i, cur);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float xn = xv[j] * rs;
+        cur[j] = cur[j] + rs * (dy[j] * g[j] - xn * dot);
+        nx[j] = scale * rnd(cur[j], dx);
+      }
+      st8(dx + r * d + i, cur);
+      if (next) st8(next + m * d + i, nx);
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < d; i += blockDim.x) part[(size_t)blockIdx.x * d + i] = sg[i];
+}
+
+int rmsnorm_bwd_blocks(int max_rows) { return grid_for(max_rows, 8, device_sm_count() * 2); }
+
+template <typename T>
+cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, T* dx,
+                               const int* kept_idx, const int* cnt, int S, int d, int max_rows, float scale,
+                               T* next, float* part, int nblocks, cudaStream_t st) {
+  const size_t smem = (size_t)d * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(rmsnorm_bwd_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  rmsnorm_bwd_kernel<T><<<nblocks, 256, smem, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next,
+                                                   part);
+  return cudaGetLastError();
+}
+
+__global__ void colsum_kernel(const float* __restrict__ part, int nrows, int d, float* __restrict__ out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= d) return;
+  float s = 0.f;
+  for (int b = 0; b < nrows; ++b) s += part[(size_t)b * d + i];
+  out[i] = s;
+}
+
+cudaError_t launch_colsum(const float* part, int nrows, int d, float* out, cudaStream_t st) {
+  colsum_kernel<<<(d + 255) / 256, 256, 0, st>>>(part, nrows, d, out);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------- scaled gather
+template <typename T>
+__global__ void gather_scale_kernel(const T* __restrict__ dx, const int* __restrict__ kept_idx,
+                                    const int* __restrict__ cnt, int S, int d, float scale, T* __restrict__ out) {
+  const long long M = (long long)(*cnt) * S;
+  const int per_row = d / 8;
+  const long long total = M * per_row;
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
+       w += (long long)gridDim.x * blockDim.x) {
+    const long long m = w / per_row;
+    const int i = (int)(w % per_row) * 8;
+    float v[8];
+    ld8(dx + src_row(kept_idx, S, m) * d + i, v);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] *= scale;
+    st8(out + m * d + i, v);
+  }
+}
+
+template <typename T>
+cudaError_t launch_gather_scale(const T* dx, const int* kept_idx, const int* cnt, int S, int d, int max_rows,
+                                float scale, T* out, cudaStream_t st) {
+  const int grid = grid_for((long long)max_rows * (d / 8), 256, device_sm_count() * 8);
+  gather_scale_kernel<T><<<grid, 256, 0, st>>>(dx, kept_idx, cnt, S, d, scale, out);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------- RoPE
+// cos/sin of pos * theta^(-2i/Dh), angles formed in double precision.
+__global__ void rope_table_kernel(float* cos_t, float* sin_t, int S, int Dh, double theta) {
+  const int half = Dh / 2;
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= S * half) return;
+  const int pos = idx / half, i = idx % half;
+  const double ang = (double)pos * pow(theta, -(2.0 * i) / (double)Dh);
+  double s, c;
+  sincos(ang, &s, &c);
+  cos_t[idx] = (float)c;
+  sin_t[idx] = (float)s;
+}
+
+cudaError_t launch_rope_table(float* cos_t, float* sin_t, int S, int Dh, double theta, cudaStream_t st) {
+  const int n = S * (Dh / 2);
+  rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(cos_t, sin_t, S, Dh, theta);
+  return cudaGetLastError();
+}
+
+// Rotate pairs (i, i+Dh/2) of the first `nheads` heads of each row, at the
+// row's position in its sequence; inverse = 1 applies the transpose.
+template <typename T>
+__global__ void rope_apply_kernel(T* __restrict__ qkv, int ld, int nheads, int Dh, const float* __restrict__ cos_t,
+                                  const float* __restrict__ sin_t, const int* __restrict__ cnt, int S,
+                                  int inverse) {
+  const long long M = (long long)(*cnt) * S;
+  const int half = Dh / 2;
+  const long long per_row = (long long)nheads * half;
+  const long long total = M * per_row;
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
+       w += (long long)gridDim.x * blockDim.x) {
+    const long long m = w / per_row;
+    const int rem = (int)(w % per_row);
+    const int h = rem / half, i = rem % half;
+    const int pos = (int)(m % S);
+    const float c = cos_t[pos * half + i], s = sin_t[pos * half + i];
+    T* p = qkv + m * ld + (long long)h * Dh;
+    const float a = to_f(p[i]), b = to_f(p[i + half]);
+    float na, nb;
+    if (!inverse) {
+      na = a * c - b * s;
+      nb = b * c + a * s;
+    } else {
+      na = a * c + b * s;
+      nb = b * c - a * s;
+    }
+    p[i] = from_f<T>(na);
+    p[i + half] = from_f<T>(nb);
+  }
+}
+
+template <typename T>
+cudaError_t launch_rope_apply(T* qkv, int ld, int nheads, int Dh, const float* cos_t, const float* sin_t,
+                              const int* cnt, int S, int max_rows, int inverse, cudaStream_t st) {
+  const int grid = grid_for((long long)max_rows * nheads * (Dh / 2), 256, device_sm_count() * 8);
+  rope_apply_kernel<T><<<grid, 256, 0, st>>>(qkv, ld, nheads, Dh, cos_t, sin_t, cnt, S, inverse);
+  return cudaGetLastError();
+}
+
+// -------------------------------------------------------------------- SwiGLU
+__device__ __forceinline__ float sigmoidf_(float g) { return 1.0f / (1.0f + expf(-g)); }
+
+template <typename T>
+__global__ void swiglu_fwd_kernel(const T* __restrict__ gu, T* __restrict__ h, const int* __restrict__ cnt, int S,
+                                  int F) {
+  const long long M = (long long)(*cnt) * S;
+  const long long total = M * F;
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
+       w += (long long)gridDim.x * blockDim.x) {
+    const long long m = w / F;
+    const int j = (int)(w % F);
+    const float g = to_f(gu[m * 2 * F + j]), u = to_f(gu[m * 2 * F + F + j]);
+    h[w] = from_f<T>(g * sigmoidf_(g) * u);
+  }
+}
+
+template <typename T>
+cudaError_t launch_swiglu_fwd(const T* gu, T* h, const int* cnt, int S, int F, int max_rows, cudaStream_t st) {
+  const int grid = grid_for((long long)max_rows * F, 256, device_sm_count() * 8);
+  swiglu_fwd_kernel<T><<<grid, 256, 0, st>>>(gu, h, cnt, S, F);
+  return cudaGetLastError();
+}
+
+template <typename T>
+__global__ void swiglu_bwd_kernel(const T* __restrict__ dh, const T* __restrict__ gu, T* __restrict__ dgu,
+                                  const int* __restrict__ cnt, int S, int F) {
+  const long long M = (long long)(*cnt) * S;
+  const long long total = M * F;
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
+       w += (long long)gridDim.x * blockDim.x) {
+    const long long m = w / F;
+    const int j = (int)(w % F);
+    const float g = to_f(gu[m * 2 * F + j]), u = to_f(gu[m * 2 * F + F + j]);
+    const float sg = sigmoidf_(g), dv = to_f(dh[w]);
+    dgu[m * 2 * F + j] = from_f<T>(dv * u * sg * (1.0f + g * (1.0f - sg)));
+    dgu[m * 2 * F + F + j] = from_f<T>(dv * g * sg);
+  }
+}
+
+template <typename T>
+cudaError_t launch_swiglu_bwd(const T* dh, const T* gu, T* dgu, const int* cnt, int S, int F, int max_rows,
+                              cudaStream_t st) {
+  const int grid = grid_for((long long)max_rows * F, 256, device_sm_count() * 8);
+  swiglu_bwd_kernel<T><<<grid, 256, 0, st>>>(dh, gu, dgu, cnt, S, F);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------- attention backward preprocess
+// Dvec[h][m] = sum_i dO[m, h*Dh+i] * O[m, h*Dh+i]  (row sum of dP * P).
+template <typename T>
+__global__ void attn_rowdot_kernel(const T* __restrict__ dO, const T* __restrict__ O, int ld, int H, int Dh,
+                                   const int* __restrict__ cnt, int S, int max_rows, float* __restrict__ Dvec) {
+  const long long M = (long long)(*cnt) * S;
+  const int lane = threadIdx.x & 31;
+  const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
+  for (long long it = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); it < M * H; it += nwarps) {
+    const long long m = it / H;
+    const int h = (int)(it % H);
+    float s = 0.f;
+    for (int i = lane; i < Dh; i += 32) s += to_f(dO[m * ld + h * Dh + i]) * to_f(O[m * ld + h * Dh + i]);
+    s = warp_sum(s);
+    if (lane == 0) Dvec[(size_t)h * max_rows + m] = s;
+  }
+}
+
+template <typename T>
+cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, const int* cnt, int S, int max_rows,
+                               float* Dvec, cudaStream_t st) {
+  const int grid = grid_for((long long)max_rows * H, 8, device_sm_count() * 16);
+  attn_rowdot_kernel<T><<<grid, 256, 0, st>>>(dO, O, ld, H, Dh, cnt, S, max_rows, Dvec);
+  return cudaGetLastError();
+}
+
+#define LD_INST(T)                                                                                              \
+  template cudaError_t launch_rmsnorm_fwd<T>(const T*, int, const int*, const int*, int, int, int, const T*,    \
+                                             float, T*, T*, float*, cudaStream_t);                              \
+  template cudaError_t launch_rmsnorm_bwd<T>(const T*, const T*, const float*, const T*, T*, const int*,        \
+                                             const int*, int, int, int, float, T*, float*, int, cudaStream_t);  \
+  template cudaError_t launch_gather_scale<T>(const T*, const int*, const int*, int, int, int, float, T*,        \
+                                              cudaStream_t);                                                    \
+  template cudaError_t launch_rope_apply<T>(T*, int, int, int, const float*, const float*, const int*, int, int, \
+                                            int, cudaStream_t);                                                 \
+  template cudaError_t launch_swiglu_fwd<T>(const T*, T*, const int*, int, int, int, cudaStream_t);             \
+  template cudaError_t launch_swiglu_bwd<T>(const T*, const T*, T*, const int*, int, int, int, cudaStream_t);   \
+  template cudaError_t launch_attn_rowdot<T>(const T*, const T*, int, int, int, const int*, int, int, float*,   \
+                                             cudaStream_t);
+LD_INST(float)
+LD_INST(bf16)
+
+}  // namespace ldk
