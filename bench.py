@@ -1,0 +1,437 @@
+#!/usr/bin/env python3
+"""Throughput of the layer-dropout decoder stack, forward + backward, on GB300.
+
+One step = ld_forward + ld_backward of the whole stack (every layer: mask
+draw, kept-row RMSNorm, QKV + RoPE, causal GQA attention, O projection with
+the 1/(1-p) residual update, RMSNorm, SwiGLU, down projection, and the
+mirrored backward) over one batch of synthetic activations, through the C ABI.
+
+Default workload: the Llama-3-8B-shaped stack (32 layers, d 4096, 32 query /
+8 key-value heads of 128, SwiGLU 14336, 4 x 4096 tokens, ILD p_max 0.4,
+per-sequence masks).  Reported:
+  value          effective tokens/s = B*S / step time (inputs resident in HBM)
+  e2e            the same with the step's inputs copied host->device from
+                 pinned memory and dX copied back, inside the timed region
+  pct_bf16_peak  executed FLOPs / time / measured bf16 peak (sustained)
+  skip_speedup   t(p=0) / t(p), next to the ideal 1/(1 - p_bar)
+  roofline       the tcgen05 GEMM class (the dominant kernel), timed with CUDA
+                 events around its launches inside the timed region
+  cpu_baseline   the CPU oracle on a bounded sample of the same workload
+
+--impl reference times the CPU oracle alone (this workload has no runnable
+reference implementation; the oracle is the reference arm).
+Multi-GPU (torchrun): replicas only, one batch per rank, no collective on
+the data path (weak scaling).
+"""
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "effective tokens/s (fwd+bwd) under layer dropout; % bf16 peak; skip-speedup vs ideal"
+PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
+
+
+def load_peaks():
+    try:
+        with open(PEAKS) as f:
+            p = json.load(f)
+        return dict(bf16=p["bf16_tflops"], bf16_sustained=p["bf16_tflops_sustained"], hbm=p["hbm_gbs"],
+                    source="measured")
+    except Exception:
+        return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
+
+
+def flops_per_token(cfg):
+    """Forward FLOPs per token per layer (2 x MACs; causal attention counted
+    as S/2 keys per query) and the part of it in the projections."""
+    d, H, Hkv, Dh, F, S = cfg["d"], cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"], cfg["S"]
+    proj = 2 * d * (H + 2 * Hkv) * Dh + 2 * d * H * Dh + 6 * d * F
+    attn = 2 * H * Dh * S
+    return proj + attn, proj
+
+
+def max_over_ranks(ms, world, device="cuda"):
+    """Step time of the whole job: the slowest rank's."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+class Clocks:
+    """nvidia-smi clock/throttle sampling while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                rows.append((float(f[1]), float(f[2]), f[5], f[6], f[7], f[8]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[2 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def cpu_baseline(cfg, host_w0, x_seq, dy_seq, rows, kept_units_per_step, s_l0):
+    """The oracle (float64 numpy) on a bounded sample: layer 0, sequence 0,
+    its first `rows` rows, forward + backward.  Extrapolated to a step by the
+    kept tokens of the step (every kept (layer, sequence) processes S rows)."""
+    import numpy as np
+    from oracle import stack as OK
+
+    W = {n: v.double().numpy() for n, v in host_w0.items()}
+    x = x_seq[:rows].double().numpy()
+    dy = dy_seq[:rows].double().numpy()
+    rope = OK._rope_cs(cfg, rows)
+    t0 = time.perf_counter()
+    out, cache = OK.layer_forward(x, W, cfg, s_l0, rope)
+    G = {n: np.zeros(OK.shape_of(cfg, n)) for n in OK.WEIGHT_NAMES}
+    OK.layer_backward(dy, W, cfg, s_l0, cache, G, rope)
+    dt = time.perf_counter() - t0
+    per_token = dt / rows
+    step_time = per_token * kept_units_per_step * cfg["S"]
+    return {"value": cfg["B"] * cfg["S"] / step_time, "unit": "tokens/s", "cores": os.cpu_count(),
+            "kind": "oracle", "sample": f"layer 0, sequence 0, rows 0..{rows - 1} of {cfg['S']}, fwd+bwd, float64 "
+            f"numpy ({dt:.1f} s); extrapolated by the step's kept tokens (attention cost of later rows "
+            f"under-represented, so the CPU figure is optimistic)", "sample_seconds": dt}
+
+
+def run_reference(args):
+    import torch
+    from paper_2609_05275_gb300 import synth
+    from oracle import masks as OM, schedule as OS
+
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    cfg, sched = synth.CONFIGS[args.config], synth.SCHEDULES[args.config]
+    rows = args.cpu_rows
+    w0 = synth.layer_weights(cfg, 0, seed=0)
+    x = synth.activations(cfg, seed=0, B=1)[0]
+    dy = synth.upstream_grad(cfg, B=1)[0]
+    osched = dict(dist=sched["dist"], p_max=sched.get("p_max", 0.0), p_explicit=sched.get("p_explicit"),
+                  time=sched.get("time", "const"), T=sched.get("T"), ramp=sched.get("ramp"))
+    times, units = [], []
+    for k in range(args.warmup + args.steps):
+        t = k
+        rates = OS.layer_rates(osched, cfg["L"], t)
+        mk = OM.draw_masks(sched["seed"], t, [OS.drop_threshold(p) for p in rates], cfg["B"])
+        r = cpu_baseline(cfg, w0, x, dy, rows, int(mk.sum()), OS.residual_scale(rates[0]))
+        if k >= args.warmup:
+            times.append(cfg["B"] * cfg["S"] / r["value"])
+            units.append(int(mk.sum()))
+    step = sum(times) / len(times)
+    value = cfg["B"] * cfg["S"] / step
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.config, **{k: cfg[k] for k in ("L", "d", "H", "Hkv", "Dh", "F", "B", "S")},
+                       "schedule": sched},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": f"per step: layer 0, sequence 0, rows 0..{rows - 1}, fwd+bwd, extrapolated "
+                                       f"by the step's kept tokens"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_sweep(args):
+    """Throughput against the ideal 1/(1 - p_bar) over the sweep grid: for
+    every (p_max, distribution, granularity) cell, one timed step per seed at
+    step 0 (after one warm-up step), CUDA events around each step."""
+    import torch
+
+    import paper_2609_05275_gb300 as P
+    from paper_2609_05275_gb300 import synth
+
+    sw = synth.SWEEP
+    cfg = dict(synth.CONFIGS[sw["base"]])
+    L, B, S = cfg["L"], cfg["B"], cfg["S"]
+    layers = synth.stack_weights(cfg, seed=0, device="cuda")
+    wtab = P.weight_table(layers)
+    grads = [{n: torch.empty(v.shape, device="cuda", dtype=torch.float32) for n, v in W.items()} for W in layers]
+    gtab = P.grad_table(grads)
+    x0 = synth.activations(cfg, seed=0, device="cuda")
+    dy0 = synth.upstream_grad(cfg, device="cuda")
+    x, dx = torch.empty_like(x0), torch.empty_like(dy0)
+    f_tok, _ = flops_per_token(cfg)
+    stacks = {g: P.LayerDropStack(cfg, dict(dist="uniform", p_max=0.0, seed=1), granularity=g)
+              for g in sw["granularity"]}
+    seeds = sw["seeds"][: args.steps] if args.steps < len(sw["seeds"]) else sw["seeds"]
+
+    def step(st, t):
+        x.copy_(x0)
+        dx.copy_(dy0)
+        st.forward(t, wtab, x)
+        st.backward(wtab, dx, gtab)
+
+    def time_cell(st, sched):
+        ms, kept = [], []
+        for seed in seeds:
+            st.schedule = P.make_schedule(dict(sched, seed=seed))
+            P.ld_set_schedule(st.h, st.schedule)
+            step(st, 0)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            step(st, 0)
+            e1.record()
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+            kept.append(int(st.masks()[2].sum()))
+        return ms, kept
+
+    dense_ms, _ = time_cell(stacks["per_sequence"], dict(dist="uniform", p_max=0.0, time="const"))
+    t_dense = statistics.median(dense_ms)
+    cells = []
+    for gran in sw["granularity"]:
+        for dist in sw["dist"]:
+            for p_max in sw["p_max"]:
+                sched = dict(dist=dist, p_max=p_max, time="const")
+                ms, kept = time_cell(stacks[gran], sched)
+                p_real = 1.0 - sum(kept) / (len(kept) * L * B)
+                t = sum(ms) / len(ms)
+                speed = t_dense / t
+                ideal = 1.0 / (1.0 - p_real)
+                cell = {"granularity": gran, "dist": dist, "p_max": p_max, "seeds": len(seeds),
+                        "ms_per_step": t, "tokens_per_s": B * S / (t / 1e3),
+                        "executed_tflops": 3.0 * f_tok * S * sum(kept) / len(kept) / (t / 1e3) / 1e12,
+                        "p_bar_realized": p_real, "speedup": speed, "ideal_speedup": ideal,
+                        "frac_of_ideal": speed / ideal}
+                cells.append(cell)
+                print(json.dumps({"sweep_cell": cell}), flush=True)
+    for st in stacks.values():
+        st.close()
+    print(json.dumps({"sweep": sw["base"], "dense_ms_per_step": t_dense,
+                      "min_frac_of_ideal": min(c["frac_of_ideal"] for c in cells if c["p_max"] > 0),
+                      "mean_frac_of_ideal": statistics.mean(c["frac_of_ideal"] for c in cells if c["p_max"] > 0)}),
+          flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="llama8b")
+    ap.add_argument("--step0", type=int, default=None, help="first step index (default: the workload's)")
+    ap.add_argument("--no-dense", action="store_true", help="skip the p=0 run (no skip_speedup)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-rows", type=int, default=1024)
+    ap.add_argument("--layers", type=int, default=None, help="override L (profiling captures only)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="drop-rate / distribution / granularity / seed sweep on the 1.3B shape (one JSON line "
+                         "per cell, then a summary line)")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
+
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_05275_gb300 as P
+    from paper_2609_05275_gb300 import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    cfg, sched = dict(synth.CONFIGS[args.config]), dict(synth.SCHEDULES[args.config])
+    if args.layers:
+        cfg["L"] = args.layers
+    L, B, S, d = cfg["L"], cfg["B"], cfg["S"], cfg["d"]
+    step0 = args.step0 if args.step0 is not None else synth.STEPS[args.config][-1]
+    peaks = load_peaks()
+
+    st = P.LayerDropStack(cfg, sched)
+    layers = synth.stack_weights(cfg, seed=0, device="cuda")
+    wtab = P.weight_table(layers)
+    grads = [{n: torch.empty(v.shape, device="cuda", dtype=torch.float32) for n, v in W.items()} for W in layers]
+    gtab = P.grad_table(grads)
+    x0 = synth.activations(cfg, seed=rank, device="cuda")
+    dy0 = synth.upstream_grad(cfg, seed=2 + 1000 * rank, device="cuda")
+    x = torch.empty_like(x0)
+    dx = torch.empty_like(dy0)
+    stream = torch.cuda.current_stream()
+
+    def step(t):
+        x.copy_(x0)
+        dx.copy_(dy0)
+        st.forward(t, wtab, x)
+        st.backward(wtab, dx, gtab)
+
+    def timed(nsteps, first, fn):
+        barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for k in range(nsteps):
+            fn(first + k)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        return max_over_ranks(e0.elapsed_time(e1) / nsteps, world)
+
+    # ---- main timed region (p as scheduled)
+    for k in range(args.warmup):
+        step(step0 + k)
+    st.sync()
+    P.ld_set_timing(st.h, 1)
+    clocks = Clocks(local)
+    clocks.start()
+    ms = timed(args.steps, step0 + args.warmup, step)
+    clk = clocks.stop()
+    gemm_ms, gemm_launches = P.ld_get_timing(st.h, P.LD_KCLASS_GEMM)
+    attn_ms, attn_launches = P.ld_get_timing(st.h, P.LD_KCLASS_ATTN)
+    row_ms, row_launches = P.ld_get_timing(st.h, P.LD_KCLASS_ROWWISE)
+    P.ld_set_timing(st.h, 0)
+    st.sync()
+
+    # kept counts of the timed steps (masks redrawn through the library)
+    kept = []
+    for k in range(args.steps):
+        _, _, cnt = st.draw_masks(step0 + args.warmup + k)
+        kept.append([int(c) for c in cnt])
+    f_tok, f_proj = flops_per_token(cfg)
+    kept_units = sum(sum(c) for c in kept)
+    exec_flops = 3.0 * f_tok * S * kept_units / args.steps  # per step, this rank
+    gemm_flops = 3.0 * f_proj * S * kept_units / args.steps
+    p_real = 1.0 - kept_units / (args.steps * L * B)
+    _, thr, _ = st.rates(step0 + args.warmup)
+    p_exp = sum(t / 2 ** 32 for t in thr) / L
+    tflops = exec_flops / (ms / 1e3) / 1e12
+
+    # ---- dense reference point (p = 0 everywhere, same shapes)
+    dense_ms = None
+    if not args.no_dense:
+        st.schedule = P.make_schedule(dict(dist="uniform", p_max=0.0, time="const", seed=sched["seed"]))
+        P.ld_set_schedule(st.h, st.schedule)
+        step(0)
+        dense_ms = timed(args.steps, 0, step)
+        P.ld_set_schedule(st.h, P.make_schedule(sched))
+
+    # ---- end to end: host inputs in pinned memory, dX read back every step
+    e2e = None
+    if not args.no_e2e:
+        xh = x0.cpu().pin_memory()
+        dyh = dy0.cpu().pin_memory()
+        dxh = torch.empty(dx.shape, dtype=dx.dtype).pin_memory()
+
+        def step_e2e(t):
+            x.copy_(xh, non_blocking=True)
+            dx.copy_(dyh, non_blocking=True)
+            st.forward(t, wtab, x)
+            st.backward(wtab, dx, gtab)
+            dxh.copy_(dx, non_blocking=True)
+
+        step_e2e(step0)
+        e2e_ms = timed(args.steps, step0 + args.warmup, step_e2e)
+        nb = x.numel() * x.element_size()
+        e2e = {"value": world * B * S / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": 2 * nb,
+               "d2h_bytes_per_step": nb, "ms_per_step": e2e_ms}
+    st.sync()
+
+    # ---- CPU oracle on a bounded sample (rank 0, one GPU only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        w0 = {n: v.cpu() for n, v in layers[0].items()}
+        _, _, sc = st.rates(step0 + args.warmup)
+        cpu = cpu_baseline(cfg, w0, x0[0].cpu(), dy0[0].cpu(), min(args.cpu_rows, S), kept_units / args.steps, sc[0])
+
+    gemm_achieved = gemm_flops * args.steps / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
+    roof = {"kernel": "gemm_tc_kernel (tcgen05 projections, fwd dgrad wgrad)", "bound": "tensor",
+            "achieved": gemm_achieved, "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
+            "frac": gemm_achieved / peaks["bf16_sustained"] if gemm_achieved else None, "traffic": None,
+            "peak_kind": f"bf16 sustained ({peaks['source']})", "launches_per_step": gemm_launches / args.steps,
+            "avg_launch_ms": gemm_ms / max(gemm_launches, 1)}
+    line = {
+        "metric": METRIC, "value": world * B * S / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.config, **{k: cfg[k] for k in ("L", "d", "H", "Hkv", "Dh", "F", "B", "S")},
+                   "schedule": sched, "granularity": "per_sequence", "first_step": step0 + args.warmup,
+                   "parallelism": f"replicas x{world}", "l2": "inputs and weights larger than L2 (no flush)"},
+        "executed_tflops": tflops, "pct_bf16_peak": 100.0 * tflops / peaks["bf16"],
+        "pct_bf16_peak_sustained": 100.0 * tflops / peaks["bf16_sustained"],
+        "p_bar_expected": p_exp, "p_bar_realized": p_real,
+        "skip_speedup": (dense_ms / ms) if dense_ms else None,
+        "ideal_speedup": 1.0 / (1.0 - p_real), "dense_ms_per_step": dense_ms,
+        "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "attention": attn_ms / args.steps,
+                               "rowwise": row_ms / args.steps},
+        "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+        "gpu_launches": None,
+    }
+    # kernels of this library launched in the timed region: per step the mask
+    # kernel and the RoPE table, then per layer 4 GEMMs + attention + 4
+    # row-wise kernels forward, 8 GEMMs + 3 attention kernels + 7 row-wise
+    # kernels backward (RoPE kernels drop out when theta = 0)
+    rope = 1 if cfg.get("rope_theta") else 0
+    line["gpu_launches"] = args.steps * (1 + rope + L * (4 + 1 + 3 + rope + 8 + 3 + 6 + rope))
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    st.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

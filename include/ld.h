@@ -90,6 +90,9 @@ typedef struct {
                        alpha / (1 - p)                                    */
   int granularity;  /* ld_granularity                                     */
   int fp32_debug;   /* 1: float32 storage and SIMT float32 kernels        */
+  int b_offset;     /* global index of this batch's sequence 0 (data-
+                       parallel shards draw the masks of their global
+                       sequences; 0 for an unsharded batch)               */
 } ld_config;
 
 typedef struct {
@@ -138,13 +141,16 @@ ld_status ld_get_rates(void* handle, long long step, double* p, unsigned long lo
 /* Draw the masks of step t into the workspace (the first kernel of
  * ld_forward, alone).  Philox4x32-10 (Salmon et al., SC'11): key = (seed
  * low 32 bits, seed high 32 bits), counter = (b', l, t low, t high) with
- * b' = b per sequence and b' = 0 per batch; word 0 is u.  Kept lists are
- * ascending in b. */
+ * b' = b_offset + b per sequence and b' = 0 per batch; word 0 is u.  Kept
+ * lists are ascending in b (local indices). */
 ld_status ld_draw_masks(void* handle, long long step, void* workspace, void* stream);
 
 /* Forward of step t, in place on x [B*S, d] (sequence b = rows b*S..b*S+S-1).
- * W points to L host structs of device pointers.  Rows of dropped sequences
- * are not touched.  Saves what the backward needs in `workspace`. */
+ * W points to L host structs of device pointers.  On the bf16 path the
+ * residual stream is carried in a float32 workspace buffer between the
+ * layers (x is read once at the start and written once at the end); rows of
+ * sequences dropped at every layer come back bit for bit.  Saves what the
+ * backward needs in `workspace` and clears the workspace status word. */
 ld_status ld_forward(void* handle, long long step, const ld_layer_w* W, void* x, void* workspace,
                      void* stream);
 
@@ -163,7 +169,8 @@ ld_status ld_backward(void* handle, const ld_layer_w* W, void* dx, ld_layer_g* G
 ld_status ld_get_masks(void* handle, unsigned char* mask, int* kept_idx, int* kept_cnt);
 
 /* Synchronise the stream of the last call and return the device status word
- * (LD_OK or LD_ERR_TIMEOUT), clearing it. */
+ * (LD_OK or LD_ERR_TIMEOUT) accumulated since the last ld_forward /
+ * ld_draw_masks on that workspace, clearing it. */
 ld_status ld_sync(void* handle);
 
 /* Release the handle (host memory only). */
@@ -171,6 +178,26 @@ ld_status ld_destroy(void* handle);
 
 /* Static description of a status code. */
 const char* ld_status_str(ld_status status);
+
+/* Kernel classes of the device-time accounting below. */
+typedef enum {
+  LD_KCLASS_GEMM = 0,    /* tcgen05 (or debug SIMT) projections and their gradients */
+  LD_KCLASS_ATTN = 1,    /* causal GQA attention, forward and backward              */
+  LD_KCLASS_ROWWISE = 2, /* RMSNorm, gathers, RoPE, SwiGLU, reductions              */
+  LD_KCLASS_COUNT = 3
+} ld_kclass;
+
+/* Device-time accounting (not in the paper; instrumentation for the
+ * roofline of each kernel class).  enable = 1 starts recording a CUDA event
+ * pair on the call's stream around every launch of ld_forward / ld_backward
+ * and resets the totals; enable = 0 stops recording.  The events add no
+ * synchronisation. */
+ld_status ld_set_timing(void* handle, int enable);
+
+/* Sum of the device time (ms) and number of launch groups of class `kclass`
+ * recorded since the last ld_set_timing(handle, 1).  Waits for the recorded
+ * events to complete. */
+ld_status ld_get_timing(void* handle, int kclass, double* ms, long long* launches);
 
 /* Dense contraction used by every projection of the block (the linear maps
  * inside f_attn and f_ffn), exposed for testing and reuse:

@@ -33,13 +33,14 @@ def mask_word(seed, step, layer, b):
     return philox4x32_10(ctr, key)[0]
 
 
-def draw_masks(seed, step, thresholds, B, granularity=PER_SEQUENCE):
-    """mask[l][b] in {0,1} (1 = keep) for every layer l (uint8, shape [L, B])."""
+def draw_masks(seed, step, thresholds, B, granularity=PER_SEQUENCE, b_offset=0):
+    """mask[l][b] in {0,1} (1 = keep) for every layer l (uint8, shape [L, B]);
+    the batch holds the global sequences b_offset .. b_offset + B - 1."""
     L = len(thresholds)
     mask = np.zeros((L, B), dtype=np.uint8)
     for layer in range(L):
         for b in range(B):
-            bb = b if granularity == PER_SEQUENCE else 0
+            bb = b_offset + b if granularity == PER_SEQUENCE else 0
             u = mask_word(seed, step, layer, bb)
             mask[layer, b] = 0 if u < thresholds[layer] else 1
     return mask

@@ -33,7 +33,7 @@ GRAN = {"per_sequence": LD_PER_SEQUENCE, "per_batch": LD_PER_BATCH}
 class ld_config(ctypes.Structure):
     _fields_ = [("L", c_int), ("d", c_int), ("H", c_int), ("Hkv", c_int), ("Dh", c_int), ("F", c_int),
                 ("B", c_int), ("S", c_int), ("eps", c_float), ("rope_theta", c_float), ("alpha", c_float),
-                ("granularity", c_int), ("fp32_debug", c_int)]
+                ("granularity", c_int), ("fp32_debug", c_int), ("b_offset", c_int)]
 
 
 class ld_schedule(ctypes.Structure):
@@ -82,6 +82,8 @@ def lib():
             "ld_sync": (c_int, [c_void_p]),
             "ld_destroy": (c_int, [c_void_p]),
             "ld_status_str": (c_char_p, [c_int]),
+            "ld_set_timing": (c_int, [c_void_p, c_int]),
+            "ld_get_timing": (c_int, [c_void_p, c_int, POINTER(c_double), POINTER(c_longlong)]),
             "ld_gemm_bf16": (c_int, [c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_int, c_void_p,
                                      c_int, c_int, c_float, c_void_p, c_void_p]),
         }
@@ -120,10 +122,11 @@ def ld_status_str(status):
     return lib().ld_status_str(int(status)).decode()
 
 
-def make_config(cfg, granularity="per_sequence", fp32_debug=False):
+def make_config(cfg, granularity="per_sequence", fp32_debug=False, b_offset=0):
     return ld_config(cfg["L"], cfg["d"], cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"], cfg["B"], cfg["S"],
                      cfg.get("eps", 1e-6), cfg.get("rope_theta", 0.0), cfg.get("alpha", 1.0),
-                     GRAN[granularity] if isinstance(granularity, str) else int(granularity), int(fp32_debug))
+                     GRAN[granularity] if isinstance(granularity, str) else int(granularity), int(fp32_debug),
+                     int(b_offset))
 
 
 def ld_create(config):
@@ -204,6 +207,20 @@ def ld_destroy(h):
     _check(lib().ld_destroy(h), "ld_destroy")
 
 
+LD_KCLASS_GEMM, LD_KCLASS_ATTN, LD_KCLASS_ROWWISE = 0, 1, 2
+
+
+def ld_set_timing(h, enable):
+    _check(lib().ld_set_timing(h, int(enable)), "ld_set_timing")
+
+
+def ld_get_timing(h, kclass):
+    ms = c_double()
+    n = c_longlong()
+    _check(lib().ld_get_timing(h, kclass, ctypes.byref(ms), ctypes.byref(n)), "ld_get_timing")
+    return ms.value, n.value
+
+
 def ld_gemm_bf16(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, alpha=1.0, status=None, stream=None):
     import torch
     d_f32 = 1 if D.dtype == torch.float32 else 0
@@ -233,10 +250,10 @@ def grad_table(grads):
 class LayerDropStack:
     """A handle with its workspace: forward / backward of the whole stack."""
 
-    def __init__(self, cfg, sched, granularity="per_sequence", fp32_debug=False, device="cuda"):
+    def __init__(self, cfg, sched, granularity="per_sequence", fp32_debug=False, device="cuda", b_offset=0):
         import torch
         self.cfg = dict(cfg)
-        self.config = make_config(cfg, granularity, fp32_debug)
+        self.config = make_config(cfg, granularity, fp32_debug, b_offset)
         self.h = ld_create(self.config)
         self.schedule = make_schedule(sched)
         ld_set_schedule(self.h, self.schedule)

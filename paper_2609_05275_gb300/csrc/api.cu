@@ -31,6 +31,7 @@ struct Layout {
   size_t layer0, per_layer;
   size_t xin, xh, qkv, o, lse, z, zh, gu, h, rstd1, rstd2;  // offsets inside a layer block
   size_t dy, dh, dgu, dzh, dz, dO, dqkv, dxh, Dvec, dqacc, part;
+  size_t xres, dres;  // float32 residual stream and its gradient (bf16 path)
   size_t total;
 };
 
@@ -48,6 +49,34 @@ struct Handle {
   bool fwd_valid = false;
   void* fwd_ws = nullptr;
   std::vector<float> fwd_scale;
+  // device-time accounting (ld_set_timing): event pairs around launches
+  bool timing = false;
+  std::vector<cudaEvent_t> ev[LD_KCLASS_COUNT];
+  size_t ev_used[LD_KCLASS_COUNT] = {};
+  ~Handle() {
+    for (auto& v : ev)
+      for (cudaEvent_t e : v) cudaEventDestroy(e);
+  }
+};
+
+// Records an event pair around the launches of its scope when timing is on.
+struct Timed {
+  Handle* h;
+  int cls;
+  cudaStream_t st;
+  Timed(Handle* h_, int cls_, cudaStream_t st_) : h(h_), cls(cls_), st(st_) { mark(); }
+  ~Timed() { mark(); }
+  void mark() {
+    if (!h->timing) return;
+    auto& v = h->ev[cls];
+    size_t& u = h->ev_used[cls];
+    if (u == v.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return;
+      v.push_back(e);
+    }
+    cudaEventRecord(v[u++], st);
+  }
 };
 
 Handle* H(void* h) { return static_cast<Handle*>(h); }
@@ -143,6 +172,8 @@ void make_layout(Handle* h) {
   y.Dvec = take((size_t)c.H * R * 4);
   y.dqacc = take(R * c.H * c.Dh * 4);
   y.part = take((size_t)h->part_blocks * c.d * 4);
+  y.xres = c.fp32_debug ? 0 : take(R * c.d * 4);
+  y.dres = c.fp32_debug ? 0 : take(R * c.d * 4);
   y.total = off;
 }
 
@@ -153,9 +184,9 @@ T* at(void* ws, size_t off) {
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
 
-#define LD_CHECK(expr)                      \
-  do {                                      \
-    if ((expr) != cudaSuccess) return LD_ERR_CUDA; \
+#define LD_CHECK(...)                              \
+  do {                                             \
+    if ((__VA_ARGS__) != cudaSuccess) return LD_ERR_CUDA; \
   } while (0)
 
 ld_status check_device() {
@@ -239,10 +270,24 @@ cudaError_t gemm<float>(const GemmArgs& a, cudaStream_t st) {
   return gemm_simt(a, st);
 }
 
+// Attention: tensor-core flash attention on the bf16 path, SIMT float32 on
+// the debug path.
 template <typename T>
-cudaError_t attn_fwd(const Handle* h, const T* qkv, T* o, float* lse, const int* cnt, cudaStream_t st) {
+cudaError_t attn_fwd(const Handle* h, void* ws, const T* qkv, T* o, float* lse, const int* cnt, cudaStream_t st);
+template <>
+cudaError_t attn_fwd<float>(const Handle* h, void* ws, const float* qkv, float* o, float* lse, const int* cnt,
+                            cudaStream_t st) {
   const ld_config& c = h->cfg;
-  return launch_attn_fwd_simt<T>(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, h->max_rows, st);
+  return launch_attn_fwd_simt<float>(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, h->max_rows, st);
+}
+template <>
+cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, float* lse, const int* cnt,
+                           cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  if (attn_tc_supported(c.S, c.Dh))
+    return launch_attn_fwd_tc(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B,
+                              at<int>(ws, h->lay.status), st);
+  return launch_attn_fwd_mma(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, st);
 }
 
 template <typename T>
@@ -251,15 +296,31 @@ cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const 
   const ld_config& c = h->cfg;
   cudaError_t e = launch_attn_rowdot<T>(dO, o, c.H * c.Dh, c.H, c.Dh, cnt, c.S, h->max_rows, Dvec, st);
   if (e != cudaSuccess) return e;
-  return launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, cnt, c.S, c.H, c.Hkv, c.Dh,
-                                 h->max_rows, st);
+  if (sizeof(T) == 4)
+    return launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, cnt, c.S, c.H, c.Hkv, c.Dh,
+                                   h->max_rows, st);
+  float* dq_acc = at<float>(ws, h->lay.dqacc);
+  const bf16* q16 = reinterpret_cast<const bf16*>(qkv);
+  bf16* d16 = reinterpret_cast<bf16*>(dqkv);
+  if (attn_bwd_tc_supported(c.S, c.Dh))
+    e = launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt,
+                           c.S, c.H, c.Hkv, c.B, at<int>(ws, h->lay.status), st);
+  else
+    e = launch_attn_bwd_mma(q16, h->nqkv, reinterpret_cast<const bf16*>(o), reinterpret_cast<const bf16*>(dO),
+                          c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, st);
+  if (e != cudaSuccess) return e;
+  return launch_dq_finish(dq_acc, d16, h->nqkv, c.H, c.Dh, cnt, c.S, h->max_rows, st);
 }
 
 template <typename T>
 ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv, void* ws, cudaStream_t st) {
   const ld_config& c = h->cfg;
   const Layout& y = h->lay;
-  T* x = static_cast<T*>(xv);
+  // The residual stream is carried in float32 through the layers (bf16 in
+  // and out at the boundary): 2*L in-place bf16 roundings of X would
+  // otherwise accumulate to several per cent of |X| at 32 layers.
+  const bool f32 = sizeof(T) == 4;
+  float* x = f32 ? static_cast<float*>(xv) : at<float>(ws, y.xres);
   int* status = at<int>(ws, y.status);
   unsigned char* mask = at<unsigned char>(ws, y.mask);
   int* kidx = at<int>(ws, y.kidx);
@@ -274,10 +335,16 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
   P.L = c.L;
   P.B = c.B;
   P.granularity = c.granularity;
+  P.b_offset = c.b_offset;
   std::vector<float> scale(c.L);
   step_rates(h, step, nullptr, P.thr, scale.data());
-  LD_CHECK(launch_mask_compact(P, mask, kidx, kcnt, st));
-  if (c.rope_theta != 0.0f) LD_CHECK(launch_rope_table(rcos, rsin, c.S, c.Dh, (double)c.rope_theta, st));
+  {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(cudaMemsetAsync(status, 0, sizeof(int), st));
+    if (!f32) LD_CHECK(launch_convert(xv, 0, x, 1, (long long)h->max_rows * c.d, st));
+    LD_CHECK(launch_mask_compact(P, mask, kidx, kcnt, st));
+    if (c.rope_theta != 0.0f) LD_CHECK(launch_rope_table(rcos, rsin, c.S, c.Dh, (double)c.rope_theta, st));
+  }
 
   const int HD = c.H * c.Dh;
   for (int l = 0; l < c.L; ++l) {
@@ -299,15 +366,15 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     const T* g2 = static_cast<const T*>(W[l].g2);
     const float s = scale[l];
 
-    LD_CHECK(launch_rmsnorm_fwd<T>(x, 1, ki, cnt, c.S, c.d, h->max_rows, g1, c.eps, xin, xh, rstd1, st));
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, ki, cnt, c.S, c.d, h->max_rows, g1, c.eps, xin, xh, rstd1, st)); }
     GemmArgs a = rows_gemm(h, cnt, h->nqkv, c.d, xh, c.d, W[l].w_qkv, c.d, 0);
     a.epi = EPI_STORE;
     a.D = qkv;
     a.ldd = h->nqkv;
-    LD_CHECK(gemm<T>(a, st));
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
     if (c.rope_theta != 0.0f)
-      LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 0, st));
-    LD_CHECK(attn_fwd<T>(h, qkv, o, lse, cnt, st));
+      { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 0, st)); }
+    { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_fwd<T>(h, ws, qkv, o, lse, cnt, st)); }
     a = rows_gemm(h, cnt, c.d, HD, o, HD, W[l].w_o, HD, 0);
     a.epi = EPI_RESID;
     a.alpha = s;
@@ -317,14 +384,14 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     a.S = c.S;
     a.save = z;
     a.ld_save = c.d;
-    LD_CHECK(gemm<T>(a, st));
-    LD_CHECK(launch_rmsnorm_fwd<T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, nullptr, zh, rstd2, st));
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<T, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (T*)nullptr, zh, rstd2, st)); }
     a = rows_gemm(h, cnt, 2 * c.F, c.d, zh, c.d, W[l].w_gu, c.d, 0);
     a.epi = EPI_STORE;
     a.D = gu;
     a.ldd = 2 * c.F;
-    LD_CHECK(gemm<T>(a, st));
-    LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cnt, c.S, c.F, h->max_rows, st));
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cnt, c.S, c.F, h->max_rows, st)); }
     a = rows_gemm(h, cnt, c.d, c.F, hh, c.F, W[l].w_d, c.F, 0);
     a.epi = EPI_RESID;
     a.alpha = s;
@@ -333,7 +400,11 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     a.kept_idx = ki;
     a.S = c.S;
     a.save = nullptr;
-    LD_CHECK(gemm<T>(a, st));
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+  }
+  if (!f32) {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(launch_convert(x, 1, xv, 0, (long long)h->max_rows * c.d, st));
   }
   h->fwd_scale = scale;
   return LD_OK;
@@ -343,7 +414,8 @@ template <typename T>
 ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G, void* ws, cudaStream_t st) {
   const ld_config& c = h->cfg;
   const Layout& y = h->lay;
-  T* dx = static_cast<T*>(dxv);
+  const bool f32 = sizeof(T) == 4;
+  float* dx = f32 ? static_cast<float*>(dxv) : at<float>(ws, y.dres);  // float32 residual gradient
   int* kidx = at<int>(ws, y.kidx);
   int* kcnt = at<int>(ws, y.kcnt);
   float* rcos = at<float>(ws, y.rcos);
@@ -359,6 +431,10 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
   float* Dvec = at<float>(ws, y.Dvec);
   float* part = at<float>(ws, y.part);
   const int HD = c.H * c.Dh;
+  if (!f32) {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(launch_convert(dxv, 0, dx, 1, (long long)h->max_rows * c.d, st));
+  }
 
   for (int l = c.L - 1; l >= 0; --l) {
     const int* cnt = kcnt + l;
@@ -380,44 +456,54 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     const float s = h->fwd_scale[l];
 
     // FFN branch: dy = r * dX^{l+1} on the kept rows.
-    LD_CHECK(launch_gather_scale<T>(dx, ki, cnt, c.S, c.d, h->max_rows, s, dy, st));
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, ki, cnt, c.S, c.d, h->max_rows, s, dy, st)); }
     GemmArgs a = rows_gemm(h, cnt, c.F, c.d, dy, c.d, W[l].w_d, c.F, 1);  // dh = dy W_d
     a.epi = EPI_STORE;
     a.D = dh;
     a.ldd = c.F;
-    LD_CHECK(gemm<T>(a, st));
-    LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cnt, c.S, c.F, h->max_rows, st));
-    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st));  // dW_d = dy^T h
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cnt, c.S, c.F, h->max_rows, st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
     a = rows_gemm(h, cnt, c.d, 2 * c.F, dgu, 2 * c.F, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
     a.epi = EPI_STORE;
     a.D = dzh;
     a.ldd = c.d;
-    LD_CHECK(gemm<T>(a, st));
-    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, 2 * c.F, c.d, dgu, 2 * c.F, zh, c.d, G[l].w_gu), st));
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, 2 * c.F, c.d, dgu, 2 * c.F, zh, c.d, G[l].w_gu), st)); }
     // dZ = dX^{l+1} + RMSNorm_2 backward; dz = r * dZ for the attention branch
-    LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, ki, cnt, c.S, c.d, h->max_rows, s, dz, part,
-                                   h->part_blocks, st));
-    LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g2, st));
+    {
+      Timed tm_(h, LD_KCLASS_ROWWISE, st);
+      LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, ki, cnt, c.S, c.d, h->max_rows, s, dz, part,
+                                     h->part_blocks, st));
+    }
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g2, st)); }
     // attention branch
     a = rows_gemm(h, cnt, HD, c.d, dz, c.d, W[l].w_o, HD, 1);  // dO = dz W_o
     a.epi = EPI_STORE;
     a.D = dO;
     a.ldd = HD;
-    LD_CHECK(gemm<T>(a, st));
-    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, HD, dz, c.d, o, HD, G[l].w_o), st));  // dW_o = dz^T o
-    LD_CHECK(attn_bwd<T>(h, ws, qkv, o, dO, lse, Dvec, dqkv, cnt, st));
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, HD, dz, c.d, o, HD, G[l].w_o), st)); }  // dW_o = dz^T o
+    { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_bwd<T>(h, ws, qkv, o, dO, lse, Dvec, dqkv, cnt, st)); }
     if (c.rope_theta != 0.0f)
-      LD_CHECK(launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1, st));
+      { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1, st)); }
     a = rows_gemm(h, cnt, c.d, h->nqkv, dqkv, h->nqkv, W[l].w_qkv, c.d, 1);  // dxh = dqkv W_qkv
     a.epi = EPI_STORE;
     a.D = dxh;
     a.ldd = c.d;
-    LD_CHECK(gemm<T>(a, st));
-    LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, h->nqkv, c.d, dqkv, h->nqkv, xh, c.d, G[l].w_qkv), st));
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, h->nqkv, c.d, dqkv, h->nqkv, xh, c.d, G[l].w_qkv), st)); }
     // dX^l = dZ + RMSNorm_1 backward
-    LD_CHECK(launch_rmsnorm_bwd<T>(dxh, xin, rstd1, g1, dx, ki, cnt, c.S, c.d, h->max_rows, 1.0f, (T*)nullptr,
-                                   part, h->part_blocks, st));
-    LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g1, st));
+    {
+      Timed tm_(h, LD_KCLASS_ROWWISE, st);
+      LD_CHECK(launch_rmsnorm_bwd<T>(dxh, xin, rstd1, g1, dx, ki, cnt, c.S, c.d, h->max_rows, 1.0f, (T*)nullptr,
+                                     part, h->part_blocks, st));
+    }
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g1, st)); }
+  }
+  if (!f32) {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(launch_convert(dx, 1, dxv, 0, (long long)h->max_rows * c.d, st));
   }
   return LD_OK;
 }
@@ -451,6 +537,7 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   if (c.Dh != 32 && c.Dh != 64 && c.Dh != 128) return LD_ERR_SHAPE;
   if (c.H < 1 || c.Hkv < 1 || c.H % c.Hkv || (c.H * c.Dh) % 64) return LD_ERR_SHAPE;
   if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH) return LD_ERR_ARG;
+  if (c.b_offset < 0 || (long long)c.b_offset + c.B > 0x7fffffffll) return LD_ERR_ARG;
   if ((long long)c.B * c.S > (1ll << 30)) return LD_ERR_SHAPE;
   Handle* h = new (std::nothrow) Handle();
   if (!h) return LD_ERR_OOM;
@@ -514,8 +601,10 @@ ld_status ld_draw_masks(void* handle, long long step, void* ws, void* stream) {
   P.L = h->cfg.L;
   P.B = h->cfg.B;
   P.granularity = h->cfg.granularity;
+  P.b_offset = h->cfg.b_offset;
   step_rates(h, step, nullptr, P.thr, nullptr);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  LD_CHECK(cudaMemsetAsync(at<int>(ws, y.status), 0, sizeof(int), st));
   LD_CHECK(launch_mask_compact(P, at<unsigned char>(ws, y.mask), at<int>(ws, y.kidx), at<int>(ws, y.kcnt), st));
   h->last_ws = ws;
   h->last_stream = st;
@@ -590,6 +679,30 @@ ld_status ld_sync(void* handle) {
 ld_status ld_destroy(void* handle) {
   if (!handle) return LD_ERR_ARG;
   delete H(handle);
+  return LD_OK;
+}
+
+ld_status ld_set_timing(void* handle, int enable) {
+  if (!handle) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  h->timing = enable != 0;
+  for (auto& u : h->ev_used) u = 0;
+  return LD_OK;
+}
+
+ld_status ld_get_timing(void* handle, int kclass, double* ms, long long* launches) {
+  if (!handle || kclass < 0 || kclass >= LD_KCLASS_COUNT) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  const size_t pairs = h->ev_used[kclass] / 2;
+  double tot = 0.0;
+  for (size_t i = 0; i < pairs; ++i) {
+    float t = 0.f;
+    LD_CHECK(cudaEventSynchronize(h->ev[kclass][2 * i + 1]));
+    LD_CHECK(cudaEventElapsedTime(&t, h->ev[kclass][2 * i], h->ev[kclass][2 * i + 1]));
+    tot += t;
+  }
+  if (ms) *ms = tot;
+  if (launches) *launches = (long long)pairs;
   return LD_OK;
 }
 

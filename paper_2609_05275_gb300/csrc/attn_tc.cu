@@ -1,0 +1,603 @@
+// Causal grouped-query flash attention, forward, on the tcgen05 tensor cores
+// (sm_103a), head sizes 64 and 128, sequence lengths that are multiples of
+// 128.
+//
+// f_attn of Eq. (transformer_layer_dropout_train) for one kept sequence and
+// query head h (key/value head g = floor(h*Hkv/H)):
+//   o_i = sum_{j<=i} softmax_j(c q_i . k_j) v_j,  c = 1/sqrt(Dh);
+// lse_i = log sum_j exp(c q_i . k_j) is kept for the backward.
+//
+// One CTA per (128-query tile, head, kept sequence); 192 threads:
+//   warp 0      TMA: the Q tile once, then K_j / V_j tiles (128 keys) into a
+//               two-stage ring (128-byte swizzled, 64-column slabs);
+//   warp 1      TMEM allocation and the MMAs: S_j = Q K_j^T into one of two
+//               TMEM score buffers, then O += P_{j-1} V_{j-1} (O in TMEM);
+//   warps 2..5  softmax, one query row per thread: S_j from TMEM, running
+//               max in base 2, P = exp2(S c log2e - m) written as bf16 into a
+//               swizzled shared-memory tile (the A operand of the PV MMA).
+// The running max is only moved (and O rescaled in TMEM) when it grows by
+// more than 2^8, so most tiles need no O round trip; P <= 2^8 stays well
+// inside bf16/fp32 range.  All waits are bounded (status word on expiry).
+#include "tc_common.cuh"
+
+namespace ldk {
+namespace {
+using namespace tc;
+
+constexpr uint32_t SLAB = 128 * 128;  // bytes of a 128-row x 64-column bf16 slab
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kRescale = 8.0f;  // move the running max only when it grows by > 2^8
+
+// byte offset of element (row r, 16-byte chunk i) in a 128B-swizzled
+// K-major slab of 128-byte rows
+__device__ __forceinline__ uint32_t swz(int r, int i) {
+  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + (((i & 7) ^ (r & 7)) << 4));
+}
+
+template <int DH>
+__global__ void __launch_bounds__(192, 1)
+    attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
+                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv, int* status) {
+  constexpr int NSLAB = DH / 64;
+  constexpr uint32_t TILE = NSLAB * SLAB;  // one 128 x DH bf16 tile
+  constexpr int NS = 2;                    // K/V stages
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Qs = smem;
+  uint8_t* Ks = Qs + TILE;
+  uint8_t* Vs = Ks + NS * TILE;
+  uint8_t* Ps = Vs + NS * TILE;  // 128 x 128 bf16, two slabs
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Ps + 2 * SLAB);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;
+  uint64_t* kv_empty = kv_full + NS;
+  uint64_t* s_full = kv_empty + NS;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* pv_done = p_full + 1;
+  uint64_t* o_full = pv_done + 1;
+  uint64_t* drain = o_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int seq = blockIdx.z;
+  if (seq >= *cnt) return;
+  const int nqt = S / 128;
+  const int qt = nqt - 1 - blockIdx.x;  // heaviest tiles first
+  const int h = blockIdx.y, g = (h * Hkv) / H;
+  const int row0 = seq * S;
+  const int nkt = qt + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_free[b], 4);
+    }
+    mbar_init(p_full, 4);
+    mbar_init(pv_done, 1);
+    mbar_init(o_full, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_o = tmem + 256;  // O accumulator: columns 256 .. 256+DH
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      const int qcol = h * DH, kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
+      mbar_arrive_expect_tx(q_full, TILE);
+      for (int c = 0; c < NSLAB; ++c) tma_load_2d(Qs + c * SLAB, &tm, qcol + 64 * c, row0 + qt * 128, q_full);
+      int issued = 0;
+      for (int j = 0; j < nkt; ++j) {
+        const int s = j % NS;
+        if (!mbar_wait(&kv_empty[s], ((j / NS) & 1) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&kv_full[s], 2 * TILE);
+        for (int c = 0; c < NSLAB; ++c) {
+          tma_load_2d(Ks + s * TILE + c * SLAB, &tm, kcol + 64 * c, row0 + j * 128, &kv_full[s]);
+          tma_load_2d(Vs + s * TILE + c * SLAB, &tm, vcol + 64 * c, row0 + j * 128, &kv_full[s]);
+        }
+        ++issued;
+      }
+      if (*abort_flag) {
+        mbar_drain(q_full, 0);
+        for (int j = issued > NS ? issued - NS : 0; j < issued; ++j) mbar_drain(&kv_full[j % NS], (j / NS) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
+      constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
+      const uint32_t qa = smem_u32(Qs), ka = smem_u32(Ks), va = smem_u32(Vs), pa = smem_u32(Ps);
+      bool ok = mbar_wait(q_full, 0, abort_flag, status);
+      for (int j = 0; ok && j <= nkt; ++j) {
+        if (j < nkt) {
+          const int s = j % NS;
+          if (!mbar_wait(&kv_full[s], (j / NS) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t kb = ka + s * TILE;
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * SLAB + (kk & 3) * 32;
+            mma_bf16(tmem + (j & 1) * 128, sdesc(qa + off, 16, 1024), sdesc(kb + off, 16, 1024), ID_S, kk > 0);
+          }
+          mma_commit(&s_full[j & 1]);
+        }
+        if (j >= 1) {
+          const int jp = j - 1, s = jp % NS;
+          if (!mbar_wait(p_full, jp & 1, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t vb = va + s * TILE;
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            // A = P (K-major, 128 keys in two slabs); B = V as MN-major
+            // (dh contiguous): 64-dh chunks one slab apart, 8-key groups 1 KB
+            mma_bf16(t_o, sdesc(pa + (kk >> 2) * SLAB + (kk & 3) * 32, 16, 1024),
+                     sdesc(vb + kk * 2048, SLAB, 1024), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
+          }
+          mma_commit(pv_done);
+          mma_commit(&kv_empty[s]);
+        }
+      }
+      if (ok) {
+        mma_commit(o_full);
+      } else {
+        mma_commit(drain);
+        mbar_drain(drain, 0);
+      }
+    }
+  } else {
+    // ------------------------------------------------ softmax (warps 2..5)
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;  // query row of this thread within the tile
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const float sl2 = kLog2e * rsqrtf((float)DH);
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkt; ++j) {
+      if (!warp_wait(&s_full[j & 1], (j >> 1) & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      float sv[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        float t[32];
+        tmem_ld32(tmem + (j & 1) * 128 + c * 32 + lane_off, t);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) sv[c * 32 + e] = t[e];
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[j & 1]);
+      float mt = -INFINITY;
+      const bool diag = (j == qt);
+#pragma unroll
+      for (int e = 0; e < 128; ++e) {
+        float v = sv[e] * sl2;
+        if (diag && e > r) v = -INFINITY;
+        sv[e] = v;
+        mt = fmaxf(mt, v);
+      }
+      bool rescale = mt > m_used + kRescale;
+      const float m_new = rescale ? mt : m_used;
+      float ls = 0.f;
+      uint32_t pk[64];
+#pragma unroll
+      for (int e = 0; e < 64; ++e) {
+        const float p0 = exp2f(sv[2 * e] - m_new), p1 = exp2f(sv[2 * e + 1] - m_new);
+        ls += p0 + p1;
+        __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
+        pk[e] = *reinterpret_cast<uint32_t*>(&b);
+      }
+      // P_{j-1} V_{j-1} must be done before P and O are touched
+      if (j >= 1 && !warp_wait(pv_done, (j - 1) & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      // tcgen05.ld/st are warp-wide: the warp rescales O together when any
+      // lane moved its max; lanes that did not multiply by 1
+      if (j >= 1 && __any_sync(0xffffffffu, rescale)) {
+        const float corr = rescale ? exp2f(m_used - m_new) : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < DH / 32; ++c) {
+          float t[32];
+          tmem_ld32(t_o + c * 32 + lane_off, t);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) t[e] *= corr;
+          tmem_st32(t_o + c * 32 + lane_off, t);
+        }
+      }
+      if (rescale) {
+        l *= exp2f(m_used - m_new);
+        m_used = m_new;
+      }
+      l += ls;
+      // P row r -> swizzled K-major tile (two 64-key slabs)
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        uint4 q = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        *reinterpret_cast<uint4*>(Ps + (i >> 3) * SLAB + swz(r, i)) = q;
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (ok && warp_wait(o_full, 0, abort_flag, status)) {
+      tc_fence_after();
+      const float inv = 1.0f / l;
+      bf16* orow = o + (long long)(row0 + qt * 128 + r) * ldo + (long long)h * DH;
+#pragma unroll 1
+      for (int c = 0; c < DH / 32; ++c) {
+        float t[32];
+        tmem_ld32(t_o + c * 32 + lane_off, t);
+        uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          uint4 q;
+          __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&q);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) hb[k] = __floats2bfloat162_rn(t[8 * i + 2 * k] * inv, t[8 * i + 2 * k + 1] * inv);
+          dst[i] = q;
+        }
+      }
+      lse[(size_t)h * lse_ld + row0 + qt * 128 + r] = (m_used + log2f(l)) * kLn2;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+template <int DH>
+cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
+                   int max_seqs, int* status, cudaStream_t st) {
+  constexpr size_t smem = (size_t)(DH / 64) * SLAB * 5 + 2 * SLAB + 1024 + 256;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e =
+        cudaFuncSetAttribute(attn_fwd_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  CUtensorMap tm;
+  if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
+  dim3 grid(S / 128, H, max_seqs);
+  attn_fwd_tc_kernel<DH><<<grid, 192, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, status);
+  return cudaGetLastError();
+}
+
+
+// ---------------------------------------------------------------------------
+// Backward, head size 128.  One CTA per (128-key tile, kv head, kept
+// sequence), looping over the query heads of the group and the 64-query
+// tiles at or after the key tile.  320 threads:
+//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (2 stages)
+//   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
+//               (M = 128 keys, N = 64 queries); then for step i-1
+//               dV += P^T dO, dK += dS^T Q (M = 128 keys, N = 128) and
+//               dQ^T = K^T dS^T (M = 128 head dims, N = 64 queries)
+//   warps 2..5  one key per thread: P^T = exp2(S^T c log2e - lse log2e),
+//               dS^T = P^T (dP^T - D), both to swizzled bf16 tiles; at the
+//               end dK (times c) and dV from TMEM to dqkv
+//   warps 6..9  dQ^T from TMEM, added into the float32 dQ buffer
+// TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447.
+constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
+
+__global__ void __launch_bounds__(320, 1)
+    attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
+                       const __grid_constant__ CUtensorMap tmo,
+                       const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
+                       float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
+                       int S, int H, int Hkv, int* status) {
+  constexpr int DH = 128;
+  constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
+  constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Ks = smem;
+  uint8_t* Vs = Ks + KT;
+  uint8_t* Qs = Vs + KT;         // [2][QT]
+  uint8_t* dOs = Qs + 2 * QT;    // [2][QT]
+  uint8_t* PTs = dOs + 2 * QT;   // 128 keys x 64 queries, one slab of 128-byte rows
+  uint8_t* DSs = PTs + SLAB;
+  float* vecs = reinterpret_cast<float*>(DSs + SLAB);  // [2][lse 64 | D 64]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + 256);
+  uint64_t* kv_full = bars;
+  uint64_t* ld_full = bars + 1;  // [2]
+  uint64_t* ld_empty = bars + 3; // [2]
+  uint64_t* sdp_full = bars + 5;
+  uint64_t* sdp_free = bars + 6;
+  uint64_t* p_ready = bars + 7;
+  uint64_t* mm_done = bars + 8;
+  uint64_t* dq_free = bars + 9;
+  uint64_t* acc_done = bars + 10;
+  uint64_t* drain = bars + 11;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int seq = blockIdx.z;
+  if (seq >= *cnt) return;
+  const int kt = blockIdx.x, g = blockIdx.y, grp = H / Hkv;
+  const int row0 = seq * S;
+  const int nq = S / 64, q0 = 2 * kt;          // query tiles q0 .. nq-1 overlap or follow the keys
+  const int n_it = grp * (nq - q0);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int HD = H * DH;
+
+  if (threadIdx.x == 0) {
+    mbar_init(kv_full, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&ld_full[b], 1);
+      mbar_init(&ld_empty[b], 1);
+    }
+    mbar_init(sdp_full, 1);
+    mbar_init(sdp_free, 4);
+    mbar_init(p_ready, 4);
+    mbar_init(mm_done, 1);
+    mbar_init(dq_free, 4);
+    mbar_init(acc_done, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_s = tmem, t_dp = tmem + 64, t_dv = tmem + 128, t_dk = tmem + 256, t_dq = tmem + 384;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
+      mbar_arrive_expect_tx(kv_full, 2 * KT);
+      for (int c = 0; c < 2; ++c) {
+        tma_load_2d(Ks + c * SLAB, &tmkv, kcol + 64 * c, row0 + kt * 128, kv_full);
+        tma_load_2d(Vs + c * SLAB, &tmkv, vcol + 64 * c, row0 + kt * 128, kv_full);
+      }
+      int issued = 0;
+      for (int i = 0; i < n_it; ++i) {
+        const int b = i & 1;
+        const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
+        if (!mbar_wait(&ld_empty[b], ((i >> 1) & 1) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 512);
+        for (int c = 0; c < 2; ++c) {
+          tma_load_2d(Qs + b * QT + c * HSLAB, &tmq, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
+          tma_load_2d(dOs + b * QT + c * HSLAB, &tmo, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
+        }
+        const size_t vo = (size_t)h * lse_ld + row0 + qt * 64;
+        bulk_load(vecs + b * 128, lse + vo, 256, &ld_full[b]);
+        bulk_load(vecs + b * 128 + 64, Dvec + vo, 256, &ld_full[b]);
+        ++issued;
+      }
+      if (*abort_flag) {
+        mbar_drain(kv_full, 0);
+        for (int i = issued > 2 ? issued - 2 : 0; i < issued; ++i) mbar_drain(&ld_full[i & 1], (i >> 1) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
+      constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
+      constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
+      const uint32_t ka = smem_u32(Ks), va = smem_u32(Vs), qa = smem_u32(Qs), oa = smem_u32(dOs);
+      const uint32_t pa = smem_u32(PTs), da = smem_u32(DSs);
+      bool ok = mbar_wait(kv_full, 0, abort_flag, status);
+      for (int i = 0; ok && i <= n_it; ++i) {
+        if (i < n_it) {
+          const int b = i & 1;
+          if (!mbar_wait(&ld_full[b], (i >> 1) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
+            const uint32_t qoff = b * QT + (kk >> 2) * HSLAB + (kk & 3) * 32;
+            mma_bf16(t_s, sdesc(ka + koff, 16, 1024), sdesc(qa + qoff, 16, 1024), ID_SP, kk > 0);
+            mma_bf16(t_dp, sdesc(va + koff, 16, 1024), sdesc(oa + qoff, 16, 1024), ID_SP, kk > 0);
+          }
+          mma_commit(sdp_full);
+        }
+        if (i >= 1) {
+          const int ip = i - 1, b = ip & 1;
+          if (!mbar_wait(p_ready, ip & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
+            const uint32_t aoff = kk * 32;                       // P^T / dS^T, K-major
+            const uint32_t boff = b * QT + kk * 2048;            // dO / Q as MN-major
+            mma_bf16(t_dv, sdesc(pa + aoff, 16, 1024), sdesc(oa + boff, HSLAB, 1024), ID_KV, (ip > 0 || kk > 0));
+            mma_bf16(t_dk, sdesc(da + aoff, 16, 1024), sdesc(qa + boff, HSLAB, 1024), ID_KV, (ip > 0 || kk > 0));
+          }
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
+            mma_bf16(t_dq, sdesc(ka + kk * 2048, SLAB, 1024), sdesc(da + kk * 2048, 16, 1024), ID_Q, kk > 0);
+          }
+          mma_commit(mm_done);
+          mma_commit(&ld_empty[b]);
+        }
+      }
+      if (ok) {
+        mma_commit(acc_done);
+      } else {
+        mma_commit(drain);
+        mbar_drain(drain, 0);
+      }
+    }
+  } else if (warp < 6) {
+    // ------------------------------------------------ P / dS (warps 2..5)
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;  // key within the tile
+    const int key = kt * 128 + r;
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const float sl2 = kLog2e * rsqrtf((float)DH);
+    bool ok = true;
+    for (int i = 0; i < n_it; ++i) {
+      const int b = i & 1;
+      const int qt = q0 + i % (nq - q0);
+      if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
+      if (!warp_wait(&ld_full[b], (i >> 1) & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      float sv[64], dp[64];
+      {
+        float t[32];
+        tmem_ld32(t_s + lane_off, t);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) sv[e] = t[e];
+        tmem_ld32(t_s + 32 + lane_off, t);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) sv[32 + e] = t[e];
+        tmem_ld32(t_dp + lane_off, t);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) dp[e] = t[e];
+        tmem_ld32(t_dp + 32 + lane_off, t);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) dp[32 + e] = t[e];
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sdp_free);
+      const float* lv = vecs + b * 128;
+      uint32_t pk[32], dk[32];
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        float p[2], d[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int c = 2 * e + u;
+          const bool vis = qt * 64 + c >= key;
+          const float pv = vis ? exp2f(sv[c] * sl2 - lv[c] * kLog2e) : 0.f;
+          p[u] = pv;
+          d[u] = pv * (dp[c] - lv[64 + c]);
+        }
+        __nv_bfloat162 bp = __floats2bfloat162_rn(p[0], p[1]), bd = __floats2bfloat162_rn(d[0], d[1]);
+        pk[e] = *reinterpret_cast<uint32_t*>(&bp);
+        dk[e] = *reinterpret_cast<uint32_t*>(&bd);
+      }
+      // the MMAs of step i-1 must be done with P^T / dS^T before they are rewritten
+      if (i >= 1 && !warp_wait(mm_done, (i - 1) & 1, abort_flag, status)) { ok = false; break; }
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        *reinterpret_cast<uint4*>(PTs + swz(r, c)) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        *reinterpret_cast<uint4*>(DSs + swz(r, c)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_ready);
+    }
+    if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
+      tc_fence_after();
+      const float c = rsqrtf((float)DH);
+      bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
+      bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
+#pragma unroll 1
+      for (int cc = 0; cc < DH / 32; ++cc) {
+        float t[32], u[32];
+        tmem_ld32(t_dk + cc * 32 + lane_off, t);
+        tmem_ld32(t_dv + cc * 32 + lane_off, u);
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          uint4 a, bq;
+          __nv_bfloat162* ha = reinterpret_cast<__nv_bfloat162*>(&a);
+          __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&bq);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            ha[k] = __floats2bfloat162_rn(c * t[8 * q4 + 2 * k], c * t[8 * q4 + 2 * k + 1]);
+            hb[k] = __floats2bfloat162_rn(u[8 * q4 + 2 * k], u[8 * q4 + 2 * k + 1]);
+          }
+          reinterpret_cast<uint4*>(krow + cc * 32)[q4] = a;
+          reinterpret_cast<uint4*>(vrow + cc * 32)[q4] = bq;
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------ dQ (warps 6..9)
+    const int quad = warp & 3;
+    const int dd = quad * 32 + lane;  // head dimension of this thread
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    for (int i = 0; i < n_it; ++i) {
+      const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
+      if (!warp_wait(mm_done, i & 1, abort_flag, status)) break;
+      tc_fence_after();
+      float t0[32], t1[32];
+      tmem_ld32(t_dq + lane_off, t0);
+      tmem_ld32(t_dq + 32 + lane_off, t1);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(dq_free);
+      float* dst = dq_acc + (size_t)(row0 + qt * 64) * HD + (size_t)h * DH + dd;
+#pragma unroll
+      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)e * HD, t0[e]);
+#pragma unroll
+      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(32 + e) * HD, t1[e]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
+                   float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, int* status,
+                   cudaStream_t st) {
+  constexpr size_t smem = 6 * SLAB + 8 * HSLAB + 256 * 4 + 1024 + 256;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(attn_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  CUtensorMap tkv, tq, to;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows
+  if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
+  if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
+  if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
+  dim3 grid(S / 128, Hkv, max_seqs);
+  attn_bwd_tc_kernel<<<grid, 320, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H, Hkv,
+                                              status);
+  return cudaGetLastError();
+}
+}  // namespace
+
+bool attn_tc_supported(int S, int Dh) { return S % 128 == 0 && (Dh == 64 || Dh == 128); }
+
+bool attn_bwd_tc_supported(int S, int Dh) { return S % 128 == 0 && Dh == 128; }
+
+cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
+                               const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
+                               int max_seqs, int* status, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)max_seqs * S * H * 128 * sizeof(float), st);
+  if (e != cudaSuccess) return e;
+  return bwd_tc(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, status, st);
+}
+
+cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
+                               int Hkv, int Dh, int max_seqs, int* status, cudaStream_t st) {
+  if (Dh == 64) return fwd_tc<64>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, status, st);
+  return fwd_tc<128>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, status, st);
+}
+
+}  // namespace ldk

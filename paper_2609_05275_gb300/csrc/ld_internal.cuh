@@ -51,37 +51,42 @@ __device__ __forceinline__ long long src_row(const int* kept_idx, int S, long lo
 struct MaskParams {
   unsigned long long seed;
   long long step;
-  int L, B, granularity;
+  int L, B, granularity, b_offset;
   unsigned long long thr[LD_MAX_L];
 };
 cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* kept_idx, int* kept_cnt,
                                 cudaStream_t st);
 
+// Elementwise copy with conversion between float32 and bf16 (n % 8 == 0).
+cudaError_t launch_convert(const void* src, int src_f32, void* dst, int dst_f32, long long n, cudaStream_t st);
+
 cudaError_t launch_rope_table(float* cos_t, float* sin_t, int S, int Dh, double theta, cudaStream_t st);
 
 // RMSNorm forward over the rows of layer l (M = *cnt * S rows).  When
-// `gather` is set the source row of compact row m is src_row(kept_idx, S, m),
-// else m.  Writes the normalised rows (out), the reciprocal rms (rstd) and,
-// if copy != null, a compact copy of the source rows.
-template <typename T>
-cudaError_t launch_rmsnorm_fwd(const T* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
+// `gather` is set the source row of compact row m is src_row(kept_idx, S, m)
+// of the float32 residual stream, else row m of a compact buffer.  Writes
+// the normalised rows (out), the reciprocal rms (rstd) and, if copy != null,
+// a compact copy of the source rows.
+template <typename TS, typename T>
+cudaError_t launch_rmsnorm_fwd(const TS* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
                                int max_rows, const T* gamma, float eps, T* copy, T* out, float* rstd,
                                cudaStream_t st);
 
 // RMSNorm backward + residual: for compact row m with source row r,
 //   dx[r] += rstd (dyn*g - xn * mean(dyn*g*xn)),  xn = xs[m] * rstd[m]
-// then, if next != null, next[m] = scale * dx[r] (compact, for the next
-// branch).  Partial gain gradients go to part[blockIdx][d]; the number of
-// blocks is returned in *nblocks (a launch constant).
+// on the float32 residual gradient dx, then, if next != null,
+// next[m] = scale * dx[r] (compact, for the next branch).  Partial gain
+// gradients go to part[blockIdx][d] (nblocks blocks, a launch constant).
 template <typename T>
-cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, T* dx,
+cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, float* dx,
                                const int* kept_idx, const int* cnt, int S, int d, int max_rows, float scale,
                                T* next, float* part, int nblocks, cudaStream_t st);
 int rmsnorm_bwd_blocks(int max_rows);
 cudaError_t launch_colsum(const float* part, int nrows, int d, float* out, cudaStream_t st);
 
+// out[m] = scale * dx[src_row(m)] from the float32 residual gradient.
 template <typename T>
-cudaError_t launch_gather_scale(const T* dx, const int* kept_idx, const int* cnt, int S, int d, int max_rows,
+cudaError_t launch_gather_scale(const float* dx, const int* kept_idx, const int* cnt, int S, int d, int max_rows,
                                 float scale, T* out, cudaStream_t st);
 
 template <typename T>
@@ -114,6 +119,16 @@ cudaError_t launch_attn_fwd_mma(const bf16* qkv, int ldqkv, bf16* o, int ldo, fl
 cudaError_t launch_attn_bwd_mma(const bf16* qkv, int ldqkv, const bf16* o, const bf16* dO, int ldo,
                                 const float* lse, const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt,
                                 int S, int H, int Hkv, int Dh, int max_seqs, cudaStream_t st);
+// tcgen05 flash attention forward (head size 64 or 128, S % 128 == 0).
+bool attn_tc_supported(int S, int Dh);
+cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
+                               int Hkv, int Dh, int max_seqs, int* status, cudaStream_t st);
+// tcgen05 flash attention backward (head size 128, S % 128 == 0); zeroes
+// dq_acc and accumulates dQ (unscaled) into it.
+bool attn_bwd_tc_supported(int S, int Dh);
+cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
+                               const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
+                               int max_seqs, int* status, cudaStream_t st);
 cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const int* cnt, int S,
                              int max_rows, cudaStream_t st);
 
@@ -142,8 +157,9 @@ struct GemmArgs {
   void* D;
   int ldd;
   float alpha;
-  // EPI_RESID: x[r] = x[r] + alpha*acc for r = src_row(kept_idx, S, m); save[m] = new x[r]
-  void* x;
+  // EPI_RESID: x[r] = x[r] + alpha*acc for r = src_row(kept_idx, S, m) on the
+  // float32 residual stream x; save[m] = new x[r] in the operand type
+  float* x;
   int ldx;
   const int* kept_idx;
   int S;

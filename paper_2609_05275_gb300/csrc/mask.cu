@@ -3,7 +3,8 @@
 // Eq. (layer_dropout_train): M^{l,t} in {0,1}^B ~ Bernoulli(1 - p^{l,t});
 // Tensor Granularity subsection: one draw per sequence, or one per layer
 // and step for the whole batch; Preliminary section: the layer then runs on
-// {b : M[b] = 1} only, which this kernel lists in ascending b.
+// {b : M[b] = 1} only, which this kernel lists in ascending b.  A shard of a
+// data-parallel batch draws with its global sequence indices (b_offset + b).
 //
 // Draw: u = word 0 of Philox4x32-10 (Salmon et al., SC'11) with key
 // (seed lo, seed hi) and counter (b', l, t lo, t hi), b' = b per sequence
@@ -44,7 +45,7 @@ __global__ void mask_compact_kernel(const MaskParams P, unsigned char* __restric
     const int b = b0 + threadIdx.x;
     int keep = 0;
     if (b < P.B) {
-      const uint32_t bb = P.granularity == LD_PER_BATCH ? 0u : (uint32_t)b;
+      const uint32_t bb = P.granularity == LD_PER_BATCH ? 0u : (uint32_t)(P.b_offset + b);
       const uint32_t u = philox4x32_10(make_uint4(bb, (uint32_t)l, t_lo, t_hi), key).x;
       keep = (unsigned long long)u >= thr;
       mask[(size_t)l * P.B + b] = (unsigned char)keep;

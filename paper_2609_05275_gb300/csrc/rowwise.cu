@@ -64,8 +64,8 @@ int device_sm_count() {
 }
 
 // ---------------------------------------------------------------- RMSNorm fwd
-template <typename T>
-__global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const T* __restrict__ src, int gather,
+template <typename TS, typename T>
+__global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const TS* __restrict__ src, int gather,
                                                           const int* __restrict__ kept_idx,
                                                           const int* __restrict__ cnt, int S, int d,
                                                           const T* __restrict__ gamma, float eps,
@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const T* __restrict__ 
   const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
   for (long long m = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); m < M; m += nwarps) {
     const long long r = gather ? src_row(kept_idx, S, m) : m;
-    const T* xr = src + r * d;
+    const TS* xr = src + r * d;
     float ss = 0.f;
     for (int i = lane * 8; i < d; i += 256) {
       float v[8];
@@ -99,12 +99,12 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const T* __restrict__ 
   }
 }
 
-template <typename T>
-cudaError_t launch_rmsnorm_fwd(const T* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
+template <typename TS, typename T>
+cudaError_t launch_rmsnorm_fwd(const TS* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
                                int max_rows, const T* gamma, float eps, T* copy, T* out, float* rstd,
                                cudaStream_t st) {
   const int grid = grid_for(max_rows, 8, device_sm_count() * 16);
-  rmsnorm_fwd_kernel<T><<<grid, 256, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy, out, rstd);
+  rmsnorm_fwd_kernel<TS, T><<<grid, 256, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy, out, rstd);
   return cudaGetLastError();
 }
 
@@ -112,7 +112,7 @@ cudaError_t launch_rmsnorm_fwd(const T* src, int gather, const int* kept_idx, co
 template <typename T>
 __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const T* __restrict__ dyn, const T* __restrict__ xs,
                                                           const float* __restrict__ rstd,
-                                                          const T* __restrict__ gamma, T* __restrict__ dx,
+                                                          const T* __restrict__ gamma, float* __restrict__ dx,
                                                           const int* __restrict__ kept_idx,
                                                           const int* __restrict__ cnt, int S, int d, float scale,
                                                           T* __restrict__ next, float* __restrict__ part) {
@@ -149,7 +149,7 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const T* __restrict__ 
       for (int j = 0; j < 8; ++j) {
         const float xn = xv[j] * rs;
         cur[j] = cur[j] + rs * (dy[j] * g[j] - xn * dot);
-        nx[j] = scale * rnd(cur[j], dx);
+        nx[j] = scale * cur[j];
       }
       st8(dx + r * d + i, cur);
       if (next) st8(next + m * d + i, nx);
@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const T* __restrict__ 
 int rmsnorm_bwd_blocks(int max_rows) { return grid_for(max_rows, 8, device_sm_count() * 2); }
 
 template <typename T>
-cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, T* dx,
+cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, float* dx,
                                const int* kept_idx, const int* cnt, int S, int d, int max_rows, float scale,
                                T* next, float* part, int nblocks, cudaStream_t st) {
   const size_t smem = (size_t)d * sizeof(float);
@@ -191,7 +191,7 @@ cudaError_t launch_colsum(const float* part, int nrows, int d, float* out, cudaS
 
 // ------------------------------------------------------------- scaled gather
 template <typename T>
-__global__ void gather_scale_kernel(const T* __restrict__ dx, const int* __restrict__ kept_idx,
+__global__ void gather_scale_kernel(const float* __restrict__ dx, const int* __restrict__ kept_idx,
                                     const int* __restrict__ cnt, int S, int d, float scale, T* __restrict__ out) {
   const long long M = (long long)(*cnt) * S;
   const int per_row = d / 8;
@@ -209,10 +209,32 @@ __global__ void gather_scale_kernel(const T* __restrict__ dx, const int* __restr
 }
 
 template <typename T>
-cudaError_t launch_gather_scale(const T* dx, const int* kept_idx, const int* cnt, int S, int d, int max_rows,
+cudaError_t launch_gather_scale(const float* dx, const int* kept_idx, const int* cnt, int S, int d, int max_rows,
                                 float scale, T* out, cudaStream_t st) {
   const int grid = grid_for((long long)max_rows * (d / 8), 256, device_sm_count() * 8);
   gather_scale_kernel<T><<<grid, 256, 0, st>>>(dx, kept_idx, cnt, S, d, scale, out);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- conversion
+template <typename TI, typename TO>
+__global__ void convert_kernel(const TI* __restrict__ src, TO* __restrict__ dst, long long n8) {
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < n8; w += (long long)gridDim.x * blockDim.x) {
+    float v[8];
+    ld8(src + w * 8, v);
+    st8(dst + w * 8, v);
+  }
+}
+
+cudaError_t launch_convert(const void* src, int src_f32, void* dst, int dst_f32, long long n, cudaStream_t st) {
+  const long long n8 = n / 8;
+  const int grid = grid_for(n8, 256, device_sm_count() * 8);
+  if (src_f32 && !dst_f32)
+    convert_kernel<float, bf16><<<grid, 256, 0, st>>>(static_cast<const float*>(src), static_cast<bf16*>(dst), n8);
+  else if (!src_f32 && dst_f32)
+    convert_kernel<bf16, float><<<grid, 256, 0, st>>>(static_cast<const bf16*>(src), static_cast<float*>(dst), n8);
+  else
+    return cudaMemcpyAsync(dst, src, n * (src_f32 ? 4 : 2), cudaMemcpyDeviceToDevice, st);
   return cudaGetLastError();
 }
 
@@ -237,41 +259,45 @@ cudaError_t launch_rope_table(float* cos_t, float* sin_t, int S, int Dh, double 
 }
 
 // Rotate pairs (i, i+Dh/2) of the first `nheads` heads of each row, at the
-// row's position in its sequence; inverse = 1 applies the transpose.
+// row's position in its sequence; inverse = 1 applies the transpose.  One
+// thread per 8 consecutive pairs (16-byte accesses).
 template <typename T>
 __global__ void rope_apply_kernel(T* __restrict__ qkv, int ld, int nheads, int Dh, const float* __restrict__ cos_t,
                                   const float* __restrict__ sin_t, const int* __restrict__ cnt, int S,
                                   int inverse) {
   const long long M = (long long)(*cnt) * S;
-  const int half = Dh / 2;
-  const long long per_row = (long long)nheads * half;
+  const int half = Dh / 2, g8 = half / 8;
+  const int per_row = nheads * g8;
   const long long total = M * per_row;
   for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
        w += (long long)gridDim.x * blockDim.x) {
     const long long m = w / per_row;
-    const int rem = (int)(w % per_row);
-    const int h = rem / half, i = rem % half;
+    const int rem = (int)(w - m * per_row);
+    const int h = rem / g8, i = (rem - h * g8) * 8;
     const int pos = (int)(m % S);
-    const float c = cos_t[pos * half + i], s = sin_t[pos * half + i];
     T* p = qkv + m * ld + (long long)h * Dh;
-    const float a = to_f(p[i]), b = to_f(p[i + half]);
-    float na, nb;
-    if (!inverse) {
-      na = a * c - b * s;
-      nb = b * c + a * s;
-    } else {
-      na = a * c + b * s;
-      nb = b * c - a * s;
+    float a[8], b[8], c[8], sn[8];
+    ld8(p + i, a);
+    ld8(p + half + i, b);
+    ld8(cos_t + pos * half + i, c);
+    ld8(sin_t + pos * half + i, sn);
+    float na[8], nb[8];
+    const float sg = inverse ? -1.f : 1.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float s = sg * sn[j];
+      na[j] = a[j] * c[j] - b[j] * s;
+      nb[j] = b[j] * c[j] + a[j] * s;
     }
-    p[i] = from_f<T>(na);
-    p[i + half] = from_f<T>(nb);
+    st8(p + i, na);
+    st8(p + half + i, nb);
   }
 }
 
 template <typename T>
 cudaError_t launch_rope_apply(T* qkv, int ld, int nheads, int Dh, const float* cos_t, const float* sin_t,
                               const int* cnt, int S, int max_rows, int inverse, cudaStream_t st) {
-  const int grid = grid_for((long long)max_rows * nheads * (Dh / 2), 256, device_sm_count() * 8);
+  const int grid = grid_for((long long)max_rows * nheads * (Dh / 16), 256, device_sm_count() * 8);
   rope_apply_kernel<T><<<grid, 256, 0, st>>>(qkv, ld, nheads, Dh, cos_t, sin_t, cnt, S, inverse);
   return cudaGetLastError();
 }
@@ -279,47 +305,63 @@ cudaError_t launch_rope_apply(T* qkv, int ld, int nheads, int Dh, const float* c
 // -------------------------------------------------------------------- SwiGLU
 __device__ __forceinline__ float sigmoidf_(float g) { return 1.0f / (1.0f + expf(-g)); }
 
+// h = silu(g) * u with g = gu[:, j], u = gu[:, F + j]; 8 columns per thread.
 template <typename T>
 __global__ void swiglu_fwd_kernel(const T* __restrict__ gu, T* __restrict__ h, const int* __restrict__ cnt, int S,
                                   int F) {
   const long long M = (long long)(*cnt) * S;
-  const long long total = M * F;
+  const int F8 = F / 8;
+  const long long total = M * F8;
   for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
        w += (long long)gridDim.x * blockDim.x) {
-    const long long m = w / F;
-    const int j = (int)(w % F);
-    const float g = to_f(gu[m * 2 * F + j]), u = to_f(gu[m * 2 * F + F + j]);
-    h[w] = from_f<T>(g * sigmoidf_(g) * u);
+    const long long m = w / F8;
+    const int j = (int)(w - m * F8) * 8;
+    float g[8], u[8], o[8];
+    ld8(gu + m * 2 * F + j, g);
+    ld8(gu + m * 2 * F + F + j, u);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) o[k] = g[k] * sigmoidf_(g[k]) * u[k];
+    st8(h + m * F + j, o);
   }
 }
 
 template <typename T>
 cudaError_t launch_swiglu_fwd(const T* gu, T* h, const int* cnt, int S, int F, int max_rows, cudaStream_t st) {
-  const int grid = grid_for((long long)max_rows * F, 256, device_sm_count() * 8);
+  const int grid = grid_for((long long)max_rows * (F / 8), 256, device_sm_count() * 8);
   swiglu_fwd_kernel<T><<<grid, 256, 0, st>>>(gu, h, cnt, S, F);
   return cudaGetLastError();
 }
 
+// dg = dh * u * s (1 + g (1 - s)), du = dh * g * s with s = sigmoid(g).
 template <typename T>
 __global__ void swiglu_bwd_kernel(const T* __restrict__ dh, const T* __restrict__ gu, T* __restrict__ dgu,
                                   const int* __restrict__ cnt, int S, int F) {
   const long long M = (long long)(*cnt) * S;
-  const long long total = M * F;
+  const int F8 = F / 8;
+  const long long total = M * F8;
   for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
        w += (long long)gridDim.x * blockDim.x) {
-    const long long m = w / F;
-    const int j = (int)(w % F);
-    const float g = to_f(gu[m * 2 * F + j]), u = to_f(gu[m * 2 * F + F + j]);
-    const float sg = sigmoidf_(g), dv = to_f(dh[w]);
-    dgu[m * 2 * F + j] = from_f<T>(dv * u * sg * (1.0f + g * (1.0f - sg)));
-    dgu[m * 2 * F + F + j] = from_f<T>(dv * g * sg);
+    const long long m = w / F8;
+    const int j = (int)(w - m * F8) * 8;
+    float g[8], u[8], dv[8], dg[8], du[8];
+    ld8(gu + m * 2 * F + j, g);
+    ld8(gu + m * 2 * F + F + j, u);
+    ld8(dh + m * F + j, dv);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float sg = sigmoidf_(g[k]);
+      dg[k] = dv[k] * u[k] * sg * (1.0f + g[k] * (1.0f - sg));
+      du[k] = dv[k] * g[k] * sg;
+    }
+    st8(dgu + m * 2 * F + j, dg);
+    st8(dgu + m * 2 * F + F + j, du);
   }
 }
 
 template <typename T>
 cudaError_t launch_swiglu_bwd(const T* dh, const T* gu, T* dgu, const int* cnt, int S, int F, int max_rows,
                               cudaStream_t st) {
-  const int grid = grid_for((long long)max_rows * F, 256, device_sm_count() * 8);
+  const int grid = grid_for((long long)max_rows * (F / 8), 256, device_sm_count() * 8);
   swiglu_bwd_kernel<T><<<grid, 256, 0, st>>>(dh, gu, dgu, cnt, S, F);
   return cudaGetLastError();
 }
@@ -351,11 +393,13 @@ cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, c
 }
 
 #define LD_INST(T)                                                                                              \
-  template cudaError_t launch_rmsnorm_fwd<T>(const T*, int, const int*, const int*, int, int, int, const T*,    \
-                                             float, T*, T*, float*, cudaStream_t);                              \
-  template cudaError_t launch_rmsnorm_bwd<T>(const T*, const T*, const float*, const T*, T*, const int*,        \
+  template cudaError_t launch_rmsnorm_fwd<float, T>(const float*, int, const int*, const int*, int, int, int,   \
+                                                    const T*, float, T*, T*, float*, cudaStream_t);             \
+  template cudaError_t launch_rmsnorm_fwd<T, T>(const T*, int, const int*, const int*, int, int, int, const T*, \
+                                                float, T*, T*, float*, cudaStream_t);                           \
+  template cudaError_t launch_rmsnorm_bwd<T>(const T*, const T*, const float*, const T*, float*, const int*,    \
                                              const int*, int, int, int, float, T*, float*, int, cudaStream_t);  \
-  template cudaError_t launch_gather_scale<T>(const T*, const int*, const int*, int, int, int, float, T*,        \
+  template cudaError_t launch_gather_scale<T>(const float*, const int*, const int*, int, int, int, float, T*,    \
                                               cudaStream_t);                                                    \
   template cudaError_t launch_rope_apply<T>(T*, int, int, int, const float*, const float*, const int*, int, int, \
                                             int, cudaStream_t);                                                 \
@@ -363,7 +407,20 @@ cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, c
   template cudaError_t launch_swiglu_bwd<T>(const T*, const T*, T*, const int*, int, int, int, cudaStream_t);   \
   template cudaError_t launch_attn_rowdot<T>(const T*, const T*, int, int, int, const int*, int, int, float*,   \
                                              cudaStream_t);
-LD_INST(float)
 LD_INST(bf16)
+template cudaError_t launch_rmsnorm_fwd<float, float>(const float*, int, const int*, const int*, int, int, int,
+                                                      const float*, float, float*, float*, float*, cudaStream_t);
+template cudaError_t launch_rmsnorm_bwd<float>(const float*, const float*, const float*, const float*, float*,
+                                               const int*, const int*, int, int, int, float, float*, float*, int,
+                                               cudaStream_t);
+template cudaError_t launch_gather_scale<float>(const float*, const int*, const int*, int, int, int, float, float*,
+                                                cudaStream_t);
+template cudaError_t launch_rope_apply<float>(float*, int, int, int, const float*, const float*, const int*, int, int,
+                                              int, cudaStream_t);
+template cudaError_t launch_swiglu_fwd<float>(const float*, float*, const int*, int, int, int, cudaStream_t);
+template cudaError_t launch_swiglu_bwd<float>(const float*, const float*, float*, const int*, int, int, int,
+                                              cudaStream_t);
+template cudaError_t launch_attn_rowdot<float>(const float*, const float*, int, int, int, const int*, int, int,
+                                               float*, cudaStream_t);
 
 }  // namespace ldk

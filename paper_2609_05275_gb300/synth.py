@@ -8,7 +8,10 @@ Recipe (the paper trains on a private corpus on Cerebras CS-3; token values
 do not change the work done, so activations stand in for embedded tokens):
   * activations x ~ N(0, 1) drawn in float32, rounded to bf16;
   * weights N(0, 0.02) per matrix, RMSNorm gains gamma = 1 (optionally
-    1 + N(0, 0.1) to exercise the gain gradient), rounded to bf16;
+    1 + N(0, 0.1) to exercise the gain gradient), rounded to bf16; workloads
+    with init "depth_scaled" draw the residual output projections (w_o, w_d)
+    with std 0.02 / sqrt(2 L), the depth-scaled init of deep pre-norm
+    decoders, so that the residual branches do not grow with depth;
   * upstream gradient dY ~ N(0, 1) in float32, rounded to bf16.
 Every tensor comes from its own ``torch.Generator`` seeded from (seed, tag,
 layer), so any one of them can be regenerated alone.
@@ -21,8 +24,10 @@ import torch
 CONFIGS = {
     "tiny": dict(L=2, d=128, H=4, Hkv=4, Dh=32, F=512, B=8, S=64, eps=1e-6, rope_theta=1e4, alpha=1.0),
     "gpt2": dict(L=12, d=768, H=12, Hkv=12, Dh=64, F=2048, B=16, S=1024, eps=1e-6, rope_theta=1e4, alpha=1.0),
-    "1.3b": dict(L=24, d=2048, H=16, Hkv=16, Dh=128, F=5632, B=8, S=2048, eps=1e-6, rope_theta=1e4, alpha=1.0),
-    "llama8b": dict(L=32, d=4096, H=32, Hkv=8, Dh=128, F=14336, B=4, S=4096, eps=1e-6, rope_theta=5e5, alpha=1.0),
+    "1.3b": dict(L=24, d=2048, H=16, Hkv=16, Dh=128, F=5632, B=8, S=2048, eps=1e-6, rope_theta=1e4, alpha=1.0,
+                 init="depth_scaled"),
+    "llama8b": dict(L=32, d=4096, H=32, Hkv=8, Dh=128, F=14336, B=4, S=4096, eps=1e-6, rope_theta=5e5, alpha=1.0,
+                    init="depth_scaled"),
 }
 
 # Drop-rate schedules the workloads name (distribution x time schedule, seed).
@@ -71,7 +76,10 @@ def layer_weights(cfg, layer, seed=0, device="cpu", dtype=torch.bfloat16, std=0.
             if gamma_noise:
                 t += gamma_noise * torch.randn(shape, generator=g, device=device, dtype=torch.float32)
         else:
-            t = std * torch.randn(shape, generator=g, device=device, dtype=torch.float32)
+            sd = std
+            if cfg.get("init") == "depth_scaled" and name in ("w_o", "w_d"):
+                sd = std / (2.0 * cfg["L"]) ** 0.5
+            t = sd * torch.randn(shape, generator=g, device=device, dtype=torch.float32)
         out[name] = t.to(torch.bfloat16).to(dtype)
     return out
 

@@ -1,0 +1,93 @@
+"""Parity at the workloads' full sizes, in the launch configuration the
+benchmark times (full B x S, all layers, bf16 tensor-core path).
+
+The oracle cannot run a full Llama-sized step, so the comparison uses two
+properties of the stack that hold at any size (both pinned on the oracle in
+test_oracle_stack.py):
+  * causality: output row i of a sequence depends only on its rows <= i, so
+    the first R output rows equal the output of the sequence cut to R rows;
+  * with dY zero outside the first R rows of two chosen sequences, every
+    weight gradient and dX come from those rows only (and dX is exactly zero
+    elsewhere).
+The oracle therefore runs the two chosen sequences cut to R rows (one kept
+at most layers, one dropped at one layer or more), and the GPU output/dX on
+those rows and the full weight gradients are compared with it.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_05275_gb300 import synth
+from parity import check_close, gpu_run, oracle_masks, oracle_run, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+def _pick(mask):
+    kept = mask.sum(axis=0)
+    a = int(np.argmax(kept))
+    order = np.argsort(kept, kind="stable")
+    b = int(next(s for s in order if s != a))
+    return sorted({a, b})
+
+
+def _run(name, step, R, granularity="per_sequence", sched=None, fp32=False, seqs=None):
+    cfg = synth.CONFIGS[name]
+    sched = sched or synth.SCHEDULES[name]
+    dtype = torch.float32 if fp32 else torch.bfloat16
+    mask, _, _ = oracle_masks(cfg, sched, step, granularity)
+    seqs = seqs if seqs is not None else _pick(mask)
+    dev = synth.stack_weights(cfg, seed=0, device="cuda")
+    x = synth.activations(cfg, seed=0, device="cuda")
+    dy = synth.upstream_grad(cfg, device="cuda")
+    keep = torch.zeros_like(dy)
+    for s in seqs:
+        keep[s, :R] = 1
+    dy = dy * keep
+    devT = [{n: v.to(dtype) for n, v in W.items()} for W in dev]
+    out, dX, grads, (gmask, idx, cnt) = gpu_run(cfg, sched, step, devT, x.to(dtype), dy.to(dtype), granularity, fp32)
+    assert (gmask == mask).all()
+    host = [{n: v.cpu() for n, v in W.items()} for W in dev]
+    del devT
+    B, S = cfg["B"], cfg["S"]
+    out = out.view(B, S, -1)
+    dX = dX.view(B, S, -1)
+    # gradient rows outside the sampled region are exactly zero
+    rest = torch.ones(B, S, dtype=torch.bool, device=dX.device)
+    for s in seqs:
+        rest[s, :R] = False
+    assert (dX[rest] == 0).all()
+    rout, rdX, rgrads, _ = oracle_run(cfg, sched, step, host, x.cpu(), dy.cpu(), granularity, rows=R, seqs=seqs)
+    check_close(f"{name} out", to_np(out[seqs, :R]), rout, fp32)
+    check_close(f"{name} dX", to_np(dX[seqs, :R]), rdX, fp32)
+    for l in range(cfg["L"]):
+        for n in grads[l]:
+            check_close(f"{name} layer{l}.{n}", to_np(grads[l][n]), rgrads[l][n], fp32)
+    return mask, seqs
+
+
+def test_gpt2_full():
+    mask, seqs = _run("gpt2", 0, R=64)
+    assert mask[0].all()
+
+
+def test_gpt2_full_fp32_debug():
+    _run("gpt2", 0, R=64, fp32=True)
+
+
+@pytest.mark.parametrize("step", [0, 500, 2000])
+def test_1p3b_full_ramp(step):
+    mask, _ = _run("1.3b", step, R=64)
+    if step == 0:
+        assert mask.all()  # ramp factor 0 at step 0: nothing dropped
+
+
+def test_1p3b_sweep_per_batch():
+    sched = dict(dist="uniform", p_max=0.5, time="const", seed=7)
+    _run("1.3b", 0, R=64, granularity="per_batch", sched=sched)
+
+
+def test_llama8b_full():
+    mask, seqs = _run("llama8b", 0, R=32)
+    assert mask[0].all() and not mask.all()

@@ -80,3 +80,18 @@ def test_ragged_kept_tiles(fp32):
         cfg = dict(synth.CONFIGS["tiny"], S=S, B=B, L=2, F=320, d=192, H=6, Hkv=3)
         sched = dict(dist="explicit", p_explicit=[0.3, 0.6], time="const", seed=5)
         _compare(cfg, sched, 1, fp32, gamma_noise=0.05)
+
+
+MULTI = [
+    dict(L=2, d=256, H=4, Hkv=2, Dh=64, F=512, B=3, S=512, eps=1e-6, rope_theta=1e4, alpha=1.0),
+    dict(L=2, d=512, H=4, Hkv=1, Dh=128, F=768, B=2, S=1024, eps=1e-6, rope_theta=5e5, alpha=0.5),
+]
+
+
+@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
+@pytest.mark.parametrize("cfg", MULTI, ids=["S512-dh64-gqa", "S1024-dh128-mqa"])
+def test_multi_tile_full_tensors(cfg, fp32):
+    # every attention and GEMM tile of several-tile sequences, compared on the
+    # full tensors (not just the first rows)
+    sched = dict(dist="explicit", p_explicit=[0.2, 0.5], time="const", seed=11)
+    _compare(cfg, sched, 2, fp32, gamma_noise=0.1)
