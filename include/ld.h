@@ -214,6 +214,27 @@ ld_status ld_gemm_bf16(int M, int N, int K, const void* A, int lda, int a_mn_maj
                        int ldb, int b_mn_major, void* D, int ldd, int d_f32, float alpha,
                        int* status_ws, void* stream);
 
+/* RMSNorm backward with the residual-gradient update on the kept rows of one
+ * layer: the last step of each branch of ld_backward (derivative of the
+ * pre-norm block of Eq. (transformer_layer_dropout_train) w.r.t. its input
+ * through RMSNorm(x) = x / sqrt(mean(x^2) + eps) * gamma).  For compact row
+ * m < kept_cnt[0] * S, stored at residual row r = kept_idx[m / S] * S + m % S:
+ *   xn = xs[m] * rstd[m],  gd = dyn[m] * gamma
+ *   dx[r] += rstd[m] * (gd - xn * mean(gd * xn))            (float32)
+ *   next[m] = scale * dx[r]                      (bf16; skipped if NULL)
+ *   dgamma  = sum over the kept rows of dyn[m] * xn          (float32)
+ * dyn: float [kept*S, d]; xs: float [kept*S, d] (the normalised input's
+ * source rows, compact); rstd: float [kept*S]; gamma: bf16 [d]; kept_idx: int [B],
+ * kept_cnt: int [1] (device; read by the kernels, so they may be produced
+ * on the same stream); dx: float [B*S, d] in/out; dgamma: float [d] out.
+ * scratch: float device buffer of scratch_bytes >= nb * d * 4 bytes, nb =
+ * min(ceil(B*S / 8), 320), for the per-block partial sums of dgamma.
+ * Requires d % 8 == 0, d <= 16384, B, S >= 1; LD_ERR_ARG for null or
+ * misaligned pointers or a short scratch buffer.  Async on `stream`. */
+ld_status ld_rmsnorm_backward(int B, int S, int d, const float* dyn, const void* xs, const float* rstd,
+                              const void* gamma, const int* kept_idx, const int* kept_cnt, float* dx, void* next,
+                              float scale, float* dgamma, float* scratch, size_t scratch_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -84,6 +84,9 @@ def lib():
             "ld_status_str": (c_char_p, [c_int]),
             "ld_set_timing": (c_int, [c_void_p, c_int]),
             "ld_get_timing": (c_int, [c_void_p, c_int, POINTER(c_double), POINTER(c_longlong)]),
+            "ld_rmsnorm_backward": (c_int, [c_int, c_int, c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                            c_void_p, c_void_p, c_void_p, c_float, c_void_p, c_void_p, c_size_t,
+                                            c_void_p]),
             "ld_gemm_bf16": (c_int, [c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_int, c_void_p,
                                      c_int, c_int, c_float, c_void_p, c_void_p]),
         }
@@ -226,6 +229,19 @@ def ld_gemm_bf16(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, alpha=1.0, status=
     d_f32 = 1 if D.dtype == torch.float32 else 0
     _check(lib().ld_gemm_bf16(M, N, K, _ptr(A), lda, int(a_mn), _ptr(B), ldb, int(b_mn), _ptr(D), ldd, d_f32,
                               float(alpha), _ptr(status), _stream(stream)), "ld_gemm_bf16")
+
+
+def rmsnorm_backward_scratch_bytes(B, S, d):
+    nb = min((B * S + 7) // 8, 320)
+    return nb * d * 4
+
+
+def ld_rmsnorm_backward(B, S, d, dyn, xs, rstd, gamma, kept_idx, kept_cnt, dx, nxt, scale, dgamma, scratch,
+                        stream=None):
+    _check(lib().ld_rmsnorm_backward(B, S, d, _ptr(dyn), _ptr(xs), _ptr(rstd), _ptr(gamma), _ptr(kept_idx),
+                                     _ptr(kept_cnt), _ptr(dx), _ptr(nxt), float(scale), _ptr(dgamma), _ptr(scratch),
+                                     scratch.numel() * scratch.element_size(), _stream(stream)),
+           "ld_rmsnorm_backward")
 
 
 def weight_table(layers):

@@ -146,12 +146,12 @@ void make_layout(Handle* h) {
     lo = align_up(lo + bytes);
     return at;
   };
-  y.xin = ltake(R * c.d * e);
+  y.xin = ltake(R * c.d * 4);  // float32 copies of X and Z (RMSNorm backward)
   y.xh = ltake(R * c.d * e);
   y.qkv = ltake(R * h->nqkv * e);
   y.o = ltake(R * c.H * c.Dh * e);
   y.lse = ltake((size_t)c.H * R * 4);
-  y.z = ltake(R * c.d * e);
+  y.z = ltake(R * c.d * 4);
   y.zh = ltake(R * c.d * e);
   y.gu = ltake(R * 2 * c.F * e);
   y.h = ltake(R * c.F * e);
@@ -164,11 +164,11 @@ void make_layout(Handle* h) {
   y.dy = take(R * c.d * e);
   y.dh = take(R * c.F * e);
   y.dgu = take(R * 2 * c.F * e);
-  y.dzh = take(R * c.d * e);
+  y.dzh = take(R * c.d * 4);  // float32: inputs of the RMSNorm backward
   y.dz = take(R * c.d * e);
   y.dO = take(R * c.H * c.Dh * e);
   y.dqkv = take(R * h->nqkv * e);
-  y.dxh = take(R * c.d * e);
+  y.dxh = take(R * c.d * 4);
   y.Dvec = take((size_t)c.H * R * 4);
   y.dqacc = take(R * c.H * c.Dh * 4);
   y.part = take((size_t)h->part_blocks * c.d * 4);
@@ -290,32 +290,46 @@ cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, 
   return launch_attn_fwd_mma(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, st);
 }
 
+// Attention backward: dq, dk, dv into dqkv with the inverse RoPE applied to
+// dq and dk (fused into dq_finish and the tcgen05 kernel's dK epilogue on
+// the bf16 path; a separate rotation otherwise).
 template <typename T>
 cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const T* dO, const float* lse, float* Dvec,
                      T* dqkv, const int* cnt, cudaStream_t st) {
   const ld_config& c = h->cfg;
+  const bool rope = c.rope_theta != 0.0f;
+  const float* rcos = rope ? at<float>(ws, h->lay.rcos) : nullptr;
+  const float* rsin = rope ? at<float>(ws, h->lay.rsin) : nullptr;
   cudaError_t e = launch_attn_rowdot<T>(dO, o, c.H * c.Dh, c.H, c.Dh, cnt, c.S, h->max_rows, Dvec, st);
   if (e != cudaSuccess) return e;
-  if (sizeof(T) == 4)
-    return launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, cnt, c.S, c.H, c.Hkv, c.Dh,
-                                   h->max_rows, st);
+  if (sizeof(T) == 4) {
+    e = launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, cnt, c.S, c.H, c.Hkv, c.Dh,
+                                h->max_rows, st);
+    if (e != cudaSuccess || !rope) return e;
+    return launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1, st);
+  }
   float* dq_acc = at<float>(ws, h->lay.dqacc);
   const bf16* q16 = reinterpret_cast<const bf16*>(qkv);
   bf16* d16 = reinterpret_cast<bf16*>(dqkv);
-  if (attn_bwd_tc_supported(c.S, c.Dh))
+  if (attn_bwd_tc_supported(c.S, c.Dh)) {
     e = launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt,
-                           c.S, c.H, c.Hkv, c.B, at<int>(ws, h->lay.status), st);
-  else
+                           c.S, c.H, c.Hkv, c.B, rcos, rsin, at<int>(ws, h->lay.status), st);
+  } else {
     e = launch_attn_bwd_mma(q16, h->nqkv, reinterpret_cast<const bf16*>(o), reinterpret_cast<const bf16*>(dO),
-                          c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, st);
+                            c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, st);
+    if (e == cudaSuccess && rope)  // the k heads of dqkv
+      e = launch_rope_apply<bf16>(d16 + (size_t)c.H * c.Dh, h->nqkv, c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1,
+                                  st);
+  }
   if (e != cudaSuccess) return e;
-  return launch_dq_finish(dq_acc, d16, h->nqkv, c.H, c.Dh, cnt, c.S, h->max_rows, st);
+  return launch_dq_finish(dq_acc, d16, h->nqkv, c.H, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, st);
 }
 
 template <typename T>
 ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv, void* ws, cudaStream_t st) {
   const ld_config& c = h->cfg;
   const Layout& y = h->lay;
+  const bool fused_rope = sizeof(T) == 2 && c.rope_theta != 0.0f && c.Dh >= 64;
   // The residual stream is carried in float32 through the layers (bf16 in
   // and out at the boundary): 2*L in-place bf16 roundings of X would
   // otherwise accumulate to several per cent of |X| at 32 layers.
@@ -351,12 +365,12 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     const int* cnt = kcnt + l;
     const int* ki = kidx + (size_t)l * c.B;
     char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
-    T* xin = reinterpret_cast<T*>(lb + y.xin);
+    float* xin = reinterpret_cast<float*>(lb + y.xin);
     T* xh = reinterpret_cast<T*>(lb + y.xh);
     T* qkv = reinterpret_cast<T*>(lb + y.qkv);
     T* o = reinterpret_cast<T*>(lb + y.o);
     float* lse = reinterpret_cast<float*>(lb + y.lse);
-    T* z = reinterpret_cast<T*>(lb + y.z);
+    float* z = reinterpret_cast<float*>(lb + y.z);
     T* zh = reinterpret_cast<T*>(lb + y.zh);
     T* gu = reinterpret_cast<T*>(lb + y.gu);
     T* hh = reinterpret_cast<T*>(lb + y.h);
@@ -371,8 +385,16 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     a.epi = EPI_STORE;
     a.D = qkv;
     a.ldd = h->nqkv;
+    if (fused_rope) {  // RoPE on the q / k heads in the projection's epilogue
+      a.epi = EPI_ROPE;
+      a.rope_cos = rcos;
+      a.rope_sin = rsin;
+      a.Dh = c.Dh;
+      a.S = c.S;
+      a.rope_cols = (c.H + c.Hkv) * c.Dh;
+    }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (c.rope_theta != 0.0f)
+    if (c.rope_theta != 0.0f && !fused_rope)
       { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 0, st)); }
     { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_fwd<T>(h, ws, qkv, o, lse, cnt, st)); }
     a = rows_gemm(h, cnt, c.d, HD, o, HD, W[l].w_o, HD, 0);
@@ -385,13 +407,18 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     a.save = z;
     a.ld_save = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<T, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (T*)nullptr, zh, rstd2, st)); }
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st)); }
     a = rows_gemm(h, cnt, 2 * c.F, c.d, zh, c.d, W[l].w_gu, c.d, 0);
     a.epi = EPI_STORE;
     a.D = gu;
     a.ldd = 2 * c.F;
+    if (!f32) {  // h = silu(g) u in the projection's epilogue
+      a.epi = EPI_SWIGLU;
+      a.h_out = hh;
+      a.F = c.F;
+    }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cnt, c.S, c.F, h->max_rows, st)); }
+    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cnt, c.S, c.F, h->max_rows, st)); }
     a = rows_gemm(h, cnt, c.d, c.F, hh, c.F, W[l].w_d, c.F, 0);
     a.epi = EPI_RESID;
     a.alpha = s;
@@ -423,11 +450,11 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
   T* dy = at<T>(ws, y.dy);
   T* dh = at<T>(ws, y.dh);
   T* dgu = at<T>(ws, y.dgu);
-  T* dzh = at<T>(ws, y.dzh);
+  float* dzh = at<float>(ws, y.dzh);
   T* dz = at<T>(ws, y.dz);
   T* dO = at<T>(ws, y.dO);
   T* dqkv = at<T>(ws, y.dqkv);
-  T* dxh = at<T>(ws, y.dxh);
+  float* dxh = at<float>(ws, y.dxh);
   float* Dvec = at<float>(ws, y.Dvec);
   float* part = at<float>(ws, y.part);
   const int HD = c.H * c.Dh;
@@ -440,12 +467,12 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     const int* cnt = kcnt + l;
     const int* ki = kidx + (size_t)l * c.B;
     char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
-    T* xin = reinterpret_cast<T*>(lb + y.xin);
+    float* xin = reinterpret_cast<float*>(lb + y.xin);
     T* xh = reinterpret_cast<T*>(lb + y.xh);
     T* qkv = reinterpret_cast<T*>(lb + y.qkv);
     T* o = reinterpret_cast<T*>(lb + y.o);
     float* lse = reinterpret_cast<float*>(lb + y.lse);
-    T* z = reinterpret_cast<T*>(lb + y.z);
+    float* z = reinterpret_cast<float*>(lb + y.z);
     T* zh = reinterpret_cast<T*>(lb + y.zh);
     T* gu = reinterpret_cast<T*>(lb + y.gu);
     T* hh = reinterpret_cast<T*>(lb + y.h);
@@ -461,11 +488,17 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     a.epi = EPI_STORE;
     a.D = dh;
     a.ldd = c.F;
+    if (!f32) {  // SwiGLU backward in the epilogue: dg, du straight from dh
+      a.epi = EPI_SWIGLU_BWD;
+      a.D = dgu;
+      a.gu = gu;
+      a.F = c.F;
+    }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cnt, c.S, c.F, h->max_rows, st)); }
+    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cnt, c.S, c.F, h->max_rows, st)); }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
     a = rows_gemm(h, cnt, c.d, 2 * c.F, dgu, 2 * c.F, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
-    a.epi = EPI_STORE;
+    a.epi = EPI_STORE_F32;
     a.D = dzh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
@@ -485,10 +518,8 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, HD, dz, c.d, o, HD, G[l].w_o), st)); }  // dW_o = dz^T o
     { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_bwd<T>(h, ws, qkv, o, dO, lse, Dvec, dqkv, cnt, st)); }
-    if (c.rope_theta != 0.0f)
-      { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1, st)); }
     a = rows_gemm(h, cnt, c.d, h->nqkv, dqkv, h->nqkv, W[l].w_qkv, c.d, 1);  // dxh = dqkv W_qkv
-    a.epi = EPI_STORE;
+    a.epi = EPI_STORE_F32;
     a.D = dxh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
@@ -703,6 +734,25 @@ ld_status ld_get_timing(void* handle, int kclass, double* ms, long long* launche
   }
   if (ms) *ms = tot;
   if (launches) *launches = (long long)pairs;
+  return LD_OK;
+}
+
+ld_status ld_rmsnorm_backward(int B, int S, int d, const float* dyn, const void* xs, const float* rstd,
+                              const void* gamma, const int* kept_idx, const int* kept_cnt, float* dx, void* next,
+                              float scale, float* dgamma, float* scratch, size_t scratch_bytes, void* stream) {
+  if (B < 1 || S < 1 || d < 8 || d % 8 || d > 16384 || (long long)B * S > (1ll << 30)) return LD_ERR_SHAPE;
+  const void* ps[] = {dyn, xs, rstd, gamma, dx, dgamma, scratch};
+  for (const void* p : ps)
+    if (!p || !aligned16(p)) return LD_ERR_ARG;
+  if (!kept_idx || !kept_cnt || (next && !aligned16(next))) return LD_ERR_ARG;
+  long long nb = ((long long)B * S + 7) / 8;
+  if (nb > 320) nb = 320;
+  if (scratch_bytes < (size_t)nb * d * sizeof(float)) return LD_ERR_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  LD_CHECK(launch_rmsnorm_bwd<bf16>(dyn, static_cast<const float*>(xs), rstd, static_cast<const bf16*>(gamma), dx,
+                                    kept_idx, kept_cnt, S, d, B * S, scale, static_cast<bf16*>(next), scratch,
+                                    (int)nb, st));
+  LD_CHECK(launch_colsum(scratch, (int)nb, d, dgamma, st));
   return LD_OK;
 }
 

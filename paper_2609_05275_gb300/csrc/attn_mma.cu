@@ -374,19 +374,44 @@ __global__ void __launch_bounds__(128) attn_bwd_kernel(const bf16* __restrict__ 
   }
 }
 
-__global__ void dq_finish_kernel(const float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, int HD, float c,
+// dq = c * dq_acc, then the inverse rotary rotation of each q head (pairs
+// (i, i + Dh/2) at the row's position), written as bf16 into dqkv.
+__global__ void dq_finish_kernel(const float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, int H, int Dh,
+                                 float c, const float* __restrict__ rcos, const float* __restrict__ rsin,
                                  const int* __restrict__ cnt, int S) {
   const long long M = (long long)(*cnt) * S;
-  const long long total = M * (HD / 4);
+  const int half = Dh / 2, HD = H * Dh;
+  const int per_row = H * (half / 4);
+  const long long total = M * per_row;
   for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
        w += (long long)gridDim.x * blockDim.x) {
-    const long long m = w / (HD / 4);
-    const int i = (int)(w % (HD / 4)) * 4;
-    const float4 v = *reinterpret_cast<const float4*>(dq_acc + m * HD + i);
-    uint2 out;
-    out.x = pack(c * v.x, c * v.y);
-    out.y = pack(c * v.z, c * v.w);
-    *reinterpret_cast<uint2*>(dqkv + m * ldq + i) = out;
+    const long long m = w / per_row;
+    const int rem = (int)(w - m * per_row);
+    const int h = rem / (half / 4), i = (rem - h * (half / 4)) * 4;
+    const float* src = dq_acc + m * HD + (long long)h * Dh + i;
+    const float4 a = *reinterpret_cast<const float4*>(src);
+    const float4 b = *reinterpret_cast<const float4*>(src + half);
+    float x1[4] = {c * a.x, c * a.y, c * a.z, c * a.w}, x2[4] = {c * b.x, c * b.y, c * b.z, c * b.w};
+    if (rcos) {
+      const int pos = (int)(m % S);
+      const float4 cv = *reinterpret_cast<const float4*>(rcos + (size_t)pos * half + i);
+      const float4 sv = *reinterpret_cast<const float4*>(rsin + (size_t)pos * half + i);
+      const float cs[4] = {cv.x, cv.y, cv.z, cv.w}, sn[4] = {sv.x, sv.y, sv.z, sv.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float p1 = x1[k], p2 = x2[k];
+        x1[k] = p1 * cs[k] + p2 * sn[k];
+        x2[k] = p2 * cs[k] - p1 * sn[k];
+      }
+    }
+    bf16* dst = dqkv + m * ldq + (long long)h * Dh + i;
+    uint2 o1, o2;
+    o1.x = pack(x1[0], x1[1]);
+    o1.y = pack(x1[2], x1[3]);
+    o2.x = pack(x2[0], x2[1]);
+    o2.y = pack(x2[2], x2[3]);
+    *reinterpret_cast<uint2*>(dst) = o1;
+    *reinterpret_cast<uint2*>(dst + half) = o2;
   }
 }
 
@@ -442,15 +467,14 @@ cudaError_t launch_attn_bwd_mma(const bf16* qkv, int ldqkv, const bf16* o, const
   return bwd_launch<128>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, st);
 }
 
-cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const int* cnt, int S,
-                             int max_rows, cudaStream_t st) {
-  const int HD = H * Dh;
-  long long work = (long long)max_rows * (HD / 4);
+cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const float* rcos,
+                             const float* rsin, const int* cnt, int S, int max_rows, cudaStream_t st) {
+  long long work = (long long)max_rows * H * (Dh / 8);
   long long grid = (work + 255) / 256;
   const long long cap = (long long)device_sm_count() * 8;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  dq_finish_kernel<<<(int)grid, 256, 0, st>>>(dq_acc, dqkv, ldqkv, HD, rsqrtf((float)Dh), cnt, S);
+  dq_finish_kernel<<<(int)grid, 256, 0, st>>>(dq_acc, dqkv, ldqkv, H, Dh, rsqrtf((float)Dh), rcos, rsin, cnt, S);
   return cudaGetLastError();
 }
 

@@ -29,6 +29,18 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescale = 8.0f;  // move the running max only when it grows by > 2^8
 
+__device__ __forceinline__ void st_bf16x32_(bf16* dst, const float* v) {
+  uint4* p = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    uint4 q;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&q);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) h[j] = __floats2bfloat162_rn(v[8 * i + 2 * j], v[8 * i + 2 * j + 1]);
+    p[i] = q;
+  }
+}
+
 // byte offset of element (row r, 16-byte chunk i) in a 128B-swizzled
 // K-major slab of 128-byte rows
 __device__ __forceinline__ uint32_t swz(int r, int i) {
@@ -304,7 +316,8 @@ __global__ void __launch_bounds__(320, 1)
                        const __grid_constant__ CUtensorMap tmo,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
-                       int S, int H, int Hkv, int* status) {
+                       int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
+                       int* status) {
   constexpr int DH = 128;
   constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
   constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
@@ -511,23 +524,31 @@ __global__ void __launch_bounds__(320, 1)
       bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
       bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
 #pragma unroll 1
-      for (int cc = 0; cc < DH / 32; ++cc) {
-        float t[32], u[32];
-        tmem_ld32(t_dk + cc * 32 + lane_off, t);
-        tmem_ld32(t_dv + cc * 32 + lane_off, u);
+      for (int cc = 0; cc < 2; ++cc) {
+        // dK pairs (i, i + 64), i = 32cc .. 32cc+31: scale, inverse rotation at
+        // the key's position, bf16
+        float k1[32], k2[32];
+        tmem_ld32(t_dk + cc * 32 + lane_off, k1);
+        tmem_ld32(t_dk + 64 + cc * 32 + lane_off, k2);
 #pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          uint4 a, bq;
-          __nv_bfloat162* ha = reinterpret_cast<__nv_bfloat162*>(&a);
-          __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&bq);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            ha[k] = __floats2bfloat162_rn(c * t[8 * q4 + 2 * k], c * t[8 * q4 + 2 * k + 1]);
-            hb[k] = __floats2bfloat162_rn(u[8 * q4 + 2 * k], u[8 * q4 + 2 * k + 1]);
+        for (int e = 0; e < 32; ++e) {
+          const float p1 = c * k1[e], p2 = c * k2[e];
+          float cs = 1.f, sn = 0.f;
+          if (rcos) {
+            cs = rcos[(size_t)key * 64 + cc * 32 + e];
+            sn = rsin[(size_t)key * 64 + cc * 32 + e];
           }
-          reinterpret_cast<uint4*>(krow + cc * 32)[q4] = a;
-          reinterpret_cast<uint4*>(vrow + cc * 32)[q4] = bq;
+          k1[e] = p1 * cs + p2 * sn;
+          k2[e] = p2 * cs - p1 * sn;
         }
+        st_bf16x32_(krow + cc * 32, k1);
+        st_bf16x32_(krow + 64 + cc * 32, k2);
+      }
+#pragma unroll 1
+      for (int cc = 0; cc < DH / 32; ++cc) {
+        float u[32];
+        tmem_ld32(t_dv + cc * 32 + lane_off, u);
+        st_bf16x32_(vrow + cc * 32, u);
       }
     }
   } else {
@@ -562,8 +583,8 @@ __global__ void __launch_bounds__(320, 1)
 }
 
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
-                   float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, int* status,
-                   cudaStream_t st) {
+                   float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
+                   const float* rsin, int* status, cudaStream_t st) {
   constexpr size_t smem = 6 * SLAB + 8 * HSLAB + 256 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
@@ -577,7 +598,7 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
   dim3 grid(S / 128, Hkv, max_seqs);
   attn_bwd_tc_kernel<<<grid, 320, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H, Hkv,
-                                              status);
+                                              rcos, rsin, status);
   return cudaGetLastError();
 }
 }  // namespace
@@ -588,10 +609,10 @@ bool attn_bwd_tc_supported(int S, int Dh) { return S % 128 == 0 && Dh == 128; }
 
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, int* status, cudaStream_t st) {
+                               int max_seqs, const float* rcos, const float* rsin, int* status, cudaStream_t st) {
   cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)max_seqs * S * H * 128 * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  return bwd_tc(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, status, st);
+  return bwd_tc(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, status, st);
 }
 
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,

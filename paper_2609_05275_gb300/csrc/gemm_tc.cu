@@ -67,13 +67,17 @@ constexpr int BM = 128, BK = 64;
 using namespace tc;
 
 // --------------------------------------------------------------- epilogue
+__device__ __forceinline__ void swiglu_bwd_chunk(const GemmArgs& a, int row, int j, const float (&dh)[32]);
+
 __device__ __forceinline__ void store_chunk(const GemmArgs& a, int row, int col, const float (&v)[32]) {
-  if (a.epi == EPI_STORE_F32) {
+  if (a.epi == EPI_SWIGLU_BWD) {
+    swiglu_bwd_chunk(a, row, col, v);
+  } else if (a.epi == EPI_STORE_F32) {
     float4* p = reinterpret_cast<float4*>(static_cast<float*>(a.D) + (size_t)row * a.ldd + col);
 #pragma unroll
     for (int i = 0; i < 8; ++i)
       p[i] = make_float4(a.alpha * v[4 * i], a.alpha * v[4 * i + 1], a.alpha * v[4 * i + 2], a.alpha * v[4 * i + 3]);
-  } else if (a.epi == EPI_STORE) {
+  } else if (a.epi == EPI_STORE || a.epi == EPI_ROPE) {
     uint4* p = reinterpret_cast<uint4*>(static_cast<bf16*>(a.D) + (size_t)row * a.ldd + col);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -83,35 +87,67 @@ __device__ __forceinline__ void store_chunk(const GemmArgs& a, int row, int col,
       for (int j = 0; j < 4; ++j) h[j] = __floats2bfloat162_rn(a.alpha * v[8 * i + 2 * j], a.alpha * v[8 * i + 2 * j + 1]);
       p[i] = q;
     }
-  } else {  // EPI_RESID: x[r] += alpha * acc on the kept row r (float32); save bf16
+  } else {  // EPI_RESID: x[r] += alpha * acc on the kept row r (float32); compact float32 copy
     const long long r = src_row(a.kept_idx, a.S, row);
     float4* px = reinterpret_cast<float4*>(a.x + r * a.ldx + col);
-    uint4* ps = a.save ? reinterpret_cast<uint4*>(static_cast<bf16*>(a.save) + (size_t)row * a.ld_save + col)
-                       : nullptr;
+    float4* ps = a.save ? reinterpret_cast<float4*>(static_cast<float*>(a.save) + (size_t)row * a.ld_save + col)
+                        : nullptr;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float4 o0 = px[2 * i], o1 = px[2 * i + 1];
-      o0.x += a.alpha * v[8 * i + 0];
-      o0.y += a.alpha * v[8 * i + 1];
-      o0.z += a.alpha * v[8 * i + 2];
-      o0.w += a.alpha * v[8 * i + 3];
-      o1.x += a.alpha * v[8 * i + 4];
-      o1.y += a.alpha * v[8 * i + 5];
-      o1.z += a.alpha * v[8 * i + 6];
-      o1.w += a.alpha * v[8 * i + 7];
-      px[2 * i] = o0;
-      px[2 * i + 1] = o1;
-      if (ps) {
-        uint4 q;
-        __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&q);
-        h[0] = __floats2bfloat162_rn(o0.x, o0.y);
-        h[1] = __floats2bfloat162_rn(o0.z, o0.w);
-        h[2] = __floats2bfloat162_rn(o1.x, o1.y);
-        h[3] = __floats2bfloat162_rn(o1.z, o1.w);
-        ps[i] = q;
-      }
+    for (int i = 0; i < 8; ++i) {
+      float4 o = px[i];
+      o.x += a.alpha * v[4 * i + 0];
+      o.y += a.alpha * v[4 * i + 1];
+      o.z += a.alpha * v[4 * i + 2];
+      o.w += a.alpha * v[4 * i + 3];
+      px[i] = o;
+      if (ps) ps[i] = o;
     }
   }
+}
+
+__device__ __forceinline__ float silu_mul(float g, float u) { return g / (1.0f + expf(-g)) * u; }
+
+__device__ __forceinline__ void st_bf16x32(bf16* dst, const float* v) {
+  uint4* p = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    uint4 q;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&q);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) h[j] = __floats2bfloat162_rn(v[8 * i + 2 * j], v[8 * i + 2 * j + 1]);
+    p[i] = q;
+  }
+}
+__device__ __forceinline__ void ld_bf16x32(const bf16* src, float* v) {
+  const uint4* p = reinterpret_cast<const uint4*>(src);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint4 q = p[i];
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(h[j]);
+      v[8 * i + 2 * j] = f.x;
+      v[8 * i + 2 * j + 1] = f.y;
+    }
+  }
+}
+
+// SwiGLU backward on a 32-column chunk of dh (hidden units j .. j+31).
+__device__ __forceinline__ void swiglu_bwd_chunk(const GemmArgs& a, int row, int j, const float (&dh)[32]) {
+  const bf16* gp = static_cast<const bf16*>(a.gu) + (size_t)row * 2 * a.F + j;
+  float g[32], u[32], dg[32], du[32];
+  ld_bf16x32(gp, g);
+  ld_bf16x32(gp + a.F, u);
+#pragma unroll
+  for (int e = 0; e < 32; ++e) {
+    const float sg = 1.0f / (1.0f + expf(-g[e]));
+    dg[e] = dh[e] * u[e] * sg * (1.0f + g[e] * (1.0f - sg));
+    du[e] = dh[e] * g[e] * sg;
+  }
+  bf16* dp = static_cast<bf16*>(a.D) + (size_t)row * 2 * a.F + j;
+  st_bf16x32(dp, dg);
+  st_bf16x32(dp + a.F, du);
 }
 
 // Tile order: groups of 8 N-blocks; inside a group consecutive tiles walk
@@ -216,7 +252,11 @@ __global__ void __launch_bounds__(192, 1)
             tma_load_2d(sa, &tmA, mb * BM, kb * BK, &full[stage]);
             tma_load_2d(sa + 8192, &tmA, mb * BM + 64, kb * BK, &full[stage]);
           }
-          if (!B_MN) {
+          if (!B_MN && a.epi == EPI_SWIGLU) {
+            // gate rows and up rows of the same hidden units side by side
+            tma_load_2d(sb, &tmB, kb * BK, nb * (BN / 2), &full[stage]);
+            tma_load_2d(sb + (BN / 2) * 128, &tmB, kb * BK, a.F + nb * (BN / 2), &full[stage]);
+          } else if (!B_MN) {
             tma_load_2d(sb, &tmB, kb * BK, nb * BN, &full[stage]);
           } else {
 #pragma unroll
@@ -302,11 +342,65 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int row = mb * BM + q * 32 + lane;
       const uint32_t tbase = tmem_base + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
+      if (a.epi == EPI_SWIGLU) {
+        // columns [0, BN/2) hold g, [BN/2, BN) hold u of hidden units j0 + c
+        const int j0 = nb * (BN / 2);
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        float v[32];
-        tmem_ld32(tbase + (uint32_t)c, v);
-        if (row < M && nb * BN + c < N) store_chunk(a, row, nb * BN + c, v);
+        for (int c = 0; c < BN / 2; c += 32) {
+          float g[32], u[32], hv[32];
+          tmem_ld32(tbase + (uint32_t)c, g);
+          tmem_ld32(tbase + (uint32_t)(BN / 2 + c), u);
+          if (row < M) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) hv[e] = silu_mul(g[e], u[e]);
+            bf16* gp = static_cast<bf16*>(a.D) + (size_t)row * 2 * a.F + j0 + c;
+            st_bf16x32(gp, g);
+            st_bf16x32(gp + a.F, u);
+            st_bf16x32(static_cast<bf16*>(a.h_out) + (size_t)row * a.F + j0 + c, hv);
+          }
+        }
+      } else if (a.epi == EPI_ROPE) {
+        // rotate pairs (i, i + Dh/2) of every q / k head in the tile
+        const int half = a.Dh / 2;
+        const int pos = row % a.S;
+#pragma unroll 1
+        for (int hb = 0; hb < BN; hb += a.Dh) {
+          const int col = nb * BN + hb;
+#pragma unroll 1
+          for (int c0 = 0; c0 < half; c0 += 32) {
+            float x1[32], x2[32];
+            tmem_ld32(tbase + (uint32_t)(hb + c0), x1);
+            tmem_ld32(tbase + (uint32_t)(hb + half + c0), x2);
+            if (row < M && col < N) {
+              if (col < a.rope_cols) {
+                const float4* cp = reinterpret_cast<const float4*>(a.rope_cos + (size_t)pos * half + c0);
+                const float4* sp = reinterpret_cast<const float4*>(a.rope_sin + (size_t)pos * half + c0);
+#pragma unroll
+                for (int q4 = 0; q4 < 8; ++q4) {
+                  const float4 cv = cp[q4], sv = sp[q4];
+                  const float cs[4] = {cv.x, cv.y, cv.z, cv.w}, sn[4] = {sv.x, sv.y, sv.z, sv.w};
+#pragma unroll
+                  for (int k = 0; k < 4; ++k) {
+                    const int e = 4 * q4 + k;
+                    const float p1 = x1[e], p2 = x2[e];
+                    x1[e] = p1 * cs[k] - p2 * sn[k];
+                    x2[e] = p2 * cs[k] + p1 * sn[k];
+                  }
+                }
+              }
+              bf16* dp = static_cast<bf16*>(a.D) + (size_t)row * a.ldd + col;
+              st_bf16x32(dp + c0, x1);
+              st_bf16x32(dp + half + c0, x2);
+            }
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(tbase + (uint32_t)c, v);
+          if (row < M && nb * BN + c < N) store_chunk(a, row, nb * BN + c, v);
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -366,7 +460,7 @@ cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st) {
     ok = make_map(&ta, a.A, mcap, kcap ? kcap : 64, a.lda, 64, 64);
   if (!ok) return cudaErrorInvalidValue;
   if (!a.b_mn)
-    ok = make_map(&tb, a.B, kcap ? kcap : 64, a.N, a.ldb, 64, (uint32_t)BN);
+    ok = make_map(&tb, a.B, kcap ? kcap : 64, a.N, a.ldb, 64, (uint32_t)(a.epi == EPI_SWIGLU ? BN / 2 : BN));
   else
     ok = make_map(&tb, a.B, a.N, kcap ? kcap : 64, a.ldb, 64, 64);
   if (!ok) return cudaErrorInvalidValue;

@@ -69,16 +69,16 @@ cudaError_t launch_rope_table(float* cos_t, float* sin_t, int S, int Dh, double 
 // a compact copy of the source rows.
 template <typename TS, typename T>
 cudaError_t launch_rmsnorm_fwd(const TS* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
-                               int max_rows, const T* gamma, float eps, T* copy, T* out, float* rstd,
+                               int max_rows, const T* gamma, float eps, TS* copy, T* out, float* rstd,
                                cudaStream_t st);
 
 // RMSNorm backward + residual: for compact row m with source row r,
 //   dx[r] += rstd (dyn*g - xn * mean(dyn*g*xn)),  xn = xs[m] * rstd[m]
-// on the float32 residual gradient dx, then, if next != null,
+// on the float32 residual gradient dx (dyn is float32), then, if next != null,
 // next[m] = scale * dx[r] (compact, for the next branch).  Partial gain
 // gradients go to part[blockIdx][d] (nblocks blocks, a launch constant).
 template <typename T>
-cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, float* dx,
+cudaError_t launch_rmsnorm_bwd(const float* dyn, const float* xs, const float* rstd, const T* gamma, float* dx,
                                const int* kept_idx, const int* cnt, int S, int d, int max_rows, float scale,
                                T* next, float* part, int nblocks, cudaStream_t st);
 int rmsnorm_bwd_blocks(int max_rows);
@@ -126,16 +126,26 @@ cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, flo
 // tcgen05 flash attention backward (head size 128, S % 128 == 0); zeroes
 // dq_acc and accumulates dQ (unscaled) into it.
 bool attn_bwd_tc_supported(int S, int Dh);
+// dK leaves with the inverse RoPE applied (rcos = null: no rotation).
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, int* status, cudaStream_t st);
-cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const int* cnt, int S,
-                             int max_rows, cudaStream_t st);
+                               int max_seqs, const float* rcos, const float* rsin, int* status, cudaStream_t st);
+// dqkv[:, q heads] = inverse-RoPE(dq_acc / sqrt(Dh)) as bf16 (rcos = null: no rotation)
+cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const float* rcos,
+                             const float* rsin, const int* cnt, int S, int max_rows, cudaStream_t st);
 
 // ------------------------------------------------------------------------
 // GEMM: D(m,n) = alpha * sum_k A(m,k) B(n,k) with a fused epilogue.
 // ------------------------------------------------------------------------
-enum EpiMode { EPI_STORE = 0, EPI_STORE_F32 = 1, EPI_RESID = 2 };
+// EPI_STORE       D = alpha*acc (bf16)        EPI_STORE_F32  D = alpha*acc (float)
+// EPI_RESID       x[kept row] += alpha*acc (float32 residual), save = new x (bf16)
+// EPI_ROPE        D = rope(acc) on the first rope_cols columns (q and k heads of
+//                 the QKV projection, position = row % S), plain store after
+// EPI_SWIGLU      B is read as matching halves of the gate and up rows; writes
+//                 g, u to D (row stride 2F, columns j and F+j) and
+//                 h = silu(g) u to h_out (row stride F)
+// EPI_SWIGLU_BWD  acc = dh; with g, u from `gu` writes dg, du to D (stride 2F)
+enum EpiMode { EPI_STORE = 0, EPI_STORE_F32 = 1, EPI_RESID = 2, EPI_ROPE = 3, EPI_SWIGLU = 4, EPI_SWIGLU_BWD = 5 };
 
 struct GemmArgs {
   // problem size; a non-null *_cnt makes the extent device-side: (*cnt) * mul
@@ -158,13 +168,21 @@ struct GemmArgs {
   int ldd;
   float alpha;
   // EPI_RESID: x[r] = x[r] + alpha*acc for r = src_row(kept_idx, S, m) on the
-  // float32 residual stream x; save[m] = new x[r] in the operand type
+  // float32 residual stream x; save[m] = new x[r] (float32, compact)
   float* x;
   int ldx;
   const int* kept_idx;
   int S;
   void* save;
   int ld_save;
+  // EPI_ROPE
+  const float* rope_cos;
+  const float* rope_sin;
+  int Dh, rope_cols;
+  // EPI_SWIGLU / EPI_SWIGLU_BWD
+  const void* gu;
+  void* h_out;
+  int F;
   int* status;
 };
 

@@ -69,7 +69,7 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const TS* __restrict__
                                                           const int* __restrict__ kept_idx,
                                                           const int* __restrict__ cnt, int S, int d,
                                                           const T* __restrict__ gamma, float eps,
-                                                          T* __restrict__ copy, T* __restrict__ out,
+                                                          TS* __restrict__ copy, T* __restrict__ out,
                                                           float* __restrict__ rstd) {
   const long long M = (long long)(*cnt) * S;
   const int lane = threadIdx.x & 31;
@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const TS* __restrict__
 
 template <typename TS, typename T>
 cudaError_t launch_rmsnorm_fwd(const TS* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
-                               int max_rows, const T* gamma, float eps, T* copy, T* out, float* rstd,
+                               int max_rows, const T* gamma, float eps, TS* copy, T* out, float* rstd,
                                cudaStream_t st) {
   const int grid = grid_for(max_rows, 8, device_sm_count() * 16);
   rmsnorm_fwd_kernel<TS, T><<<grid, 256, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy, out, rstd);
@@ -110,7 +110,7 @@ cudaError_t launch_rmsnorm_fwd(const TS* src, int gather, const int* kept_idx, c
 
 // ---------------------------------------------------------------- RMSNorm bwd
 template <typename T>
-__global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const T* __restrict__ dyn, const T* __restrict__ xs,
+__global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const float* __restrict__ dyn, const float* __restrict__ xs,
                                                           const float* __restrict__ rstd,
                                                           const T* __restrict__ gamma, float* __restrict__ dx,
                                                           const int* __restrict__ kept_idx,
@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const T* __restrict__ 
 int rmsnorm_bwd_blocks(int max_rows) { return grid_for(max_rows, 8, device_sm_count() * 2); }
 
 template <typename T>
-cudaError_t launch_rmsnorm_bwd(const T* dyn, const T* xs, const float* rstd, const T* gamma, float* dx,
+cudaError_t launch_rmsnorm_bwd(const float* dyn, const float* xs, const float* rstd, const T* gamma, float* dx,
                                const int* kept_idx, const int* cnt, int S, int d, int max_rows, float scale,
                                T* next, float* part, int nblocks, cudaStream_t st) {
   const size_t smem = (size_t)d * sizeof(float);
@@ -394,10 +394,9 @@ cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, c
 
 #define LD_INST(T)                                                                                              \
   template cudaError_t launch_rmsnorm_fwd<float, T>(const float*, int, const int*, const int*, int, int, int,   \
-                                                    const T*, float, T*, T*, float*, cudaStream_t);             \
-  template cudaError_t launch_rmsnorm_fwd<T, T>(const T*, int, const int*, const int*, int, int, int, const T*, \
-                                                float, T*, T*, float*, cudaStream_t);                           \
-  template cudaError_t launch_rmsnorm_bwd<T>(const T*, const T*, const float*, const T*, float*, const int*,    \
+                                                    const T*, float, float*, T*, float*, cudaStream_t);         \
+  template cudaError_t launch_rmsnorm_bwd<T>(const float*, const float*, const float*, const T*, float*,         \
+                                             const int*,                                                         \
                                              const int*, int, int, int, float, T*, float*, int, cudaStream_t);  \
   template cudaError_t launch_gather_scale<T>(const float*, const int*, const int*, int, int, int, float, T*,    \
                                               cudaStream_t);                                                    \
