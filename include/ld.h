@@ -235,6 +235,25 @@ ld_status ld_rmsnorm_backward(int B, int S, int d, const float* dyn, const void*
                               const void* gamma, const int* kept_idx, const int* kept_cnt, float* dx, void* next,
                               float scale, float* dgamma, float* scratch, size_t scratch_bytes, void* stream);
 
+/* The same step as ld_rmsnorm_backward for callers that cannot allocate
+ * device memory where they need it (a CUDA graph captured in global mode,
+ * where allocation calls are refused during capture; a runtime whose device
+ * memory is owned by an allocator this library cannot reach; a path that must
+ * not enter an allocator).  The paper has no counterpart: this is a property
+ * of the library, not of the method.  Arguments are those of
+ * ld_rmsnorm_backward without the scratch buffer: the partial sums of dgamma
+ * live in a fixed 10 MiB device array inside the library, which every GPU that
+ * loads the library holds until the process exits.  Limit:
+ * min(ceil(B*S / 8), 320) * d <= 2,621,440 (e.g. d <= 8192 once B*S >= 2560);
+ * larger sizes return LD_ERR_SHAPE.  The first call on each device looks up
+ * the array's address with that device current, so make it before any stream
+ * capture.  All calls share the array: nothing in it needs clearing (each
+ * call overwrites every partial sum it reads), but calls that overlap on the
+ * GPU race on it and must be serialised by the caller.  Allocates nothing. */
+ld_status ld_rmsnorm_backward_noalloc(int B, int S, int d, const float* dyn, const void* xs, const float* rstd,
+                                      const void* gamma, const int* kept_idx, const int* kept_cnt, float* dx,
+                                      void* next, float scale, float* dgamma, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -87,6 +87,9 @@ def lib():
             "ld_rmsnorm_backward": (c_int, [c_int, c_int, c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                             c_void_p, c_void_p, c_void_p, c_float, c_void_p, c_void_p, c_size_t,
                                             c_void_p]),
+            "ld_rmsnorm_backward_noalloc": (c_int, [c_int, c_int, c_int, c_void_p, c_void_p, c_void_p, c_void_p,
+                                                    c_void_p, c_void_p, c_void_p, c_void_p, c_float, c_void_p,
+                                                    c_void_p]),
             "ld_gemm_bf16": (c_int, [c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_int, c_void_p,
                                      c_int, c_int, c_float, c_void_p, c_void_p]),
         }
@@ -242,6 +245,14 @@ def ld_rmsnorm_backward(B, S, d, dyn, xs, rstd, gamma, kept_idx, kept_cnt, dx, n
                                      _ptr(kept_cnt), _ptr(dx), _ptr(nxt), float(scale), _ptr(dgamma), _ptr(scratch),
                                      scratch.numel() * scratch.element_size(), _stream(stream)),
            "ld_rmsnorm_backward")
+
+
+def ld_rmsnorm_backward_noalloc(B, S, d, dyn, xs, rstd, gamma, kept_idx, kept_cnt, dx, nxt, scale, dgamma,
+                                stream=None):
+    _check(lib().ld_rmsnorm_backward_noalloc(B, S, d, _ptr(dyn), _ptr(xs), _ptr(rstd), _ptr(gamma), _ptr(kept_idx),
+                                             _ptr(kept_cnt), _ptr(dx), _ptr(nxt), float(scale), _ptr(dgamma),
+                                             _stream(stream)),
+           "ld_rmsnorm_backward_noalloc")
 
 
 def weight_table(layers):
