@@ -576,9 +576,11 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   h->esz = c.fp32_debug ? 4 : 2;
   h->max_rows = c.B * c.S;
   h->nqkv = (c.H + 2 * c.Hkv) * c.Dh;
-  // number of partial-sum blocks of the gain gradient (a launch constant)
+  // number of blocks (and partial-sum rows of the gain gradient) of the
+  // RMSNorm backward inside ld_backward: enough to keep ~8 blocks per SM of
+  // a 152-SM GPU streaming (a launch constant; no CUDA call here)
   h->part_blocks = (h->max_rows + 7) / 8;
-  if (h->part_blocks > 2 * 160) h->part_blocks = 2 * 160;
+  if (h->part_blocks > 8 * 152) h->part_blocks = 8 * 152;
   make_layout(h);
   *handle = h;
   return LD_OK;

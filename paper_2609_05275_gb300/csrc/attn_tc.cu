@@ -183,36 +183,36 @@ __global__ void __launch_bounds__(192, 1)
     for (int j = 0; j < nkt; ++j) {
       if (!warp_wait(&s_full[j & 1], (j >> 1) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      float sv[128];
+      uint32_t sr[4][32];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        float t[32];
-        tmem_ld32(tmem + (j & 1) * 128 + c * 32 + lane_off, t);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) sv[c * 32 + e] = t[e];
-      }
+      for (int c = 0; c < 4; ++c) tmem_ld32_nw(tmem + (j & 1) * 128 + c * 32 + lane_off, sr[c]);
+      tmem_wait_ld();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_free[j & 1]);
-      float mt = -INFINITY;
-      const bool diag = (j == qt);
+      // running max on the raw scores (the scale is positive); keys after
+      // the query (diagonal tile only) are left out
+      const int lim = (j == qt) ? r : 127;
+      float mraw = -INFINITY;
 #pragma unroll
       for (int e = 0; e < 128; ++e) {
-        float v = sv[e] * sl2;
-        if (diag && e > r) v = -INFINITY;
-        sv[e] = v;
-        mt = fmaxf(mt, v);
+        const float v = __uint_as_float(sr[e >> 5][e & 31]);
+        mraw = fmaxf(mraw, e <= lim ? v : -INFINITY);
       }
+      const float mt = mraw * sl2;
       bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
       float ls = 0.f;
       uint32_t pk[64];
 #pragma unroll
       for (int e = 0; e < 64; ++e) {
-        const float p0 = exp2f(sv[2 * e] - m_new), p1 = exp2f(sv[2 * e + 1] - m_new);
+        float p0 = ex2(fmaf(__uint_as_float(sr[(2 * e) >> 5][(2 * e) & 31]), sl2, -m_new));
+        float p1 = ex2(fmaf(__uint_as_float(sr[(2 * e + 1) >> 5][(2 * e + 1) & 31]), sl2, -m_new));
+        p0 = (2 * e <= lim) ? p0 : 0.f;
+        p1 = (2 * e + 1 <= lim) ? p1 : 0.f;
         ls += p0 + p1;
-        __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
-        pk[e] = *reinterpret_cast<uint32_t*>(&b);
+        __nv_bfloat162 bq = __floats2bfloat162_rn(p0, p1);
+        pk[e] = *reinterpret_cast<uint32_t*>(&bq);
       }
       // P_{j-1} V_{j-1} must be done before P and O are touched
       if (j >= 1 && !warp_wait(pv_done, (j - 1) & 1, abort_flag, status)) { ok = false; break; }
@@ -313,7 +313,7 @@ constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
 __global__ void __launch_bounds__(320, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
-                       const __grid_constant__ CUtensorMap tmo,
+                       const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
@@ -329,7 +329,8 @@ __global__ void __launch_bounds__(320, 1)
   uint8_t* dOs = Qs + 2 * QT;    // [2][QT]
   uint8_t* PTs = dOs + 2 * QT;   // 128 keys x 64 queries, one slab of 128-byte rows
   uint8_t* DSs = PTs + SLAB;
-  float* vecs = reinterpret_cast<float*>(DSs + SLAB);  // [2][lse 64 | D 64]
+  float* dqs = reinterpret_cast<float*>(DSs + SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
+  float* vecs = dqs + 64 * DH;                         // [2][lse 64 | D 64]
   uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + 256);
   uint64_t* kv_full = bars;
   uint64_t* ld_full = bars + 1;  // [2]
@@ -470,26 +471,17 @@ __global__ void __launch_bounds__(320, 1)
       if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
       if (!warp_wait(&ld_full[b], (i >> 1) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      float sv[64], dp[64];
-      {
-        float t[32];
-        tmem_ld32(t_s + lane_off, t);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) sv[e] = t[e];
-        tmem_ld32(t_s + 32 + lane_off, t);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) sv[32 + e] = t[e];
-        tmem_ld32(t_dp + lane_off, t);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) dp[e] = t[e];
-        tmem_ld32(t_dp + 32 + lane_off, t);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) dp[32 + e] = t[e];
-      }
+      uint32_t sr[2][32], dr[2][32];
+      tmem_ld32_nw(t_s + lane_off, sr[0]);
+      tmem_ld32_nw(t_s + 32 + lane_off, sr[1]);
+      tmem_ld32_nw(t_dp + lane_off, dr[0]);
+      tmem_ld32_nw(t_dp + 32 + lane_off, dr[1]);
+      tmem_wait_ld();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
       const float* lv = vecs + b * 128;
+      const int qbase = qt * 64 - key;  // query c is visible iff qbase + c >= 0
       uint32_t pk[32], dk[32];
 #pragma unroll
       for (int e = 0; e < 32; ++e) {
@@ -497,10 +489,12 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
           const int c = 2 * e + u;
-          const bool vis = qt * 64 + c >= key;
-          const float pv = vis ? exp2f(sv[c] * sl2 - lv[c] * kLog2e) : 0.f;
+          const float s_ = __uint_as_float(sr[c >> 5][c & 31]);
+          const float dpv = __uint_as_float(dr[c >> 5][c & 31]);
+          float pv = ex2(fmaf(s_, sl2, -lv[c] * kLog2e));
+          pv = (qbase + c >= 0) ? pv : 0.f;
           p[u] = pv;
-          d[u] = pv * (dp[c] - lv[64 + c]);
+          d[u] = pv * (dpv - lv[64 + c]);
         }
         __nv_bfloat162 bp = __floats2bfloat162_rn(p[0], p[1]), bd = __floats2bfloat162_rn(d[0], d[1]);
         pk[e] = *reinterpret_cast<uint32_t*>(&bp);
@@ -553,9 +547,12 @@ __global__ void __launch_bounds__(320, 1)
     }
   } else {
     // ------------------------------------------------ dQ (warps 6..9)
+    // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
+    // into dq_acc by one bulk tensor reduce per step.
     const int quad = warp & 3;
     const int dd = quad * 32 + lane;  // head dimension of this thread
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const bool leader = (warp == 6 && lane == 0);
     for (int i = 0; i < n_it; ++i) {
       const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
       if (!warp_wait(mm_done, i & 1, abort_flag, status)) break;
@@ -566,12 +563,20 @@ __global__ void __launch_bounds__(320, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(dq_free);
-      float* dst = dq_acc + (size_t)(row0 + qt * 64) * HD + (size_t)h * DH + dd;
+      if (leader && i > 0) bulk_wait_read();  // the previous reduce has read the tile
+      named_barrier(1, 128);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)e * HD, t0[e]);
+      for (int e = 0; e < 32; ++e) dqs[e * DH + dd] = t0[e];
 #pragma unroll
-      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(32 + e) * HD, t1[e]);
+      for (int e = 0; e < 32; ++e) dqs[(32 + e) * DH + dd] = t1[e];
+      fence_proxy_async();
+      named_barrier(1, 128);
+      if (leader) {
+        tma_reduce_add_2d(&tmdq, h * DH, row0 + qt * 64, dqs);
+        bulk_commit();
+      }
     }
+    if (leader) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -585,19 +590,21 @@ __global__ void __launch_bounds__(320, 1)
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, int* status, cudaStream_t st) {
-  constexpr size_t smem = 6 * SLAB + 8 * HSLAB + 256 * 4 + 1024 + 256;
+  constexpr size_t smem = 6 * SLAB + 8 * HSLAB + 256 * 4 + 64 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(attn_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  CUtensorMap tkv, tq, to;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows
+  CUtensorMap tkv, tq, to, tdq;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows; dQ reduce boxes
+  if (!make_map_f32(&tdq, dq_acc, (uint64_t)H * 128, (uint64_t)max_seqs * S, (uint64_t)H * 128, 128, 64))
+    return cudaErrorInvalidValue;
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
   dim3 grid(S / 128, Hkv, max_seqs);
-  attn_bwd_tc_kernel<<<grid, 320, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H, Hkv,
+  attn_bwd_tc_kernel<<<grid, 320, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H, Hkv,
                                               rcos, rsin, status);
   return cudaGetLastError();
 }

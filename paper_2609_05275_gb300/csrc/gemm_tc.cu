@@ -59,6 +59,19 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, 
   return r == CUDA_SUCCESS;
 }
 
+bool make_map_f32(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld, uint32_t box_inner,
+                  uint32_t box_outer) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * 4};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
 }  // namespace tc
 
 namespace {
@@ -391,6 +404,45 @@ __global__ void __launch_bounds__(192, 1)
               bf16* dp = static_cast<bf16*>(a.D) + (size_t)row * a.ldd + col;
               st_bf16x32(dp + c0, x1);
               st_bf16x32(dp + half + c0, x2);
+            }
+          }
+        }
+      } else if (a.epi == EPI_RESID) {
+        // residual rows are read ahead (the next chunk while this one is
+        // finished) so their latency overlaps the TMEM loads and the adds
+        const bool rok = row < M;
+        const long long r = rok ? src_row(a.kept_idx, a.S, row) : 0;
+        float* xrow = a.x + r * a.ldx + (size_t)nb * BN;
+        float* srow = a.save ? static_cast<float*>(a.save) + (size_t)row * a.ld_save + (size_t)nb * BN : nullptr;
+        float4 xv[8];
+        if (rok && nb * BN < N) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) xv[i] = reinterpret_cast<const float4*>(xrow)[i];
+        }
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(tbase + (uint32_t)c, v);
+          const bool ok = rok && nb * BN + c < N;
+          float4 o[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            o[i] = xv[i];
+            o[i].x += a.alpha * v[4 * i + 0];
+            o[i].y += a.alpha * v[4 * i + 1];
+            o[i].z += a.alpha * v[4 * i + 2];
+            o[i].w += a.alpha * v[4 * i + 3];
+          }
+          if (rok && c + 32 < BN && nb * BN + c + 32 < N) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) xv[i] = reinterpret_cast<const float4*>(xrow + c + 32)[i];
+          }
+          if (ok) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(xrow + c)[i] = o[i];
+            if (srow) {
+#pragma unroll
+              for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(srow + c)[i] = o[i];
             }
           }
         }

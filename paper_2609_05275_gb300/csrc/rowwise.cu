@@ -161,18 +161,120 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const float* __restric
 
 int rmsnorm_bwd_blocks(int max_rows) { return grid_for(max_rows, 8, device_sm_count() * 2); }
 
+// Same operation with the block spread over the columns: thread t owns the
+// 8-column chunks t, t + 256, ... (MAXJ of them), keeps its share of gamma and
+// of the gain gradient in registers, and the block reduces the dot products of
+// RPB rows at once (their loads are all in flight together).  No
+// shared-memory atomics; all global accesses coalesced.
+template <typename T, int MAXJ, int RPB>
+__global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __restrict__ dyn,
+                                                               const float* __restrict__ xs,
+                                                               const float* __restrict__ rstd,
+                                                               const T* __restrict__ gamma, float* __restrict__ dx,
+                                                               const int* __restrict__ kept_idx,
+                                                               const int* __restrict__ cnt, int S, int d, float scale,
+                                                               T* __restrict__ next, float* __restrict__ part) {
+  __shared__ float red[RPB][8];
+  __shared__ float tot[RPB];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  const int d8 = d / 8;
+  float g[MAXJ][8], gacc[MAXJ][8];
+#pragma unroll
+  for (int j = 0; j < MAXJ; ++j) {
+    const int c8 = tid + 256 * j;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      g[j][e] = 0.f;
+      gacc[j][e] = 0.f;
+    }
+    if (c8 < d8) ld8(gamma + c8 * 8, g[j]);
+  }
+  const long long M = (long long)(*cnt) * S;
+  for (long long m0 = (long long)blockIdx.x * RPB; m0 < M; m0 += (long long)gridDim.x * RPB) {
+    float dy[RPB][MAXJ][8], xv[RPB][MAXJ][8];
+    float pd[RPB];
+#pragma unroll
+    for (int q = 0; q < RPB; ++q) {
+      const long long m = m0 + q;
+      pd[q] = 0.f;
+#pragma unroll
+      for (int j = 0; j < MAXJ; ++j) {
+        const int c8 = tid + 256 * j;
+        if (m < M && c8 < d8) {
+          ld8(dyn + m * d + c8 * 8, dy[q][j]);
+          ld8(xs + m * d + c8 * 8, xv[q][j]);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) pd[q] += dy[q][j][e] * g[j][e] * xv[q][j][e];
+        }
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < RPB; ++q) {
+      const float v = warp_sum(pd[q]);
+      if (lane == 0) red[q][w] = v;
+    }
+    __syncthreads();
+    if (w < RPB) {
+      float v = lane < 8 ? red[w][lane] : 0.f;
+      v = warp_sum(v);
+      if (lane == 0) tot[w] = v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < RPB; ++q) {
+      const long long m = m0 + q;
+      if (m >= M) break;
+      const long long r = src_row(kept_idx, S, m);
+      const float rs = rstd[m];
+      const float dot = tot[q] * rs / (float)d;  // mean(dyn * gamma * xn)
+#pragma unroll
+      for (int j = 0; j < MAXJ; ++j) {
+        const int c8 = tid + 256 * j;
+        if (c8 < d8) {
+          float cur[8], nx[8];
+          ld8(dx + r * d + c8 * 8, cur);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float xn = xv[q][j][e] * rs;
+            cur[e] = cur[e] + rs * (dy[q][j][e] * g[j][e] - xn * dot);
+            nx[e] = scale * cur[e];
+            gacc[j][e] += dy[q][j][e] * xn;
+          }
+          st8(dx + r * d + c8 * 8, cur);
+          if (next) st8(next + m * d + c8 * 8, nx);
+        }
+      }
+    }
+    __syncthreads();  // red / tot are rewritten by the next group
+  }
+#pragma unroll
+  for (int j = 0; j < MAXJ; ++j) {
+    const int c8 = tid + 256 * j;
+    if (c8 < d8) st8(part + (size_t)blockIdx.x * d + c8 * 8, gacc[j]);
+  }
+}
+
 template <typename T>
 cudaError_t launch_rmsnorm_bwd(const float* dyn, const float* xs, const float* rstd, const T* gamma, float* dx,
                                const int* kept_idx, const int* cnt, int S, int d, int max_rows, float scale,
                                T* next, float* part, int nblocks, cudaStream_t st) {
-  const size_t smem = (size_t)d * sizeof(float);
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(rmsnorm_bwd_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
+  (void)max_rows;
+  if (d <= 2048) {
+    rmsnorm_bwd_cols_kernel<T, 1, 4><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
+  } else if (d <= 4096) {
+    rmsnorm_bwd_cols_kernel<T, 2, 2><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
+  } else if (d <= 8192) {
+    rmsnorm_bwd_cols_kernel<T, 4, 1><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
+  } else {
+    const size_t smem = (size_t)d * sizeof(float);
+    if (smem > 48 * 1024) {
+      cudaError_t e = cudaFuncSetAttribute(rmsnorm_bwd_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem);
+      if (e != cudaSuccess) return e;
+    }
+    rmsnorm_bwd_kernel<T><<<nblocks, 256, smem, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next,
+                                                     part);
   }
-  rmsnorm_bwd_kernel<T><<<nblocks, 256, smem, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next,
-                                                   part);
   return cudaGetLastError();
 }
 
