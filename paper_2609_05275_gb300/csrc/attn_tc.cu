@@ -7,14 +7,16 @@
 //   o_i = sum_{j<=i} softmax_j(c q_i . k_j) v_j,  c = 1/sqrt(Dh);
 // lse_i = log sum_j exp(c q_i . k_j) is kept for the backward.
 //
-// One CTA per (128-query tile, head, kept sequence); 192 threads:
-//   warp 0      TMA: the Q tile once, then K_j / V_j tiles (128 keys) into a
-//               two-stage ring (128-byte swizzled, 64-column slabs);
+// One CTA per (128-query tile, head, kept sequence); 320 threads:
+//   warp 0      TMA: the Q tile once, then K_j and V_j tiles (128 keys) into
+//               two two-stage rings (128-byte swizzled, 64-column slabs), K
+//               one tile ahead of V;
 //   warp 1      TMEM allocation and the MMAs: S_j = Q K_j^T into one of two
 //               TMEM score buffers, then O += P_{j-1} V_{j-1} (O in TMEM);
-//   warps 2..5  softmax, one query row per thread: S_j from TMEM, running
-//               max in base 2, P = exp2(S c log2e - m) written as bf16 into a
-//               swizzled shared-memory tile (the A operand of the PV MMA).
+//   warps 2..9  softmax, one query row and 64 keys per thread (two warps
+//               per row): S_j from TMEM, running max in base 2,
+//               P = exp2(S c log2e - m) written as bf16 into a swizzled
+//               shared-memory tile (the A operand of the PV MMA).
 // The running max is only moved (and O rescaled in TMEM) when it grows by
 // more than 2^8, so most tiles need no O round trip; P <= 2^8 stays well
 // inside bf16/fp32 range.  All waits are bounded (status word on expiry).
@@ -48,7 +50,7 @@ __device__ __forceinline__ uint32_t swz(int r, int i) {
 }
 
 template <int DH>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
                        int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv, int* status) {
   constexpr int NSLAB = DH / 64;
@@ -60,24 +62,29 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* Ks = Qs + TILE;
   uint8_t* Vs = Ks + NS * TILE;
   uint8_t* Ps = Vs + NS * TILE;  // 128 x 128 bf16, two slabs
-  uint64_t* bars = reinterpret_cast<uint64_t*>(Ps + 2 * SLAB);
+  float(*xmax)[2][128] = reinterpret_cast<float(*)[2][128]>(Ps + 2 * SLAB);  // [tile parity][half][row]
+  float(*xsum)[128] = reinterpret_cast<float(*)[128]>(Ps + 2 * SLAB + 2 * 2 * 128 * 4);  // [half][row]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Ps + 2 * SLAB + 6 * 128 * 4);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;
-  uint64_t* kv_empty = kv_full + NS;
-  uint64_t* s_full = kv_empty + NS;
+  uint64_t* k_full = bars + 1;        // [NS] K ring: a stage frees once S_j has read it
+  uint64_t* k_empty = k_full + NS;
+  uint64_t* v_full = k_empty + NS;    // [NS] V ring: a stage frees once P_j V_j has read it
+  uint64_t* v_empty = v_full + NS;
+  uint64_t* s_full = v_empty + NS;
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
   uint64_t* pv_done = p_full + 1;
   uint64_t* o_full = pv_done + 1;
   uint64_t* drain = o_full + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* xbar = drain + 1;  // [4]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 4);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  const int seq = blockIdx.z;
+  const int seq = blockIdx.y;
   if (seq >= *cnt) return;
   const int nqt = S / 128;
-  const int qt = nqt - 1 - blockIdx.x;  // heaviest tiles first
-  const int h = blockIdx.y, g = (h * Hkv) / H;
+  const int qt = nqt - 1 - blockIdx.z;  // slowest grid dimension: heaviest tiles are dispatched first
+  const int h = blockIdx.x, g = (h * Hkv) / H;
   const int row0 = seq * S;
   const int nkt = qt + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -85,17 +92,20 @@ __global__ void __launch_bounds__(192, 1)
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < NS; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&s_full[b], 1);
-      mbar_init(&s_free[b], 4);
+      mbar_init(&s_free[b], 8);
     }
-    mbar_init(p_full, 4);
+    mbar_init(p_full, 8);
     mbar_init(pv_done, 1);
     mbar_init(o_full, 1);
     mbar_init(drain, 1);
+    for (int q = 0; q < 4; ++q) mbar_init(&xbar[q], 2);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -112,20 +122,30 @@ __global__ void __launch_bounds__(192, 1)
       const int qcol = h * DH, kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
       mbar_arrive_expect_tx(q_full, TILE);
       for (int c = 0; c < NSLAB; ++c) tma_load_2d(Qs + c * SLAB, &tm, qcol + 64 * c, row0 + qt * 128, q_full);
-      int issued = 0;
-      for (int j = 0; j < nkt; ++j) {
-        const int s = j % NS;
-        if (!mbar_wait(&kv_empty[s], ((j / NS) & 1) ^ 1u, abort_flag, status)) break;
-        mbar_arrive_expect_tx(&kv_full[s], 2 * TILE);
-        for (int c = 0; c < NSLAB; ++c) {
-          tma_load_2d(Ks + s * TILE + c * SLAB, &tm, kcol + 64 * c, row0 + j * 128, &kv_full[s]);
-          tma_load_2d(Vs + s * TILE + c * SLAB, &tm, vcol + 64 * c, row0 + j * 128, &kv_full[s]);
+      // K runs one tile ahead of V: S_{j+1} is issued before P_j V_j
+      int nk = 0, nv = 0;
+      for (int j = 0; j <= nkt; ++j) {
+        if (j < nkt) {
+          const int s = j % NS;
+          if (!mbar_wait(&k_empty[s], ((j / NS) & 1) ^ 1u, abort_flag, status)) break;
+          mbar_arrive_expect_tx(&k_full[s], TILE);
+          for (int c = 0; c < NSLAB; ++c)
+            tma_load_2d(Ks + s * TILE + c * SLAB, &tm, kcol + 64 * c, row0 + j * 128, &k_full[s]);
+          ++nk;
         }
-        ++issued;
+        if (j >= 1) {
+          const int jv = j - 1, s = jv % NS;
+          if (!mbar_wait(&v_empty[s], ((jv / NS) & 1) ^ 1u, abort_flag, status)) break;
+          mbar_arrive_expect_tx(&v_full[s], TILE);
+          for (int c = 0; c < NSLAB; ++c)
+            tma_load_2d(Vs + s * TILE + c * SLAB, &tm, vcol + 64 * c, row0 + jv * 128, &v_full[s]);
+          ++nv;
+        }
       }
       if (*abort_flag) {
         mbar_drain(q_full, 0);
-        for (int j = issued > NS ? issued - NS : 0; j < issued; ++j) mbar_drain(&kv_full[j % NS], (j / NS) & 1);
+        for (int j = nk > NS ? nk - NS : 0; j < nk; ++j) mbar_drain(&k_full[j % NS], (j / NS) & 1);
+        for (int j = nv > NS ? nv - NS : 0; j < nv; ++j) mbar_drain(&v_full[j % NS], (j / NS) & 1);
       }
     }
   } else if (warp == 1) {
@@ -138,7 +158,7 @@ __global__ void __launch_bounds__(192, 1)
       for (int j = 0; ok && j <= nkt; ++j) {
         if (j < nkt) {
           const int s = j % NS;
-          if (!mbar_wait(&kv_full[s], (j / NS) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(&k_full[s], (j / NS) & 1, abort_flag, status)) { ok = false; break; }
           if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t kb = ka + s * TILE;
@@ -148,10 +168,12 @@ __global__ void __launch_bounds__(192, 1)
             mma_bf16(tmem + (j & 1) * 128, sdesc(qa + off, 16, 1024), sdesc(kb + off, 16, 1024), ID_S, kk > 0);
           }
           mma_commit(&s_full[j & 1]);
+          mma_commit(&k_empty[s]);
         }
         if (j >= 1) {
           const int jp = j - 1, s = jp % NS;
           if (!mbar_wait(p_full, jp & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(&v_full[s], (jp / NS) & 1, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t vb = va + s * TILE;
 #pragma unroll
@@ -162,7 +184,7 @@ __global__ void __launch_bounds__(192, 1)
                      sdesc(vb + kk * 2048, SLAB, 1024), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
           }
           mma_commit(pv_done);
-          mma_commit(&kv_empty[s]);
+          mma_commit(&v_empty[s]);
         }
       }
       if (ok) {
@@ -173,39 +195,48 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else {
-    // ------------------------------------------------ softmax (warps 2..5)
+    // ------------------------------------------------ softmax (warps 2..9)
+    // two warps per TMEM lane quadrant, one query row per thread: warps 2..5
+    // take keys 0..63 of the tile (and O columns 0..DH/2), warps 6..9 keys
+    // 64..127 (and the rest of O); the pair exchanges row maxima and sums
+    // through shared memory
     const int quad = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int r = quad * 32 + lane;  // query row of this thread within the tile
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    uint64_t* xb = &xbar[quad];      // exchange barrier of the two warps of this quadrant (2 arrivals a phase)
     const float sl2 = kLog2e * rsqrtf((float)DH);
+    constexpr int OC = DH / 64;      // 32-column chunks of O per half
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nkt; ++j) {
       if (!warp_wait(&s_full[j & 1], (j >> 1) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t sr[4][32];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32_nw(tmem + (j & 1) * 128 + c * 32 + lane_off, sr[c]);
+      uint32_t sr[2][32];
+      tmem_ld32_nw(tmem + (j & 1) * 128 + half * 64 + lane_off, sr[0]);
+      tmem_ld32_nw(tmem + (j & 1) * 128 + half * 64 + 32 + lane_off, sr[1]);
       tmem_wait_ld();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_free[j & 1]);
       // running max on the raw scores (the scale is positive); keys after
       // the query (diagonal tile only) are left out
-      const int lim = (j == qt) ? r : 127;
+      const int lim = ((j == qt) ? r : 127) - half * 64;  // last visible local column
       float mraw = -INFINITY;
 #pragma unroll
-      for (int e = 0; e < 128; ++e) {
-        const float v = __uint_as_float(sr[e >> 5][e & 31]);
-        mraw = fmaxf(mraw, e <= lim ? v : -INFINITY);
-      }
+      for (int e = 0; e < 64; ++e) mraw = fmaxf(mraw, e <= lim ? __uint_as_float(sr[e >> 5][e & 31]) : -INFINITY);
+      xmax[j & 1][half][r] = mraw;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(xb);
+      if (!warp_wait(xb, j & 1, abort_flag, status)) { ok = false; break; }
+      mraw = fmaxf(mraw, xmax[j & 1][half ^ 1][r]);
       const float mt = mraw * sl2;
-      bool rescale = mt > m_used + kRescale;
+      const bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
       float ls = 0.f;
-      uint32_t pk[64];
+      uint32_t pk[32];
 #pragma unroll
-      for (int e = 0; e < 64; ++e) {
+      for (int e = 0; e < 32; ++e) {
         float p0 = ex2(fmaf(__uint_as_float(sr[(2 * e) >> 5][(2 * e) & 31]), sl2, -m_new));
         float p1 = ex2(fmaf(__uint_as_float(sr[(2 * e + 1) >> 5][(2 * e + 1) & 31]), sl2, -m_new));
         p0 = (2 * e <= lim) ? p0 : 0.f;
@@ -217,17 +248,17 @@ __global__ void __launch_bounds__(192, 1)
       // P_{j-1} V_{j-1} must be done before P and O are touched
       if (j >= 1 && !warp_wait(pv_done, (j - 1) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      // tcgen05.ld/st are warp-wide: the warp rescales O together when any
-      // lane moved its max; lanes that did not multiply by 1
+      // tcgen05.ld/st are warp-wide: the warp rescales its half of O together
+      // when any lane moved its max; lanes that did not multiply by 1
       if (j >= 1 && __any_sync(0xffffffffu, rescale)) {
         const float corr = rescale ? exp2f(m_used - m_new) : 1.f;
 #pragma unroll 1
-        for (int c = 0; c < DH / 32; ++c) {
+        for (int c = 0; c < OC; ++c) {
           float t[32];
-          tmem_ld32(t_o + c * 32 + lane_off, t);
+          tmem_ld32(t_o + half * (DH / 2) + c * 32 + lane_off, t);
 #pragma unroll
           for (int e = 0; e < 32; ++e) t[e] *= corr;
-          tmem_st32(t_o + c * 32 + lane_off, t);
+          tmem_st32(t_o + half * (DH / 2) + c * 32 + lane_off, t);
         }
       }
       if (rescale) {
@@ -235,11 +266,11 @@ __global__ void __launch_bounds__(192, 1)
         m_used = m_new;
       }
       l += ls;
-      // P row r -> swizzled K-major tile (two 64-key slabs)
+      // this half's 64 keys of row r -> slab `half` of the swizzled K-major P tile
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
+      for (int i = 0; i < 8; ++i) {
         uint4 q = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-        *reinterpret_cast<uint4*>(Ps + (i >> 3) * SLAB + swz(r, i)) = q;
+        *reinterpret_cast<uint4*>(Ps + half * SLAB + swz(r, i)) = q;
       }
       fence_proxy_async();
       tc_fence_before();
@@ -248,12 +279,17 @@ __global__ void __launch_bounds__(192, 1)
     }
     if (ok && warp_wait(o_full, 0, abort_flag, status)) {
       tc_fence_after();
-      const float inv = 1.0f / l;
-      bf16* orow = o + (long long)(row0 + qt * 128 + r) * ldo + (long long)h * DH;
+      xsum[half][r] = l;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(xb);
+      const bool got = warp_wait(xb, nkt & 1, abort_flag, status);
+      const float lt = l + (got ? xsum[half ^ 1][r] : 0.f);
+      const float inv = 1.0f / lt;
+      bf16* orow = o + (long long)(row0 + qt * 128 + r) * ldo + (long long)h * DH + half * (DH / 2);
 #pragma unroll 1
-      for (int c = 0; c < DH / 32; ++c) {
+      for (int c = 0; c < OC; ++c) {
         float t[32];
-        tmem_ld32(t_o + c * 32 + lane_off, t);
+        tmem_ld32(t_o + half * (DH / 2) + c * 32 + lane_off, t);
         uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -264,7 +300,7 @@ __global__ void __launch_bounds__(192, 1)
           dst[i] = q;
         }
       }
-      lse[(size_t)h * lse_ld + row0 + qt * 128 + r] = (m_used + log2f(l)) * kLn2;
+      if (half == 0) lse[(size_t)h * lse_ld + row0 + qt * 128 + r] = (m_used + log2f(lt)) * kLn2;
     }
   }
 
@@ -279,7 +315,7 @@ __global__ void __launch_bounds__(192, 1)
 template <int DH>
 cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
                    int max_seqs, int* status, cudaStream_t st) {
-  constexpr size_t smem = (size_t)(DH / 64) * SLAB * 5 + 2 * SLAB + 1024 + 256;
+  constexpr size_t smem = (size_t)(DH / 64) * SLAB * 5 + 2 * SLAB + 6 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
@@ -289,8 +325,8 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
   }
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
-  dim3 grid(S / 128, H, max_seqs);
-  attn_fwd_tc_kernel<DH><<<grid, 192, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, status);
+  dim3 grid(H, max_seqs, S / 128);
+  attn_fwd_tc_kernel<DH><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, status);
   return cudaGetLastError();
 }
 
@@ -298,20 +334,20 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // ---------------------------------------------------------------------------
 // Backward, head size 128.  One CTA per (128-key tile, kv head, kept
 // sequence), looping over the query heads of the group and the 64-query
-// tiles at or after the key tile.  320 threads:
-//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (2 stages)
+// tiles at or after the key tile.  448 threads:
+//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
 //   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
 //               (M = 128 keys, N = 64 queries); then for step i-1
 //               dV += P^T dO, dK += dS^T Q (M = 128 keys, N = 128) and
 //               dQ^T = K^T dS^T (M = 128 head dims, N = 64 queries)
-//   warps 2..5  one key per thread: P^T = exp2(S^T c log2e - lse log2e),
+//   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e),
 //               dS^T = P^T (dP^T - D), both to swizzled bf16 tiles; at the
 //               end dK (times c) and dV from TMEM to dqkv
-//   warps 6..9  dQ^T from TMEM, added into the float32 dQ buffer
+//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
 // TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(448, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
                        const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
@@ -321,33 +357,34 @@ __global__ void __launch_bounds__(320, 1)
   constexpr int DH = 128;
   constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
   constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
+  constexpr int NST = 3;               // stages of the Q / dO / lse / D ring
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Ks = smem;
   uint8_t* Vs = Ks + KT;
-  uint8_t* Qs = Vs + KT;         // [2][QT]
-  uint8_t* dOs = Qs + 2 * QT;    // [2][QT]
-  uint8_t* PTs = dOs + 2 * QT;   // 128 keys x 64 queries, one slab of 128-byte rows
+  uint8_t* Qs = Vs + KT;         // [NST][QT]
+  uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
+  uint8_t* PTs = dOs + NST * QT; // 128 keys x 64 queries, one slab of 128-byte rows
   uint8_t* DSs = PTs + SLAB;
   float* dqs = reinterpret_cast<float*>(DSs + SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
-  float* vecs = dqs + 64 * DH;                         // [2][lse 64 | D 64]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + 256);
+  float* vecs = dqs + 64 * DH;                         // [NST][lse 64 | D 64]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * 128);
   uint64_t* kv_full = bars;
-  uint64_t* ld_full = bars + 1;  // [2]
-  uint64_t* ld_empty = bars + 3; // [2]
-  uint64_t* sdp_full = bars + 5;
-  uint64_t* sdp_free = bars + 6;
-  uint64_t* p_ready = bars + 7;
-  uint64_t* mm_done = bars + 8;
-  uint64_t* dq_free = bars + 9;
-  uint64_t* acc_done = bars + 10;
-  uint64_t* drain = bars + 11;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  uint64_t* ld_full = bars + 1;          // [NST]
+  uint64_t* ld_empty = ld_full + NST;    // [NST]
+  uint64_t* sdp_full = ld_empty + NST;
+  uint64_t* sdp_free = sdp_full + 1;
+  uint64_t* p_ready = sdp_full + 2;
+  uint64_t* mm_done = sdp_full + 3;
+  uint64_t* dq_free = sdp_full + 4;
+  uint64_t* acc_done = sdp_full + 5;
+  uint64_t* drain = sdp_full + 6;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sdp_full + 7);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  const int seq = blockIdx.z;
+  const int seq = blockIdx.y;
   if (seq >= *cnt) return;
-  const int kt = blockIdx.x, g = blockIdx.y, grp = H / Hkv;
+  const int kt = blockIdx.z, g = blockIdx.x, grp = H / Hkv;  // heaviest key tiles (kt = 0) dispatched first
   const int row0 = seq * S;
   const int nq = S / 64, q0 = 2 * kt;          // query tiles q0 .. nq-1 overlap or follow the keys
   const int n_it = grp * (nq - q0);
@@ -356,13 +393,13 @@ __global__ void __launch_bounds__(320, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < NST; ++b) {
       mbar_init(&ld_full[b], 1);
       mbar_init(&ld_empty[b], 1);
     }
     mbar_init(sdp_full, 1);
-    mbar_init(sdp_free, 4);
-    mbar_init(p_ready, 4);
+    mbar_init(sdp_free, 8);
+    mbar_init(p_ready, 8);
     mbar_init(mm_done, 1);
     mbar_init(dq_free, 4);
     mbar_init(acc_done, 1);
@@ -388,9 +425,9 @@ __global__ void __launch_bounds__(320, 1)
       }
       int issued = 0;
       for (int i = 0; i < n_it; ++i) {
-        const int b = i & 1;
+        const int b = i % NST;
         const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
-        if (!mbar_wait(&ld_empty[b], ((i >> 1) & 1) ^ 1u, abort_flag, status)) break;
+        if (!mbar_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
         mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 512);
         for (int c = 0; c < 2; ++c) {
           tma_load_2d(Qs + b * QT + c * HSLAB, &tmq, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
@@ -403,7 +440,7 @@ __global__ void __launch_bounds__(320, 1)
       }
       if (*abort_flag) {
         mbar_drain(kv_full, 0);
-        for (int i = issued > 2 ? issued - 2 : 0; i < issued; ++i) mbar_drain(&ld_full[i & 1], (i >> 1) & 1);
+        for (int i = issued > NST ? issued - NST : 0; i < issued; ++i) mbar_drain(&ld_full[i % NST], (i / NST) & 1);
       }
     }
   } else if (warp == 1) {
@@ -417,8 +454,8 @@ __global__ void __launch_bounds__(320, 1)
       bool ok = mbar_wait(kv_full, 0, abort_flag, status);
       for (int i = 0; ok && i <= n_it; ++i) {
         if (i < n_it) {
-          const int b = i & 1;
-          if (!mbar_wait(&ld_full[b], (i >> 1) & 1, abort_flag, status)) { ok = false; break; }
+          const int b = i % NST;
+          if (!mbar_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
           if (!mbar_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
 #pragma unroll
@@ -431,7 +468,7 @@ __global__ void __launch_bounds__(320, 1)
           mma_commit(sdp_full);
         }
         if (i >= 1) {
-          const int ip = i - 1, b = ip & 1;
+          const int ip = i - 1, b = ip % NST;
           if (!mbar_wait(p_ready, ip & 1, abort_flag, status)) { ok = false; break; }
           if (!mbar_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
@@ -457,44 +494,43 @@ __global__ void __launch_bounds__(320, 1)
         mbar_drain(drain, 0);
       }
     }
-  } else if (warp < 6) {
-    // ------------------------------------------------ P / dS (warps 2..5)
+  } else if (warp < 10) {
+    // ------------------------------------------------ P / dS (warps 2..9)
+    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..31 of the
+    // step, warps 6..9 queries 32..63, one key per thread
     const int quad = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
     const float sl2 = kLog2e * rsqrtf((float)DH);
     bool ok = true;
     for (int i = 0; i < n_it; ++i) {
-      const int b = i & 1;
+      const int b = i % NST;
       const int qt = q0 + i % (nq - q0);
       if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
-      if (!warp_wait(&ld_full[b], (i >> 1) & 1, abort_flag, status)) { ok = false; break; }
+      if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t sr[2][32], dr[2][32];
-      tmem_ld32_nw(t_s + lane_off, sr[0]);
-      tmem_ld32_nw(t_s + 32 + lane_off, sr[1]);
-      tmem_ld32_nw(t_dp + lane_off, dr[0]);
-      tmem_ld32_nw(t_dp + 32 + lane_off, dr[1]);
+      uint32_t sr[32], dr[32];
+      tmem_ld32_nw(t_s + half * 32 + lane_off, sr);
+      tmem_ld32_nw(t_dp + half * 32 + lane_off, dr);
       tmem_wait_ld();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
-      const float* lv = vecs + b * 128;
-      const int qbase = qt * 64 - key;  // query c is visible iff qbase + c >= 0
-      uint32_t pk[32], dk[32];
+      const float* lv = vecs + b * 128 + half * 32;
+      const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
+      uint32_t pk[16], dk[16];
 #pragma unroll
-      for (int e = 0; e < 32; ++e) {
+      for (int e = 0; e < 16; ++e) {
         float p[2], d[2];
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
           const int c = 2 * e + u;
-          const float s_ = __uint_as_float(sr[c >> 5][c & 31]);
-          const float dpv = __uint_as_float(dr[c >> 5][c & 31]);
-          float pv = ex2(fmaf(s_, sl2, -lv[c] * kLog2e));
+          float pv = ex2(fmaf(__uint_as_float(sr[c]), sl2, -lv[c] * kLog2e));
           pv = (qbase + c >= 0) ? pv : 0.f;
           p[u] = pv;
-          d[u] = pv * (dpv - lv[64 + c]);
+          d[u] = pv * (__uint_as_float(dr[c]) - lv[64 + c]);
         }
         __nv_bfloat162 bp = __floats2bfloat162_rn(p[0], p[1]), bd = __floats2bfloat162_rn(d[0], d[1]);
         pk[e] = *reinterpret_cast<uint32_t*>(&bp);
@@ -503,9 +539,10 @@ __global__ void __launch_bounds__(320, 1)
       // the MMAs of step i-1 must be done with P^T / dS^T before they are rewritten
       if (i >= 1 && !warp_wait(mm_done, (i - 1) & 1, abort_flag, status)) { ok = false; break; }
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        *reinterpret_cast<uint4*>(PTs + swz(r, c)) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-        *reinterpret_cast<uint4*>(DSs + swz(r, c)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
+      for (int c = 0; c < 4; ++c) {
+        const int chunk = half * 4 + c;
+        *reinterpret_cast<uint4*>(PTs + swz(r, chunk)) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        *reinterpret_cast<uint4*>(DSs + swz(r, chunk)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
       }
       fence_proxy_async();
       tc_fence_before();
@@ -514,45 +551,47 @@ __global__ void __launch_bounds__(320, 1)
     }
     if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
       tc_fence_after();
-      const float c = rsqrtf((float)DH);
-      bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
-      bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
+      if (half == 0) {
+        // dK (times c) with the inverse rotation at the key's position
+        const float c = rsqrtf((float)DH);
+        bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
 #pragma unroll 1
-      for (int cc = 0; cc < 2; ++cc) {
-        // dK pairs (i, i + 64), i = 32cc .. 32cc+31: scale, inverse rotation at
-        // the key's position, bf16
-        float k1[32], k2[32];
-        tmem_ld32(t_dk + cc * 32 + lane_off, k1);
-        tmem_ld32(t_dk + 64 + cc * 32 + lane_off, k2);
+        for (int cc = 0; cc < 2; ++cc) {
+          float k1[32], k2[32];
+          tmem_ld32(t_dk + cc * 32 + lane_off, k1);
+          tmem_ld32(t_dk + 64 + cc * 32 + lane_off, k2);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const float p1 = c * k1[e], p2 = c * k2[e];
-          float cs = 1.f, sn = 0.f;
-          if (rcos) {
-            cs = rcos[(size_t)key * 64 + cc * 32 + e];
-            sn = rsin[(size_t)key * 64 + cc * 32 + e];
+          for (int e = 0; e < 32; ++e) {
+            const float p1 = c * k1[e], p2 = c * k2[e];
+            float cs = 1.f, sn = 0.f;
+            if (rcos) {
+              cs = rcos[(size_t)key * 64 + cc * 32 + e];
+              sn = rsin[(size_t)key * 64 + cc * 32 + e];
+            }
+            k1[e] = p1 * cs + p2 * sn;
+            k2[e] = p2 * cs - p1 * sn;
           }
-          k1[e] = p1 * cs + p2 * sn;
-          k2[e] = p2 * cs - p1 * sn;
+          st_bf16x32_(krow + cc * 32, k1);
+          st_bf16x32_(krow + 64 + cc * 32, k2);
         }
-        st_bf16x32_(krow + cc * 32, k1);
-        st_bf16x32_(krow + 64 + cc * 32, k2);
-      }
+      } else {
+        bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
 #pragma unroll 1
-      for (int cc = 0; cc < DH / 32; ++cc) {
-        float u[32];
-        tmem_ld32(t_dv + cc * 32 + lane_off, u);
-        st_bf16x32_(vrow + cc * 32, u);
+        for (int cc = 0; cc < DH / 32; ++cc) {
+          float u[32];
+          tmem_ld32(t_dv + cc * 32 + lane_off, u);
+          st_bf16x32_(vrow + cc * 32, u);
+        }
       }
     }
   } else {
-    // ------------------------------------------------ dQ (warps 6..9)
+    // ------------------------------------------------ dQ (warps 10..13)
     // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
     // into dq_acc by one bulk tensor reduce per step.
     const int quad = warp & 3;
     const int dd = quad * 32 + lane;  // head dimension of this thread
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const bool leader = (warp == 6 && lane == 0);
+    const bool leader = (warp == 10 && lane == 0);
     for (int i = 0; i < n_it; ++i) {
       const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
       if (!warp_wait(mm_done, i & 1, abort_flag, status)) break;
@@ -590,7 +629,9 @@ __global__ void __launch_bounds__(320, 1)
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, int* status, cudaStream_t st) {
-  constexpr size_t smem = 6 * SLAB + 8 * HSLAB + 256 * 4 + 64 * 128 * 4 + 1024 + 256;
+  // K, V, P^T, dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
+  // vectors + dQ staging + alignment + barriers = 232,192 bytes (of 232,448)
+  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 128 * 4 + 64 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(attn_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -603,8 +644,8 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
-  dim3 grid(S / 128, Hkv, max_seqs);
-  attn_bwd_tc_kernel<<<grid, 320, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H, Hkv,
+  dim3 grid(Hkv, max_seqs, S / 128);
+  attn_bwd_tc_kernel<<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H, Hkv,
                                               rcos, rsin, status);
   return cudaGetLastError();
 }
