@@ -37,6 +37,13 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "effective tokens/s (fwd+bwd) under layer dropout; % bf16 peak; skip-speedup vs ideal"
+
+# DRAM read + write of the tcgen05 GEMM per kept row of a launch, from one
+# ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the 24 GEMM
+# launches of a 2-layer stack with the Llama-3-8B shapes and 12288 kept rows
+# per launch; command and per-launch table in
+# profiles/gemm_tc_llama8b_traffic.md.  Scaled by the kept rows per launch.
+GEMM_DRAM_BYTES_PER_ROW = 159899.0
 PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 
 
@@ -397,9 +404,15 @@ def main():
         cpu = cpu_baseline(cfg, w0, x0[0].cpu(), dy0[0].cpu(), min(args.cpu_rows, S), kept_units / args.steps, sc[0])
 
     gemm_achieved = gemm_flops * args.steps / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
+    # 12 GEMM launches per executed layer (4 forward, 8 backward)
+    traffic = None
+    if args.config == "llama8b" and gemm_launches > 0:
+        rows_per_launch = kept_units * S / (gemm_launches / 12.0)
+        traffic = GEMM_DRAM_BYTES_PER_ROW * rows_per_launch
     roof = {"kernel": "gemm_tc_kernel (tcgen05 projections, fwd dgrad wgrad)", "bound": "tensor",
             "achieved": gemm_achieved, "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
-            "frac": gemm_achieved / peaks["bf16_sustained"] if gemm_achieved else None, "traffic": None,
+            "frac": gemm_achieved / peaks["bf16_sustained"] if gemm_achieved else None, "traffic": traffic,
+            "traffic_source": "ncu DRAM bytes of a 2-layer capture per kept row, times kept rows per launch",
             "peak_kind": f"bf16 sustained ({peaks['source']})", "launches_per_step": gemm_launches / args.steps,
             "avg_launch_ms": gemm_ms / max(gemm_launches, 1)}
     line = {

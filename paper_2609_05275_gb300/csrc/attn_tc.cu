@@ -20,6 +20,8 @@
 // The running max is only moved (and O rescaled in TMEM) when it grows by
 // more than 2^8, so most tiles need no O round trip; P <= 2^8 stays well
 // inside bf16/fp32 range.  All waits are bounded (status word on expiry).
+#include <type_traits>
+
 #include "tc_common.cuh"
 
 namespace ldk {
@@ -221,10 +223,17 @@ __global__ void __launch_bounds__(320, 1)
       if (lane == 0) mbar_arrive(&s_free[j & 1]);
       // running max on the raw scores (the scale is positive); keys after
       // the query (diagonal tile only) are left out
-      const int lim = ((j == qt) ? r : 127) - half * 64;  // last visible local column
+      const bool diag = (j == qt);                       // the only tile with masked keys (block-uniform)
+      const int lim = (diag ? r : 127) - half * 64;      // last visible local column
       float mraw = -INFINITY;
+      if (diag) {
 #pragma unroll
-      for (int e = 0; e < 64; ++e) mraw = fmaxf(mraw, e <= lim ? __uint_as_float(sr[e >> 5][e & 31]) : -INFINITY);
+        for (int e = 0; e < 64; ++e) mraw = fmaxf(mraw, e <= lim ? __uint_as_float(sr[e >> 5][e & 31]) : -INFINITY);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 64; e += 2)
+          mraw = fmax3(mraw, __uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1]));
+      }
       xmax[j & 1][half][r] = mraw;
       __syncwarp();
       if (lane == 0) mbar_arrive(xb);
@@ -233,18 +242,33 @@ __global__ void __launch_bounds__(320, 1)
       const float mt = mraw * sl2;
       const bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
-      float ls = 0.f;
+      // P = exp2(S c log2e - m) on pairs of keys (packed fp32 pipe); the
+      // causal mask only on the diagonal tile
       uint32_t pk[32];
+      uint64_t ls2 = f2_pack(0.f, 0.f);
+      auto pass = [&](auto masked) {
+        constexpr bool MASK = decltype(masked)::value;
+        const uint64_t sl2x2 = f2_pack(sl2, sl2), nm2 = f2_pack(-m_new, -m_new);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        float p0 = ex2(fmaf(__uint_as_float(sr[(2 * e) >> 5][(2 * e) & 31]), sl2, -m_new));
-        float p1 = ex2(fmaf(__uint_as_float(sr[(2 * e + 1) >> 5][(2 * e + 1) & 31]), sl2, -m_new));
-        p0 = (2 * e <= lim) ? p0 : 0.f;
-        p1 = (2 * e + 1 <= lim) ? p1 : 0.f;
-        ls += p0 + p1;
-        __nv_bfloat162 bq = __floats2bfloat162_rn(p0, p1);
-        pk[e] = *reinterpret_cast<uint32_t*>(&bq);
-      }
+        for (int e = 0; e < 32; ++e) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e >> 4][(2 * e) & 31]), __uint_as_float(sr[e >> 4][(2 * e + 1) & 31])),
+                           sl2x2, nm2),
+                    x0, x1);
+          float p0 = ex2(x0), p1 = ex2(x1);
+          if constexpr (MASK) {
+            p0 = (2 * e <= lim) ? p0 : 0.f;
+            p1 = (2 * e + 1 <= lim) ? p1 : 0.f;
+          }
+          ls2 = f2_add(ls2, f2_pack(p0, p1));
+          pk[e] = bf16x2_bits(p0, p1);
+        }
+      };
+      if (diag) pass(std::true_type{});
+      else pass(std::false_type{});
+      float ls_a, ls_b;
+      f2_unpack(ls2, ls_a, ls_b);
+      const float ls = ls_a + ls_b;
       // P_{j-1} V_{j-1} must be done before P and O are touched
       if (j >= 1 && !warp_wait(pv_done, (j - 1) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
@@ -389,7 +413,6 @@ __global__ void __launch_bounds__(448, 1)
   const int nq = S / 64, q0 = 2 * kt;          // query tiles q0 .. nq-1 overlap or follow the keys
   const int n_it = grp * (nq - q0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int HD = H * DH;
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
@@ -518,24 +541,40 @@ __global__ void __launch_bounds__(448, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
-      const float* lv = vecs + b * 128 + half * 32;
+      const float4* lv4 = reinterpret_cast<const float4*>(vecs + b * 128 + half * 32);       // lse of the 32 queries
+      const float4* dv4 = reinterpret_cast<const float4*>(vecs + b * 128 + 64 + half * 32);  // D of the 32 queries
       const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
       uint32_t pk[16], dk[16];
+      // pairs of queries on the packed fp32 pipe; the causal mask only on
+      // warps whose 32 keys are not all visible to the 32 queries (warp-uniform)
+      auto pass = [&](auto masked) {
+        constexpr bool MASK = decltype(masked)::value;
+        const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
 #pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        float p[2], d[2];
+        for (int e4 = 0; e4 < 8; ++e4) {
+          const float4 lq = lv4[e4], dq = dv4[e4];
+          const uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
+          const uint64_t dd[2] = {f2_pack(dq.x, dq.y), f2_pack(dq.z, dq.w)};
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int c = 2 * e + u;
-          float pv = ex2(fmaf(__uint_as_float(sr[c]), sl2, -lv[c] * kLog2e));
-          pv = (qbase + c >= 0) ? pv : 0.f;
-          p[u] = pv;
-          d[u] = pv * (__uint_as_float(dr[c]) - lv[64 + c]);
+          for (int h2 = 0; h2 < 2; ++h2) {
+            const int c = 4 * e4 + 2 * h2;
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2, nl[h2]), x0, x1);
+            float p0 = ex2(x0), p1 = ex2(x1);
+            if constexpr (MASK) {
+              p0 = (qbase + c >= 0) ? p0 : 0.f;
+              p1 = (qbase + c + 1 >= 0) ? p1 : 0.f;
+            }
+            const uint64_t pp = f2_pack(p0, p1);
+            float d0, d1;
+            f2_unpack(f2_mul(pp, f2_sub(f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1])), dd[h2])), d0, d1);
+            pk[c >> 1] = bf16x2_bits(p0, p1);
+            dk[c >> 1] = bf16x2_bits(d0, d1);
+          }
         }
-        __nv_bfloat162 bp = __floats2bfloat162_rn(p[0], p[1]), bd = __floats2bfloat162_rn(d[0], d[1]);
-        pk[e] = *reinterpret_cast<uint32_t*>(&bp);
-        dk[e] = *reinterpret_cast<uint32_t*>(&bd);
-      }
+      };
+      if (__shfl_sync(0xffffffffu, qbase, 31) >= 0) pass(std::false_type{});
+      else pass(std::true_type{});
       // the MMAs of step i-1 must be done with P^T / dS^T before they are rewritten
       if (i >= 1 && !warp_wait(mm_done, (i - 1) & 1, abort_flag, status)) { ok = false; break; }
 #pragma unroll

@@ -166,7 +166,9 @@ int rmsnorm_bwd_blocks(int max_rows) { return grid_for(max_rows, 8, device_sm_co
 // of the gain gradient in registers, and the block reduces the dot products of
 // RPB rows at once (their loads are all in flight together).  No
 // shared-memory atomics; all global accesses coalesced.
-template <typename T, int MAXJ, int RPB>
+// PF: the residual-gradient rows dx are read together with dyn and xs (one
+// memory round trip per row group instead of two; costs 8 MAXJ RPB registers).
+template <typename T, int MAXJ, int RPB, bool PF>
 __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __restrict__ dyn,
                                                                const float* __restrict__ xs,
                                                                const float* __restrict__ rstd,
@@ -191,8 +193,11 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __re
   }
   const long long M = (long long)(*cnt) * S;
   for (long long m0 = (long long)blockIdx.x * RPB; m0 < M; m0 += (long long)gridDim.x * RPB) {
-    float dy[RPB][MAXJ][8], xv[RPB][MAXJ][8];
+    float dy[RPB][MAXJ][8], xv[RPB][MAXJ][8], cur[PF ? RPB : 1][MAXJ][8];
     float pd[RPB];
+    long long rr[RPB];
+#pragma unroll
+    for (int q = 0; q < RPB; ++q) rr[q] = (m0 + q < M) ? src_row(kept_idx, S, m0 + q) : 0;
 #pragma unroll
     for (int q = 0; q < RPB; ++q) {
       const long long m = m0 + q;
@@ -203,6 +208,7 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __re
         if (m < M && c8 < d8) {
           ld8(dyn + m * d + c8 * 8, dy[q][j]);
           ld8(xs + m * d + c8 * 8, xv[q][j]);
+          if constexpr (PF) ld8(dx + rr[q] * d + c8 * 8, cur[q][j]);
 #pragma unroll
           for (int e = 0; e < 8; ++e) pd[q] += dy[q][j][e] * g[j][e] * xv[q][j][e];
         }
@@ -224,23 +230,28 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __re
     for (int q = 0; q < RPB; ++q) {
       const long long m = m0 + q;
       if (m >= M) break;
-      const long long r = src_row(kept_idx, S, m);
+      const long long r = rr[q];
       const float rs = rstd[m];
       const float dot = tot[q] * rs / (float)d;  // mean(dyn * gamma * xn)
 #pragma unroll
       for (int j = 0; j < MAXJ; ++j) {
         const int c8 = tid + 256 * j;
         if (c8 < d8) {
-          float cur[8], nx[8];
-          ld8(dx + r * d + c8 * 8, cur);
+          float cr[8], nx[8];
+          if constexpr (PF) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) cr[e] = cur[q][j][e];
+          } else {
+            ld8(dx + r * d + c8 * 8, cr);
+          }
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             const float xn = xv[q][j][e] * rs;
-            cur[e] = cur[e] + rs * (dy[q][j][e] * g[j][e] - xn * dot);
-            nx[e] = scale * cur[e];
+            cr[e] = cr[e] + rs * (dy[q][j][e] * g[j][e] - xn * dot);
+            nx[e] = scale * cr[e];
             gacc[j][e] += dy[q][j][e] * xn;
           }
-          st8(dx + r * d + c8 * 8, cur);
+          st8(dx + r * d + c8 * 8, cr);
           if (next) st8(next + m * d + c8 * 8, nx);
         }
       }
@@ -260,11 +271,11 @@ cudaError_t launch_rmsnorm_bwd(const float* dyn, const float* xs, const float* r
                                T* next, float* part, int nblocks, cudaStream_t st) {
   (void)max_rows;
   if (d <= 2048) {
-    rmsnorm_bwd_cols_kernel<T, 1, 4><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
+    rmsnorm_bwd_cols_kernel<T, 1, 2, true><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
   } else if (d <= 4096) {
-    rmsnorm_bwd_cols_kernel<T, 2, 2><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
+    rmsnorm_bwd_cols_kernel<T, 2, 1, true><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
   } else if (d <= 8192) {
-    rmsnorm_bwd_cols_kernel<T, 4, 1><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
+    rmsnorm_bwd_cols_kernel<T, 4, 1, false><<<nblocks, 256, 0, st>>>(dyn, xs, rstd, gamma, dx, kept_idx, cnt, S, d, scale, next, part);
   } else {
     const size_t smem = (size_t)d * sizeof(float);
     if (smem > 48 * 1024) {
