@@ -362,13 +362,18 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 //   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
 //   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
 //               (M = 128 keys, N = 64 queries); then for step i-1
-//               dV += P^T dO, dK += dS^T Q (M = 128 keys, N = 128) and
-//               dQ^T = K^T dS^T (M = 128 head dims, N = 64 queries)
-//   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e),
-//               dS^T = P^T (dP^T - D), both to swizzled bf16 tiles; at the
-//               end dK (times c) and dV from TMEM to dqkv
+//               dV += P^T dO (P^T read from TMEM), dK += dS^T Q (M = 128
+//               keys, N = 128) and dQ^T = K^T dS^T (M = 128 head dims,
+//               N = 64 queries)
+//   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e)
+//               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
+//               swizzled shared-memory tile; at the end dK (times c) and dV
+//               from TMEM to dqkv
 //   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
-// TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447.
+// P^T and dS^T are double-buffered (step i uses buffer i & 1), so the
+// softmax warps write step i while the MMAs of step i-1 still read theirs.
+// TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447,
+// P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
 __global__ void __launch_bounds__(448, 1)
@@ -388,9 +393,8 @@ __global__ void __launch_bounds__(448, 1)
   uint8_t* Vs = Ks + KT;
   uint8_t* Qs = Vs + KT;         // [NST][QT]
   uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
-  uint8_t* PTs = dOs + NST * QT; // 128 keys x 64 queries, one slab of 128-byte rows
-  uint8_t* DSs = PTs + SLAB;
-  float* dqs = reinterpret_cast<float*>(DSs + SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
+  uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
+  float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
   float* vecs = dqs + 64 * DH;                         // [NST][lse 64 | D 64]
   uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * 128);
   uint64_t* kv_full = bars;
@@ -398,12 +402,12 @@ __global__ void __launch_bounds__(448, 1)
   uint64_t* ld_empty = ld_full + NST;    // [NST]
   uint64_t* sdp_full = ld_empty + NST;
   uint64_t* sdp_free = sdp_full + 1;
-  uint64_t* p_ready = sdp_full + 2;
-  uint64_t* mm_done = sdp_full + 3;
-  uint64_t* dq_free = sdp_full + 4;
-  uint64_t* acc_done = sdp_full + 5;
-  uint64_t* drain = sdp_full + 6;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sdp_full + 7);
+  uint64_t* p_ready = sdp_full + 2;  // [2] per P^T / dS^T buffer
+  uint64_t* mm_done = sdp_full + 4;  // [2] per P^T / dS^T buffer
+  uint64_t* dq_free = sdp_full + 6;
+  uint64_t* acc_done = sdp_full + 7;
+  uint64_t* drain = sdp_full + 8;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sdp_full + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int seq = blockIdx.y;
@@ -422,8 +426,10 @@ __global__ void __launch_bounds__(448, 1)
     }
     mbar_init(sdp_full, 1);
     mbar_init(sdp_free, 8);
-    mbar_init(p_ready, 8);
-    mbar_init(mm_done, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&p_ready[b], 8);
+      mbar_init(&mm_done[b], 1);
+    }
     mbar_init(dq_free, 4);
     mbar_init(acc_done, 1);
     mbar_init(drain, 1);
@@ -436,6 +442,7 @@ __global__ void __launch_bounds__(448, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t t_s = tmem, t_dp = tmem + 64, t_dv = tmem + 128, t_dk = tmem + 256, t_dq = tmem + 384;
+  const uint32_t t_p = tmem + 448;  // [2] x 32 columns: P^T as bf16 pairs
 
   if (warp == 0) {
     if (lane == 0) {
@@ -473,7 +480,7 @@ __global__ void __launch_bounds__(448, 1)
       constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
       constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
       const uint32_t ka = smem_u32(Ks), va = smem_u32(Vs), qa = smem_u32(Qs), oa = smem_u32(dOs);
-      const uint32_t pa = smem_u32(PTs), da = smem_u32(DSs);
+      const uint32_t da0 = smem_u32(DSs);
       bool ok = mbar_wait(kv_full, 0, abort_flag, status);
       for (int i = 0; ok && i <= n_it; ++i) {
         if (i < n_it) {
@@ -491,22 +498,23 @@ __global__ void __launch_bounds__(448, 1)
           mma_commit(sdp_full);
         }
         if (i >= 1) {
-          const int ip = i - 1, b = ip % NST;
-          if (!mbar_wait(p_ready, ip & 1, abort_flag, status)) { ok = false; break; }
+          const int ip = i - 1, b = ip % NST, pb = ip & 1;
+          if (!mbar_wait(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
           if (!mbar_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
+          const uint32_t da = da0 + pb * SLAB;
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
-            const uint32_t aoff = kk * 32;                       // P^T / dS^T, K-major
+            const uint32_t aoff = kk * 32;                       // dS^T, K-major
             const uint32_t boff = b * QT + kk * 2048;            // dO / Q as MN-major
-            mma_bf16(t_dv, sdesc(pa + aoff, 16, 1024), sdesc(oa + boff, HSLAB, 1024), ID_KV, (ip > 0 || kk > 0));
+            mma_bf16_ta(t_dv, t_p + pb * 32 + kk * 8, sdesc(oa + boff, HSLAB, 1024), ID_KV, (ip > 0 || kk > 0));
             mma_bf16(t_dk, sdesc(da + aoff, 16, 1024), sdesc(qa + boff, HSLAB, 1024), ID_KV, (ip > 0 || kk > 0));
           }
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
             mma_bf16(t_dq, sdesc(ka + kk * 2048, SLAB, 1024), sdesc(da + kk * 2048, 16, 1024), ID_Q, kk > 0);
           }
-          mma_commit(mm_done);
+          mma_commit(&mm_done[pb]);
           mma_commit(&ld_empty[b]);
         }
       }
@@ -575,18 +583,22 @@ __global__ void __launch_bounds__(448, 1)
       };
       if (__shfl_sync(0xffffffffu, qbase, 31) >= 0) pass(std::false_type{});
       else pass(std::true_type{});
-      // the MMAs of step i-1 must be done with P^T / dS^T before they are rewritten
-      if (i >= 1 && !warp_wait(mm_done, (i - 1) & 1, abort_flag, status)) { ok = false; break; }
+      // the MMAs of step i-2 must be done with buffer i & 1 before it is rewritten
+      const int pb = i & 1;
+      if (i >= 2 && !warp_wait(&mm_done[pb], ((i >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      tmem_st16(t_p + pb * 32 + half * 16 + lane_off, pk);
+      uint8_t* ds = DSs + pb * SLAB;
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         const int chunk = half * 4 + c;
-        *reinterpret_cast<uint4*>(PTs + swz(r, chunk)) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-        *reinterpret_cast<uint4*>(DSs + swz(r, chunk)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
+        *reinterpret_cast<uint4*>(ds + swz(r, chunk)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
       }
       fence_proxy_async();
+      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(p_ready);
+      if (lane == 0) mbar_arrive(&p_ready[pb]);
     }
     if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
       tc_fence_after();
@@ -633,7 +645,7 @@ __global__ void __launch_bounds__(448, 1)
     const bool leader = (warp == 10 && lane == 0);
     for (int i = 0; i < n_it; ++i) {
       const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
-      if (!warp_wait(mm_done, i & 1, abort_flag, status)) break;
+      if (!warp_wait(&mm_done[i & 1], (i >> 1) & 1, abort_flag, status)) break;
       tc_fence_after();
       float t0[32], t1[32];
       tmem_ld32(t_dq + lane_off, t0);
@@ -668,7 +680,7 @@ __global__ void __launch_bounds__(448, 1)
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, int* status, cudaStream_t st) {
-  // K, V, P^T, dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
+  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
   // vectors + dQ staging + alignment + barriers = 232,192 bytes (of 232,448)
   constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 128 * 4 + 64 * 128 * 4 + 1024 + 256;
   static bool attr = false;
