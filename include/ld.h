@@ -11,6 +11,8 @@
  *   Eq. (transformer_layer_dropout_train), one mask for both sub-blocks
  *   (layer granularity, Model Granularity subsection):
  *     Z^l = X^l + r M^l f_attn(X^l),   X^{l+1} = Z^l + r M^l f_ffn(Z^l)
+ *   or, with sub-layer granularity (same subsection), independent masks
+ *   M^l_attn and M^l_ffn in place of M^l in those two updates;
  *   r = alpha / (1 - p) (Dropout Scale paragraph; parameterization table).
  *
  * and, as the Preliminary section's "more efficient implementation" asks, it
@@ -93,6 +95,9 @@ typedef struct {
   int b_offset;     /* global index of this batch's sequence 0 (data-
                        parallel shards draw the masks of their global
                        sequences; 0 for an unsharded batch)               */
+  int sublayer;     /* 0: one mask per (layer, sequence) for both blocks;
+                       1: sub-layer granularity, independent attention and
+                       FFN masks, each Bernoulli(1 - p^{l,t})             */
 } ld_config;
 
 typedef struct {
@@ -141,8 +146,9 @@ ld_status ld_get_rates(void* handle, long long step, double* p, unsigned long lo
 /* Draw the masks of step t into the workspace (the first kernel of
  * ld_forward, alone).  Philox4x32-10 (Salmon et al., SC'11): key = (seed
  * low 32 bits, seed high 32 bits), counter = (b', l, t low, t high) with
- * b' = b_offset + b per sequence and b' = 0 per batch; word 0 is u.  Kept
- * lists are ascending in b (local indices). */
+ * b' = b_offset + b per sequence and b' = 0 per batch; word 0 is u (with
+ * sub-layer granularity word 0 draws the attention mask and word 1 the FFN
+ * mask).  Kept lists are ascending in b (local indices). */
 ld_status ld_draw_masks(void* handle, long long step, void* workspace, void* stream);
 
 /* Forward of step t, in place on x [B*S, d] (sequence b = rows b*S..b*S+S-1).
@@ -165,7 +171,9 @@ ld_status ld_backward(void* handle, const ld_layer_w* W, void* dx, ld_layer_g* G
 
 /* Copy the masks of the last ld_forward / ld_draw_masks to host memory:
  * mask [L*B] (1 = keep), kept_idx [L*B] (ascending, -1 padded), kept_cnt
- * [L].  Synchronises that call's stream.  Any output may be NULL. */
+ * [L]; with sub-layer granularity the attention tables followed by the FFN
+ * tables: mask and kept_idx [2*L*B], kept_cnt [2*L].  Synchronises that
+ * call's stream.  Any output may be NULL. */
 ld_status ld_get_masks(void* handle, unsigned char* mask, int* kept_idx, int* kept_cnt);
 
 /* Synchronise the stream of the last call and return the device status word

@@ -14,6 +14,10 @@ Reading of the draw (the paper names no generator):
       b' = 0 per batch (so a per-batch mask is the per-sequence draw of
       sequence 0, broadcast);
   the layer is dropped for that sequence iff u < thr_l, thr_l = floor(p 2^32).
+Sub-layer granularity (Model Granularity subsection: M_attn and M_ffn drawn
+independently, each Bernoulli(1 - p^{l,t})): the attention mask uses word 0
+of the same Philox output and the FFN mask word 1, so the attention mask is
+the layer-granularity mask.
 Kept lists are in ascending b.
 """
 
@@ -24,32 +28,41 @@ from .philox import philox4x32_10, philox4x32_10_np
 PER_SEQUENCE, PER_BATCH = "per_sequence", "per_batch"
 
 
-def mask_word(seed, step, layer, b):
-    """The 32-bit uniform word for (seed, step, layer, sequence)."""
+def mask_word(seed, step, layer, b, word=0):
+    """The 32-bit uniform word for (seed, step, layer, sequence): output word
+    `word` of Philox4x32-10."""
     seed = int(seed)
     step = int(step)
     key = (seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
     ctr = (b, layer, step & 0xFFFFFFFF, (step >> 32) & 0xFFFFFFFF)
-    return philox4x32_10(ctr, key)[0]
+    return philox4x32_10(ctr, key)[word]
 
 
-def draw_masks(seed, step, thresholds, B, granularity=PER_SEQUENCE, b_offset=0):
+def draw_masks(seed, step, thresholds, B, granularity=PER_SEQUENCE, b_offset=0, sublayer=False):
     """mask[l][b] in {0,1} (1 = keep) for every layer l (uint8, shape [L, B]);
-    the batch holds the global sequences b_offset .. b_offset + B - 1."""
+    with ``sublayer`` the pair (M_attn, M_ffn) as uint8 [2, L, B].  The batch
+    holds the global sequences b_offset .. b_offset + B - 1."""
     L = len(thresholds)
-    mask = np.zeros((L, B), dtype=np.uint8)
-    for layer in range(L):
-        for b in range(B):
-            bb = b_offset + b if granularity == PER_SEQUENCE else 0
-            u = mask_word(seed, step, layer, bb)
-            mask[layer, b] = 0 if u < thresholds[layer] else 1
-    return mask
+    nw = 2 if sublayer else 1
+    mask = np.zeros((nw, L, B), dtype=np.uint8)
+    for w in range(nw):
+        for layer in range(L):
+            for b in range(B):
+                bb = b_offset + b if granularity == PER_SEQUENCE else 0
+                u = mask_word(seed, step, layer, bb, w)
+                mask[w, layer, b] = 0 if u < thresholds[layer] else 1
+    return mask if sublayer else mask[0]
 
 
 def kept_lists(mask):
     """kept_idx[l] = ascending b with mask[l][b] = 1; kept_cnt[l] = its length.
 
-    Returned as (int32 [L, B] padded with -1, int32 [L])."""
+    Returned as (int32 [L, B] padded with -1, int32 [L]); a sub-layer mask
+    [2, L, B] gives ([2, L, B], [2, L])."""
+    mask = np.asarray(mask)
+    if mask.ndim == 3:
+        pairs = [kept_lists(m) for m in mask]
+        return np.stack([p[0] for p in pairs]), np.stack([p[1] for p in pairs])
     L, B = mask.shape
     idx = np.full((L, B), -1, dtype=np.int32)
     cnt = np.zeros(L, dtype=np.int32)

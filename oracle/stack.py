@@ -8,6 +8,10 @@ both sub-blocks (layer granularity, Model Granularity subsection):
     Z^l      = X^l + r M^l f_attn(X^l)
     X^{l+1}  = Z^l + r M^l f_ffn(Z^l)
 
+or, with sub-layer granularity (same subsection), independent masks
+M^l_attn and M^l_ffn in place of M^l in the two lines: a sequence may run
+either block alone, both or neither.
+
 and the per-sequence case form of the Preliminary section: a dropped
 sequence keeps X^{l+1}[b] = X^l[b]; a kept one gets the residual update with
 r = alpha / (1 - p^{l,t}) (Dropout Scale paragraph and the parameterization
@@ -153,12 +157,10 @@ def _split_qkv(qkv, cfg):
     return q, k, v
 
 
-def layer_forward(x, W, cfg, s, rope_cs):
-    """Kept sequence x [S, d] -> X^{l+1}[b] and the values the backward needs."""
+def attn_forward(x, W, cfg, s, rope_cs):
+    """Attention residual block of a kept sequence: Z = X + s f_attn(X)."""
     S = x.shape[0]
-    F = cfg["F"]
-    eps = cfg["eps"]
-    xh, xn, r1 = rmsnorm(x, W["g1"], eps)
+    xh, xn, r1 = rmsnorm(x, W["g1"], cfg["eps"])
     q, k, v = _split_qkv(xh @ W["w_qkv"].T, cfg)
     if rope_cs is not None:
         cos, sin = rope_cs
@@ -166,22 +168,38 @@ def layer_forward(x, W, cfg, s, rope_cs):
         k = rope(k, cos[:S], sin[:S])
     o = attention(q, k, v).reshape(S, -1)
     z = x + s * (o @ W["w_o"].T)
-    zh, zn, r2 = rmsnorm(z, W["g2"], eps)
+    return z, dict(xh=xh, xn=xn, r1=r1, q=q, k=k, v=v, o=o)
+
+
+def ffn_forward(z, W, cfg, s):
+    """FFN residual block of a kept sequence: X' = Z + s f_ffn(Z)."""
+    F = cfg["F"]
+    zh, zn, r2 = rmsnorm(z, W["g2"], cfg["eps"])
     gu = zh @ W["w_gu"].T
     g, u = gu[:, :F], gu[:, F:]
     h = g * sigmoid(g) * u
     out = z + s * (h @ W["w_d"].T)
-    cache = dict(xh=xh, xn=xn, r1=r1, q=q, k=k, v=v, o=o, zh=zh, zn=zn, r2=r2, g=g, u=u, h=h)
-    return out, cache
+    return out, dict(zh=zh, zn=zn, r2=r2, g=g, u=u, h=h)
+
+
+def layer_forward(x, W, cfg, s, rope_cs):
+    """Kept sequence x [S, d] -> X^{l+1}[b] and the values the backward needs."""
+    z, ca = attn_forward(x, W, cfg, s, rope_cs)
+    out, cf = ffn_forward(z, W, cfg, s)
+    return out, {**ca, **cf}
 
 
 def layer_backward(dout, W, cfg, s, cache, G, rope_cs):
     """d X^{l+1}[b] -> d X^l[b] for a kept sequence; adds into the layer's
     weight gradients G."""
-    S = dout.shape[0]
-    H, Hkv, Dh = cfg["H"], cfg["Hkv"], cfg["Dh"]
+    dz = ffn_backward(dout, W, cfg, s, cache, G)
+    return attn_backward(dz, W, cfg, s, cache, G, rope_cs)
+
+
+def ffn_backward(dout, W, cfg, s, cache, G):
+    """d X'[b] -> d Z[b] through the FFN block; adds into G."""
     c = cache
-    # FFN branch: out = z + s * (h w_d^T), h = silu(g) u.
+    # out = z + s * (h w_d^T), h = silu(g) u.
     dy = s * dout
     G["w_d"] += dy.T @ c["h"]
     dh = dy @ W["w_d"]
@@ -193,8 +211,15 @@ def layer_backward(dout, W, cfg, s, cache, G, rope_cs):
     dzh = dgu @ W["w_gu"]
     dz_norm, dg2 = rmsnorm_backward(dzh, c["zn"], c["r2"], W["g2"])
     G["g2"] += dg2
-    dz = dout + dz_norm
-    # attention branch: z = x + s * (o w_o^T).
+    return dout + dz_norm
+
+
+def attn_backward(dz, W, cfg, s, cache, G, rope_cs):
+    """d Z[b] -> d X[b] through the attention block; adds into G."""
+    S = dz.shape[0]
+    H, Dh = cfg["H"], cfg["Dh"]
+    c = cache
+    # z = x + s * (o w_o^T).
     da = s * dz
     G["w_o"] += da.T @ c["o"]
     do = (da @ W["w_o"]).reshape(S, H, Dh)
@@ -231,39 +256,61 @@ def _rope_cs(cfg, S):
     return rope_tables(S, cfg["Dh"], theta)
 
 
+def _branch_masks(masks):
+    """(attention mask [L, B], FFN mask [L, B]) from a layer mask [L, B]
+    (both blocks share it, layer granularity) or a sub-layer pair [2, L, B]
+    (independent M_attn and M_ffn, Model Granularity subsection)."""
+    masks = np.asarray(masks)
+    if masks.ndim == 3:
+        return masks[0], masks[1]
+    return masks, masks
+
+
 def stack_forward(x, layers, cfg, masks, scales):
-    """x [B, S, d] -> (X^L, caches).  masks [L, B] (1 = keep), scales [L]."""
+    """x [B, S, d] -> (X^L, caches).  masks [L, B] or [2, L, B] (1 = keep),
+    scales [L]."""
     X = np.array(x, dtype=np.float64, copy=True)
     B, S, _ = X.shape
-    L = masks.shape[0]
+    ma, mf = _branch_masks(masks)
+    L = ma.shape[0]
     rope_cs = _rope_cs(cfg, S)
     caches = [[None] * B for _ in range(L)]
     for l in range(L):
-        if not masks[l].any():
+        if not (ma[l].any() or mf[l].any()):
             continue
         W = _layer(layers, l)
         for b in range(B):
-            if masks[l, b]:
-                X[b], caches[l][b] = layer_forward(X[b], W, cfg, scales[l], rope_cs)
+            c = {}
+            if ma[l, b]:
+                X[b], ca = attn_forward(X[b], W, cfg, scales[l], rope_cs)
+                c.update(ca)
+            if mf[l, b]:
+                X[b], cf = ffn_forward(X[b], W, cfg, scales[l])
+                c.update(cf)
+            if c:
+                caches[l][b] = c
     return X, caches
 
 
 def stack_backward(dy, layers, cfg, masks, scales, caches):
     """d X^L -> (d X^0, per-layer weight gradients).
 
-    Dropped sequences pass their gradient through unchanged; a layer's weight
+    Dropped sequences pass their gradient through unchanged; a block's weight
     gradients sum over its kept sequences only (zero if none is kept)."""
     dX = np.array(dy, dtype=np.float64, copy=True)
     B, S, _ = dX.shape
-    L = masks.shape[0]
+    ma, mf = _branch_masks(masks)
+    L = ma.shape[0]
     rope_cs = _rope_cs(cfg, S)
     grads = [None] * L
     for l in reversed(range(L)):
-        W = _layer(layers, l) if masks[l].any() else None
+        W = _layer(layers, l) if (ma[l].any() or mf[l].any()) else None
         G = {n: np.zeros(shape_of(cfg, n)) for n in WEIGHT_NAMES}
         for b in range(B):
-            if masks[l, b]:
-                dX[b] = layer_backward(dX[b], W, cfg, scales[l], caches[l][b], G, rope_cs)
+            if mf[l, b]:
+                dX[b] = ffn_backward(dX[b], W, cfg, scales[l], caches[l][b], G)
+            if ma[l, b]:
+                dX[b] = attn_backward(dX[b], W, cfg, scales[l], caches[l][b], G, rope_cs)
         grads[l] = G
     return dX, grads
 

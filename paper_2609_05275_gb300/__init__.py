@@ -33,7 +33,7 @@ GRAN = {"per_sequence": LD_PER_SEQUENCE, "per_batch": LD_PER_BATCH}
 class ld_config(ctypes.Structure):
     _fields_ = [("L", c_int), ("d", c_int), ("H", c_int), ("Hkv", c_int), ("Dh", c_int), ("F", c_int),
                 ("B", c_int), ("S", c_int), ("eps", c_float), ("rope_theta", c_float), ("alpha", c_float),
-                ("granularity", c_int), ("fp32_debug", c_int), ("b_offset", c_int)]
+                ("granularity", c_int), ("fp32_debug", c_int), ("b_offset", c_int), ("sublayer", c_int)]
 
 
 class ld_schedule(ctypes.Structure):
@@ -128,11 +128,11 @@ def ld_status_str(status):
     return lib().ld_status_str(int(status)).decode()
 
 
-def make_config(cfg, granularity="per_sequence", fp32_debug=False, b_offset=0):
+def make_config(cfg, granularity="per_sequence", fp32_debug=False, b_offset=0, sublayer=False):
     return ld_config(cfg["L"], cfg["d"], cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"], cfg["B"], cfg["S"],
                      cfg.get("eps", 1e-6), cfg.get("rope_theta", 0.0), cfg.get("alpha", 1.0),
                      GRAN[granularity] if isinstance(granularity, str) else int(granularity), int(fp32_debug),
-                     int(b_offset))
+                     int(b_offset), int(sublayer))
 
 
 def ld_create(config):
@@ -196,12 +196,17 @@ def ld_backward(h, wtab, dx, gtab, workspace, stream=None):
     _check(lib().ld_backward(h, wtab, _ptr(dx), gtab, _ptr(workspace), _stream(stream)), "ld_backward")
 
 
-def ld_get_masks(h, L, B):
+def ld_get_masks(h, L, B, sublayer=False):
+    """(mask, kept_idx, kept_cnt) as [L, B], [L, B], [L]; with sub-layer
+    granularity [2, L, B], [2, L, B], [2, L] (attention, then FFN)."""
     import numpy as np
-    mask = np.zeros(L * B, dtype=np.uint8)
-    idx = np.zeros(L * B, dtype=np.int32)
-    cnt = np.zeros(L, dtype=np.int32)
+    nm = 2 if sublayer else 1
+    mask = np.zeros(nm * L * B, dtype=np.uint8)
+    idx = np.zeros(nm * L * B, dtype=np.int32)
+    cnt = np.zeros(nm * L, dtype=np.int32)
     _check(lib().ld_get_masks(h, mask.ctypes.data, idx.ctypes.data, cnt.ctypes.data), "ld_get_masks")
+    if sublayer:
+        return mask.reshape(2, L, B), idx.reshape(2, L, B), cnt.reshape(2, L)
     return mask.reshape(L, B), idx.reshape(L, B), cnt
 
 
@@ -277,10 +282,12 @@ def grad_table(grads):
 class LayerDropStack:
     """A handle with its workspace: forward / backward of the whole stack."""
 
-    def __init__(self, cfg, sched, granularity="per_sequence", fp32_debug=False, device="cuda", b_offset=0):
+    def __init__(self, cfg, sched, granularity="per_sequence", fp32_debug=False, device="cuda", b_offset=0,
+                 sublayer=False):
         import torch
         self.cfg = dict(cfg)
-        self.config = make_config(cfg, granularity, fp32_debug, b_offset)
+        self.sublayer = bool(sublayer)
+        self.config = make_config(cfg, granularity, fp32_debug, b_offset, sublayer)
         self.h = ld_create(self.config)
         self.schedule = make_schedule(sched)
         ld_set_schedule(self.h, self.schedule)
@@ -293,10 +300,10 @@ class LayerDropStack:
 
     def draw_masks(self, step, stream=None):
         ld_draw_masks(self.h, step, self.workspace, stream)
-        return ld_get_masks(self.h, self.cfg["L"], self.cfg["B"])
+        return ld_get_masks(self.h, self.cfg["L"], self.cfg["B"], self.sublayer)
 
     def masks(self):
-        return ld_get_masks(self.h, self.cfg["L"], self.cfg["B"])
+        return ld_get_masks(self.h, self.cfg["L"], self.cfg["B"], self.sublayer)
 
     def forward(self, step, wtab, x, stream=None):
         ld_forward(self.h, step, wtab, x, self.workspace, stream)

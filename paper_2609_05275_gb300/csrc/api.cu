@@ -134,9 +134,10 @@ void make_layout(Handle* h) {
     return at;
   };
   y.status = take(64);
-  y.mask = take((size_t)c.L * c.B);
-  y.kidx = take((size_t)c.L * c.B * 4);
-  y.kcnt = take((size_t)c.L * 4);
+  const size_t nm = c.sublayer ? 2 : 1;  // attention and FFN tables with sub-layer granularity
+  y.mask = take(nm * c.L * c.B);
+  y.kidx = take(nm * c.L * c.B * 4);
+  y.kcnt = take(nm * c.L * 4);
   y.rcos = take((size_t)c.S * (c.Dh / 2) * 4);
   y.rsin = take((size_t)c.S * (c.Dh / 2) * 4);
   // per-layer saved activations
@@ -350,6 +351,7 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
   P.B = c.B;
   P.granularity = c.granularity;
   P.b_offset = c.b_offset;
+  P.nmask = c.sublayer ? 2 : 1;
   std::vector<float> scale(c.L);
   step_rates(h, step, nullptr, P.thr, scale.data());
   {
@@ -362,8 +364,12 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
 
   const int HD = c.H * c.Dh;
   for (int l = 0; l < c.L; ++l) {
+    // kept lists of the attention block (cnt, ki) and of the FFN block
+    // (cntf, kif); the same list unless the masks are drawn per sub-layer
     const int* cnt = kcnt + l;
     const int* ki = kidx + (size_t)l * c.B;
+    const int* cntf = c.sublayer ? kcnt + c.L + l : cnt;
+    const int* kif = c.sublayer ? kidx + (size_t)(c.L + l) * c.B : ki;
     char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
     float* xin = reinterpret_cast<float*>(lb + y.xin);
     T* xh = reinterpret_cast<T*>(lb + y.xh);
@@ -404,11 +410,17 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     a.ldx = c.d;
     a.kept_idx = ki;
     a.S = c.S;
-    a.save = z;
+    a.save = c.sublayer ? nullptr : z;  // same rows feed the FFN block: keep a compact copy of Z
     a.ld_save = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st)); }
-    a = rows_gemm(h, cnt, 2 * c.F, c.d, zh, c.d, W[l].w_gu, c.d, 0);
+    if (c.sublayer) {  // the FFN block gathers its own rows of Z from the residual stream
+      Timed tm_(h, LD_KCLASS_ROWWISE, st);
+      LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, kif, cntf, c.S, c.d, h->max_rows, g2, c.eps, z, zh, rstd2, st));
+    } else {
+      Timed tm_(h, LD_KCLASS_ROWWISE, st);
+      LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st));
+    }
+    a = rows_gemm(h, cntf, 2 * c.F, c.d, zh, c.d, W[l].w_gu, c.d, 0);
     a.epi = EPI_STORE;
     a.D = gu;
     a.ldd = 2 * c.F;
@@ -418,13 +430,13 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
       a.F = c.F;
     }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cnt, c.S, c.F, h->max_rows, st)); }
-    a = rows_gemm(h, cnt, c.d, c.F, hh, c.F, W[l].w_d, c.F, 0);
+    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cntf, c.S, c.F, h->max_rows, st)); }
+    a = rows_gemm(h, cntf, c.d, c.F, hh, c.F, W[l].w_d, c.F, 0);
     a.epi = EPI_RESID;
     a.alpha = s;
     a.x = x;
     a.ldx = c.d;
-    a.kept_idx = ki;
+    a.kept_idx = kif;
     a.S = c.S;
     a.save = nullptr;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
@@ -464,8 +476,10 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
   }
 
   for (int l = c.L - 1; l >= 0; --l) {
-    const int* cnt = kcnt + l;
+    const int* cnt = kcnt + l;  // attention block's kept list; FFN block's below
     const int* ki = kidx + (size_t)l * c.B;
+    const int* cntf = c.sublayer ? kcnt + c.L + l : cnt;
+    const int* kif = c.sublayer ? kidx + (size_t)(c.L + l) * c.B : ki;
     char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
     float* xin = reinterpret_cast<float*>(lb + y.xin);
     T* xh = reinterpret_cast<T*>(lb + y.xh);
@@ -483,8 +497,8 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     const float s = h->fwd_scale[l];
 
     // FFN branch: dy = r * dX^{l+1} on the kept rows.
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, ki, cnt, c.S, c.d, h->max_rows, s, dy, st)); }
-    GemmArgs a = rows_gemm(h, cnt, c.F, c.d, dy, c.d, W[l].w_d, c.F, 1);  // dh = dy W_d
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, kif, cntf, c.S, c.d, h->max_rows, s, dy, st)); }
+    GemmArgs a = rows_gemm(h, cntf, c.F, c.d, dy, c.d, W[l].w_d, c.F, 1);  // dh = dy W_d
     a.epi = EPI_STORE;
     a.D = dh;
     a.ldd = c.F;
@@ -495,21 +509,23 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
       a.F = c.F;
     }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cnt, c.S, c.F, h->max_rows, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
-    a = rows_gemm(h, cnt, c.d, 2 * c.F, dgu, 2 * c.F, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
+    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cntf, c.S, c.F, h->max_rows, st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cntf, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
+    a = rows_gemm(h, cntf, c.d, 2 * c.F, dgu, 2 * c.F, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
     a.epi = EPI_STORE_F32;
     a.D = dzh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, 2 * c.F, c.d, dgu, 2 * c.F, zh, c.d, G[l].w_gu), st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cntf, 2 * c.F, c.d, dgu, 2 * c.F, zh, c.d, G[l].w_gu), st)); }
     // dZ = dX^{l+1} + RMSNorm_2 backward; dz = r * dZ for the attention branch
+    // (written by the same kernel when both blocks keep the same rows)
     {
       Timed tm_(h, LD_KCLASS_ROWWISE, st);
-      LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, ki, cnt, c.S, c.d, h->max_rows, s, dz, part,
-                                     h->part_blocks, st));
+      LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, kif, cntf, c.S, c.d, h->max_rows, s,
+                                     c.sublayer ? (T*)nullptr : dz, part, h->part_blocks, st));
     }
     { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g2, st)); }
+    if (c.sublayer) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, ki, cnt, c.S, c.d, h->max_rows, s, dz, st)); }
     // attention branch
     a = rows_gemm(h, cnt, HD, c.d, dz, c.d, W[l].w_o, HD, 1);  // dO = dz W_o
     a.epi = EPI_STORE;
@@ -568,6 +584,7 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   if (c.Dh != 32 && c.Dh != 64 && c.Dh != 128) return LD_ERR_SHAPE;
   if (c.H < 1 || c.Hkv < 1 || c.H % c.Hkv || (c.H * c.Dh) % 64) return LD_ERR_SHAPE;
   if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH) return LD_ERR_ARG;
+  if (c.sublayer != 0 && c.sublayer != 1) return LD_ERR_ARG;
   if (c.b_offset < 0 || (long long)c.b_offset + c.B > 0x7fffffffll) return LD_ERR_ARG;
   if ((long long)c.B * c.S > (1ll << 30)) return LD_ERR_SHAPE;
   Handle* h = new (std::nothrow) Handle();
@@ -635,6 +652,7 @@ ld_status ld_draw_masks(void* handle, long long step, void* ws, void* stream) {
   P.B = h->cfg.B;
   P.granularity = h->cfg.granularity;
   P.b_offset = h->cfg.b_offset;
+  P.nmask = h->cfg.sublayer ? 2 : 1;
   step_rates(h, step, nullptr, P.thr, nullptr);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   LD_CHECK(cudaMemsetAsync(at<int>(ws, y.status), 0, sizeof(int), st));
@@ -688,11 +706,12 @@ ld_status ld_get_masks(void* handle, unsigned char* mask, int* kept_idx, int* ke
   Handle* h = H(handle);
   if (!h->have_masks) return LD_ERR_STATE;
   const Layout& y = h->lay;
-  const size_t LB = (size_t)h->cfg.L * h->cfg.B;
+  const size_t nm = h->cfg.sublayer ? 2 : 1;
+  const size_t LB = nm * h->cfg.L * h->cfg.B;
   LD_CHECK(cudaStreamSynchronize(h->last_stream));
   if (mask) LD_CHECK(cudaMemcpy(mask, at<unsigned char>(h->last_ws, y.mask), LB, cudaMemcpyDeviceToHost));
   if (kept_idx) LD_CHECK(cudaMemcpy(kept_idx, at<int>(h->last_ws, y.kidx), LB * 4, cudaMemcpyDeviceToHost));
-  if (kept_cnt) LD_CHECK(cudaMemcpy(kept_cnt, at<int>(h->last_ws, y.kcnt), (size_t)h->cfg.L * 4, cudaMemcpyDeviceToHost));
+  if (kept_cnt) LD_CHECK(cudaMemcpy(kept_cnt, at<int>(h->last_ws, y.kcnt), nm * h->cfg.L * 4, cudaMemcpyDeviceToHost));
   return LD_OK;
 }
 

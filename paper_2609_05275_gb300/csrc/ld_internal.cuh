@@ -52,6 +52,7 @@ struct MaskParams {
   unsigned long long seed;
   long long step;
   int L, B, granularity, b_offset;
+  int nmask;  // 1: one mask per (layer, sequence); 2: attention (word 0) and FFN (word 1) masks
   unsigned long long thr[LD_MAX_L];
 };
 cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* kept_idx, int* kept_cnt,

@@ -9,6 +9,9 @@
 // Draw: u = word 0 of Philox4x32-10 (Salmon et al., SC'11) with key
 // (seed lo, seed hi) and counter (b', l, t lo, t hi), b' = b per sequence
 // and 0 per batch.  Sequence b drops layer l iff u < thr_l = floor(p 2^32).
+// Sub-layer granularity (Model Granularity subsection): the attention mask
+// takes word 0 and the FFN mask word 1 of the same draw; their tables follow
+// each other ([2][L][B], counts [2][L]).
 #include "ld_internal.cuh"
 
 namespace ldk {
@@ -34,8 +37,8 @@ __global__ void mask_compact_kernel(const MaskParams P, unsigned char* __restric
                                     int* __restrict__ kept_idx, int* __restrict__ kept_cnt) {
   __shared__ int warp_off[32];
   __shared__ int base;
-  const int l = blockIdx.x;
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int w = blockIdx.x / P.L, l = blockIdx.x % P.L;  // mask w of layer l
+  const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5, nw = blockDim.x >> 5;
   const unsigned long long thr = P.thr[l];
   const uint2 key = make_uint2((uint32_t)P.seed, (uint32_t)(P.seed >> 32));
   const uint32_t t_lo = (uint32_t)(unsigned long long)P.step, t_hi = (uint32_t)((unsigned long long)P.step >> 32);
@@ -46,14 +49,15 @@ __global__ void mask_compact_kernel(const MaskParams P, unsigned char* __restric
     int keep = 0;
     if (b < P.B) {
       const uint32_t bb = P.granularity == LD_PER_BATCH ? 0u : (uint32_t)(P.b_offset + b);
-      const uint32_t u = philox4x32_10(make_uint4(bb, (uint32_t)l, t_lo, t_hi), key).x;
+      const uint4 r = philox4x32_10(make_uint4(bb, (uint32_t)l, t_lo, t_hi), key);
+      const uint32_t u = w == 0 ? r.x : r.y;
       keep = (unsigned long long)u >= thr;
-      mask[(size_t)l * P.B + b] = (unsigned char)keep;
+      mask[(size_t)blockIdx.x * P.B + b] = (unsigned char)keep;
     }
     const unsigned bal = __ballot_sync(0xffffffffu, keep);
-    if (lane == 0) warp_off[w] = __popc(bal);
+    if (lane == 0) warp_off[wp] = __popc(bal);
     __syncthreads();
-    if (w == 0) {
+    if (wp == 0) {
       // exclusive scan of the per-warp counts
       int v = lane < nw ? warp_off[lane] : 0;
       int incl = v;
@@ -66,13 +70,13 @@ __global__ void mask_compact_kernel(const MaskParams P, unsigned char* __restric
       if (lane == 31) warp_off[31] = incl;  // chunk total (nw <= 31 slots used above)
     }
     __syncthreads();
-    if (keep) kept_idx[(size_t)l * P.B + base + warp_off[w] + __popc(bal & ((1u << lane) - 1u))] = b;
+    if (keep) kept_idx[(size_t)blockIdx.x * P.B + base + warp_off[wp] + __popc(bal & ((1u << lane) - 1u))] = b;
     __syncthreads();
     if (threadIdx.x == 0) base += warp_off[31];
     __syncthreads();
   }
-  for (int i = base + threadIdx.x; i < P.B; i += blockDim.x) kept_idx[(size_t)l * P.B + i] = -1;
-  if (threadIdx.x == 0) kept_cnt[l] = base;
+  for (int i = base + threadIdx.x; i < P.B; i += blockDim.x) kept_idx[(size_t)blockIdx.x * P.B + i] = -1;
+  if (threadIdx.x == 0) kept_cnt[blockIdx.x] = base;
 }
 
 cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* kept_idx, int* kept_cnt,
@@ -80,7 +84,7 @@ cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* k
   // at most 31 warps so that slot 31 of warp_off can hold the chunk total
   int threads = ((P.B + 31) / 32) * 32;
   if (threads > 992) threads = 992;
-  mask_compact_kernel<<<P.L, threads, 0, st>>>(P, mask, kept_idx, kept_cnt);
+  mask_compact_kernel<<<P.L * P.nmask, threads, 0, st>>>(P, mask, kept_idx, kept_cnt);
   return cudaGetLastError();
 }
 

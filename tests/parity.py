@@ -26,12 +26,12 @@ def oracle_sched(sched):
     return d
 
 
-def oracle_masks(cfg, sched, step, granularity="per_sequence"):
+def oracle_masks(cfg, sched, step, granularity="per_sequence", sublayer=False):
     rates = OS.layer_rates(oracle_sched(sched), cfg["L"], step)
     thr = [OS.drop_threshold(p) for p in rates]
     scales = [OS.residual_scale(p, cfg.get("alpha", 1.0)) for p in rates]
     gran = OM.PER_SEQUENCE if granularity == "per_sequence" else OM.PER_BATCH
-    mask = OM.draw_masks(sched.get("seed", 0), step, thr, cfg["B"], gran)
+    mask = OM.draw_masks(sched.get("seed", 0), step, thr, cfg["B"], gran, sublayer=sublayer)
     return mask, thr, scales
 
 
@@ -52,9 +52,9 @@ def to_np(t):
 
 
 def gpu_run(cfg, sched, step, layers_dev, x_dev, dy_dev, granularity="per_sequence", fp32_debug=False,
-            backward=True):
+            backward=True, sublayer=False):
     """Forward (+ backward) through the C ABI.  Returns (out, dX, grads, masks)."""
-    st = P.LayerDropStack(cfg, sched, granularity=granularity, fp32_debug=fp32_debug)
+    st = P.LayerDropStack(cfg, sched, granularity=granularity, fp32_debug=fp32_debug, sublayer=sublayer)
     try:
         wtab = P.weight_table(layers_dev)
         x = x_dev.clone()
@@ -74,15 +74,15 @@ def gpu_run(cfg, sched, step, layers_dev, x_dev, dy_dev, granularity="per_sequen
 
 
 def oracle_run(cfg, sched, step, layers_host, x_host, dy_host, granularity="per_sequence", rows=None,
-               seqs=None):
+               seqs=None, sublayer=False):
     """The oracle on (optionally) the first `rows` rows of the sequences
     `seqs`; returns (out, dX, grads, mask)."""
-    mask, thr, scales = oracle_masks(cfg, sched, step, granularity)
+    mask, thr, scales = oracle_masks(cfg, sched, step, granularity, sublayer)
     x = x_host.double().numpy()
     dy = dy_host.double().numpy()
     mk = mask
     if seqs is not None:
-        x, dy, mk = x[seqs], dy[seqs], mask[:, seqs]
+        x, dy, mk = x[seqs], dy[seqs], mask[..., seqs]
     if rows is not None:
         x, dy = x[:, :rows], dy[:, :rows]
 

@@ -45,6 +45,21 @@ def test_create_rejects(change, status):
     assert P.ld_create_status(P.make_config(cfg)) == status
 
 
+def test_sublayer_flag():
+    cfg = synth.CONFIGS["tiny"]
+    bad = P.make_config(cfg)
+    bad.sublayer = 2
+    assert P.ld_create_status(bad) == P.LD_ERR_ARG
+    h1, h2 = P.ld_create(P.make_config(cfg)), P.ld_create(P.make_config(cfg, sublayer=True))
+    try:
+        # the attention and FFN mask tables take twice the mask space, nothing else changes
+        n1, n2 = P.ld_workspace_size(h1), P.ld_workspace_size(h2)
+        assert n1 <= n2 <= n1 + 3 * 256 + cfg["L"] * cfg["B"] * 5 + cfg["L"] * 4
+    finally:
+        P.ld_destroy(h1)
+        P.ld_destroy(h2)
+
+
 def test_schedule_validation_and_state():
     h = P.ld_create(P.make_config(synth.CONFIGS["tiny"]))
     try:

@@ -14,12 +14,12 @@ from oracle import masks as OM
 pytestmark = pytest.mark.gpu
 
 
-def _check(cfg, sched, steps, granularity):
-    st = P.LayerDropStack(cfg, sched, granularity=granularity)
+def _check(cfg, sched, steps, granularity, sublayer=False):
+    st = P.LayerDropStack(cfg, sched, granularity=granularity, sublayer=sublayer)
     try:
         for t in steps:
             mask, idx, cnt = st.draw_masks(t)
-            ref, _, _ = oracle_masks(cfg, sched, t, granularity)
+            ref, _, _ = oracle_masks(cfg, sched, t, granularity, sublayer)
             ridx, rcnt = OM.kept_lists(ref)
             assert (mask == ref).all(), t
             assert (cnt == rcnt).all(), t
@@ -53,3 +53,12 @@ def test_large_and_ragged_batches(B):
     cfg = dict(synth.CONFIGS["tiny"], B=B, L=5)
     sched = dict(dist="explicit", p_explicit=[0.0, 1.0, 0.5, 0.1, 0.9], time="const", seed=2 ** 40 + 3)
     _check(cfg, sched, [0, 7], "per_sequence")
+
+
+@pytest.mark.parametrize("granularity", ["per_sequence", "per_batch"])
+@pytest.mark.parametrize("B", [4, 33, 4096])
+def test_sublayer_masks(granularity, B):
+    # attention (word 0) and FFN (word 1) tables, bit for bit
+    cfg = dict(synth.CONFIGS["tiny"], B=B, L=7)
+    sched = dict(dist="ild", p_max=0.8, time="const", seed=2 ** 35 + 9)
+    _check(cfg, sched, [0, 5, 2 ** 33 + 1], granularity, sublayer=True)

@@ -22,11 +22,12 @@ def _inputs(cfg, dtype, gamma_noise=0.0, seed=0):
     return host, x, dy, dev, x.to(dtype).cuda(), dy.to(dtype).cuda()
 
 
-def _compare(cfg, sched, step, fp32, granularity="per_sequence", gamma_noise=0.0):
+def _compare(cfg, sched, step, fp32, granularity="per_sequence", gamma_noise=0.0, sublayer=False):
     dtype = torch.float32 if fp32 else torch.bfloat16
     host, x, dy, dev, xd, dyd = _inputs(cfg, dtype, gamma_noise)
-    out, dX, grads, (mask, idx, cnt) = gpu_run(cfg, sched, step, dev, xd, dyd, granularity, fp32)
-    rout, rdX, rgrads, rmask = oracle_run(cfg, sched, step, host, x, dy, granularity)
+    out, dX, grads, (mask, idx, cnt) = gpu_run(cfg, sched, step, dev, xd, dyd, granularity, fp32,
+                                               sublayer=sublayer)
+    rout, rdX, rgrads, rmask = oracle_run(cfg, sched, step, host, x, dy, granularity, sublayer=sublayer)
     assert (mask == rmask).all()
     ridx, rcnt = OM.kept_lists(rmask)
     assert (idx == ridx).all() and (cnt == rcnt).all()
@@ -37,7 +38,7 @@ def _compare(cfg, sched, step, fp32, granularity="per_sequence", gamma_noise=0.0
             check_close(f"layer{l}.{n}", to_np(grads[l][n]), rgrads[l][n], fp32)
     # dropped sequences: output and gradient pass through bit for bit
     for b in range(cfg["B"]):
-        if not rmask[:, b].any():
+        if not rmask[..., b].any():
             assert torch.equal(out.view(cfg["B"], cfg["S"], -1)[b].cpu(), xd.view(cfg["B"], cfg["S"], -1)[b].cpu())
             assert torch.equal(dX.view(cfg["B"], cfg["S"], -1)[b].cpu(), dyd.view(cfg["B"], cfg["S"], -1)[b].cpu())
     return mask
@@ -95,3 +96,23 @@ def test_multi_tile_full_tensors(cfg, fp32):
     # full tensors (not just the first rows)
     sched = dict(dist="explicit", p_explicit=[0.2, 0.5], time="const", seed=11)
     _compare(cfg, sched, 2, fp32, gamma_noise=0.1)
+
+
+@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
+def test_sublayer_granularity(fp32):
+    # independent attention / FFN masks (Model Granularity subsection): every
+    # combination of (attention kept, FFN kept) occurs; a block's gradients
+    # sum over its own kept sequences
+    cfg = dict(synth.CONFIGS["tiny"], L=3, B=8, H=4, Hkv=2)
+    sched = dict(dist="uniform", p_max=0.5, time="const", seed=3)
+    mask = _compare(cfg, sched, 5, fp32, gamma_noise=0.1, sublayer=True)
+    assert mask.shape == (2, 3, 8)
+    combos = {(int(a), int(f)) for a, f in zip(mask[0].ravel(), mask[1].ravel())}
+    assert combos == {(0, 0), (0, 1), (1, 0), (1, 1)}
+
+
+@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
+def test_sublayer_multi_tile(fp32):
+    cfg = MULTI[1]
+    sched = dict(dist="explicit", p_explicit=[0.5, 0.5], time="const", seed=21)
+    _compare(cfg, sched, 0, fp32, gamma_noise=0.1, sublayer=True, granularity="per_sequence")

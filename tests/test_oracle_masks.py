@@ -127,3 +127,33 @@ def test_tie_at_threshold_keeps():
         u = M.mask_word(2024, 9, 0, b)
         assert M.draw_masks(2024, 9, [u], 5)[0, b] == 1
         assert M.draw_masks(2024, 9, [u + 1], 5)[0, b] == 0
+
+
+def test_sublayer_masks():
+    # Sub-layer granularity: M_attn is the layer-granularity mask (word 0),
+    # M_ffn an independent Bernoulli(1 - p) draw (word 1); p = 0 / 1 and the
+    # per-batch case behave as for one mask; kept lists per block.
+    thr = [S.drop_threshold(p) for p in (0.0, 0.3, 0.5, 1.0)]
+    for gran in (M.PER_SEQUENCE, M.PER_BATCH):
+        pair = M.draw_masks(11, 42, thr, 64, gran, sublayer=True)
+        assert pair.shape == (2, 4, 64) and pair.dtype == np.uint8
+        assert (pair[0] == M.draw_masks(11, 42, thr, 64, gran)).all()
+        assert (pair[:, 0] == 1).all() and (pair[:, 3] == 0).all()
+        if gran == M.PER_BATCH:
+            assert (pair == pair[:, :, :1]).all()
+        idx, cnt = M.kept_lists(pair)
+        assert idx.shape == (2, 4, 64) and cnt.shape == (2, 4)
+        for w in range(2):
+            i1, c1 = M.kept_lists(pair[w])
+            assert (idx[w] == i1).all() and (cnt[w] == c1).all()
+    # joint frequencies of (attn, ffn) at p = 0.5 over 2 * 10^5 draws: each
+    # of the four outcomes within 4 sigma of 1/4
+    t2 = [S.drop_threshold(0.5)] * 50
+    both = np.stack([M.draw_masks(3, t, t2, 400, sublayer=True) for t in range(10)], axis=1)  # [2, 10, 50, 400]
+    a, f = both[0].ravel().astype(np.int64), both[1].ravel().astype(np.int64)
+    n = a.size
+    sigma = math.sqrt(0.25 * 0.75 / n)
+    for va in (0, 1):
+        for vf in (0, 1):
+            assert abs(((a == va) & (f == vf)).mean() - 0.25) < 4 * sigma
+    assert abs(np.corrcoef(a, f)[0, 1]) < 4 / math.sqrt(n)

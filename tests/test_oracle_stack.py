@@ -88,6 +88,54 @@ def test_all_masks_brute_force():
                 assert (out[b] == x[b]).all()
 
 
+def test_sublayer_matches_torch_autograd():
+    # Independent attention / FFN masks (every combination occurs): forward
+    # and hand-derived backward against the dense composition + autograd.
+    cfg = MICRO
+    layers = _layers(cfg, seed=8)
+    x, dy = _inputs(cfg, seed=9)
+    masks = np.array([[[1, 0, 1], [0, 1, 1]],     # M_attn [L, B]
+                      [[0, 0, 1], [1, 1, 0]]],    # M_ffn
+                     dtype=np.uint8)
+    scales = [1.0 / (1 - 0.4), 1.3]
+    out, caches = O.stack_forward(x, layers, cfg, masks, scales)
+    dX, grads = O.stack_backward(dy, layers, cfg, masks, scales, caches)
+    tl = to_torch_layers(layers, requires_grad=True)
+    tx = torch.tensor(x, requires_grad=True)
+    tout = masked_stack(tx, tl, cfg, masks, scales)
+    np.testing.assert_allclose(out, tout.detach().numpy(), rtol=0, atol=1e-11)
+    (tout * torch.tensor(dy)).sum().backward()
+    np.testing.assert_allclose(dX, tx.grad.numpy(), rtol=0, atol=1e-10)
+    for l in range(cfg["L"]):
+        for n in O.WEIGHT_NAMES:
+            ref = tl[l][n].grad
+            ref = np.zeros(O.shape_of(cfg, n)) if ref is None else ref.numpy()
+            np.testing.assert_allclose(grads[l][n], ref, rtol=0, atol=1e-10, err_msg=f"layer {l} {n}")
+
+
+def test_sublayer_brute_force_and_layer_reduction():
+    # Every (M_attn, M_ffn) of B = 1, L = 2 (16 cases) against the dense
+    # composition; equal masks reproduce the layer-granularity stack exactly.
+    cfg = dict(MICRO, B=1)
+    layers = _layers(cfg, seed=10)
+    x, dy = _inputs(cfg, seed=11)
+    tl = to_torch_layers(layers)
+    scales = [1.25, 2.0]
+    for bits in itertools.product([0, 1], repeat=4):
+        masks = np.array(bits, dtype=np.uint8).reshape(2, 2, 1)
+        out, _ = O.stack_forward(x, layers, cfg, masks, scales)
+        ref = masked_stack(torch.tensor(x), tl, cfg, masks, scales).numpy()
+        np.testing.assert_allclose(out, ref, rtol=0, atol=1e-11)
+    for bits in itertools.product([0, 1], repeat=2):
+        m = np.array(bits, dtype=np.uint8).reshape(2, 1)
+        o1, c1 = O.stack_forward(x, layers, cfg, m, scales)
+        o2, c2 = O.stack_forward(x, layers, cfg, np.stack([m, m]), scales)
+        d1, g1 = O.stack_backward(dy, layers, cfg, m, scales, c1)
+        d2, g2 = O.stack_backward(dy, layers, cfg, np.stack([m, m]), scales, c2)
+        assert (o1 == o2).all() and (d1 == d2).all()
+        assert all((g1[l][n] == g2[l][n]).all() for l in range(2) for n in O.WEIGHT_NAMES)
+
+
 def test_p1_is_identity():
     cfg = MICRO
     layers = _layers(cfg)

@@ -57,18 +57,19 @@ def dense_layer(x, W, cfg):
 
 def masked_stack(x, layers, cfg, masks, scales):
     """Stack with per-sequence masks, composed from dense layers:
-    a kept sequence gets z = x + s f_attn(x), x' = z + s f_ffn(z); a dropped
-    one is left as it is."""
+    z = x + s M_attn f_attn(x), x' = z + s M_ffn f_ffn(z), where masks is
+    [L, B] (M_attn = M_ffn = masks, layer granularity) or [2, L, B]
+    (M_attn = masks[0], M_ffn = masks[1], sub-layer granularity)."""
+    ma, mf = (masks[0], masks[1]) if masks.ndim == 3 else (masks, masks)
     B = x.shape[0]
     outs = []
     for b in range(B):
         xb = x[b]
-        for l in range(masks.shape[0]):
-            if masks[l, b]:
-                f_attn, f_ffn = dense_layer(xb, layers[l], cfg)
-                s = float(scales[l])
-                zb = xb + s * f_attn(xb)
-                xb = zb + s * f_ffn(zb)
+        for l in range(ma.shape[0]):
+            f_attn, f_ffn = dense_layer(xb, layers[l], cfg)
+            s = float(scales[l])
+            zb = xb + s * f_attn(xb) if ma[l, b] else xb
+            xb = zb + s * f_ffn(zb) if mf[l, b] else zb
         outs.append(xb)
     return torch.stack(outs)
 
