@@ -61,7 +61,8 @@ def flops_per_token(cfg):
     """Forward FLOPs per token per layer (2 x MACs; causal attention counted
     as S/2 keys per query) and the part of it in the projections."""
     d, H, Hkv, Dh, F, S = cfg["d"], cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"], cfg["S"]
-    proj = 2 * d * (H + 2 * Hkv) * Dh + 2 * d * H * Dh + 6 * d * F
+    ffn = 4 * d * F if cfg.get("act") == "relu2" else 6 * d * F  # up (+ gate) and down
+    proj = 2 * d * (H + 2 * Hkv) * Dh + 2 * d * H * Dh + ffn
     attn = 2 * H * Dh * S
     return proj + attn, proj
 

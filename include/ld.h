@@ -22,6 +22,8 @@
  * Block: RMSNorm -> fused QKV projection -> RoPE -> causal grouped-query
  * attention -> output projection -> scaled residual; RMSNorm -> SwiGLU
  * gate/up -> down projection -> scaled residual.  No biases, no final norm.
+ * The paper's own models (Methodology section) use ALiBi in place of RoPE
+ * and a squared-ReLU feed-forward: ld_config.alibi and ld_config.act.
  *
  * Conventions for every entry point
  *   - Device pointers are plain CUDA device addresses owned by the caller;
@@ -78,6 +80,11 @@ typedef enum { LD_DIST_UNIFORM = 0, LD_DIST_ILD = 1, LD_DIST_ALD = 2, LD_DIST_EX
  *         in the paper).  The product is clamped to [0, 1].              */
 typedef enum { LD_TIME_CONST = 0, LD_TIME_ITS = 1, LD_TIME_DTS = 2, LD_TIME_RAMP = 3 } ld_time;
 
+/* Feed-forward activation.  SwiGLU: h = silu(g) * u with w_gu = [gate;
+ * up] (2F rows).  Squared ReLU (the paper's architecture, Methodology
+ * section): h = max(u, 0)^2 with w_gu = up only (F rows). */
+typedef enum { LD_ACT_SWIGLU = 0, LD_ACT_RELU2 = 1 } ld_act;
+
 typedef struct {
   int L;            /* layers                                             */
   int d;            /* model width; multiple of 64                        */
@@ -98,6 +105,10 @@ typedef struct {
   int sublayer;     /* 0: one mask per (layer, sequence) for both blocks;
                        1: sub-layer granularity, independent attention and
                        FFN masks, each Bernoulli(1 - p^{l,t})             */
+  int alibi;        /* 1: ALiBi position bias, scores of query head h get
+                       + m_h (j - i) with the slopes of Press et al. (ICLR
+                       2022); requires rope_theta = 0                      */
+  int act;          /* ld_act: feed-forward activation                    */
 } ld_config;
 
 typedef struct {
@@ -114,7 +125,8 @@ typedef struct {
 /* Weights of one layer (device pointers, bf16 or float32):
  *   w_qkv [(H+2Hkv)*Dh, d]  rows: Q heads, then K heads, then V heads
  *   w_o   [d, H*Dh]
- *   w_gu  [2F, d]           rows: gate (F), then up (F)
+ *   w_gu  [2F, d]           rows: gate (F), then up (F); [F, d] (up) with
+ *                           LD_ACT_RELU2
  *   w_d   [d, F]
  *   g1, g2 [d]              RMSNorm gains before attention / FFN          */
 typedef struct { const void *w_qkv, *w_o, *w_gu, *w_d, *g1, *g2; } ld_layer_w;
@@ -124,7 +136,8 @@ typedef struct { float *w_qkv, *w_o, *w_gu, *w_d, *g1, *g2; } ld_layer_g;
 
 /* Validate `cfg` and create a handle.  Allocates host memory only (no CUDA
  * call), so it can run without a GPU.  LD_ERR_SHAPE for an unsupported
- * shape, LD_ERR_ARG for null pointers or a non-finite eps/alpha. */
+ * shape, LD_ERR_ARG for null pointers, a non-finite eps/alpha, a flag out of
+ * range or ALiBi together with a rotary embedding. */
 ld_status ld_create(const ld_config* cfg, void** handle);
 
 /* Bytes of device workspace ld_forward/ld_backward need: the mask tables,

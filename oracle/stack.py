@@ -22,7 +22,11 @@ The paper leaves the block internals open (its footnote to the transformer
 form); the block here is the one the workloads name: RMSNorm (eps inside the
 square root, gain gamma), rotary position embedding on q and k, causal
 grouped-query attention with scale 1/sqrt(Dh), SwiGLU feed-forward
-h = silu(g) * u, no biases.  Weights use the [out, in] layout: w_qkv rows are
+h = silu(g) * u, no biases.  The paper's own models (Methodology section)
+use ALiBi position biases and squared-ReLU activations instead: with
+cfg["alibi"] the scores of head h get + m_h (j - i) (no rotary embedding),
+with cfg["act"] == "relu2" the feed-forward is h = max(u, 0)^2 of one up
+projection (w_gu then holds only the F "up" rows).  Weights use the [out, in] layout: w_qkv rows are
 [Q heads; K heads; V heads], w_gu rows are [gate; up].  Query head h reads
 key/value head floor(h * Hkv / H).  RoPE rotates the pairs (i, i + Dh/2) by
 angle pos * theta^(-2i/Dh) at in-sequence position pos; theta = 0 disables it.
@@ -91,10 +95,28 @@ def kv_head(h, H, Hkv):
     return (h * Hkv) // H
 
 
-def attention_probs(qh, kh):
-    """Causal softmax(q k^T / sqrt(Dh)) for one head: [S, S]."""
+def alibi_slopes(H):
+    """Per-head ALiBi slopes (Press et al., "Train Short, Test Long", ICLR
+    2022): for a power of two n, the geometric sequence 2^(-8 k / n),
+    k = 1..n; otherwise the n0 = 2^floor(log2 H) slopes of that sequence
+    followed by every other slope (the 1st, 3rd, ...) of the sequence for
+    2 n0, H - n0 of them."""
+    def geometric(n):
+        return [2.0 ** (-8.0 * k / n) for k in range(1, n + 1)]
+
+    n0 = 2 ** int(math.floor(math.log2(H)))
+    if n0 == H:
+        return np.array(geometric(H))
+    return np.array(geometric(n0) + geometric(2 * n0)[0::2][: H - n0])
+
+
+def attention_probs(qh, kh, slope=None):
+    """Causal softmax(q k^T / sqrt(Dh) [+ slope (j - i)]) for one head: [S, S]."""
     S, Dh = qh.shape
     sc = (qh @ kh.T) / math.sqrt(Dh)
+    if slope is not None:
+        pos = np.arange(S, dtype=np.float64)
+        sc = sc + slope * (pos[None, :] - pos[:, None])
     causal = np.tril(np.ones((S, S), dtype=bool))
     sc = np.where(causal, sc, -np.inf)
     sc = sc - np.max(sc, axis=1, keepdims=True)
@@ -102,25 +124,27 @@ def attention_probs(qh, kh):
     return e / np.sum(e, axis=1, keepdims=True)
 
 
-def attention(q, k, v):
-    """Causal grouped-query attention. q [S,H,Dh], k/v [S,Hkv,Dh] -> [S,H,Dh]."""
+def attention(q, k, v, slopes=None):
+    """Causal grouped-query attention. q [S,H,Dh], k/v [S,Hkv,Dh] -> [S,H,Dh];
+    ``slopes`` [H] adds the ALiBi bias."""
     S, H, Dh = q.shape
     Hkv = k.shape[1]
     o = np.zeros_like(q)
     for h in range(H):
         j = kv_head(h, H, Hkv)
-        P = attention_probs(q[:, h, :], k[:, j, :])
+        P = attention_probs(q[:, h, :], k[:, j, :], None if slopes is None else slopes[h])
         o[:, h, :] = P @ v[:, j, :]
     return o
 
 
-def attention_backward(do, q, k, v):
+def attention_backward(do, q, k, v, slopes=None):
     """Gradients of ``attention`` w.r.t. q, k, v given d(out) = do.
 
     Per head, with P the probabilities and c = 1/sqrt(Dh):
       dv += P^T do;  dP = do v^T;  dS = P * (dP - rowsum(dP * P));
       dq = c dS k;   dk += c dS^T q
-    (key/value gradients summed over the query heads that share them)."""
+    (key/value gradients summed over the query heads that share them; the
+    ALiBi bias is constant in q and k and only enters through P)."""
     S, H, Dh = q.shape
     Hkv = k.shape[1]
     c = 1.0 / math.sqrt(Dh)
@@ -129,7 +153,7 @@ def attention_backward(do, q, k, v):
     dv = np.zeros_like(v)
     for h in range(H):
         j = kv_head(h, H, Hkv)
-        P = attention_probs(q[:, h, :], k[:, j, :])
+        P = attention_probs(q[:, h, :], k[:, j, :], None if slopes is None else slopes[h])
         doh = do[:, h, :]
         dv[:, j, :] += P.T @ doh
         dP = doh @ v[:, j, :].T
@@ -137,6 +161,10 @@ def attention_backward(do, q, k, v):
         dq[:, h, :] = c * (dS @ k[:, j, :])
         dk[:, j, :] += c * (dS.T @ q[:, h, :])
     return dq, dk, dv
+
+
+def relu(x):
+    return np.maximum(x, 0.0)
 
 
 def sigmoid(x):
@@ -157,6 +185,10 @@ def _split_qkv(qkv, cfg):
     return q, k, v
 
 
+def _slopes(cfg):
+    return alibi_slopes(cfg["H"]) if cfg.get("alibi") else None
+
+
 def attn_forward(x, W, cfg, s, rope_cs):
     """Attention residual block of a kept sequence: Z = X + s f_attn(X)."""
     S = x.shape[0]
@@ -166,18 +198,23 @@ def attn_forward(x, W, cfg, s, rope_cs):
         cos, sin = rope_cs
         q = rope(q, cos[:S], sin[:S])
         k = rope(k, cos[:S], sin[:S])
-    o = attention(q, k, v).reshape(S, -1)
+    o = attention(q, k, v, _slopes(cfg)).reshape(S, -1)
     z = x + s * (o @ W["w_o"].T)
     return z, dict(xh=xh, xn=xn, r1=r1, q=q, k=k, v=v, o=o)
 
 
 def ffn_forward(z, W, cfg, s):
-    """FFN residual block of a kept sequence: X' = Z + s f_ffn(Z)."""
+    """FFN residual block of a kept sequence: X' = Z + s f_ffn(Z), with
+    f_ffn = w_d silu(g) u (SwiGLU) or w_d max(u, 0)^2 (squared ReLU)."""
     F = cfg["F"]
     zh, zn, r2 = rmsnorm(z, W["g2"], cfg["eps"])
     gu = zh @ W["w_gu"].T
-    g, u = gu[:, :F], gu[:, F:]
-    h = g * sigmoid(g) * u
+    if cfg.get("act") == "relu2":
+        g, u = None, gu
+        h = relu(u) ** 2
+    else:
+        g, u = gu[:, :F], gu[:, F:]
+        h = g * sigmoid(g) * u
     out = z + s * (h @ W["w_d"].T)
     return out, dict(zh=zh, zn=zn, r2=r2, g=g, u=u, h=h)
 
@@ -203,10 +240,13 @@ def ffn_backward(dout, W, cfg, s, cache, G):
     dy = s * dout
     G["w_d"] += dy.T @ c["h"]
     dh = dy @ W["w_d"]
-    sg = sigmoid(c["g"])
-    dg = dh * c["u"] * sg * (1.0 + c["g"] * (1.0 - sg))
-    du = dh * c["g"] * sg
-    dgu = np.concatenate([dg, du], axis=1)
+    if cfg.get("act") == "relu2":
+        dgu = dh * 2.0 * relu(c["u"])      # d/du max(u, 0)^2 = 2 max(u, 0)
+    else:
+        sg = sigmoid(c["g"])
+        dg = dh * c["u"] * sg * (1.0 + c["g"] * (1.0 - sg))
+        du = dh * c["g"] * sg
+        dgu = np.concatenate([dg, du], axis=1)
     G["w_gu"] += dgu.T @ c["zh"]
     dzh = dgu @ W["w_gu"]
     dz_norm, dg2 = rmsnorm_backward(dzh, c["zn"], c["r2"], W["g2"])
@@ -223,7 +263,7 @@ def attn_backward(dz, W, cfg, s, cache, G, rope_cs):
     da = s * dz
     G["w_o"] += da.T @ c["o"]
     do = (da @ W["w_o"]).reshape(S, H, Dh)
-    dq, dk, dv = attention_backward(do, c["q"], c["k"], c["v"])
+    dq, dk, dv = attention_backward(do, c["q"], c["k"], c["v"], _slopes(cfg))
     if rope_cs is not None:
         cos, sin = rope_cs
         dq = rope_backward(dq, cos[:S], sin[:S])
@@ -251,7 +291,7 @@ def _layer(layers, l):
 
 def _rope_cs(cfg, S):
     theta = cfg.get("rope_theta", 0.0)
-    if not theta:
+    if not theta or cfg.get("alibi"):
         return None
     return rope_tables(S, cfg["Dh"], theta)
 
@@ -320,7 +360,7 @@ def shape_of(cfg, name):
     return {
         "w_qkv": ((H + 2 * Hkv) * Dh, d),
         "w_o": (d, H * Dh),
-        "w_gu": (2 * F, d),
+        "w_gu": ((F if cfg.get("act") == "relu2" else 2 * F), d),
         "w_d": (d, F),
         "g1": (d,),
         "g2": (d,),

@@ -27,13 +27,15 @@ LD_DIST_UNIFORM, LD_DIST_ILD, LD_DIST_ALD, LD_DIST_EXPLICIT = 0, 1, 2, 3
 LD_TIME_CONST, LD_TIME_ITS, LD_TIME_DTS, LD_TIME_RAMP = 0, 1, 2, 3
 DIST = {"uniform": LD_DIST_UNIFORM, "ild": LD_DIST_ILD, "ald": LD_DIST_ALD, "explicit": LD_DIST_EXPLICIT}
 TIME = {"const": LD_TIME_CONST, "its": LD_TIME_ITS, "dts": LD_TIME_DTS, "ramp": LD_TIME_RAMP}
+ACT = {"swiglu": 0, "relu2": 1}
 GRAN = {"per_sequence": LD_PER_SEQUENCE, "per_batch": LD_PER_BATCH}
 
 
 class ld_config(ctypes.Structure):
     _fields_ = [("L", c_int), ("d", c_int), ("H", c_int), ("Hkv", c_int), ("Dh", c_int), ("F", c_int),
                 ("B", c_int), ("S", c_int), ("eps", c_float), ("rope_theta", c_float), ("alpha", c_float),
-                ("granularity", c_int), ("fp32_debug", c_int), ("b_offset", c_int), ("sublayer", c_int)]
+                ("granularity", c_int), ("fp32_debug", c_int), ("b_offset", c_int), ("sublayer", c_int),
+                ("alibi", c_int), ("act", c_int)]
 
 
 class ld_schedule(ctypes.Structure):
@@ -132,7 +134,8 @@ def make_config(cfg, granularity="per_sequence", fp32_debug=False, b_offset=0, s
     return ld_config(cfg["L"], cfg["d"], cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"], cfg["B"], cfg["S"],
                      cfg.get("eps", 1e-6), cfg.get("rope_theta", 0.0), cfg.get("alpha", 1.0),
                      GRAN[granularity] if isinstance(granularity, str) else int(granularity), int(fp32_debug),
-                     int(b_offset), int(sublayer))
+                     int(b_offset), int(sublayer), int(bool(cfg.get("alibi", False))),
+                     ACT[cfg.get("act", "swiglu")])
 
 
 def ld_create(config):

@@ -27,7 +27,7 @@ namespace {
 size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
 
 struct Layout {
-  size_t status, mask, kidx, kcnt, rcos, rsin;
+  size_t status, mask, kidx, kcnt, rcos, rsin, alibi;
   size_t layer0, per_layer;
   size_t xin, xh, qkv, o, lse, z, zh, gu, h, rstd1, rstd2;  // offsets inside a layer block
   size_t dy, dh, dgu, dzh, dz, dO, dqkv, dxh, Dvec, dqacc, part;
@@ -42,7 +42,7 @@ struct Handle {
   std::vector<float> p_expl;
   Layout lay;
   size_t esz = 2;
-  int max_rows = 0, nqkv = 0, part_blocks = 0;
+  int max_rows = 0, nqkv = 0, nf = 0, part_blocks = 0;  // nf: columns of the gate/up projection
   void* last_ws = nullptr;
   cudaStream_t last_stream = nullptr;
   bool have_masks = false;
@@ -140,6 +140,7 @@ void make_layout(Handle* h) {
   y.kcnt = take(nm * c.L * 4);
   y.rcos = take((size_t)c.S * (c.Dh / 2) * 4);
   y.rsin = take((size_t)c.S * (c.Dh / 2) * 4);
+  y.alibi = take((size_t)c.H * 4);
   // per-layer saved activations
   size_t lo = 0;
   auto ltake = [&](size_t bytes) {
@@ -154,7 +155,7 @@ void make_layout(Handle* h) {
   y.lse = ltake((size_t)c.H * R * 4);
   y.z = ltake(R * c.d * 4);
   y.zh = ltake(R * c.d * e);
-  y.gu = ltake(R * 2 * c.F * e);
+  y.gu = ltake(R * h->nf * e);  // g || u (SwiGLU) or u (squared ReLU)
   y.h = ltake(R * c.F * e);
   y.rstd1 = ltake(R * 4);
   y.rstd2 = ltake(R * 4);
@@ -164,7 +165,7 @@ void make_layout(Handle* h) {
   // backward scratch (shared by all layers)
   y.dy = take(R * c.d * e);
   y.dh = take(R * c.F * e);
-  y.dgu = take(R * 2 * c.F * e);
+  y.dgu = take(R * h->nf * e);
   y.dzh = take(R * c.d * 4);  // float32: inputs of the RMSNorm backward
   y.dz = take(R * c.d * e);
   y.dO = take(R * c.H * c.Dh * e);
@@ -271,6 +272,9 @@ cudaError_t gemm<float>(const GemmArgs& a, cudaStream_t st) {
   return gemm_simt(a, st);
 }
 
+// The ALiBi slope table in the workspace, or null without ALiBi.
+const float* alibi_table(const Handle* h, void* ws) { return h->cfg.alibi ? at<float>(ws, h->lay.alibi) : nullptr; }
+
 // Attention: tensor-core flash attention on the bf16 path, SIMT float32 on
 // the debug path.
 template <typename T>
@@ -279,16 +283,17 @@ template <>
 cudaError_t attn_fwd<float>(const Handle* h, void* ws, const float* qkv, float* o, float* lse, const int* cnt,
                             cudaStream_t st) {
   const ld_config& c = h->cfg;
-  return launch_attn_fwd_simt<float>(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, h->max_rows, st);
+  return launch_attn_fwd_simt<float>(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, h->max_rows,
+                                     alibi_table(h, ws), st);
 }
 template <>
 cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, float* lse, const int* cnt,
                            cudaStream_t st) {
   const ld_config& c = h->cfg;
   if (attn_tc_supported(c.S, c.Dh))
-    return launch_attn_fwd_tc(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B,
+    return launch_attn_fwd_tc(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
                               at<int>(ws, h->lay.status), st);
-  return launch_attn_fwd_mma(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, st);
+  return launch_attn_fwd_mma(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws), st);
 }
 
 // Attention backward: dq, dk, dv into dqkv with the inverse RoPE applied to
@@ -305,7 +310,7 @@ cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const 
   if (e != cudaSuccess) return e;
   if (sizeof(T) == 4) {
     e = launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, cnt, c.S, c.H, c.Hkv, c.Dh,
-                                h->max_rows, st);
+                                h->max_rows, alibi_table(h, ws), st);
     if (e != cudaSuccess || !rope) return e;
     return launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1, st);
   }
@@ -314,10 +319,11 @@ cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const 
   bf16* d16 = reinterpret_cast<bf16*>(dqkv);
   if (attn_bwd_tc_supported(c.S, c.Dh)) {
     e = launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt,
-                           c.S, c.H, c.Hkv, c.B, rcos, rsin, at<int>(ws, h->lay.status), st);
+                           c.S, c.H, c.Hkv, c.B, rcos, rsin, alibi_table(h, ws), at<int>(ws, h->lay.status), st);
   } else {
     e = launch_attn_bwd_mma(q16, h->nqkv, reinterpret_cast<const bf16*>(o), reinterpret_cast<const bf16*>(dO),
-                            c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, st);
+                            c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
+                            st);
     if (e == cudaSuccess && rope)  // the k heads of dqkv
       e = launch_rope_apply<bf16>(d16 + (size_t)c.H * c.Dh, h->nqkv, c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1,
                                   st);
@@ -360,6 +366,7 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     if (!f32) LD_CHECK(launch_convert(xv, 0, x, 1, (long long)h->max_rows * c.d, st));
     LD_CHECK(launch_mask_compact(P, mask, kidx, kcnt, st));
     if (c.rope_theta != 0.0f) LD_CHECK(launch_rope_table(rcos, rsin, c.S, c.Dh, (double)c.rope_theta, st));
+    if (c.alibi) LD_CHECK(launch_alibi_table(at<float>(ws, y.alibi), c.H, st));
   }
 
   const int HD = c.H * c.Dh;
@@ -420,17 +427,21 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
       Timed tm_(h, LD_KCLASS_ROWWISE, st);
       LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st));
     }
-    a = rows_gemm(h, cntf, 2 * c.F, c.d, zh, c.d, W[l].w_gu, c.d, 0);
+    a = rows_gemm(h, cntf, h->nf, c.d, zh, c.d, W[l].w_gu, c.d, 0);
     a.epi = EPI_STORE;
     a.D = gu;
-    a.ldd = 2 * c.F;
-    if (!f32) {  // h = silu(g) u in the projection's epilogue
-      a.epi = EPI_SWIGLU;
+    a.ldd = h->nf;
+    if (!f32) {  // h = silu(g) u or max(u, 0)^2 in the projection's epilogue
+      a.epi = c.act ? EPI_RELU2 : EPI_SWIGLU;
       a.h_out = hh;
       a.F = c.F;
     }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cntf, c.S, c.F, h->max_rows, st)); }
+    if (f32) {
+      Timed tm_(h, LD_KCLASS_ROWWISE, st);
+      if (c.act) LD_CHECK(launch_relu2<T>(gu, (const T*)nullptr, hh, cntf, c.S, c.F, h->max_rows, st));
+      else LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cntf, c.S, c.F, h->max_rows, st));
+    }
     a = rows_gemm(h, cntf, c.d, c.F, hh, c.F, W[l].w_d, c.F, 0);
     a.epi = EPI_RESID;
     a.alpha = s;
@@ -502,21 +513,25 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     a.epi = EPI_STORE;
     a.D = dh;
     a.ldd = c.F;
-    if (!f32) {  // SwiGLU backward in the epilogue: dg, du straight from dh
-      a.epi = EPI_SWIGLU_BWD;
+    if (!f32) {  // activation backward in the epilogue: dg, du (or du) straight from dh
+      a.epi = c.act ? EPI_RELU2_BWD : EPI_SWIGLU_BWD;
       a.D = dgu;
       a.gu = gu;
       a.F = c.F;
     }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (f32) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cntf, c.S, c.F, h->max_rows, st)); }
+    if (f32) {
+      Timed tm_(h, LD_KCLASS_ROWWISE, st);
+      if (c.act) LD_CHECK(launch_relu2<T>(gu, dh, dgu, cntf, c.S, c.F, h->max_rows, st));
+      else LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cntf, c.S, c.F, h->max_rows, st));
+    }
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cntf, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
-    a = rows_gemm(h, cntf, c.d, 2 * c.F, dgu, 2 * c.F, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
+    a = rows_gemm(h, cntf, c.d, h->nf, dgu, h->nf, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
     a.epi = EPI_STORE_F32;
     a.D = dzh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cntf, 2 * c.F, c.d, dgu, 2 * c.F, zh, c.d, G[l].w_gu), st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cntf, h->nf, c.d, dgu, h->nf, zh, c.d, G[l].w_gu), st)); }
     // dZ = dX^{l+1} + RMSNorm_2 backward; dz = r * dZ for the attention branch
     // (written by the same kernel when both blocks keep the same rows)
     {
@@ -585,6 +600,9 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   if (c.H < 1 || c.Hkv < 1 || c.H % c.Hkv || (c.H * c.Dh) % 64) return LD_ERR_SHAPE;
   if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH) return LD_ERR_ARG;
   if (c.sublayer != 0 && c.sublayer != 1) return LD_ERR_ARG;
+  if (c.alibi != 0 && c.alibi != 1) return LD_ERR_ARG;
+  if (c.alibi && c.rope_theta != 0.0f) return LD_ERR_ARG;  // one position scheme
+  if (c.act != LD_ACT_SWIGLU && c.act != LD_ACT_RELU2) return LD_ERR_ARG;
   if (c.b_offset < 0 || (long long)c.b_offset + c.B > 0x7fffffffll) return LD_ERR_ARG;
   if ((long long)c.B * c.S > (1ll << 30)) return LD_ERR_SHAPE;
   Handle* h = new (std::nothrow) Handle();
@@ -593,6 +611,7 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   h->esz = c.fp32_debug ? 4 : 2;
   h->max_rows = c.B * c.S;
   h->nqkv = (c.H + 2 * c.Hkv) * c.Dh;
+  h->nf = c.act == LD_ACT_RELU2 ? c.F : 2 * c.F;
   // number of blocks (and partial-sum rows of the gain gradient) of the
   // RMSNorm backward inside ld_backward: enough to keep ~8 blocks per SM of
   // a 152-SM GPU streaming (a launch constant; no CUDA call here)

@@ -3,7 +3,8 @@
 //
 // f_attn of Eq. (transformer_layer_dropout_train), per kept sequence s and
 // query head h (key/value head g = floor(h*Hkv/H)):
-//   o_i = sum_{j<=i} softmax_j(c q_i . k_j) v_j,   c = 1/sqrt(Dh)
+//   o_i = sum_{j<=i} softmax_j(c q_i . k_j [+ m_h (j - i)]) v_j,   c = 1/sqrt(Dh)
+// (the bracket with an ALiBi slope table, m_h per query head).
 // Rows are compact: kept sequence s occupies rows s*S .. s*S+S-1 of qkv
 // ([Q heads | K heads | V heads] columns).  The grid covers every batch slot
 // and blocks past the layer's kept count return at once, so the launch is
@@ -88,7 +89,8 @@ __device__ __forceinline__ void frag_b_kn(const bf16* base, int ld, int k0, int 
 template <int DH>
 __global__ void __launch_bounds__(128) attn_fwd_kernel(const bf16* __restrict__ qkv, int ldq, bf16* __restrict__ o,
                                                        int ldo, float* __restrict__ lse, int lse_ld,
-                                                       const int* __restrict__ cnt, int S, int H, int Hkv) {
+                                                       const int* __restrict__ cnt, int S, int H, int Hkv,
+                                                       const float* __restrict__ alibi) {
   constexpr int LDS = DH + 8, NDT = DH / 8, NKC = DH / 16;
   extern __shared__ __align__(16) uint8_t smraw[];
   bf16* Qs = reinterpret_cast<bf16*>(smraw);
@@ -119,6 +121,7 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(const bf16* __restrict__ 
   for (int i = 0; i < NDT; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
   const float sl2 = rsqrtf((float)DH) * kLog2e;
+  const float slope2 = alibi ? alibi[h] * kLog2e : 0.f;  // ALiBi bias slope2 (key - query), base 2
   const int qr0 = qt * 64 + warp * 16 + (lane >> 2);  // this thread's rows: qr0, qr0 + 8
 
   for (int kt = 0; kt <= qt; ++kt) {
@@ -152,7 +155,7 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(const bf16* __restrict__ 
       for (int e = 0; e < 4; ++e) {
         const int key = kt * 64 + nt * 8 + 2 * (lane & 3) + (e & 1);
         const int qr = qr0 + (e >> 1) * 8;
-        float v = s[nt][e] * sl2;
+        float v = fmaf(s[nt][e], sl2, slope2 * (float)(key - qr));
         if (kt == qt && key > qr) v = -INFINITY;
         s[nt][e] = v;
         mx[e >> 1] = fmaxf(mx[e >> 1], v);
@@ -224,7 +227,7 @@ __global__ void __launch_bounds__(128) attn_bwd_kernel(const bf16* __restrict__ 
                                                        const float* __restrict__ lse, const float* __restrict__ Dvec,
                                                        int lse_ld, float* __restrict__ dq_acc,
                                                        bf16* __restrict__ dqkv, const int* __restrict__ cnt, int S,
-                                                       int H, int Hkv) {
+                                                       int H, int Hkv, const float* __restrict__ alibi) {
   constexpr int LDS = DH + 8, NDT = DH / 8, NKC = DH / 16, LDP = 64 + 8;
   extern __shared__ __align__(16) uint8_t smraw[];
   bf16* Ks = reinterpret_cast<bf16*>(smraw);
@@ -256,6 +259,7 @@ __global__ void __launch_bounds__(128) attn_bwd_kernel(const bf16* __restrict__ 
   const int kr0 = kt * 64 + warp * 16 + (lane >> 2);  // this thread's keys: kr0, kr0 + 8
 
   for (int h = g * grp; h < (g + 1) * grp; ++h) {
+    const float slope2 = alibi ? alibi[h] * kLog2e : 0.f;
     for (int qt = kt; qt < nqt; ++qt) {
       const long long qrow = row0 + qt * 64;
       load_tile<DH>(Qs, qkv + qrow * ldq + (long long)h * DH, ldq, tid);
@@ -296,7 +300,8 @@ __global__ void __launch_bounds__(128) attn_bwd_kernel(const bf16* __restrict__ 
         for (int e = 0; e < 4; ++e) {
           const int ql = nt * 8 + 2 * (lane & 3) + (e & 1);
           const int key = kr0 + (e >> 1) * 8;
-          const float p = (qt * 64 + ql >= key) ? exp2f(st[nt][e] * sl2 - lse_s[ql]) : 0.f;
+          const float x = fmaf(st[nt][e], sl2, slope2 * (float)(key - qt * 64 - ql));
+          const float p = (qt * 64 + ql >= key) ? exp2f(x - lse_s[ql]) : 0.f;
           st[nt][e] = p;
           dp[nt][e] = p * (dp[nt][e] - D_s[ql]);
         }
@@ -417,7 +422,7 @@ __global__ void dq_finish_kernel(const float* __restrict__ dq_acc, bf16* __restr
 
 template <int DH>
 cudaError_t fwd_launch(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
-                       int max_seqs, cudaStream_t st) {
+                       int max_seqs, const float* alibi, cudaStream_t st) {
   constexpr size_t smem = (size_t)5 * 64 * (DH + 8) * sizeof(bf16);
   static bool attr = false;
   if (!attr) {
@@ -426,14 +431,14 @@ cudaError_t fwd_launch(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, c
     attr = true;
   }
   dim3 grid(S / 64, H, max_seqs);
-  attn_fwd_kernel<DH><<<grid, 128, smem, st>>>(qkv, ldq, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv);
+  attn_fwd_kernel<DH><<<grid, 128, smem, st>>>(qkv, ldq, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi);
   return cudaGetLastError();
 }
 
 template <int DH>
 cudaError_t bwd_launch(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                        float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs,
-                       cudaStream_t st) {
+                       const float* alibi, cudaStream_t st) {
   constexpr size_t smem = (size_t)4 * 64 * (DH + 8) * sizeof(bf16) + 64 * 72 * sizeof(bf16) + 128 * sizeof(float);
   static bool attr = false;
   if (!attr) {
@@ -443,28 +448,28 @@ cudaError_t bwd_launch(const bf16* qkv, int ldq, const bf16* dO, int ldo, const 
   }
   dim3 grid(S / 64, Hkv, max_seqs);
   attn_bwd_kernel<DH><<<grid, 128, smem, st>>>(qkv, ldq, dO, ldo, lse, Dvec, max_seqs * S, dq_acc, dqkv, cnt, S, H,
-                                               Hkv);
+                                               Hkv, alibi);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_attn_fwd_mma(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
-                                int Hkv, int Dh, int max_seqs, cudaStream_t st) {
-  if (Dh == 32) return fwd_launch<32>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, st);
-  if (Dh == 64) return fwd_launch<64>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, st);
-  return fwd_launch<128>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, st);
+                                int Hkv, int Dh, int max_seqs, const float* alibi, cudaStream_t st) {
+  if (Dh == 32) return fwd_launch<32>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, st);
+  if (Dh == 64) return fwd_launch<64>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, st);
+  return fwd_launch<128>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, st);
 }
 
 cudaError_t launch_attn_bwd_mma(const bf16* qkv, int ldqkv, const bf16* o, const bf16* dO, int ldo, const float* lse,
                                 const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                                int Dh, int max_seqs, cudaStream_t st) {
+                                int Dh, int max_seqs, const float* alibi, cudaStream_t st) {
   (void)o;
   cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)max_seqs * S * H * Dh * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  if (Dh == 32) return bwd_launch<32>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, st);
-  if (Dh == 64) return bwd_launch<64>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, st);
-  return bwd_launch<128>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, st);
+  if (Dh == 32) return bwd_launch<32>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, alibi, st);
+  if (Dh == 64) return bwd_launch<64>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, alibi, st);
+  return bwd_launch<128>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, alibi, st);
 }
 
 cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const float* rcos,

@@ -2,8 +2,9 @@
 // attention of the float32 debug path.  One warp per (row, head).
 //
 // f_attn of Eq. (transformer_layer_dropout_train) for one kept sequence:
-//   o_i = sum_{j<=i} softmax_j(c q_i . k_j) v_j,  c = 1/sqrt(Dh),
-// query head h reads key/value head floor(h*Hkv/H).  Rows are compact: the
+//   o_i = sum_{j<=i} softmax_j(c q_i . k_j [+ m_h (j - i)]) v_j,  c = 1/sqrt(Dh),
+// (the bracket with an ALiBi slope table), query head h reads key/value head
+// floor(h*Hkv/H).  Rows are compact: the
 // kept sequence s occupies rows s*S .. s*S+S-1 of qkv, whose columns are
 // [Q heads | K heads | V heads].  lse[h][m] = log sum_j exp(c q_m . k_j).
 #include "ld_internal.cuh"
@@ -27,7 +28,7 @@ template <typename T>
 __global__ void __launch_bounds__(128) attn_fwd_simt_kernel(const T* __restrict__ qkv, int ldq, T* __restrict__ o,
                                                             int ldo, float* __restrict__ lse, int lse_ld,
                                                             const int* __restrict__ cnt, int S, int H, int Hkv,
-                                                            int Dh) {
+                                                            int Dh, const float* __restrict__ alibi) {
   __shared__ float qs[kWarps][128];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long M = (long long)(*cnt) * S;
@@ -50,7 +51,7 @@ __global__ void __launch_bounds__(128) attn_fwd_simt_kernel(const T* __restrict_
         const T* kr = qkv + (seq0 + j) * ldq + (long long)(H + g) * Dh;
         float t = 0.f;
         for (int i = 0; i < Dh; ++i) t += qs[w][i] * to_f(kr[i]);
-        s = t;
+        s = alibi ? t + alibi[h] * (float)(j - pos) : t;
       }
       const float nmx = fmaxf(mx, wmax(s));
       const float p = (j <= pos) ? expf(s - nmx) : 0.f;
@@ -78,7 +79,7 @@ __global__ void __launch_bounds__(128) attn_dq_simt_kernel(const T* __restrict__
                                                            const float* __restrict__ lse,
                                                            const float* __restrict__ Dvec, int lse_ld,
                                                            T* __restrict__ dqkv, const int* __restrict__ cnt, int S,
-                                                           int H, int Hkv, int Dh) {
+                                                           int H, int Hkv, int Dh, const float* __restrict__ alibi) {
   __shared__ float qs[kWarps][128];
   __shared__ float ds_[kWarps][128];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -110,6 +111,7 @@ __global__ void __launch_bounds__(128) attn_dq_simt_kernel(const T* __restrict__
           s += qs[w][i] * to_f(kr[i]);
           dp += ds_[w][i] * to_f(vr[i]);
         }
+        if (alibi) s += alibi[h] * (float)(j - pos);
         const float p = expf(s - L_);
         dsv = p * (dp - D_);
       }
@@ -132,7 +134,8 @@ __global__ void __launch_bounds__(128) attn_dkv_simt_kernel(const T* __restrict_
                                                             const float* __restrict__ lse,
                                                             const float* __restrict__ Dvec, int lse_ld,
                                                             T* __restrict__ dqkv, const int* __restrict__ cnt,
-                                                            int S, int H, int Hkv, int Dh) {
+                                                            int S, int H, int Hkv, int Dh,
+                                                            const float* __restrict__ alibi) {
   __shared__ float ks[kWarps][128];
   __shared__ float vs[kWarps][128];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -165,6 +168,7 @@ __global__ void __launch_bounds__(128) attn_dkv_simt_kernel(const T* __restrict_
             s += ks[w][e] * to_f(qr[e]);
             dp += vs[w][e] * to_f(dr[e]);
           }
+          if (alibi) s += alibi[h] * (float)(pos - i);
           p = expf(s - lse[(size_t)h * lse_ld + mq]);
           dsv = p * (dp - Dvec[(size_t)h * lse_ld + mq]);
         }
@@ -200,32 +204,33 @@ static int attn_grid(long long items) {
 
 template <typename T>
 cudaError_t launch_attn_fwd_simt(const T* qkv, int ldqkv, T* o, int ldo, float* lse, const int* cnt, int S, int H,
-                                 int Hkv, int Dh, int max_rows, cudaStream_t st) {
+                                 int Hkv, int Dh, int max_rows, const float* alibi, cudaStream_t st) {
   attn_fwd_simt_kernel<T><<<attn_grid((long long)max_rows * H), 128, 0, st>>>(qkv, ldqkv, o, ldo, lse, max_rows,
-                                                                               cnt, S, H, Hkv, Dh);
+                                                                               cnt, S, H, Hkv, Dh, alibi);
   return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t launch_attn_bwd_simt(const T* qkv, int ldqkv, const T* dO, int ldo, const float* lse, const float* Dvec,
                                  T* dqkv, const int* cnt, int S, int H, int Hkv, int Dh, int max_rows,
-                                 cudaStream_t st) {
+                                 const float* alibi, cudaStream_t st) {
   attn_dq_simt_kernel<T><<<attn_grid((long long)max_rows * H), 128, 0, st>>>(qkv, ldqkv, dO, ldo, lse, Dvec, max_rows,
-                                                                             dqkv, cnt, S, H, Hkv, Dh);
+                                                                             dqkv, cnt, S, H, Hkv, Dh, alibi);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   attn_dkv_simt_kernel<T><<<attn_grid((long long)max_rows * Hkv), 128, 0, st>>>(
-      qkv, ldqkv, dO, ldo, lse, Dvec, max_rows, dqkv, cnt, S, H, Hkv, Dh);
+      qkv, ldqkv, dO, ldo, lse, Dvec, max_rows, dqkv, cnt, S, H, Hkv, Dh, alibi);
   return cudaGetLastError();
 }
 
 template cudaError_t launch_attn_fwd_simt<float>(const float*, int, float*, int, float*, const int*, int, int, int,
-                                                 int, int, cudaStream_t);
+                                                 int, int, const float*, cudaStream_t);
 template cudaError_t launch_attn_fwd_simt<bf16>(const bf16*, int, bf16*, int, float*, const int*, int, int, int, int,
-                                                int, cudaStream_t);
+                                                int, const float*, cudaStream_t);
 template cudaError_t launch_attn_bwd_simt<float>(const float*, int, const float*, int, const float*, const float*,
-                                                 float*, const int*, int, int, int, int, int, cudaStream_t);
+                                                 float*, const int*, int, int, int, int, int, const float*,
+                                                 cudaStream_t);
 template cudaError_t launch_attn_bwd_simt<bf16>(const bf16*, int, const bf16*, int, const float*, const float*, bf16*,
-                                                const int*, int, int, int, int, int, cudaStream_t);
+                                                const int*, int, int, int, int, int, const float*, cudaStream_t);
 
 }  // namespace ldk

@@ -20,6 +20,10 @@
 // The running max is only moved (and O rescaled in TMEM) when it grows by
 // more than 2^8, so most tiles need no O round trip; P <= 2^8 stays well
 // inside bf16/fp32 range.  All waits are bounded (status word on expiry).
+// With ALiBi (the paper's architecture, Methodology section) head h adds
+// m_h (j - i) to the scaled score of query i and key j: the scores are first
+// turned into biased base-2 logits x = S c log2e + m_h log2e (j - i), and the
+// max and P = exp2(x - m) work on x.
 #include <type_traits>
 
 #include "tc_common.cuh"
@@ -51,10 +55,11 @@ __device__ __forceinline__ uint32_t swz(int r, int i) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + (((i & 7) ^ (r & 7)) << 4));
 }
 
-template <int DH>
+template <int DH, bool ALIBI>
 __global__ void __launch_bounds__(320, 1)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
-                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv, int* status) {
+                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv,
+                       const float* __restrict__ alibi, int* status) {
   constexpr int NSLAB = DH / 64;
   constexpr uint32_t TILE = NSLAB * SLAB;  // one 128 x DH bf16 tile
   constexpr int NS = 2;                    // K/V stages
@@ -207,7 +212,11 @@ __global__ void __launch_bounds__(320, 1)
     const int r = quad * 32 + lane;  // query row of this thread within the tile
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
     uint64_t* xb = &xbar[quad];      // exchange barrier of the two warps of this quadrant (2 arrivals a phase)
+    // logits are x = S * sl2 (+ ALiBi bias); after the ALiBi transform the
+    // scores held are already x, so the scale applied later is 1
     const float sl2 = kLog2e * rsqrtf((float)DH);
+    const float sl2e = ALIBI ? 1.f : sl2;
+    const float slope2 = ALIBI ? alibi[h] * kLog2e : 0.f;
     constexpr int OC = DH / 64;      // 32-column chunks of O per half
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
@@ -225,6 +234,20 @@ __global__ void __launch_bounds__(320, 1)
       // the query (diagonal tile only) are left out
       const bool diag = (j == qt);                       // the only tile with masked keys (block-uniform)
       const int lim = (diag ? r : 127) - half * 64;      // last visible local column
+      if constexpr (ALIBI) {
+        // x_e = S_e sl2 + slope2 (key_e - query) for the 64 keys of this half
+        const float b0 = slope2 * (float)(j * 128 + half * 64 - (qt * 128 + r));
+        const uint64_t sl2x2 = f2_pack(sl2, sl2), sx2 = f2_pack(slope2, slope2), b0x2 = f2_pack(b0, b0);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e >> 4][(2 * e) & 31]), __uint_as_float(sr[e >> 4][(2 * e + 1) & 31])),
+                           sl2x2, f2_fma(f2_pack((float)(2 * e), (float)(2 * e + 1)), sx2, b0x2)),
+                    x0, x1);
+          sr[e >> 4][(2 * e) & 31] = __float_as_uint(x0);
+          sr[e >> 4][(2 * e + 1) & 31] = __float_as_uint(x1);
+        }
+      }
       float mraw = -INFINITY;
       if (diag) {
 #pragma unroll
@@ -239,7 +262,7 @@ __global__ void __launch_bounds__(320, 1)
       if (lane == 0) mbar_arrive(xb);
       if (!warp_wait(xb, j & 1, abort_flag, status)) { ok = false; break; }
       mraw = fmaxf(mraw, xmax[j & 1][half ^ 1][r]);
-      const float mt = mraw * sl2;
+      const float mt = mraw * sl2e;
       const bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
       // P = exp2(S c log2e - m) on pairs of keys (packed fp32 pipe); the
@@ -248,7 +271,7 @@ __global__ void __launch_bounds__(320, 1)
       uint64_t ls2 = f2_pack(0.f, 0.f);
       auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
-        const uint64_t sl2x2 = f2_pack(sl2, sl2), nm2 = f2_pack(-m_new, -m_new);
+        const uint64_t sl2x2 = f2_pack(sl2e, sl2e), nm2 = f2_pack(-m_new, -m_new);
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
           float x0, x1;
@@ -336,21 +359,21 @@ __global__ void __launch_bounds__(320, 1)
   }
 }
 
-template <int DH>
+template <int DH, bool ALIBI>
 cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
-                   int max_seqs, int* status, cudaStream_t st) {
+                   int max_seqs, const float* alibi, int* status, cudaStream_t st) {
   constexpr size_t smem = (size_t)(DH / 64) * SLAB * 5 + 2 * SLAB + 6 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
-        cudaFuncSetAttribute(attn_fwd_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(attn_fwd_tc_kernel<DH, ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   dim3 grid(H, max_seqs, S / 128);
-  attn_fwd_tc_kernel<DH><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, status);
+  attn_fwd_tc_kernel<DH, ALIBI><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi, status);
   return cudaGetLastError();
 }
 
@@ -376,13 +399,14 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
+template <bool ALIBI>
 __global__ void __launch_bounds__(448, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
                        const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
-                       int* status) {
+                       const float* __restrict__ alibi, int* status) {
   constexpr int DH = 128;
   constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
   constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
@@ -539,6 +563,8 @@ __global__ void __launch_bounds__(448, 1)
     for (int i = 0; i < n_it; ++i) {
       const int b = i % NST;
       const int qt = q0 + i % (nq - q0);
+      // ALiBi: logit bias slope2 (key - query) of this step's query head
+      const float slope2 = ALIBI ? alibi[g * grp + i / (nq - q0)] * kLog2e : 0.f;
       if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
       if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
@@ -558,10 +584,20 @@ __global__ void __launch_bounds__(448, 1)
       auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
         const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
+        // bias of query c: slope2 (key - qt*64 - half*32 - c) = b0 - slope2 c
+        const float b0 = slope2 * (float)(-qbase);
+        const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
         for (int e4 = 0; e4 < 8; ++e4) {
           const float4 lq = lv4[e4], dq = dv4[e4];
-          const uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
+          uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
+          if constexpr (ALIBI) {
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+              const float c0 = (float)(4 * e4 + 2 * h2);
+              nl[h2] = f2_add(nl[h2], f2_fma(f2_pack(c0, c0 + 1.f), nsx2, b0x2));
+            }
+          }
           const uint64_t dd[2] = {f2_pack(dq.x, dq.y), f2_pack(dq.z, dq.w)};
 #pragma unroll
           for (int h2 = 0; h2 < 2; ++h2) {
@@ -677,15 +713,17 @@ __global__ void __launch_bounds__(448, 1)
   }
 }
 
+template <bool ALIBI>
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
-                   const float* rsin, int* status, cudaStream_t st) {
+                   const float* rsin, const float* alibi, int* status, cudaStream_t st) {
   // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
   // vectors + dQ staging + alignment + barriers = 232,192 bytes (of 232,448)
   constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 128 * 4 + 64 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(attn_bwd_tc_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
@@ -696,8 +734,8 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
   dim3 grid(Hkv, max_seqs, S / 128);
-  attn_bwd_tc_kernel<<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H, Hkv,
-                                              rcos, rsin, status);
+  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
+                                                     H, Hkv, rcos, rsin, alibi, status);
   return cudaGetLastError();
 }
 }  // namespace
@@ -708,16 +746,25 @@ bool attn_bwd_tc_supported(int S, int Dh) { return S % 128 == 0 && Dh == 128; }
 
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, const float* rcos, const float* rsin, int* status, cudaStream_t st) {
+                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, int* status,
+                               cudaStream_t st) {
   cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)max_seqs * S * H * 128 * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  return bwd_tc(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, status, st);
+  if (alibi)
+    return bwd_tc<true>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                        status, st);
+  return bwd_tc<false>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                       status, st);
 }
 
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
-                               int Hkv, int Dh, int max_seqs, int* status, cudaStream_t st) {
-  if (Dh == 64) return fwd_tc<64>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, status, st);
-  return fwd_tc<128>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, status, st);
+                               int Hkv, int Dh, int max_seqs, const float* alibi, int* status, cudaStream_t st) {
+  if (alibi) {
+    if (Dh == 64) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
+    return fwd_tc<128, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
+  }
+  if (Dh == 64) return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
+  return fwd_tc<128, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
 }
 
 }  // namespace ldk

@@ -81,10 +81,13 @@ using namespace tc;
 
 // --------------------------------------------------------------- epilogue
 __device__ __forceinline__ void swiglu_bwd_chunk(const GemmArgs& a, int row, int j, const float (&dh)[32]);
+__device__ __forceinline__ void relu2_chunk(const GemmArgs& a, int row, int j, const float (&v)[32]);
 
 __device__ __forceinline__ void store_chunk(const GemmArgs& a, int row, int col, const float (&v)[32]) {
   if (a.epi == EPI_SWIGLU_BWD) {
     swiglu_bwd_chunk(a, row, col, v);
+  } else if (a.epi == EPI_RELU2 || a.epi == EPI_RELU2_BWD) {
+    relu2_chunk(a, row, col, v);
   } else if (a.epi == EPI_STORE_F32) {
     float4* p = reinterpret_cast<float4*>(static_cast<float*>(a.D) + (size_t)row * a.ldd + col);
 #pragma unroll
@@ -161,6 +164,30 @@ __device__ __forceinline__ void swiglu_bwd_chunk(const GemmArgs& a, int row, int
   bf16* dp = static_cast<bf16*>(a.D) + (size_t)row * 2 * a.F + j;
   st_bf16x32(dp, dg);
   st_bf16x32(dp + a.F, du);
+}
+
+// Squared ReLU on a 32-column chunk: forward (u -> save u, h = max(u,0)^2)
+// or backward (dh -> du = dh * 2 max(u, 0) with the saved u).
+__device__ __forceinline__ void relu2_chunk(const GemmArgs& a, int row, int j, const float (&v)[32]) {
+  const size_t off = (size_t)row * a.ldd + j;
+  float w[32];
+  if (a.epi == EPI_RELU2) {
+    float u[32];
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+      u[e] = v[e];
+      const float r = fmaxf(v[e], 0.f);
+      w[e] = r * r;
+    }
+    st_bf16x32(static_cast<bf16*>(a.D) + off, u);
+    st_bf16x32(static_cast<bf16*>(a.h_out) + off, w);
+  } else {
+    float u[32];
+    ld_bf16x32(static_cast<const bf16*>(a.gu) + off, u);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) w[e] = v[e] * 2.f * fmaxf(u[e], 0.f);
+    st_bf16x32(static_cast<bf16*>(a.D) + off, w);
+  }
 }
 
 // Tile order: groups of 8 N-blocks; inside a group consecutive tiles walk

@@ -63,6 +63,9 @@ cudaError_t launch_convert(const void* src, int src_f32, void* dst, int dst_f32,
 
 cudaError_t launch_rope_table(float* cos_t, float* sin_t, int S, int Dh, double theta, cudaStream_t st);
 
+// ALiBi slopes m_h of H heads (natural units) into slopes[H].
+cudaError_t launch_alibi_table(float* slopes, int H, cudaStream_t st);
+
 // RMSNorm forward over the rows of layer l (M = *cnt * S rows).  When
 // `gather` is set the source row of compact row m is src_row(kept_idx, S, m)
 // of the float32 residual stream, else row m of a compact buffer.  Writes
@@ -101,36 +104,45 @@ template <typename T>
 cudaError_t launch_swiglu_bwd(const T* dh, const T* gu, T* dgu, const int* cnt, int S, int F, int max_rows,
                               cudaStream_t st);
 
+// Squared ReLU over [M, F] rows: out = max(u, 0)^2 if dh is null, else
+// out = dh * 2 max(u, 0).
+template <typename T>
+cudaError_t launch_relu2(const T* u, const T* dh, T* out, const int* cnt, int S, int F, int max_rows,
+                         cudaStream_t st);
+
 template <typename T>
 cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, const int* cnt, int S, int max_rows,
                                float* Dvec, cudaStream_t st);
 
+// Every attention launcher takes `alibi`: null, or the device table of the
+// H ALiBi slopes (scores of head h get + m_h (j - i)).
 // Reference (SIMT) attention, used by the float32 debug path.
 template <typename T>
 cudaError_t launch_attn_fwd_simt(const T* qkv, int ldqkv, T* o, int ldo, float* lse, const int* cnt, int S, int H,
-                                 int Hkv, int Dh, int max_rows, cudaStream_t st);
+                                 int Hkv, int Dh, int max_rows, const float* alibi, cudaStream_t st);
 template <typename T>
 cudaError_t launch_attn_bwd_simt(const T* qkv, int ldqkv, const T* dO, int ldo, const float* lse, const float* Dvec,
                                  T* dqkv, const int* cnt, int S, int H, int Hkv, int Dh, int max_rows,
-                                 cudaStream_t st);
+                                 const float* alibi, cudaStream_t st);
 
 // Tensor-core (mma.sync) flash attention for bf16.
 cudaError_t launch_attn_fwd_mma(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S,
-                                int H, int Hkv, int Dh, int max_seqs, cudaStream_t st);
+                                int H, int Hkv, int Dh, int max_seqs, const float* alibi, cudaStream_t st);
 cudaError_t launch_attn_bwd_mma(const bf16* qkv, int ldqkv, const bf16* o, const bf16* dO, int ldo,
                                 const float* lse, const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt,
-                                int S, int H, int Hkv, int Dh, int max_seqs, cudaStream_t st);
+                                int S, int H, int Hkv, int Dh, int max_seqs, const float* alibi, cudaStream_t st);
 // tcgen05 flash attention forward (head size 64 or 128, S % 128 == 0).
 bool attn_tc_supported(int S, int Dh);
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
-                               int Hkv, int Dh, int max_seqs, int* status, cudaStream_t st);
+                               int Hkv, int Dh, int max_seqs, const float* alibi, int* status, cudaStream_t st);
 // tcgen05 flash attention backward (head size 128, S % 128 == 0); zeroes
 // dq_acc and accumulates dQ (unscaled) into it.
 bool attn_bwd_tc_supported(int S, int Dh);
 // dK leaves with the inverse RoPE applied (rcos = null: no rotation).
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, const float* rcos, const float* rsin, int* status, cudaStream_t st);
+                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, int* status,
+                               cudaStream_t st);
 // dqkv[:, q heads] = inverse-RoPE(dq_acc / sqrt(Dh)) as bf16 (rcos = null: no rotation)
 cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const float* rcos,
                              const float* rsin, const int* cnt, int S, int max_rows, cudaStream_t st);
@@ -146,7 +158,18 @@ cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, 
 //                 g, u to D (row stride 2F, columns j and F+j) and
 //                 h = silu(g) u to h_out (row stride F)
 // EPI_SWIGLU_BWD  acc = dh; with g, u from `gu` writes dg, du to D (stride 2F)
-enum EpiMode { EPI_STORE = 0, EPI_STORE_F32 = 1, EPI_RESID = 2, EPI_ROPE = 3, EPI_SWIGLU = 4, EPI_SWIGLU_BWD = 5 };
+// EPI_RELU2: D = u (bf16 save), h_out = max(u, 0)^2 (both [M, N], row stride ldd);
+// EPI_RELU2_BWD: D = dh * 2 max(u, 0) with u read from `gu` ([M, N], stride ldd).
+enum EpiMode {
+  EPI_STORE = 0,
+  EPI_STORE_F32 = 1,
+  EPI_RESID = 2,
+  EPI_ROPE = 3,
+  EPI_SWIGLU = 4,
+  EPI_SWIGLU_BWD = 5,
+  EPI_RELU2 = 6,
+  EPI_RELU2_BWD = 7
+};
 
 struct GemmArgs {
   // problem size; a non-null *_cnt makes the extent device-side: (*cnt) * mul

@@ -479,6 +479,58 @@ cudaError_t launch_swiglu_bwd(const T* dh, const T* gu, T* dgu, const int* cnt, 
   return cudaGetLastError();
 }
 
+// ------------------------------------------------------------ ALiBi slopes
+// Press et al., "Train Short, Test Long" (ICLR 2022): with n0 the largest
+// power of two <= H, head h < n0 has slope 2^(-8 (h + 1) / n0); head
+// n0 + k has 2^(-4 (2k + 1) / n0), every other slope of the 2 n0 sequence.
+__global__ void alibi_table_kernel(float* __restrict__ slopes, int H) {
+  int n0 = 1;
+  while (n0 * 2 <= H) n0 *= 2;
+  for (int h = threadIdx.x; h < H; h += blockDim.x) {
+    const double e = h < n0 ? -8.0 * (h + 1) / n0 : -4.0 * (2 * (h - n0) + 1) / n0;
+    slopes[h] = (float)exp2(e);
+  }
+}
+
+cudaError_t launch_alibi_table(float* slopes, int H, cudaStream_t st) {
+  alibi_table_kernel<<<1, 256, 0, st>>>(slopes, H);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------ squared ReLU
+// h = max(u, 0)^2 (forward); du = dh * 2 max(u, 0) (backward); [M, F] rows.
+template <typename T>
+__global__ void relu2_kernel(const T* __restrict__ u, const T* __restrict__ dh, T* __restrict__ out,
+                             const int* __restrict__ cnt, int S, int F) {
+  const long long total = (long long)(*cnt) * S * (F / 8);
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
+       w += (long long)gridDim.x * blockDim.x) {
+    float uv[8], o[8];
+    ld8(u + w * 8, uv);
+    if (dh) {
+      float dv[8];
+      ld8(dh + w * 8, dv);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) o[k] = dv[k] * 2.f * fmaxf(uv[k], 0.f);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float r = fmaxf(uv[k], 0.f);
+        o[k] = r * r;
+      }
+    }
+    st8(out + w * 8, o);
+  }
+}
+
+template <typename T>
+cudaError_t launch_relu2(const T* u, const T* dh, T* out, const int* cnt, int S, int F, int max_rows,
+                         cudaStream_t st) {
+  const int grid = grid_for((long long)max_rows * (F / 8), 256, device_sm_count() * 8);
+  relu2_kernel<T><<<grid, 256, 0, st>>>(u, dh, out, cnt, S, F);
+  return cudaGetLastError();
+}
+
 // ------------------------------------------- attention backward preprocess
 // Dvec[h][m] = sum_i dO[m, h*Dh+i] * O[m, h*Dh+i]  (row sum of dP * P).
 template <typename T>
@@ -517,6 +569,7 @@ cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, c
                                             int, cudaStream_t);                                                 \
   template cudaError_t launch_swiglu_fwd<T>(const T*, T*, const int*, int, int, int, cudaStream_t);             \
   template cudaError_t launch_swiglu_bwd<T>(const T*, const T*, T*, const int*, int, int, int, cudaStream_t);   \
+  template cudaError_t launch_relu2<T>(const T*, const T*, T*, const int*, int, int, int, cudaStream_t);        \
   template cudaError_t launch_attn_rowdot<T>(const T*, const T*, int, int, int, const int*, int, int, float*,   \
                                              cudaStream_t);
 LD_INST(bf16)
@@ -532,6 +585,7 @@ template cudaError_t launch_rope_apply<float>(float*, int, int, int, const float
 template cudaError_t launch_swiglu_fwd<float>(const float*, float*, const int*, int, int, int, cudaStream_t);
 template cudaError_t launch_swiglu_bwd<float>(const float*, const float*, float*, const int*, int, int, int,
                                               cudaStream_t);
+template cudaError_t launch_relu2<float>(const float*, const float*, float*, const int*, int, int, int, cudaStream_t);
 template cudaError_t launch_attn_rowdot<float>(const float*, const float*, int, int, int, const int*, int, int,
                                                float*, cudaStream_t);
 

@@ -28,6 +28,11 @@ CONFIGS = {
                  init="depth_scaled"),
     "llama8b": dict(L=32, d=4096, H=32, Hkv=8, Dh=128, F=14336, B=4, S=4096, eps=1e-6, rope_theta=5e5, alpha=1.0,
                     init="depth_scaled"),
+    # the paper's own architecture (Methodology section; model table): ALiBi
+    # position biases, squared-ReLU feed-forward of width 8 d, 3.9B shape;
+    # batch and sequence length chosen here (16384 tokens like the others)
+    "paper-3.9b": dict(L=40, d=2048, H=16, Hkv=16, Dh=128, F=16384, B=8, S=2048, eps=1e-6, rope_theta=0.0,
+                       alpha=1.0, alibi=True, act="relu2", init="depth_scaled"),
 }
 
 # Drop-rate schedules the workloads name (distribution x time schedule, seed).
@@ -36,10 +41,11 @@ SCHEDULES = {
     "gpt2": dict(dist="ild", p_max=0.2, time="const", seed=1),
     "1.3b": dict(dist="ild", p_max=0.3, time="ramp", ramp=(0, 1000, 0.0, 1.0), seed=1),
     "llama8b": dict(dist="ild", p_max=0.4, time="const", seed=1),
+    "paper-3.9b": dict(dist="ild", p_max=0.4, time="const", seed=1),
 }
 
 # Steps at which each workload is run (the 1.3B ramp is sampled at 0/500/2000).
-STEPS = {"tiny": [0], "gpt2": [0], "1.3b": [0, 500, 2000], "llama8b": [0]}
+STEPS = {"tiny": [0], "gpt2": [0], "1.3b": [0, 500, 2000], "llama8b": [0], "paper-3.9b": [0]}
 
 # Sweep on the 1.3B shape: p_max x distribution x granularity x seeds.
 SWEEP = dict(base="1.3b", p_max=[0.0, 0.1, 0.2, 0.3, 0.5], dist=["ild", "uniform"],
@@ -59,7 +65,7 @@ def weight_shapes(cfg):
     return {
         "w_qkv": ((H + 2 * Hkv) * Dh, d),
         "w_o": (d, H * Dh),
-        "w_gu": (2 * F, d),
+        "w_gu": ((F if cfg.get("act") == "relu2" else 2 * F), d),  # [gate; up] or up alone
         "w_d": (d, F),
         "g1": (d,),
         "g2": (d,),

@@ -60,6 +60,23 @@ def test_sublayer_flag():
         P.ld_destroy(h2)
 
 
+def test_position_and_activation_flags():
+    cfg = synth.CONFIGS["tiny"]
+    assert P.ld_create_status(P.make_config(dict(cfg, alibi=True))) == P.LD_ERR_ARG  # ALiBi and RoPE together
+    assert P.ld_create_status(P.make_config(dict(cfg, alibi=True, rope_theta=0.0, act="relu2"))) == P.LD_OK
+    bad = P.make_config(cfg)
+    bad.act = 2
+    assert P.ld_create_status(bad) == P.LD_ERR_ARG
+    # the squared-ReLU stack saves u instead of g || u: a smaller workspace
+    h1 = P.ld_create(P.make_config(cfg))
+    h2 = P.ld_create(P.make_config(dict(cfg, rope_theta=0.0, alibi=True, act="relu2")))
+    try:
+        assert P.ld_workspace_size(h2) < P.ld_workspace_size(h1)
+    finally:
+        P.ld_destroy(h1)
+        P.ld_destroy(h2)
+
+
 def test_schedule_validation_and_state():
     h = P.ld_create(P.make_config(synth.CONFIGS["tiny"]))
     try:

@@ -91,3 +91,9 @@ def test_1p3b_sweep_per_batch():
 def test_llama8b_full():
     mask, seqs = _run("llama8b", 0, R=32)
     assert mask[0].all() and not mask.all()
+
+
+def test_paper_arch_3p9b_full():
+    # the paper's architecture: ALiBi (16 heads) + squared-ReLU FFN, 40 layers
+    mask, seqs = _run("paper-3.9b", 0, R=32)
+    assert mask[0].all() and not mask.all()

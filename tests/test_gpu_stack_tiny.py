@@ -116,3 +116,29 @@ def test_sublayer_multi_tile(fp32):
     cfg = MULTI[1]
     sched = dict(dist="explicit", p_explicit=[0.5, 0.5], time="const", seed=21)
     _compare(cfg, sched, 0, fp32, gamma_noise=0.1, sublayer=True, granularity="per_sequence")
+
+
+PAPER = [
+    # ALiBi + squared ReLU; tiny shape (mma.sync attention, Dh 32)
+    dict(synth.CONFIGS["tiny"], H=4, Hkv=2, rope_theta=0.0, alibi=True, act="relu2"),
+    # 6 heads (slopes of a non-power-of-two head count), tcgen05 forward, mma.sync backward
+    dict(L=2, d=384, H=6, Hkv=3, Dh=64, F=1536, B=3, S=512, eps=1e-6, rope_theta=0.0, alpha=1.0, alibi=True,
+         act="relu2"),
+    # tcgen05 forward and backward
+    dict(L=2, d=512, H=4, Hkv=1, Dh=128, F=1024, B=2, S=1024, eps=1e-6, rope_theta=0.0, alpha=1.0, alibi=True,
+         act="relu2"),
+]
+
+
+@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
+@pytest.mark.parametrize("cfg", PAPER, ids=["tiny", "S512-dh64-h6", "S1024-dh128"])
+def test_paper_architecture(cfg, fp32):
+    sched = dict(dist="explicit", p_explicit=[0.3, 0.5][: cfg["L"]], time="const", seed=13)
+    _compare(cfg, sched, 1, fp32, gamma_noise=0.1)
+
+
+@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
+def test_paper_architecture_sublayer(fp32):
+    cfg = PAPER[2]
+    sched = dict(dist="explicit", p_explicit=[0.5, 0.5], time="const", seed=21)
+    _compare(cfg, sched, 0, fp32, gamma_noise=0.1, sublayer=True)

@@ -10,6 +10,7 @@ against things fixed independently of it:
     parity protocol relies on."""
 
 import itertools
+import os
 
 import numpy as np
 import pytest
@@ -43,14 +44,22 @@ def _inputs(cfg, seed=1):
     return x, dy
 
 
+PAPER_ARCH = dict(MICRO, alibi=True, rope_theta=0.0, act="relu2")  # ALiBi + squared ReLU (Methodology)
+
 CFGS = [
     MICRO,
     dict(MICRO, H=4, Hkv=4, rope_theta=0.0),   # MHA, no rotary embedding
     dict(MICRO, H=4, Hkv=1, Dh=16, d=48),      # one key/value head
+    PAPER_ARCH,                                # ALiBi + squared ReLU, 4 heads
+    dict(PAPER_ARCH, H=6, Hkv=3),              # ALiBi slopes for a head count that is not a power of two
 ]
 
 
-@pytest.mark.parametrize("cfg", CFGS, ids=["gqa-rope", "mha-norope", "mqa"])
+def _slopes(cfg):
+    return O.alibi_slopes(cfg["H"]) if cfg.get("alibi") else None
+
+
+@pytest.mark.parametrize("cfg", CFGS, ids=["gqa-rope", "mha-norope", "mqa", "alibi-relu2", "alibi6-relu2"])
 def test_forward_and_backward_match_torch_autograd(cfg):
     layers = _layers(cfg)
     x, dy = _inputs(cfg)
@@ -61,7 +70,7 @@ def test_forward_and_backward_match_torch_autograd(cfg):
 
     tl = to_torch_layers(layers, requires_grad=True)
     tx = torch.tensor(x, requires_grad=True)
-    tout = masked_stack(tx, tl, cfg, masks, scales)
+    tout = masked_stack(tx, tl, cfg, masks, scales, _slopes(cfg))
     np.testing.assert_allclose(out, tout.detach().numpy(), rtol=0, atol=1e-11)
     (tout * torch.tensor(dy)).sum().backward()
     np.testing.assert_allclose(dX, tx.grad.numpy(), rtol=0, atol=1e-10)
@@ -147,8 +156,38 @@ def test_p1_is_identity():
     assert all((g[n] == 0).all() for g in grads for n in O.WEIGHT_NAMES)
 
 
+def test_alibi_slopes():
+    # ALiBi paper (Press et al., ICLR 2022), Section 3: 8 heads use 2^-1 ..
+    # 2^-8; 16 heads the sequence that starts at 2^-0.5 with ratio 2^-0.5
+    # (tests/golden/alibi_slopes.txt).  Other head counts: the slopes of the
+    # largest power of two n0 <= H, then geometric means of neighbouring
+    # slopes of that sequence (1 taken as the slope before the first).
+    gold = {}
+    for line in open(os.path.join(os.path.dirname(__file__), "golden", "alibi_slopes.txt")):
+        if line.strip() and not line.startswith("#"):
+            h, *v = line.split()
+            gold[int(h)] = [float(x) for x in v]
+    for H, ref in gold.items():
+        np.testing.assert_array_equal(O.alibi_slopes(H), np.array(ref))
+    for H in (3, 5, 6, 9, 10, 12, 14, 21, 24, 40):
+        m = O.alibi_slopes(H)
+        n0 = 2 ** int(np.floor(np.log2(H)))
+        base = O.alibi_slopes(n0)
+        np.testing.assert_array_equal(m[:n0], base)
+        prev = np.concatenate([[1.0], base])
+        np.testing.assert_allclose(m[n0:], np.sqrt(prev[:-1] * prev[1:])[: H - n0], rtol=1e-15)
+        assert len(set(m)) == H and (m > 0).all() and (m < 1).all()
+
+
+def test_finite_differences_paper_arch():
+    _finite_differences(dict(PAPER_ARCH, H=6, Hkv=2))
+
+
 def test_finite_differences():
-    cfg = MICRO
+    _finite_differences(MICRO)
+
+
+def _finite_differences(cfg):
     layers = _layers(cfg, seed=5)
     x, dy = _inputs(cfg, seed=6)
     masks = np.array([[1, 1, 0], [0, 1, 1]], dtype=np.uint8)

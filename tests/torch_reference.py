@@ -24,12 +24,22 @@ def _rope_complex(t, theta):
     return torch.cat([c.real, c.imag], dim=-1)
 
 
-def dense_layer(x, W, cfg):
+def dense_layer(x, W, cfg, slopes=None):
     """f for one sequence x [S, d] at rate 0 and scale 1: returns (attn, ffn)
-    callables so that masks and scales can be composed outside."""
+    callables so that masks and scales can be composed outside.  With
+    cfg["alibi"] the per-head ``slopes`` enter SDPA as an additive float mask
+    m_h (j - i) next to -inf above the diagonal; cfg["act"] == "relu2" selects
+    the squared-ReLU feed-forward."""
     H, Hkv, Dh, Fh = cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"]
     eps, theta = cfg["eps"], cfg.get("rope_theta", 0.0)
     S = x.shape[0]
+    alibi = cfg.get("alibi", False)
+    if alibi:
+        theta = 0.0
+        pos = torch.arange(S, dtype=torch.float64)
+        rel = pos[None, :] - pos[:, None]
+        bias = torch.as_tensor(slopes, dtype=torch.float64)[:, None, None] * rel[None]
+        bias = bias.masked_fill(rel[None] > 0, float("-inf"))
 
     def f_attn(xx):
         xh = F.rms_norm(xx, (xx.shape[-1],), weight=W["g1"], eps=eps)
@@ -42,20 +52,25 @@ def dense_layer(x, W, cfg):
         rep = H // Hkv
         k = k.repeat_interleave(rep, dim=1)
         v = v.repeat_interleave(rep, dim=1)
-        o = F.scaled_dot_product_attention(
-            q.transpose(0, 1)[None], k.transpose(0, 1)[None], v.transpose(0, 1)[None], is_causal=True
-        )[0].transpose(0, 1).reshape(S, H * Dh)
+        qq, kk, vv = q.transpose(0, 1)[None], k.transpose(0, 1)[None], v.transpose(0, 1)[None]
+        if alibi:
+            o = F.scaled_dot_product_attention(qq, kk, vv, attn_mask=bias[None])
+        else:
+            o = F.scaled_dot_product_attention(qq, kk, vv, is_causal=True)
+        o = o[0].transpose(0, 1).reshape(S, H * Dh)
         return o @ W["w_o"].T
 
     def f_ffn(zz):
         zh = F.rms_norm(zz, (zz.shape[-1],), weight=W["g2"], eps=eps)
         gu = zh @ W["w_gu"].T
+        if cfg.get("act") == "relu2":
+            return F.relu(gu).square() @ W["w_d"].T
         return (F.silu(gu[:, :Fh]) * gu[:, Fh:]) @ W["w_d"].T
 
     return f_attn, f_ffn
 
 
-def masked_stack(x, layers, cfg, masks, scales):
+def masked_stack(x, layers, cfg, masks, scales, slopes=None):
     """Stack with per-sequence masks, composed from dense layers:
     z = x + s M_attn f_attn(x), x' = z + s M_ffn f_ffn(z), where masks is
     [L, B] (M_attn = M_ffn = masks, layer granularity) or [2, L, B]
@@ -66,7 +81,7 @@ def masked_stack(x, layers, cfg, masks, scales):
     for b in range(B):
         xb = x[b]
         for l in range(ma.shape[0]):
-            f_attn, f_ffn = dense_layer(xb, layers[l], cfg)
+            f_attn, f_ffn = dense_layer(xb, layers[l], cfg, slopes)
             s = float(scales[l])
             zb = xb + s * f_attn(xb) if ma[l, b] else xb
             xb = zb + s * f_ffn(zb) if mf[l, b] else zb
