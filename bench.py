@@ -263,6 +263,79 @@ def run_sweep(args):
     return 0
 
 
+def run_eval(args):
+    """Depth-elastic inference forward (ld_forward_eval) on the workload's
+    weights: full depth, early exit at L/2 and alternate-layer skipping, at
+    the workload's B x S and at batch-1 shapes with S = 128 and 512.  Each
+    setting is timed eagerly and as a CUDA graph replay (CUDA events, median
+    of --steps after --warmup); one JSON line per (shape, setting)."""
+    import torch
+
+    import paper_2609_05275_gb300 as P
+    from paper_2609_05275_gb300 import synth
+
+    base = dict(synth.CONFIGS[args.config])
+    if args.layers:
+        base["L"] = args.layers
+    L = base["L"]
+    layers = synth.stack_weights(base, seed=0, device="cuda")
+    wtab = P.weight_table(layers)
+    settings = [("full depth", [1] * L), ("early exit at L/2", [1] * (L // 2) + [0] * (L - L // 2)),
+                ("alternate layers", [1 - (l % 2) for l in range(L)])]
+    shapes = [(base["B"], base["S"]), (1, 512), (1, 128)]
+    for B, S in shapes:
+        cfg = dict(base, B=B, S=S)
+        f_tok, _ = flops_per_token(cfg)
+        st = P.LayerDropStack(cfg, dict(dist="uniform", p_max=0.0, seed=1))
+        st.workspace = torch.empty(P.ld_eval_workspace_size(st.h), dtype=torch.uint8, device="cuda")
+        x0 = synth.activations(cfg, seed=0, device="cuda")
+        x = torch.empty_like(x0)
+        full_ms = None
+        for name, ex in settings:
+            def step():
+                x.copy_(x0)
+                st.forward_eval(ex, wtab, x)
+
+            res = {}
+            for mode in ("eager", "graph"):
+                run = step
+                if mode == "graph":
+                    stream = torch.cuda.Stream()
+                    stream.wait_stream(torch.cuda.current_stream())
+                    g = torch.cuda.CUDAGraph()
+                    with torch.cuda.stream(stream):
+                        step()  # first call outside the capture (one-time set-up)
+                        with torch.cuda.graph(g, stream=stream):
+                            step()
+                    torch.cuda.current_stream().wait_stream(stream)
+                    run = g.replay
+                for _ in range(max(args.warmup, 3)):
+                    run()
+                torch.cuda.synchronize()
+                times = []
+                for _ in range(args.steps):
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record()
+                    run()
+                    e1.record()
+                    e1.synchronize()
+                    times.append(e0.elapsed_time(e1))
+                res[mode] = statistics.median(times)
+            st.sync()
+            ms = min(res.values())
+            if full_ms is None:
+                full_ms = ms
+            n_exec = sum(ex)
+            print(json.dumps({"eval": {
+                "workload": args.config, "B": B, "S": S, "setting": name, "layers_executed": n_exec, "L": L,
+                "ms_eager": res["eager"], "ms_graph": res["graph"], "tokens_per_s": B * S / (ms / 1e3),
+                "executed_tflops": f_tok * B * S * n_exec / (ms / 1e3) / 1e12,
+                "speedup_vs_full_depth": full_ms / ms, "ideal_speedup": L / max(n_exec, 1),
+                "r_eval": 1.0, "dtype": "bf16", "data": "synthetic"}}), flush=True)
+        st.close()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -279,11 +352,16 @@ def main():
     ap.add_argument("--sweep", action="store_true",
                     help="drop-rate / distribution / granularity / seed sweep on the 1.3B shape (one JSON line "
                          "per cell, then a summary line)")
+    ap.add_argument("--eval", action="store_true",
+                    help="depth-elastic inference forward (full depth, early exit, layer skipping) at the "
+                         "workload shape and batch-1 shapes; one JSON line per setting")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
     if args.sweep:
         return run_sweep(args)
+    if args.eval:
+        return run_eval(args)
 
     import torch
     import torch.distributed as dist

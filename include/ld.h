@@ -173,6 +173,25 @@ ld_status ld_draw_masks(void* handle, long long step, void* workspace, void* str
 ld_status ld_forward(void* handle, long long step, const ld_layer_w* W, void* x, void* workspace,
                      void* stream);
 
+/* Depth-elastic inference forward, Eq. (transformer_layer_dropout_eval):
+ *   Z = X + r_eval[l] f_attn(X),  X' = Z + r_eval[l] f_ffn(Z)
+ * for every sequence on each layer with execute[l] = 1; layers with
+ * execute[l] = 0 are skipped (identity).  Early exit at l' (Inference
+ * Optimizations section: run layers 0 .. l'-1) is execute = 1 for l < l',
+ * intermediate layer skipping any other pattern.  execute: host [L] of 0/1;
+ * r_eval: host [L] or NULL for the paper's r_eval = 1.  x [B*S, d] in place.
+ * Needs no schedule and keeps no activations for a backward: `workspace`
+ * may be as small as ld_eval_workspace_size (one layer's activations),
+ * and a following ld_backward returns LD_ERR_STATE.  The weights of skipped
+ * layers are never read (their pointers may be NULL).  LD_ERR_ARG for a
+ * null argument, an execute entry other than 0/1, a non-finite r_eval or a
+ * missing weight of an executed layer. */
+ld_status ld_forward_eval(void* handle, const unsigned char* execute, const float* r_eval, const ld_layer_w* W,
+                          void* x, void* workspace, void* stream);
+
+/* Bytes of device workspace ld_forward_eval needs (256-byte aligned). */
+ld_status ld_eval_workspace_size(void* handle, size_t* bytes);
+
 /* Backward of the last ld_forward on this handle and workspace (same W).
  * dx [B*S, d] holds dY on entry and dX on return (in place); rows of a
  * sequence dropped at layer l pass through that layer unchanged.  G points

@@ -332,6 +332,25 @@ def stack_forward(x, layers, cfg, masks, scales):
     return X, caches
 
 
+def stack_forward_eval(x, layers, cfg, execute, r_eval=None):
+    """Depth-elastic inference, Eq. (transformer_layer_dropout_eval): every
+    sequence runs Z = X + r_eval f_attn(X), X' = Z + r_eval f_ffn(Z) on each
+    layer l with execute[l] = 1 and skips the others (early exit at l' runs
+    layers 0 .. l'-1; intermediate skipping any other pattern, Inference
+    Optimizations section).  r_eval defaults to 1, the paper's choice."""
+    X = np.array(x, dtype=np.float64, copy=True)
+    B, S, _ = X.shape
+    rope_cs = _rope_cs(cfg, S)
+    for l in range(len(execute)):
+        if not execute[l]:
+            continue
+        W = _layer(layers, l)
+        r = 1.0 if r_eval is None else float(r_eval[l])
+        for b in range(B):
+            X[b], _ = layer_forward(X[b], W, cfg, r, rope_cs)
+    return X
+
+
 def stack_backward(dy, layers, cfg, masks, scales, caches):
     """d X^L -> (d X^0, per-layer weight gradients).
 

@@ -80,6 +80,9 @@ def lib():
             "ld_draw_masks": (c_int, [c_void_p, c_longlong, c_void_p, c_void_p]),
             "ld_forward": (c_int, [c_void_p, c_longlong, POINTER(ld_layer_w), c_void_p, c_void_p, c_void_p]),
             "ld_backward": (c_int, [c_void_p, POINTER(ld_layer_w), c_void_p, POINTER(ld_layer_g), c_void_p, c_void_p]),
+            "ld_forward_eval": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(ld_layer_w), c_void_p, c_void_p,
+                                        c_void_p]),
+            "ld_eval_workspace_size": (c_int, [c_void_p, POINTER(c_size_t)]),
             "ld_get_masks": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p]),
             "ld_sync": (c_int, [c_void_p]),
             "ld_destroy": (c_int, [c_void_p]),
@@ -199,6 +202,21 @@ def ld_backward(h, wtab, dx, gtab, workspace, stream=None):
     _check(lib().ld_backward(h, wtab, _ptr(dx), gtab, _ptr(workspace), _stream(stream)), "ld_backward")
 
 
+def ld_eval_workspace_size(h):
+    n = c_size_t()
+    _check(lib().ld_eval_workspace_size(h, ctypes.byref(n)), "ld_eval_workspace_size")
+    return n.value
+
+
+def ld_forward_eval(h, execute, r_eval, wtab, x, workspace, stream=None):
+    """execute: sequence of L 0/1 flags; r_eval: sequence of L floats or None."""
+    import numpy as np
+    ex = np.ascontiguousarray(np.asarray(execute, dtype=np.uint8))
+    rv = None if r_eval is None else np.ascontiguousarray(np.asarray(r_eval, dtype=np.float32))
+    _check(lib().ld_forward_eval(h, ex.ctypes.data, None if rv is None else rv.ctypes.data, wtab, _ptr(x),
+                                 _ptr(workspace), _stream(stream)), "ld_forward_eval")
+
+
 def ld_get_masks(h, L, B, sublayer=False):
     """(mask, kept_idx, kept_cnt) as [L, B], [L, B], [L]; with sub-layer
     granularity [2, L, B], [2, L, B], [2, L] (attention, then FFN)."""
@@ -264,9 +282,12 @@ def ld_rmsnorm_backward_noalloc(B, S, d, dyn, xs, rstd, gamma, kept_idx, kept_cn
 
 
 def weight_table(layers):
-    """ld_layer_w[L] from a list of dicts of device tensors."""
+    """ld_layer_w[L] from a list of dicts of device tensors (None: a layer
+    whose weights are never read, e.g. one skipped by ld_forward_eval)."""
     tab = (ld_layer_w * len(layers))()
     for i, W in enumerate(layers):
+        if W is None:
+            continue
         for n in _WNAMES:
             setattr(tab[i], n, W[n].data_ptr())
     tab._keep = layers
@@ -313,6 +334,10 @@ class LayerDropStack:
 
     def backward(self, wtab, dx, gtab, stream=None):
         ld_backward(self.h, wtab, dx, gtab, self.workspace, stream)
+
+    def forward_eval(self, execute, wtab, x, r_eval=None, stream=None):
+        """Inference forward on the executed layers (in place on x)."""
+        ld_forward_eval(self.h, execute, r_eval, wtab, x, self.workspace, stream)
 
     def sync(self):
         st = ld_sync(self.h)

@@ -49,6 +49,7 @@ struct Handle {
   bool fwd_valid = false;
   void* fwd_ws = nullptr;
   std::vector<float> fwd_scale;
+  size_t eval_xres = 0, eval_total = 0;  // evaluation layout: residual stream offset, total bytes
   // device-time accounting (ld_set_timing): event pairs around launches
   bool timing = false;
   std::vector<cudaEvent_t> ev[LD_KCLASS_COUNT];
@@ -161,6 +162,11 @@ void make_layout(Handle* h) {
   y.rstd2 = ltake(R * 4);
   y.per_layer = lo;
   y.layer0 = off;
+  // evaluation layout (ld_forward_eval): the same header, one block of
+  // activations reused by every layer, then the float32 residual stream
+  const size_t eo = align_up(off + lo);
+  h->eval_xres = c.fp32_debug ? 0 : eo;
+  h->eval_total = c.fp32_debug ? eo : align_up(eo + R * c.d * 4);
   off = align_up(off + (size_t)c.L * lo);
   // backward scratch (shared by all layers)
   y.dy = take(R * c.d * e);
@@ -332,44 +338,141 @@ cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const 
   return launch_dq_finish(dq_acc, d16, h->nqkv, c.H, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, st);
 }
 
+// One layer of the forward on the rows of its kept lists: the attention
+// block on (cnt, ki), the FFN block on (cntf, kif), branch scale s.  `lb` is
+// the layer's block of saved activations; x the float32 (or debug-path)
+// residual stream, updated in place.
+template <typename T>
+ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, float* x, const int* cnt, const int* ki,
+                        const int* cntf, const int* kif, float s, cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  const Layout& y = h->lay;
+  const bool f32 = sizeof(T) == 4;
+  const bool fused_rope = !f32 && c.rope_theta != 0.0f && c.Dh >= 64;
+  const bool same_rows = cnt == cntf;  // both blocks keep the same rows
+  const int HD = c.H * c.Dh;
+  float* rcos = at<float>(ws, y.rcos);
+  float* rsin = at<float>(ws, y.rsin);
+  float* xin = reinterpret_cast<float*>(lb + y.xin);
+  T* xh = reinterpret_cast<T*>(lb + y.xh);
+  T* qkv = reinterpret_cast<T*>(lb + y.qkv);
+  T* o = reinterpret_cast<T*>(lb + y.o);
+  float* lse = reinterpret_cast<float*>(lb + y.lse);
+  float* z = reinterpret_cast<float*>(lb + y.z);
+  T* zh = reinterpret_cast<T*>(lb + y.zh);
+  T* gu = reinterpret_cast<T*>(lb + y.gu);
+  T* hh = reinterpret_cast<T*>(lb + y.h);
+  float* rstd1 = reinterpret_cast<float*>(lb + y.rstd1);
+  float* rstd2 = reinterpret_cast<float*>(lb + y.rstd2);
+  const T* g1 = static_cast<const T*>(Wl.g1);
+  const T* g2 = static_cast<const T*>(Wl.g2);
+
+  { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, ki, cnt, c.S, c.d, h->max_rows, g1, c.eps, xin, xh, rstd1, st)); }
+  GemmArgs a = rows_gemm(h, cnt, h->nqkv, c.d, xh, c.d, Wl.w_qkv, c.d, 0);
+  a.epi = EPI_STORE;
+  a.D = qkv;
+  a.ldd = h->nqkv;
+  if (fused_rope) {  // RoPE on the q / k heads in the projection's epilogue
+    a.epi = EPI_ROPE;
+    a.rope_cos = rcos;
+    a.rope_sin = rsin;
+    a.Dh = c.Dh;
+    a.S = c.S;
+    a.rope_cols = (c.H + c.Hkv) * c.Dh;
+  }
+  { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+  if (c.rope_theta != 0.0f && !fused_rope)
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 0, st)); }
+  { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_fwd<T>(h, ws, qkv, o, lse, cnt, st)); }
+  a = rows_gemm(h, cnt, c.d, HD, o, HD, Wl.w_o, HD, 0);
+  a.epi = EPI_RESID;
+  a.alpha = s;
+  a.x = x;
+  a.ldx = c.d;
+  a.kept_idx = ki;
+  a.S = c.S;
+  a.save = same_rows ? z : nullptr;  // same rows feed the FFN block: keep a compact copy of Z
+  a.ld_save = c.d;
+  { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+  if (!same_rows) {  // the FFN block gathers its own rows of Z from the residual stream
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, kif, cntf, c.S, c.d, h->max_rows, g2, c.eps, z, zh, rstd2, st));
+  } else {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st));
+  }
+  a = rows_gemm(h, cntf, h->nf, c.d, zh, c.d, Wl.w_gu, c.d, 0);
+  a.epi = EPI_STORE;
+  a.D = gu;
+  a.ldd = h->nf;
+  if (!f32) {  // h = silu(g) u or max(u, 0)^2 in the projection's epilogue
+    a.epi = c.act ? EPI_RELU2 : EPI_SWIGLU;
+    a.h_out = hh;
+    a.F = c.F;
+  }
+  { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+  if (f32) {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    if (c.act) LD_CHECK(launch_relu2<T>(gu, (const T*)nullptr, hh, cntf, c.S, c.F, h->max_rows, st));
+    else LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cntf, c.S, c.F, h->max_rows, st));
+  }
+  a = rows_gemm(h, cntf, c.d, c.F, hh, c.F, Wl.w_d, c.F, 0);
+  a.epi = EPI_RESID;
+  a.alpha = s;
+  a.x = x;
+  a.ldx = c.d;
+  a.kept_idx = kif;
+  a.S = c.S;
+  a.save = nullptr;
+  { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+  return LD_OK;
+}
+
+// Work shared by the training and evaluation forwards before the layers:
+// clear the status word, widen x into the float32 residual stream (bf16
+// path), draw the masks (P) and build the RoPE / ALiBi tables.
+template <typename T>
+ld_status forward_prologue(Handle* h, const MaskParams& P, void* xv, float* x, void* ws, cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  const Layout& y = h->lay;
+  Timed tm_(h, LD_KCLASS_ROWWISE, st);
+  LD_CHECK(cudaMemsetAsync(at<int>(ws, y.status), 0, sizeof(int), st));
+  if (sizeof(T) == 2) LD_CHECK(launch_convert(xv, 0, x, 1, (long long)h->max_rows * c.d, st));
+  LD_CHECK(launch_mask_compact(P, at<unsigned char>(ws, y.mask), at<int>(ws, y.kidx), at<int>(ws, y.kcnt), st));
+  if (c.rope_theta != 0.0f)
+    LD_CHECK(launch_rope_table(at<float>(ws, y.rcos), at<float>(ws, y.rsin), c.S, c.Dh, (double)c.rope_theta, st));
+  if (c.alibi) LD_CHECK(launch_alibi_table(at<float>(ws, y.alibi), c.H, st));
+  return LD_OK;
+}
+
+MaskParams mask_params(const Handle* h, long long step) {
+  MaskParams P;  // 2 KB kernel parameter, filled on the host
+  P.seed = h->sched.seed;
+  P.step = step;
+  P.L = h->cfg.L;
+  P.B = h->cfg.B;
+  P.granularity = h->cfg.granularity;
+  P.b_offset = h->cfg.b_offset;
+  P.nmask = h->cfg.sublayer ? 2 : 1;
+  return P;
+}
+
 template <typename T>
 ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv, void* ws, cudaStream_t st) {
   const ld_config& c = h->cfg;
   const Layout& y = h->lay;
-  const bool fused_rope = sizeof(T) == 2 && c.rope_theta != 0.0f && c.Dh >= 64;
   // The residual stream is carried in float32 through the layers (bf16 in
   // and out at the boundary): 2*L in-place bf16 roundings of X would
   // otherwise accumulate to several per cent of |X| at 32 layers.
   const bool f32 = sizeof(T) == 4;
   float* x = f32 ? static_cast<float*>(xv) : at<float>(ws, y.xres);
-  int* status = at<int>(ws, y.status);
-  unsigned char* mask = at<unsigned char>(ws, y.mask);
   int* kidx = at<int>(ws, y.kidx);
   int* kcnt = at<int>(ws, y.kcnt);
-  float* rcos = at<float>(ws, y.rcos);
-  float* rsin = at<float>(ws, y.rsin);
-  (void)status;
-
-  MaskParams P;  // 2 KB kernel parameter, filled on the host
-  P.seed = h->sched.seed;
-  P.step = step;
-  P.L = c.L;
-  P.B = c.B;
-  P.granularity = c.granularity;
-  P.b_offset = c.b_offset;
-  P.nmask = c.sublayer ? 2 : 1;
+  MaskParams P = mask_params(h, step);
   std::vector<float> scale(c.L);
   step_rates(h, step, nullptr, P.thr, scale.data());
-  {
-    Timed tm_(h, LD_KCLASS_ROWWISE, st);
-    LD_CHECK(cudaMemsetAsync(status, 0, sizeof(int), st));
-    if (!f32) LD_CHECK(launch_convert(xv, 0, x, 1, (long long)h->max_rows * c.d, st));
-    LD_CHECK(launch_mask_compact(P, mask, kidx, kcnt, st));
-    if (c.rope_theta != 0.0f) LD_CHECK(launch_rope_table(rcos, rsin, c.S, c.Dh, (double)c.rope_theta, st));
-    if (c.alibi) LD_CHECK(launch_alibi_table(at<float>(ws, y.alibi), c.H, st));
-  }
-
-  const int HD = c.H * c.Dh;
+  ld_status r = forward_prologue<T>(h, P, xv, x, ws, st);
+  if (r != LD_OK) return r;
   for (int l = 0; l < c.L; ++l) {
     // kept lists of the attention block (cnt, ki) and of the FFN block
     // (cntf, kif); the same list unless the masks are drawn per sub-layer
@@ -377,86 +480,47 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
     const int* ki = kidx + (size_t)l * c.B;
     const int* cntf = c.sublayer ? kcnt + c.L + l : cnt;
     const int* kif = c.sublayer ? kidx + (size_t)(c.L + l) * c.B : ki;
-    char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
-    float* xin = reinterpret_cast<float*>(lb + y.xin);
-    T* xh = reinterpret_cast<T*>(lb + y.xh);
-    T* qkv = reinterpret_cast<T*>(lb + y.qkv);
-    T* o = reinterpret_cast<T*>(lb + y.o);
-    float* lse = reinterpret_cast<float*>(lb + y.lse);
-    float* z = reinterpret_cast<float*>(lb + y.z);
-    T* zh = reinterpret_cast<T*>(lb + y.zh);
-    T* gu = reinterpret_cast<T*>(lb + y.gu);
-    T* hh = reinterpret_cast<T*>(lb + y.h);
-    float* rstd1 = reinterpret_cast<float*>(lb + y.rstd1);
-    float* rstd2 = reinterpret_cast<float*>(lb + y.rstd2);
-    const T* g1 = static_cast<const T*>(W[l].g1);
-    const T* g2 = static_cast<const T*>(W[l].g2);
-    const float s = scale[l];
-
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, ki, cnt, c.S, c.d, h->max_rows, g1, c.eps, xin, xh, rstd1, st)); }
-    GemmArgs a = rows_gemm(h, cnt, h->nqkv, c.d, xh, c.d, W[l].w_qkv, c.d, 0);
-    a.epi = EPI_STORE;
-    a.D = qkv;
-    a.ldd = h->nqkv;
-    if (fused_rope) {  // RoPE on the q / k heads in the projection's epilogue
-      a.epi = EPI_ROPE;
-      a.rope_cos = rcos;
-      a.rope_sin = rsin;
-      a.Dh = c.Dh;
-      a.S = c.S;
-      a.rope_cols = (c.H + c.Hkv) * c.Dh;
-    }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (c.rope_theta != 0.0f && !fused_rope)
-      { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 0, st)); }
-    { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_fwd<T>(h, ws, qkv, o, lse, cnt, st)); }
-    a = rows_gemm(h, cnt, c.d, HD, o, HD, W[l].w_o, HD, 0);
-    a.epi = EPI_RESID;
-    a.alpha = s;
-    a.x = x;
-    a.ldx = c.d;
-    a.kept_idx = ki;
-    a.S = c.S;
-    a.save = c.sublayer ? nullptr : z;  // same rows feed the FFN block: keep a compact copy of Z
-    a.ld_save = c.d;
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (c.sublayer) {  // the FFN block gathers its own rows of Z from the residual stream
-      Timed tm_(h, LD_KCLASS_ROWWISE, st);
-      LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, kif, cntf, c.S, c.d, h->max_rows, g2, c.eps, z, zh, rstd2, st));
-    } else {
-      Timed tm_(h, LD_KCLASS_ROWWISE, st);
-      LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st));
-    }
-    a = rows_gemm(h, cntf, h->nf, c.d, zh, c.d, W[l].w_gu, c.d, 0);
-    a.epi = EPI_STORE;
-    a.D = gu;
-    a.ldd = h->nf;
-    if (!f32) {  // h = silu(g) u or max(u, 0)^2 in the projection's epilogue
-      a.epi = c.act ? EPI_RELU2 : EPI_SWIGLU;
-      a.h_out = hh;
-      a.F = c.F;
-    }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    if (f32) {
-      Timed tm_(h, LD_KCLASS_ROWWISE, st);
-      if (c.act) LD_CHECK(launch_relu2<T>(gu, (const T*)nullptr, hh, cntf, c.S, c.F, h->max_rows, st));
-      else LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cntf, c.S, c.F, h->max_rows, st));
-    }
-    a = rows_gemm(h, cntf, c.d, c.F, hh, c.F, W[l].w_d, c.F, 0);
-    a.epi = EPI_RESID;
-    a.alpha = s;
-    a.x = x;
-    a.ldx = c.d;
-    a.kept_idx = kif;
-    a.S = c.S;
-    a.save = nullptr;
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
+    r = forward_layer<T>(h, ws, at<char>(ws, y.layer0 + (size_t)l * y.per_layer), W[l], x, cnt, ki, cntf, kif,
+                         scale[l], st);
+    if (r != LD_OK) return r;
   }
   if (!f32) {
     Timed tm_(h, LD_KCLASS_ROWWISE, st);
     LD_CHECK(launch_convert(x, 1, xv, 0, (long long)h->max_rows * c.d, st));
   }
   h->fwd_scale = scale;
+  return LD_OK;
+}
+
+// Evaluation forward, Eq. (transformer_layer_dropout_eval): every sequence
+// runs every executed layer with the branch scale r_eval[l]; skipped layers
+// are not launched.  One block of activations (reused layer after layer)
+// and the float32 residual stream at the offsets of the evaluation layout.
+template <typename T>
+ld_status forward_eval_impl(Handle* h, const unsigned char* execute, const float* r_eval, const ld_layer_w* W,
+                            void* xv, void* ws, cudaStream_t st) {
+  const ld_config& c = h->cfg;
+  const Layout& y = h->lay;
+  const bool f32 = sizeof(T) == 4;
+  float* x = f32 ? static_cast<float*>(xv) : at<float>(ws, h->eval_xres);
+  int* kidx = at<int>(ws, y.kidx);
+  int* kcnt = at<int>(ws, y.kcnt);
+  MaskParams P = mask_params(h, 0);
+  P.nmask = 1;
+  for (int l = 0; l < c.L; ++l) P.thr[l] = 0;  // p = 0: every sequence kept, lists 0 .. B-1
+  ld_status r = forward_prologue<T>(h, P, xv, x, ws, st);
+  if (r != LD_OK) return r;
+  for (int l = 0; l < c.L; ++l) {
+    if (!execute[l]) continue;
+    const int* cnt = kcnt + l;
+    const int* ki = kidx + (size_t)l * c.B;
+    r = forward_layer<T>(h, ws, at<char>(ws, y.layer0), W[l], x, cnt, ki, cnt, ki, r_eval ? r_eval[l] : 1.0f, st);
+    if (r != LD_OK) return r;
+  }
+  if (!f32) {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(launch_convert(x, 1, xv, 0, (long long)h->max_rows * c.d, st));
+  }
   return LD_OK;
 }
 
@@ -699,6 +763,36 @@ ld_status ld_forward(void* handle, long long step, const ld_layer_w* W, void* x,
     h->fwd_valid = true;
     h->fwd_ws = ws;
   }
+  return r;
+}
+
+ld_status ld_eval_workspace_size(void* handle, size_t* bytes) {
+  if (!handle || !bytes) return LD_ERR_ARG;
+  *bytes = H(handle)->eval_total;
+  return LD_OK;
+}
+
+ld_status ld_forward_eval(void* handle, const unsigned char* execute, const float* r_eval, const ld_layer_w* W,
+                          void* x, void* ws, void* stream) {
+  if (!handle || !execute || !W || !x || !ws || !aligned16(x) || !aligned16(ws)) return LD_ERR_ARG;
+  Handle* h = H(handle);
+  for (int l = 0; l < h->cfg.L; ++l) {
+    if (execute[l] > 1) return LD_ERR_ARG;
+    if (r_eval && !finite(r_eval[l])) return LD_ERR_ARG;
+    if (!execute[l]) continue;  // the weights of skipped layers are never read
+    const void* ps[6] = {W[l].w_qkv, W[l].w_o, W[l].w_gu, W[l].w_d, W[l].g1, W[l].g2};
+    for (const void* p : ps)
+      if (!p || !aligned16(p)) return LD_ERR_ARG;
+  }
+  ld_status r = LD_OK;
+  if (!h->cfg.fp32_debug && (r = check_device()) != LD_OK) return r;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  r = h->cfg.fp32_debug ? forward_eval_impl<float>(h, execute, r_eval, W, x, ws, st)
+                        : forward_eval_impl<bf16>(h, execute, r_eval, W, x, ws, st);
+  h->last_ws = ws;
+  h->last_stream = st;
+  h->have_masks = false;  // the workspace holds no training masks now
+  h->fwd_valid = false;   // nor a forward a backward could follow
   return r;
 }
 

@@ -77,6 +77,27 @@ def test_position_and_activation_flags():
         P.ld_destroy(h2)
 
 
+def test_eval_entry_points():
+    cfg = synth.CONFIGS["llama8b"]
+    h = P.ld_create(P.make_config(cfg))
+    try:
+        # one layer's activations instead of L layers' plus the backward scratch
+        assert P.ld_eval_workspace_size(h) * 8 < P.ld_workspace_size(h)
+        L = P.lib()
+        W = (P.ld_layer_w * cfg["L"])()
+        ex = (ctypes.c_ubyte * cfg["L"])(*([1] + [0] * (cfg["L"] - 1)))
+        fake = ctypes.c_void_p(1 << 20)  # aligned, never dereferenced: argument checks fail first
+        assert L.ld_forward_eval(h, ex, None, W, fake, fake, None) == P.LD_ERR_ARG  # layer 0's weights missing
+        ex2 = (ctypes.c_ubyte * cfg["L"])(*([2] + [0] * (cfg["L"] - 1)))
+        assert L.ld_forward_eval(h, ex2, None, W, fake, fake, None) == P.LD_ERR_ARG  # not 0/1
+        assert L.ld_forward_eval(h, None, None, W, fake, fake, None) == P.LD_ERR_ARG
+        zero = (ctypes.c_ubyte * cfg["L"])()
+        rv = (ctypes.c_float * cfg["L"])(*([float("nan")] * cfg["L"]))
+        assert L.ld_forward_eval(h, zero, rv, W, fake, fake, None) == P.LD_ERR_ARG  # non-finite r_eval
+    finally:
+        P.ld_destroy(h)
+
+
 def test_schedule_validation_and_state():
     h = P.ld_create(P.make_config(synth.CONFIGS["tiny"]))
     try:

@@ -145,6 +145,27 @@ def test_sublayer_brute_force_and_layer_reduction():
         assert all((g1[l][n] == g2[l][n]).all() for l in range(2) for n in O.WEIGHT_NAMES)
 
 
+@pytest.mark.parametrize("cfg", [MICRO, PAPER_ARCH], ids=["rope-swiglu", "alibi-relu2"])
+def test_eval_forward_early_exit_and_skipping(cfg):
+    # Eq. (transformer_layer_dropout_eval) against the dense torch
+    # composition: early exit at l' = the first l' layers at scale r_eval;
+    # intermediate skipping = those layers with the others left out.
+    cfg = dict(cfg, L=4)
+    layers = _layers(cfg, seed=12)
+    x, _ = _inputs(cfg, seed=13)
+    tl = to_torch_layers(layers)
+    tx = torch.tensor(x)
+    B = cfg["B"]
+    for execute, r_eval in (([1, 1, 1, 1], None), ([1, 1, 0, 0], None), ([1, 0, 1, 0], [1.0, 9.0, 0.5, 9.0]),
+                            ([0, 1, 1, 1], [1.0, 0.7, 1.3, 2.0])):
+        out = O.stack_forward_eval(x, layers, cfg, execute, r_eval)
+        masks = np.repeat(np.array(execute, dtype=np.uint8)[:, None], B, axis=1)
+        scales = [1.0] * 4 if r_eval is None else r_eval
+        ref = masked_stack(tx, tl, cfg, masks, scales, _slopes(cfg)).numpy()
+        np.testing.assert_allclose(out, ref, rtol=0, atol=1e-11)
+    assert (O.stack_forward_eval(x, layers, cfg, [0, 0, 0, 0]) == x).all()
+
+
 def test_p1_is_identity():
     cfg = MICRO
     layers = _layers(cfg)
