@@ -9,14 +9,16 @@
 //
 // One CTA per (128-query tile, head, kept sequence); 320 threads:
 //   warp 0      TMA: the Q tile once, then K_j and V_j tiles (128 keys) into
-//               two two-stage rings (128-byte swizzled, 64-column slabs), K
-//               one tile ahead of V;
+//               a three-stage K ring and a two-stage V ring (128-byte
+//               swizzled, 64-column slabs), K one tile ahead of V;
 //   warp 1      TMEM allocation and the MMAs: S_j = Q K_j^T into one of two
-//               TMEM score buffers, then O += P_{j-1} V_{j-1} (O in TMEM);
+//               TMEM score buffers, then O += P_{j-1} V_{j-1} (O in TMEM,
+//               P read from TMEM as the A operand);
 //   warps 2..9  softmax, one query row and 64 keys per thread (two warps
 //               per row): S_j from TMEM, running max in base 2,
-//               P = exp2(S c log2e - m) written as bf16 into a swizzled
-//               shared-memory tile (the A operand of the PV MMA).
+//               P = exp2(S c log2e - m) written as bf16 into one of two TMEM
+//               P buffers, so step j is written while P_{j-1} V_{j-1} runs.
+// TMEM columns: S 0-255 (two buffers), O 256-(256+DH), P 384-511 (two).
 // The running max is only moved (and O rescaled in TMEM) when it grows by
 // more than 2^8, so most tiles need no O round trip; P <= 2^8 stays well
 // inside bf16/fp32 range.  All waits are bounded (status word on expiry).
@@ -37,10 +39,10 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescale = 8.0f;  // move the running max only when it grows by > 2^8
 
-__device__ __forceinline__ void st_bf16x32_(bf16* dst, const float* v) {
+__device__ __forceinline__ void st_bf16x16_(bf16* dst, const float* v) {
   uint4* p = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
+  for (int i = 0; i < 2; ++i) {
     uint4 q;
     __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&q);
 #pragma unroll
@@ -48,7 +50,6 @@ __device__ __forceinline__ void st_bf16x32_(bf16* dst, const float* v) {
     p[i] = q;
   }
 }
-
 // byte offset of element (row r, 16-byte chunk i) in a 128B-swizzled
 // K-major slab of 128-byte rows
 __device__ __forceinline__ uint32_t swz(int r, int i) {
@@ -62,26 +63,26 @@ __global__ void __launch_bounds__(320, 1)
                        const float* __restrict__ alibi, int* status) {
   constexpr int NSLAB = DH / 64;
   constexpr uint32_t TILE = NSLAB * SLAB;  // one 128 x DH bf16 tile
-  constexpr int NS = 2;                    // K/V stages
+  constexpr int NSK = 3, NSV = 2;          // K and V stages
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Qs = smem;
   uint8_t* Ks = Qs + TILE;
-  uint8_t* Vs = Ks + NS * TILE;
-  uint8_t* Ps = Vs + NS * TILE;  // 128 x 128 bf16, two slabs
-  float(*xmax)[2][128] = reinterpret_cast<float(*)[2][128]>(Ps + 2 * SLAB);  // [tile parity][half][row]
-  float(*xsum)[128] = reinterpret_cast<float(*)[128]>(Ps + 2 * SLAB + 2 * 2 * 128 * 4);  // [half][row]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(Ps + 2 * SLAB + 6 * 128 * 4);
+  uint8_t* Vs = Ks + NSK * TILE;
+  uint8_t* xch = Vs + NSV * TILE;
+  float(*xmax)[2][128] = reinterpret_cast<float(*)[2][128]>(xch);  // [tile parity][half][row]
+  float(*xsum)[128] = reinterpret_cast<float(*)[128]>(xch + 2 * 2 * 128 * 4);  // [half][row]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xch + 6 * 128 * 4);
   uint64_t* q_full = bars;
-  uint64_t* k_full = bars + 1;        // [NS] K ring: a stage frees once S_j has read it
-  uint64_t* k_empty = k_full + NS;
-  uint64_t* v_full = k_empty + NS;    // [NS] V ring: a stage frees once P_j V_j has read it
-  uint64_t* v_empty = v_full + NS;
-  uint64_t* s_full = v_empty + NS;
+  uint64_t* k_full = bars + 1;        // [NSK] K ring: a stage frees once S_j has read it
+  uint64_t* k_empty = k_full + NSK;
+  uint64_t* v_full = k_empty + NSK;   // [NSV] V ring: a stage frees once P_j V_j has read it
+  uint64_t* v_empty = v_full + NSV;
+  uint64_t* s_full = v_empty + NSV;
   uint64_t* s_free = s_full + 2;
-  uint64_t* p_full = s_free + 2;
-  uint64_t* pv_done = p_full + 1;
-  uint64_t* o_full = pv_done + 1;
+  uint64_t* p_full = s_free + 2;      // [2] per P buffer
+  uint64_t* pv_done = p_full + 2;     // [2] per P buffer
+  uint64_t* o_full = pv_done + 2;
   uint64_t* drain = o_full + 1;
   uint64_t* xbar = drain + 1;  // [4]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 4);
@@ -98,9 +99,11 @@ __global__ void __launch_bounds__(320, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < NS; ++s) {
+    for (int s = 0; s < NSK; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < NSV; ++s) {
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
     }
@@ -108,8 +111,10 @@ __global__ void __launch_bounds__(320, 1)
       mbar_init(&s_full[b], 1);
       mbar_init(&s_free[b], 8);
     }
-    mbar_init(p_full, 8);
-    mbar_init(pv_done, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&p_full[b], 8);
+      mbar_init(&pv_done[b], 1);
+    }
     mbar_init(o_full, 1);
     mbar_init(drain, 1);
     for (int q = 0; q < 4; ++q) mbar_init(&xbar[q], 2);
@@ -122,6 +127,7 @@ __global__ void __launch_bounds__(320, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t t_o = tmem + 256;  // O accumulator: columns 256 .. 256+DH
+  const uint32_t t_p = tmem + 384;  // [2] x 64 columns: P as bf16 pairs (A operand of P V)
 
   if (warp == 0) {
     if (lane == 0) {
@@ -133,16 +139,16 @@ __global__ void __launch_bounds__(320, 1)
       int nk = 0, nv = 0;
       for (int j = 0; j <= nkt; ++j) {
         if (j < nkt) {
-          const int s = j % NS;
-          if (!mbar_wait(&k_empty[s], ((j / NS) & 1) ^ 1u, abort_flag, status)) break;
+          const int s = j % NSK;
+          if (!mbar_wait(&k_empty[s], ((j / NSK) & 1) ^ 1u, abort_flag, status)) break;
           mbar_arrive_expect_tx(&k_full[s], TILE);
           for (int c = 0; c < NSLAB; ++c)
             tma_load_2d(Ks + s * TILE + c * SLAB, &tm, kcol + 64 * c, row0 + j * 128, &k_full[s]);
           ++nk;
         }
         if (j >= 1) {
-          const int jv = j - 1, s = jv % NS;
-          if (!mbar_wait(&v_empty[s], ((jv / NS) & 1) ^ 1u, abort_flag, status)) break;
+          const int jv = j - 1, s = jv % NSV;
+          if (!mbar_wait(&v_empty[s], ((jv / NSV) & 1) ^ 1u, abort_flag, status)) break;
           mbar_arrive_expect_tx(&v_full[s], TILE);
           for (int c = 0; c < NSLAB; ++c)
             tma_load_2d(Vs + s * TILE + c * SLAB, &tm, vcol + 64 * c, row0 + jv * 128, &v_full[s]);
@@ -151,8 +157,8 @@ __global__ void __launch_bounds__(320, 1)
       }
       if (*abort_flag) {
         mbar_drain(q_full, 0);
-        for (int j = nk > NS ? nk - NS : 0; j < nk; ++j) mbar_drain(&k_full[j % NS], (j / NS) & 1);
-        for (int j = nv > NS ? nv - NS : 0; j < nv; ++j) mbar_drain(&v_full[j % NS], (j / NS) & 1);
+        for (int j = nk > NSK ? nk - NSK : 0; j < nk; ++j) mbar_drain(&k_full[j % NSK], (j / NSK) & 1);
+        for (int j = nv > NSV ? nv - NSV : 0; j < nv; ++j) mbar_drain(&v_full[j % NSV], (j / NSV) & 1);
       }
     }
   } else if (warp == 1) {
@@ -160,37 +166,38 @@ __global__ void __launch_bounds__(320, 1)
       // ------------------------------------------------ MMA issuer
       constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
       constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
-      const uint32_t qa = smem_u32(Qs), ka = smem_u32(Ks), va = smem_u32(Vs), pa = smem_u32(Ps);
+      // descriptors built once, advanced by (byte offset >> 4) per MMA
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
+      const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
       bool ok = mbar_wait(q_full, 0, abort_flag, status);
       for (int j = 0; ok && j <= nkt; ++j) {
         if (j < nkt) {
-          const int s = j % NS;
-          if (!mbar_wait(&k_full[s], (j / NS) & 1, abort_flag, status)) { ok = false; break; }
+          const int s = j % NSK;
+          if (!mbar_wait(&k_full[s], (j / NSK) & 1, abort_flag, status)) { ok = false; break; }
           if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t kb = ka + s * TILE;
+          const uint64_t kb = DK + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
           for (int kk = 0; kk < DH / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * SLAB + (kk & 3) * 32;
-            mma_bf16(tmem + (j & 1) * 128, sdesc(qa + off, 16, 1024), sdesc(kb + off, 16, 1024), ID_S, kk > 0);
+            const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+            mma_bf16(tmem + (j & 1) * 128, DQ + off, kb + off, ID_S, kk > 0);
           }
           mma_commit(&s_full[j & 1]);
           mma_commit(&k_empty[s]);
         }
         if (j >= 1) {
-          const int jp = j - 1, s = jp % NS;
-          if (!mbar_wait(p_full, jp & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(&v_full[s], (jp / NS) & 1, abort_flag, status)) { ok = false; break; }
+          const int jp = j - 1, s = jp % NSV, pb = jp & 1;
+          if (!mbar_wait(&p_full[pb], (jp >> 1) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(&v_full[s], (jp / NSV) & 1, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t vb = va + s * TILE;
+          const uint64_t vb = DV + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            // A = P (K-major, 128 keys in two slabs); B = V as MN-major
+            // A = P from TMEM (16 keys = 8 columns a step); B = V as MN-major
             // (dh contiguous): 64-dh chunks one slab apart, 8-key groups 1 KB
-            mma_bf16(t_o, sdesc(pa + (kk >> 2) * SLAB + (kk & 3) * 32, 16, 1024),
-                     sdesc(vb + kk * 2048, SLAB, 1024), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
+            mma_bf16_ta(t_o, t_p + pb * 64 + kk * 8, vb + ((kk * 2048) >> 4), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
           }
-          mma_commit(pv_done);
+          mma_commit(&pv_done[pb]);
           mma_commit(&v_empty[s]);
         }
       }
@@ -292,12 +299,16 @@ __global__ void __launch_bounds__(320, 1)
       float ls_a, ls_b;
       f2_unpack(ls2, ls_a, ls_b);
       const float ls = ls_a + ls_b;
-      // P_{j-1} V_{j-1} must be done before P and O are touched
-      if (j >= 1 && !warp_wait(pv_done, (j - 1) & 1, abort_flag, status)) { ok = false; break; }
+      // P_{j-2} V_{j-2} must be done with P buffer j & 1 before it is
+      // rewritten; O is rescaled only once P_{j-1} V_{j-1} has accumulated
+      const int pb = j & 1;
+      if (j >= 2 && !warp_wait(&pv_done[pb], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+      const bool any_rescale = j >= 1 && __any_sync(0xffffffffu, rescale);
+      if (any_rescale && !warp_wait(&pv_done[pb ^ 1], ((j - 1) >> 1) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
       // tcgen05.ld/st are warp-wide: the warp rescales its half of O together
       // when any lane moved its max; lanes that did not multiply by 1
-      if (j >= 1 && __any_sync(0xffffffffu, rescale)) {
+      if (any_rescale) {
         const float corr = rescale ? exp2f(m_used - m_new) : 1.f;
 #pragma unroll 1
         for (int c = 0; c < OC; ++c) {
@@ -313,16 +324,12 @@ __global__ void __launch_bounds__(320, 1)
         m_used = m_new;
       }
       l += ls;
-      // this half's 64 keys of row r -> slab `half` of the swizzled K-major P tile
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        uint4 q = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-        *reinterpret_cast<uint4*>(Ps + half * SLAB + swz(r, i)) = q;
-      }
-      fence_proxy_async();
+      // this half's 64 keys of row r -> columns 32 half .. 32 half + 31 of P buffer pb
+      tmem_st32u(t_p + pb * 64 + half * 32 + lane_off, pk);
+      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(p_full);
+      if (lane == 0) mbar_arrive(&p_full[pb]);
     }
     if (ok && warp_wait(o_full, 0, abort_flag, status)) {
       tc_fence_after();
@@ -362,7 +369,8 @@ __global__ void __launch_bounds__(320, 1)
 template <int DH, bool ALIBI>
 cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
                    int max_seqs, const float* alibi, int* status, cudaStream_t st) {
-  constexpr size_t smem = (size_t)(DH / 64) * SLAB * 5 + 2 * SLAB + 6 * 128 * 4 + 1024 + 256;
+  // Q, 3 K and 2 V tiles + the row max / sum exchange + alignment + barriers
+  constexpr size_t smem = (size_t)(DH / 64) * SLAB * 6 + 6 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
@@ -381,28 +389,31 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // ---------------------------------------------------------------------------
 // Backward, head size 128.  One CTA per (128-key tile, kv head, kept
 // sequence), looping over the query heads of the group and the 64-query
-// tiles at or after the key tile.  448 threads:
-//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
+// tiles at or after the key tile.  704 threads:
+//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (4 stages)
 //   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
 //               (M = 128 keys, N = 64 queries); then for step i-1
 //               dV += P^T dO (P^T read from TMEM), dK += dS^T Q (M = 128
 //               keys, N = 128) and dQ^T = K^T dS^T (M = 128 head dims,
 //               N = 64 queries)
-//   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e)
+//   warps 2..17 one key and 16 queries per thread (four warps per TMEM lane
+//               quadrant): P^T = exp2(S^T c log2e - lse log2e)
 //               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
 //               swizzled shared-memory tile; at the end dK (times c) and dV
 //               from TMEM to dqkv
-//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
+//   warps 18..21  dQ^T from TMEM, reduced into the float32 dQ buffer
 // P^T and dS^T are double-buffered (step i uses buffer i & 1), so the
 // softmax warps write step i while the MMAs of step i-1 still read theirs.
 // TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447,
 // P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
+constexpr int NSM = 16;               // softmax warps of the backward (4 per TMEM lane quadrant)
+constexpr int BWD_THREADS = 32 * (2 + NSM + 4);
 
 template <bool ALIBI>
-__global__ void __launch_bounds__(448, 1)
+__global__ void __launch_bounds__(BWD_THREADS, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
-                       const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
+                       const __grid_constant__ CUtensorMap tmo,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
@@ -410,16 +421,21 @@ __global__ void __launch_bounds__(448, 1)
   constexpr int DH = 128;
   constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
   constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
-  constexpr int NST = 3;               // stages of the Q / dO / lse / D ring
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  constexpr int NST = 4;               // stages of the Q / dO / lse / D ring
+  // 1024-byte aligned by declaration (the 128-byte swizzle needs it); the
+  // check below makes a misplaced window an error instead of wrong tiles
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
+  if (smem_u32(smem_raw) & 1023) {
+    if (threadIdx.x == 0) set_status(status, LD_ERR_UNSUPPORTED);
+    return;
+  }
   uint8_t* Ks = smem;
   uint8_t* Vs = Ks + KT;
   uint8_t* Qs = Vs + KT;         // [NST][QT]
   uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
   uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
-  float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
-  float* vecs = dqs + 64 * DH;                         // [NST][lse 64 | D 64]
+  float* vecs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [NST][lse 64 | D 64]
   uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * 128);
   uint64_t* kv_full = bars;
   uint64_t* ld_full = bars + 1;          // [NST]
@@ -449,9 +465,9 @@ __global__ void __launch_bounds__(448, 1)
       mbar_init(&ld_empty[b], 1);
     }
     mbar_init(sdp_full, 1);
-    mbar_init(sdp_free, 8);
+    mbar_init(sdp_free, NSM);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&p_ready[b], 8);
+      mbar_init(&p_ready[b], NSM);
       mbar_init(&mm_done[b], 1);
     }
     mbar_init(dq_free, 4);
@@ -503,8 +519,15 @@ __global__ void __launch_bounds__(448, 1)
       constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
       constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
       constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
-      const uint32_t ka = smem_u32(Ks), va = smem_u32(Vs), qa = smem_u32(Qs), oa = smem_u32(dOs);
-      const uint32_t da0 = smem_u32(DSs);
+      // shared-memory descriptors built once; an MMA's operand is its base
+      // plus (byte offset >> 4) in the address field (every tile lies below
+      // 256 KB, so the 14-bit field never carries), which keeps the issuing
+      // thread -- it shares its SM sub-partition with four softmax warps and
+      // a dQ warp -- at a few instructions per MMA
+      const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
+      const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
+      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
       bool ok = mbar_wait(kv_full, 0, abort_flag, status);
       for (int i = 0; ok && i <= n_it; ++i) {
         if (i < n_it) {
@@ -512,12 +535,13 @@ __global__ void __launch_bounds__(448, 1)
           if (!mbar_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
           if (!mbar_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
+          const uint64_t st = (uint64_t)((b * QT) >> 4);
 #pragma unroll
           for (int kk = 0; kk < DH / 16; ++kk) {
-            const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
-            const uint32_t qoff = b * QT + (kk >> 2) * HSLAB + (kk & 3) * 32;
-            mma_bf16(t_s, sdesc(ka + koff, 16, 1024), sdesc(qa + qoff, 16, 1024), ID_SP, kk > 0);
-            mma_bf16(t_dp, sdesc(va + koff, 16, 1024), sdesc(oa + qoff, 16, 1024), ID_SP, kk > 0);
+            const uint32_t koff = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+            const uint32_t qoff = ((kk >> 2) * HSLAB + (kk & 3) * 32) >> 4;
+            mma_bf16(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
+            mma_bf16(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
           }
           mma_commit(sdp_full);
         }
@@ -526,17 +550,18 @@ __global__ void __launch_bounds__(448, 1)
           if (!mbar_wait(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
           if (!mbar_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t da = da0 + pb * SLAB;
+          const uint64_t st = (uint64_t)((b * QT) >> 4), ds = (uint64_t)((pb * SLAB) >> 4);
+          const uint32_t first = ip > 0 ? 1u : 0u;
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
-            const uint32_t aoff = kk * 32;                       // dS^T, K-major
-            const uint32_t boff = b * QT + kk * 2048;            // dO / Q as MN-major
-            mma_bf16_ta(t_dv, t_p + pb * 32 + kk * 8, sdesc(oa + boff, HSLAB, 1024), ID_KV, (ip > 0 || kk > 0));
-            mma_bf16(t_dk, sdesc(da + aoff, 16, 1024), sdesc(qa + boff, HSLAB, 1024), ID_KV, (ip > 0 || kk > 0));
+            const uint32_t aoff = (kk * 32) >> 4;                // dS^T, K-major
+            const uint32_t boff = (kk * 2048) >> 4;              // dO / Q as MN-major
+            mma_bf16_ta(t_dv, t_p + pb * 32 + kk * 8, DOMN + st + boff, ID_KV, kk > 0 ? 1u : first);
+            mma_bf16(t_dk, DS + ds + aoff, DQMN + st + boff, ID_KV, kk > 0 ? 1u : first);
           }
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
-            mma_bf16(t_dq, sdesc(ka + kk * 2048, SLAB, 1024), sdesc(da + kk * 2048, 16, 1024), ID_Q, kk > 0);
+            mma_bf16(t_dq, DKMN + ((kk * 2048) >> 4), DS + ds + ((kk * 2048) >> 4), ID_Q, kk > 0);
           }
           mma_commit(&mm_done[pb]);
           mma_commit(&ld_empty[b]);
@@ -549,12 +574,12 @@ __global__ void __launch_bounds__(448, 1)
         mbar_drain(drain, 0);
       }
     }
-  } else if (warp < 10) {
-    // ------------------------------------------------ P / dS (warps 2..9)
-    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..31 of the
-    // step, warps 6..9 queries 32..63, one key per thread
+  } else if (warp < 2 + NSM) {
+    // ------------------------------------------------ P / dS (warps 2..17)
+    // four warps per TMEM lane quadrant, one key and 16 of the step's 64
+    // queries per thread (quarter q of the warp: queries 16q .. 16q+15)
     const int quad = warp & 3;
-    const int half = (warp - 2) >> 2;
+    const int quarter = (warp - 2) >> 2;
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
@@ -568,27 +593,27 @@ __global__ void __launch_bounds__(448, 1)
       if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
       if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t sr[32], dr[32];
-      tmem_ld32_nw(t_s + half * 32 + lane_off, sr);
-      tmem_ld32_nw(t_dp + half * 32 + lane_off, dr);
+      uint32_t sr[16], dr[16];
+      tmem_ld16_nw(t_s + quarter * 16 + lane_off, sr);
+      tmem_ld16_nw(t_dp + quarter * 16 + lane_off, dr);
       tmem_wait_ld();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
-      const float4* lv4 = reinterpret_cast<const float4*>(vecs + b * 128 + half * 32);       // lse of the 32 queries
-      const float4* dv4 = reinterpret_cast<const float4*>(vecs + b * 128 + 64 + half * 32);  // D of the 32 queries
-      const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
-      uint32_t pk[16], dk[16];
+      const float4* lv4 = reinterpret_cast<const float4*>(vecs + b * 128 + quarter * 16);       // lse of the 16 queries
+      const float4* dv4 = reinterpret_cast<const float4*>(vecs + b * 128 + 64 + quarter * 16);  // D of the 16 queries
+      const int qbase = qt * 64 + quarter * 16 - key;  // query c is visible iff qbase + c >= 0
+      uint32_t pk[8], dk[8];
       // pairs of queries on the packed fp32 pipe; the causal mask only on
-      // warps whose 32 keys are not all visible to the 32 queries (warp-uniform)
+      // warps whose 32 keys are not all visible to the 16 queries (warp-uniform)
       auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
         const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
-        // bias of query c: slope2 (key - qt*64 - half*32 - c) = b0 - slope2 c
+        // bias of query c: slope2 (key - qt*64 - quarter*16 - c) = b0 - slope2 c
         const float b0 = slope2 * (float)(-qbase);
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
-        for (int e4 = 0; e4 < 8; ++e4) {
+        for (int e4 = 0; e4 < 4; ++e4) {
           const float4 lq = lv4[e4], dq = dv4[e4];
           uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
           if constexpr (ALIBI) {
@@ -623,11 +648,11 @@ __global__ void __launch_bounds__(448, 1)
       const int pb = i & 1;
       if (i >= 2 && !warp_wait(&mm_done[pb], ((i >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      tmem_st16(t_p + pb * 32 + half * 16 + lane_off, pk);
+      tmem_st8(t_p + pb * 32 + quarter * 8 + lane_off, pk);
       uint8_t* ds = DSs + pb * SLAB;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int chunk = half * 4 + c;
+      for (int c = 0; c < 2; ++c) {
+        const int chunk = quarter * 2 + c;
         *reinterpret_cast<uint4*>(ds + swz(r, chunk)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
       }
       fence_proxy_async();
@@ -638,47 +663,51 @@ __global__ void __launch_bounds__(448, 1)
     }
     if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
       tc_fence_after();
-      if (half == 0) {
-        // dK (times c) with the inverse rotation at the key's position
+      if (quarter < 2) {
+        // dK (times c) with the inverse rotation at the key's position:
+        // quarter 0 the pairs (i, i+64) for i < 32, quarter 1 for 32 <= i < 64
         const float c = rsqrtf((float)DH);
         bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
 #pragma unroll 1
-        for (int cc = 0; cc < 2; ++cc) {
-          float k1[32], k2[32];
-          tmem_ld32(t_dk + cc * 32 + lane_off, k1);
-          tmem_ld32(t_dk + 64 + cc * 32 + lane_off, k2);
+        for (int cc = quarter * 2; cc < quarter * 2 + 2; ++cc) {
+          float k1[16], k2[16];
+          tmem_ld16(t_dk + cc * 16 + lane_off, k1);
+          tmem_ld16(t_dk + 64 + cc * 16 + lane_off, k2);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
+          for (int e = 0; e < 16; ++e) {
             const float p1 = c * k1[e], p2 = c * k2[e];
             float cs = 1.f, sn = 0.f;
             if (rcos) {
-              cs = rcos[(size_t)key * 64 + cc * 32 + e];
-              sn = rsin[(size_t)key * 64 + cc * 32 + e];
+              cs = rcos[(size_t)key * 64 + cc * 16 + e];
+              sn = rsin[(size_t)key * 64 + cc * 16 + e];
             }
             k1[e] = p1 * cs + p2 * sn;
             k2[e] = p2 * cs - p1 * sn;
           }
-          st_bf16x32_(krow + cc * 32, k1);
-          st_bf16x32_(krow + 64 + cc * 32, k2);
+          st_bf16x16_(krow + cc * 16, k1);
+          st_bf16x16_(krow + 64 + cc * 16, k2);
         }
       } else {
+        // dV: quarter 2 columns 0..63, quarter 3 columns 64..127
         bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
 #pragma unroll 1
-        for (int cc = 0; cc < DH / 32; ++cc) {
-          float u[32];
-          tmem_ld32(t_dv + cc * 32 + lane_off, u);
-          st_bf16x32_(vrow + cc * 32, u);
+        for (int cc = (quarter - 2) * 4; cc < (quarter - 2) * 4 + 4; ++cc) {
+          float u[16];
+          tmem_ld16(t_dv + cc * 16 + lane_off, u);
+          st_bf16x16_(vrow + cc * 16, u);
         }
       }
     }
   } else {
-    // ------------------------------------------------ dQ (warps 10..13)
-    // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
-    // into dq_acc by one bulk tensor reduce per step.
+    // ------------------------------------------------ dQ (warps 18..21)
+    // dQ^T from TMEM, added into the float32 dq_acc by reductions from
+    // registers: thread dd holds head dimension dd of the step's 64 queries,
+    // so each warp instruction adds 32 consecutive floats (128 bytes) of one
+    // query row.
     const int quad = warp & 3;
     const int dd = quad * 32 + lane;  // head dimension of this thread
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const bool leader = (warp == 10 && lane == 0);
+    const size_t HD = (size_t)H * DH;
     for (int i = 0; i < n_it; ++i) {
       const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
       if (!warp_wait(&mm_done[i & 1], (i >> 1) & 1, abort_flag, status)) break;
@@ -689,20 +718,12 @@ __global__ void __launch_bounds__(448, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(dq_free);
-      if (leader && i > 0) bulk_wait_read();  // the previous reduce has read the tile
-      named_barrier(1, 128);
+      float* dst = dq_acc + (size_t)(row0 + qt * 64) * HD + (size_t)h * DH + dd;
 #pragma unroll
-      for (int e = 0; e < 32; ++e) dqs[e * DH + dd] = t0[e];
+      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)e * HD, t0[e]);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) dqs[(32 + e) * DH + dd] = t1[e];
-      fence_proxy_async();
-      named_barrier(1, 128);
-      if (leader) {
-        tma_reduce_add_2d(&tmdq, h * DH, row0 + qt * 64, dqs);
-        bulk_commit();
-      }
+      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(32 + e) * HD, t1[e]);
     }
-    if (leader) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -717,9 +738,10 @@ template <bool ALIBI>
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, const float* alibi, int* status, cudaStream_t st) {
-  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
-  // vectors + dQ staging + alignment + barriers = 232,192 bytes (of 232,448)
-  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 128 * 4 + 64 * 128 * 4 + 1024 + 256;
+  // K, V, 2 x dS^T (6 slabs) + 4 stages of Q, dO (16 half slabs) + lse/D
+  // vectors + barriers = 231,680 bytes (of 232,448); the window is
+  // 1024-byte aligned by declaration, no padding
+  constexpr size_t smem = 6 * SLAB + 16 * HSLAB + 4 * 128 * 4 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
@@ -727,14 +749,12 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  CUtensorMap tkv, tq, to, tdq;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows; dQ reduce boxes
-  if (!make_map_f32(&tdq, dq_acc, (uint64_t)H * 128, (uint64_t)max_seqs * S, (uint64_t)H * 128, 128, 64))
-    return cudaErrorInvalidValue;
+  CUtensorMap tkv, tq, to;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
   dim3 grid(Hkv, max_seqs, S / 128);
-  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
+  attn_bwd_tc_kernel<ALIBI><<<grid, BWD_THREADS, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
                                                      H, Hkv, rcos, rsin, alibi, status);
   return cudaGetLastError();
 }
