@@ -39,10 +39,10 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescale = 8.0f;  // move the running max only when it grows by > 2^8
 
-__device__ __forceinline__ void st_bf16x16_(bf16* dst, const float* v) {
+__device__ __forceinline__ void st_bf16x32_(bf16* dst, const float* v) {
   uint4* p = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-  for (int i = 0; i < 2; ++i) {
+  for (int i = 0; i < 4; ++i) {
     uint4 q;
     __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&q);
 #pragma unroll
@@ -389,31 +389,28 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // ---------------------------------------------------------------------------
 // Backward, head size 128.  One CTA per (128-key tile, kv head, kept
 // sequence), looping over the query heads of the group and the 64-query
-// tiles at or after the key tile.  704 threads:
-//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (4 stages)
+// tiles at or after the key tile.  448 threads:
+//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
 //   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
 //               (M = 128 keys, N = 64 queries); then for step i-1
 //               dV += P^T dO (P^T read from TMEM), dK += dS^T Q (M = 128
 //               keys, N = 128) and dQ^T = K^T dS^T (M = 128 head dims,
 //               N = 64 queries)
-//   warps 2..17 one key and 16 queries per thread (four warps per TMEM lane
-//               quadrant): P^T = exp2(S^T c log2e - lse log2e)
+//   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e)
 //               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
 //               swizzled shared-memory tile; at the end dK (times c) and dV
 //               from TMEM to dqkv
-//   warps 18..21  dQ^T from TMEM, reduced into the float32 dQ buffer
+//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
 // P^T and dS^T are double-buffered (step i uses buffer i & 1), so the
 // softmax warps write step i while the MMAs of step i-1 still read theirs.
 // TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447,
 // P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
-constexpr int NSM = 16;               // softmax warps of the backward (4 per TMEM lane quadrant)
-constexpr int BWD_THREADS = 32 * (2 + NSM + 4);
 
 template <bool ALIBI>
-__global__ void __launch_bounds__(BWD_THREADS, 1)
+__global__ void __launch_bounds__(448, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
-                       const __grid_constant__ CUtensorMap tmo,
+                       const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
@@ -421,21 +418,16 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
   constexpr int DH = 128;
   constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
   constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
-  constexpr int NST = 4;               // stages of the Q / dO / lse / D ring
-  // 1024-byte aligned by declaration (the 128-byte swizzle needs it); the
-  // check below makes a misplaced window an error instead of wrong tiles
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* smem = smem_raw;
-  if (smem_u32(smem_raw) & 1023) {
-    if (threadIdx.x == 0) set_status(status, LD_ERR_UNSUPPORTED);
-    return;
-  }
+  constexpr int NST = 3;               // stages of the Q / dO / lse / D ring
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Ks = smem;
   uint8_t* Vs = Ks + KT;
   uint8_t* Qs = Vs + KT;         // [NST][QT]
   uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
   uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
-  float* vecs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [NST][lse 64 | D 64]
+  float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
+  float* vecs = dqs + 64 * DH;                         // [NST][lse 64 | D 64]
   uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * 128);
   uint64_t* kv_full = bars;
   uint64_t* ld_full = bars + 1;          // [NST]
@@ -465,9 +457,9 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       mbar_init(&ld_empty[b], 1);
     }
     mbar_init(sdp_full, 1);
-    mbar_init(sdp_free, NSM);
+    mbar_init(sdp_free, 8);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&p_ready[b], NSM);
+      mbar_init(&p_ready[b], 8);
       mbar_init(&mm_done[b], 1);
     }
     mbar_init(dq_free, 4);
@@ -521,9 +513,7 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
       // shared-memory descriptors built once; an MMA's operand is its base
       // plus (byte offset >> 4) in the address field (every tile lies below
-      // 256 KB, so the 14-bit field never carries), which keeps the issuing
-      // thread -- it shares its SM sub-partition with four softmax warps and
-      // a dQ warp -- at a few instructions per MMA
+      // 256 KB, so the 14-bit field never carries)
       const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
       const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
       const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
@@ -574,12 +564,12 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
         mbar_drain(drain, 0);
       }
     }
-  } else if (warp < 2 + NSM) {
-    // ------------------------------------------------ P / dS (warps 2..17)
-    // four warps per TMEM lane quadrant, one key and 16 of the step's 64
-    // queries per thread (quarter q of the warp: queries 16q .. 16q+15)
+  } else if (warp < 10) {
+    // ------------------------------------------------ P / dS (warps 2..9)
+    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..31 of the
+    // step, warps 6..9 queries 32..63, one key per thread
     const int quad = warp & 3;
-    const int quarter = (warp - 2) >> 2;
+    const int half = (warp - 2) >> 2;
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
@@ -593,27 +583,27 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
       if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t sr[16], dr[16];
-      tmem_ld16_nw(t_s + quarter * 16 + lane_off, sr);
-      tmem_ld16_nw(t_dp + quarter * 16 + lane_off, dr);
+      uint32_t sr[32], dr[32];
+      tmem_ld32_nw(t_s + half * 32 + lane_off, sr);
+      tmem_ld32_nw(t_dp + half * 32 + lane_off, dr);
       tmem_wait_ld();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
-      const float4* lv4 = reinterpret_cast<const float4*>(vecs + b * 128 + quarter * 16);       // lse of the 16 queries
-      const float4* dv4 = reinterpret_cast<const float4*>(vecs + b * 128 + 64 + quarter * 16);  // D of the 16 queries
-      const int qbase = qt * 64 + quarter * 16 - key;  // query c is visible iff qbase + c >= 0
-      uint32_t pk[8], dk[8];
+      const float4* lv4 = reinterpret_cast<const float4*>(vecs + b * 128 + half * 32);       // lse of the 32 queries
+      const float4* dv4 = reinterpret_cast<const float4*>(vecs + b * 128 + 64 + half * 32);  // D of the 32 queries
+      const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
+      uint32_t pk[16], dk[16];
       // pairs of queries on the packed fp32 pipe; the causal mask only on
-      // warps whose 32 keys are not all visible to the 16 queries (warp-uniform)
+      // warps whose 32 keys are not all visible to the 32 queries (warp-uniform)
       auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
         const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
-        // bias of query c: slope2 (key - qt*64 - quarter*16 - c) = b0 - slope2 c
+        // bias of query c: slope2 (key - qt*64 - half*32 - c) = b0 - slope2 c
         const float b0 = slope2 * (float)(-qbase);
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
-        for (int e4 = 0; e4 < 4; ++e4) {
+        for (int e4 = 0; e4 < 8; ++e4) {
           const float4 lq = lv4[e4], dq = dv4[e4];
           uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
           if constexpr (ALIBI) {
@@ -648,11 +638,11 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       const int pb = i & 1;
       if (i >= 2 && !warp_wait(&mm_done[pb], ((i >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      tmem_st8(t_p + pb * 32 + quarter * 8 + lane_off, pk);
+      tmem_st16(t_p + pb * 32 + half * 16 + lane_off, pk);
       uint8_t* ds = DSs + pb * SLAB;
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        const int chunk = quarter * 2 + c;
+      for (int c = 0; c < 4; ++c) {
+        const int chunk = half * 4 + c;
         *reinterpret_cast<uint4*>(ds + swz(r, chunk)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
       }
       fence_proxy_async();
@@ -663,51 +653,47 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
     }
     if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
       tc_fence_after();
-      if (quarter < 2) {
-        // dK (times c) with the inverse rotation at the key's position:
-        // quarter 0 the pairs (i, i+64) for i < 32, quarter 1 for 32 <= i < 64
+      if (half == 0) {
+        // dK (times c) with the inverse rotation at the key's position
         const float c = rsqrtf((float)DH);
         bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
 #pragma unroll 1
-        for (int cc = quarter * 2; cc < quarter * 2 + 2; ++cc) {
-          float k1[16], k2[16];
-          tmem_ld16(t_dk + cc * 16 + lane_off, k1);
-          tmem_ld16(t_dk + 64 + cc * 16 + lane_off, k2);
+        for (int cc = 0; cc < 2; ++cc) {
+          float k1[32], k2[32];
+          tmem_ld32(t_dk + cc * 32 + lane_off, k1);
+          tmem_ld32(t_dk + 64 + cc * 32 + lane_off, k2);
 #pragma unroll
-          for (int e = 0; e < 16; ++e) {
+          for (int e = 0; e < 32; ++e) {
             const float p1 = c * k1[e], p2 = c * k2[e];
             float cs = 1.f, sn = 0.f;
             if (rcos) {
-              cs = rcos[(size_t)key * 64 + cc * 16 + e];
-              sn = rsin[(size_t)key * 64 + cc * 16 + e];
+              cs = rcos[(size_t)key * 64 + cc * 32 + e];
+              sn = rsin[(size_t)key * 64 + cc * 32 + e];
             }
             k1[e] = p1 * cs + p2 * sn;
             k2[e] = p2 * cs - p1 * sn;
           }
-          st_bf16x16_(krow + cc * 16, k1);
-          st_bf16x16_(krow + 64 + cc * 16, k2);
+          st_bf16x32_(krow + cc * 32, k1);
+          st_bf16x32_(krow + 64 + cc * 32, k2);
         }
       } else {
-        // dV: quarter 2 columns 0..63, quarter 3 columns 64..127
         bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
 #pragma unroll 1
-        for (int cc = (quarter - 2) * 4; cc < (quarter - 2) * 4 + 4; ++cc) {
-          float u[16];
-          tmem_ld16(t_dv + cc * 16 + lane_off, u);
-          st_bf16x16_(vrow + cc * 16, u);
+        for (int cc = 0; cc < DH / 32; ++cc) {
+          float u[32];
+          tmem_ld32(t_dv + cc * 32 + lane_off, u);
+          st_bf16x32_(vrow + cc * 32, u);
         }
       }
     }
   } else {
-    // ------------------------------------------------ dQ (warps 18..21)
-    // dQ^T from TMEM, added into the float32 dq_acc by reductions from
-    // registers: thread dd holds head dimension dd of the step's 64 queries,
-    // so each warp instruction adds 32 consecutive floats (128 bytes) of one
-    // query row.
+    // ------------------------------------------------ dQ (warps 10..13)
+    // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
+    // into dq_acc by one bulk tensor reduce per step.
     const int quad = warp & 3;
     const int dd = quad * 32 + lane;  // head dimension of this thread
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const size_t HD = (size_t)H * DH;
+    const bool leader = (warp == 10 && lane == 0);
     for (int i = 0; i < n_it; ++i) {
       const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
       if (!warp_wait(&mm_done[i & 1], (i >> 1) & 1, abort_flag, status)) break;
@@ -718,12 +704,20 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(dq_free);
-      float* dst = dq_acc + (size_t)(row0 + qt * 64) * HD + (size_t)h * DH + dd;
+      if (leader && i > 0) bulk_wait_read();  // the previous reduce has read the tile
+      named_barrier(1, 128);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)e * HD, t0[e]);
+      for (int e = 0; e < 32; ++e) dqs[e * DH + dd] = t0[e];
 #pragma unroll
-      for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(32 + e) * HD, t1[e]);
+      for (int e = 0; e < 32; ++e) dqs[(32 + e) * DH + dd] = t1[e];
+      fence_proxy_async();
+      named_barrier(1, 128);
+      if (leader) {
+        tma_reduce_add_2d(&tmdq, h * DH, row0 + qt * 64, dqs);
+        bulk_commit();
+      }
     }
+    if (leader) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -738,10 +732,9 @@ template <bool ALIBI>
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, const float* alibi, int* status, cudaStream_t st) {
-  // K, V, 2 x dS^T (6 slabs) + 4 stages of Q, dO (16 half slabs) + lse/D
-  // vectors + barriers = 231,680 bytes (of 232,448); the window is
-  // 1024-byte aligned by declaration, no padding
-  constexpr size_t smem = 6 * SLAB + 16 * HSLAB + 4 * 128 * 4 + 256;
+  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
+  // vectors + dQ staging + alignment + barriers = 232,192 bytes (of 232,448)
+  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 128 * 4 + 64 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
@@ -749,12 +742,14 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  CUtensorMap tkv, tq, to;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows
+  CUtensorMap tkv, tq, to, tdq;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows; dQ reduce boxes
+  if (!make_map_f32(&tdq, dq_acc, (uint64_t)H * 128, (uint64_t)max_seqs * S, (uint64_t)H * 128, 128, 64))
+    return cudaErrorInvalidValue;
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
   dim3 grid(Hkv, max_seqs, S / 128);
-  attn_bwd_tc_kernel<ALIBI><<<grid, BWD_THREADS, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
+  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
                                                      H, Hkv, rcos, rsin, alibi, status);
   return cudaGetLastError();
 }
