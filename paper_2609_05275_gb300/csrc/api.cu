@@ -677,10 +677,11 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   h->nqkv = (c.H + 2 * c.Hkv) * c.Dh;
   h->nf = c.act == LD_ACT_RELU2 ? c.F : 2 * c.F;
   // number of blocks (and partial-sum rows of the gain gradient) of the
-  // RMSNorm backward inside ld_backward: enough to keep ~8 blocks per SM of
-  // a 152-SM GPU streaming (a launch constant; no CUDA call here)
+  // RMSNorm backward inside ld_backward: the two blocks per SM of a 152-SM
+  // GPU that its register use lets stay resident, each looping over rows
+  // (a launch constant; no CUDA call here)
   h->part_blocks = (h->max_rows + 7) / 8;
-  if (h->part_blocks > 8 * 152) h->part_blocks = 8 * 152;
+  if (h->part_blocks > 2 * 152) h->part_blocks = 2 * 152;
   make_layout(h);
   *handle = h;
   return LD_OK;

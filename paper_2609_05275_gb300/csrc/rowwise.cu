@@ -289,16 +289,29 @@ cudaError_t launch_rmsnorm_bwd(const float* dyn, const float* xs, const float* r
   return cudaGetLastError();
 }
 
-__global__ void colsum_kernel(const float* __restrict__ part, int nrows, int d, float* __restrict__ out) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= d) return;
+// out[c] = sum over rows of part[row][c]: a block owns 32 columns, its 8
+// warps take every 8th row (one coalesced 128-byte read per warp and row),
+// and the 8 partial sums are combined in shared memory.
+__global__ void __launch_bounds__(256) colsum_kernel(const float* __restrict__ part, int nrows, int d,
+                                                     float* __restrict__ out) {
+  __shared__ float red[8][33];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int c = blockIdx.x * 32 + lane;
   float s = 0.f;
-  for (int b = 0; b < nrows; ++b) s += part[(size_t)b * d + i];
-  out[i] = s;
+  if (c < d)
+    for (int r = w; r < nrows; r += 8) s += part[(size_t)r * d + c];
+  red[w][lane] = s;
+  __syncthreads();
+  if (w == 0 && c < d) {
+    float t = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) t += red[k][lane];
+    out[c] = t;
+  }
 }
 
 cudaError_t launch_colsum(const float* part, int nrows, int d, float* out, cudaStream_t st) {
-  colsum_kernel<<<(d + 255) / 256, 256, 0, st>>>(part, nrows, d, out);
+  colsum_kernel<<<(d + 31) / 32, 256, 0, st>>>(part, nrows, d, out);
   return cudaGetLastError();
 }
 
