@@ -65,7 +65,13 @@ typedef enum {
 
 /* Tensor granularity (Tensor Granularity subsection): one Bernoulli draw per
  * sequence, or one per layer and step shared by the whole batch. */
-typedef enum { LD_PER_SEQUENCE = 0, LD_PER_BATCH = 1 } ld_granularity;
+/* Tensor granularity of the masks (Tensor Granularity subsection):
+ * per sequence, per batch (one draw per layer and step, shared by every
+ * sequence), or per shard: one draw per layer and step for this batch shard
+ * alone, keyed by its first global sequence b_offset, so that data-parallel
+ * ranks drop different layers while each skips whole layers (the paper's
+ * per-device batch dropping; on one device it is the per-batch case). */
+typedef enum { LD_PER_SEQUENCE = 0, LD_PER_BATCH = 1, LD_PER_SHARD = 2 } ld_granularity;
 
 /* Layer distributions (Dropout Distribution section):
  *   UNIFORM  p^l = p_max

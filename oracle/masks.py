@@ -14,6 +14,9 @@ Reading of the draw (the paper names no generator):
       b' = 0 per batch (so a per-batch mask is the per-sequence draw of
       sequence 0, broadcast);
   the layer is dropped for that sequence iff u < thr_l, thr_l = floor(p 2^32).
+Per shard (the paper's per-device batch dropping for data parallelism, Tensor
+Granularity subsection): b' = b_offset, the shard's first global sequence,
+for every sequence of the shard -- one draw per layer and step per shard.
 Sub-layer granularity (Model Granularity subsection: M_attn and M_ffn drawn
 independently, each Bernoulli(1 - p^{l,t})): the attention mask uses word 0
 of the same Philox output and the FFN mask word 1, so the attention mask is
@@ -25,7 +28,7 @@ import numpy as np
 
 from .philox import philox4x32_10, philox4x32_10_np
 
-PER_SEQUENCE, PER_BATCH = "per_sequence", "per_batch"
+PER_SEQUENCE, PER_BATCH, PER_SHARD = "per_sequence", "per_batch", "per_shard"
 
 
 def mask_word(seed, step, layer, b, word=0):
@@ -48,7 +51,12 @@ def draw_masks(seed, step, thresholds, B, granularity=PER_SEQUENCE, b_offset=0, 
     for w in range(nw):
         for layer in range(L):
             for b in range(B):
-                bb = b_offset + b if granularity == PER_SEQUENCE else 0
+                if granularity == PER_SEQUENCE:
+                    bb = b_offset + b
+                elif granularity == PER_SHARD:
+                    bb = b_offset
+                else:
+                    bb = 0
                 u = mask_word(seed, step, layer, bb, w)
                 mask[w, layer, b] = 0 if u < thresholds[layer] else 1
     return mask if sublayer else mask[0]

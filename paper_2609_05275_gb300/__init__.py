@@ -22,13 +22,13 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "ld.h")
 
 # enums of include/ld.h
 LD_OK, LD_ERR_ARG, LD_ERR_SHAPE, LD_ERR_STATE, LD_ERR_CUDA, LD_ERR_TIMEOUT, LD_ERR_OOM, LD_ERR_UNSUPPORTED = range(8)
-LD_PER_SEQUENCE, LD_PER_BATCH = 0, 1
+LD_PER_SEQUENCE, LD_PER_BATCH, LD_PER_SHARD = 0, 1, 2
 LD_DIST_UNIFORM, LD_DIST_ILD, LD_DIST_ALD, LD_DIST_EXPLICIT = 0, 1, 2, 3
 LD_TIME_CONST, LD_TIME_ITS, LD_TIME_DTS, LD_TIME_RAMP = 0, 1, 2, 3
 DIST = {"uniform": LD_DIST_UNIFORM, "ild": LD_DIST_ILD, "ald": LD_DIST_ALD, "explicit": LD_DIST_EXPLICIT}
 TIME = {"const": LD_TIME_CONST, "its": LD_TIME_ITS, "dts": LD_TIME_DTS, "ramp": LD_TIME_RAMP}
 ACT = {"swiglu": 0, "relu2": 1}
-GRAN = {"per_sequence": LD_PER_SEQUENCE, "per_batch": LD_PER_BATCH}
+GRAN = {"per_sequence": LD_PER_SEQUENCE, "per_batch": LD_PER_BATCH, "per_shard": LD_PER_SHARD}
 
 
 class ld_config(ctypes.Structure):

@@ -662,7 +662,8 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   if (c.d < 64 || c.d % 64 || c.F < 64 || c.F % 64 || c.d > 16384) return LD_ERR_SHAPE;
   if (c.Dh != 32 && c.Dh != 64 && c.Dh != 128) return LD_ERR_SHAPE;
   if (c.H < 1 || c.Hkv < 1 || c.H % c.Hkv || (c.H * c.Dh) % 64) return LD_ERR_SHAPE;
-  if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH) return LD_ERR_ARG;
+  if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH && c.granularity != LD_PER_SHARD)
+    return LD_ERR_ARG;
   if (c.sublayer != 0 && c.sublayer != 1) return LD_ERR_ARG;
   if (c.alibi != 0 && c.alibi != 1) return LD_ERR_ARG;
   if (c.alibi && c.rope_theta != 0.0f) return LD_ERR_ARG;  // one position scheme

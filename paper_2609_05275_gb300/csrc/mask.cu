@@ -8,7 +8,8 @@
 //
 // Draw: u = word 0 of Philox4x32-10 (Salmon et al., SC'11) with key
 // (seed lo, seed hi) and counter (b', l, t lo, t hi), b' = b per sequence
-// and 0 per batch.  Sequence b drops layer l iff u < thr_l = floor(p 2^32).
+// 0 per batch and b_offset per shard.  Sequence b drops layer l iff
+// u < thr_l = floor(p 2^32).
 // Sub-layer granularity (Model Granularity subsection): the attention mask
 // takes word 0 and the FFN mask word 1 of the same draw; their tables follow
 // each other ([2][L][B], counts [2][L]).
@@ -48,7 +49,9 @@ __global__ void mask_compact_kernel(const MaskParams P, unsigned char* __restric
     const int b = b0 + threadIdx.x;
     int keep = 0;
     if (b < P.B) {
-      const uint32_t bb = P.granularity == LD_PER_BATCH ? 0u : (uint32_t)(P.b_offset + b);
+      const uint32_t bb = P.granularity == LD_PER_BATCH   ? 0u
+                          : P.granularity == LD_PER_SHARD ? (uint32_t)P.b_offset
+                                                          : (uint32_t)(P.b_offset + b);
       const uint4 r = philox4x32_10(make_uint4(bb, (uint32_t)l, t_lo, t_hi), key);
       const uint32_t u = w == 0 ? r.x : r.y;
       keep = (unsigned long long)u >= thr;

@@ -30,7 +30,7 @@ def oracle_masks(cfg, sched, step, granularity="per_sequence", sublayer=False):
     rates = OS.layer_rates(oracle_sched(sched), cfg["L"], step)
     thr = [OS.drop_threshold(p) for p in rates]
     scales = [OS.residual_scale(p, cfg.get("alpha", 1.0)) for p in rates]
-    gran = OM.PER_SEQUENCE if granularity == "per_sequence" else OM.PER_BATCH
+    gran = {"per_sequence": OM.PER_SEQUENCE, "per_batch": OM.PER_BATCH, "per_shard": OM.PER_SHARD}[granularity]
     mask = OM.draw_masks(sched.get("seed", 0), step, thr, cfg["B"], gran, sublayer=sublayer)
     return mask, thr, scales
 

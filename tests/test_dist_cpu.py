@@ -48,6 +48,9 @@ def _worker(rank, world, port, q):
         full_mask = OM.draw_masks(5, 3, thr, B)
         mask = OM.draw_masks(5, 3, thr, Bs, b_offset=rank * Bs)
         ok_mask = bool((mask == full_mask[:, rank * Bs:(rank + 1) * Bs]).all())
+        # per-shard granularity: each rank draws for its whole shard, keyed by its first global sequence
+        shard = OM.draw_masks(5, 3, thr, Bs, OM.PER_SHARD, b_offset=rank * Bs)
+        ok_mask = ok_mask and bool((shard == full_mask[:, rank * Bs:rank * Bs + 1]).all())
         layers = [{n: v.double().numpy() for n, v in W.items()} for W in synth.stack_weights(cfg, seed=0)]
         x = synth.activations(cfg, seed=0, B=B).double().numpy()
         dy = synth.upstream_grad(cfg, B=B).double().numpy()

@@ -8,8 +8,9 @@ import torch
 
 import paper_2609_05275_gb300 as P
 from paper_2609_05275_gb300 import synth
-from parity import oracle_masks
+from parity import oracle_masks, oracle_sched
 from oracle import masks as OM
+from oracle import schedule as OS
 
 pytestmark = pytest.mark.gpu
 
@@ -62,3 +63,22 @@ def test_sublayer_masks(granularity, B):
     cfg = dict(synth.CONFIGS["tiny"], B=B, L=7)
     sched = dict(dist="ild", p_max=0.8, time="const", seed=2 ** 35 + 9)
     _check(cfg, sched, [0, 5, 2 ** 33 + 1], granularity, sublayer=True)
+
+
+@pytest.mark.parametrize("b_offset", [0, 8, 1000])
+def test_per_shard_masks(b_offset):
+    # per-device batch dropping: one draw per layer and step for the shard,
+    # keyed by its first global sequence; bit-exact against the oracle
+    cfg = dict(synth.CONFIGS["tiny"], B=8, L=6)
+    sched = dict(dist="ild", p_max=0.7, time="const", seed=77)
+    st = P.LayerDropStack(cfg, sched, granularity="per_shard", b_offset=b_offset)
+    try:
+        rates = OS.layer_rates(oracle_sched(sched), cfg["L"], 3)
+        thr = [OS.drop_threshold(p) for p in rates]
+        mask, idx, cnt = st.draw_masks(3)
+        ref = OM.draw_masks(77, 3, thr, cfg["B"], OM.PER_SHARD, b_offset=b_offset)
+        ridx, rcnt = OM.kept_lists(ref)
+        assert (mask == ref).all() and (idx == ridx).all() and (cnt == rcnt).all()
+        assert ((cnt == 0) | (cnt == cfg["B"])).all()  # whole shard kept or dropped
+    finally:
+        st.close()

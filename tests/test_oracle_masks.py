@@ -157,3 +157,23 @@ def test_sublayer_masks():
         for vf in (0, 1):
             assert abs(((a == va) & (f == vf)).mean() - 0.25) < 4 * sigma
     assert abs(np.corrcoef(a, f)[0, 1]) < 4 / math.sqrt(n)
+
+
+def test_per_shard_masks():
+    # Per-shard draws (per-device batch dropping): a shard's mask is the
+    # per-sequence draw of its first global sequence, broadcast over the
+    # shard; shard 0 is the per-batch mask; distinct shards draw independently.
+    thr = [S.drop_threshold(p) for p in (0.0, 0.4, 0.7, 1.0)]
+    B = 8
+    for off in (0, 8, 24, 2 ** 31 - 9):
+        m = M.draw_masks(3, 17, thr, B, M.PER_SHARD, b_offset=off)
+        ref = M.draw_masks(3, 17, thr, 1, M.PER_SEQUENCE, b_offset=off)
+        assert (m == ref).all()
+    assert (M.draw_masks(3, 17, thr, B, M.PER_SHARD, b_offset=0) == M.draw_masks(3, 17, thr, B, M.PER_BATCH)).all()
+    # two shards at p = 0.5 over many (layer, step): they agree on half the draws (independence)
+    t2 = [S.drop_threshold(0.5)] * 40
+    a = np.stack([M.draw_masks(5, t, t2, 4, M.PER_SHARD, b_offset=0)[:, 0] for t in range(50)]).ravel()
+    b = np.stack([M.draw_masks(5, t, t2, 4, M.PER_SHARD, b_offset=4)[:, 0] for t in range(50)]).ravel()
+    n = a.size
+    assert abs((a == b).mean() - 0.5) < 4 * math.sqrt(0.25 / n)
+    assert abs(a.mean() - 0.5) < 4 * math.sqrt(0.25 / n)
