@@ -16,6 +16,9 @@
 //   warps 2..5  epilogue: tcgen05.ld of the accumulator (each warp reads
 //               its 32-lane quadrant), fused scale / residual update, and
 //               global stores, overlapped with the next tile's MMAs.
+// 256-column tiles run on CTA pairs (clusters of two on the SMs of a TPC):
+// a 256 x 256 tile per pair, each CTA loading 128 rows of A and 128 rows of
+// B, one tcgen05.mma.cta_group::2 (M=256) per K=16 step from the even CTA.
 // Operands may be K-major or MN-major (weight-gradient and data-gradient
 // products read activations and weights transposed); the shared-memory
 // descriptors and the instruction descriptor's major bits cover both, so no
@@ -203,12 +206,22 @@ __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int&
   nb = first_n + r % gn;
 }
 
-template <int BN, int STAGES, bool A_MN, bool B_MN>
+// PAIR = false: one CTA per BM x BN tile, tcgen05.mma.cta_group::1.
+// PAIR = true: a cluster of two CTAs (the two SMs of a TPC) shares a tile of
+// 2*BM x BN.  Each CTA loads its own BM rows of A and half of the BN rows of
+// B, so per k-step a CTA streams 32 KB instead of 48 KB from L2 and a stage
+// takes 32 KB of shared memory (a deeper ring fits); the even CTA issues
+// tcgen05.mma.cta_group::2 (M = 256) for both, and each CTA's TMEM receives
+// its own BM rows of the accumulator, which its epilogue warps store.
+template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR>
 __global__ void __launch_bounds__(192, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const GemmArgs a) {
+  constexpr int NCTA = PAIR ? 2 : 1;
+  constexpr int BN_L = BN / NCTA;  // rows of B this CTA loads
+  constexpr int BMT = BM * NCTA;   // rows of a tile
   constexpr uint32_t A_BYTES = BM * BK * 2;
-  constexpr uint32_t B_BYTES = BN * BK * 2;
+  constexpr uint32_t B_BYTES = BN_L * BK * 2;
   constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   constexpr uint32_t TMEM_COLS = 2 * BN;
   extern __shared__ uint8_t smem_raw[];
@@ -222,10 +235,13 @@ __global__ void __launch_bounds__(192, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR ? (cluster_rank() & 1u) : 0u;
+  const int tile0 = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int tstep = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
   const int M = a.M_cnt ? (*a.M_cnt) * a.M_mul : a.M;
   const int K = a.K_cnt ? (*a.K_cnt) * a.K_mul : a.K;
   const int N = a.N;
-  const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN;
+  const int num_m = (M + BMT - 1) / BMT, num_n = (N + BN - 1) / BN;
   const int num_tiles = num_m * num_n;
   const int num_kb = K / BK;
 
@@ -236,20 +252,21 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&tfull[s], 1);
-      mbar_init(&tempty[s], 4);
+      mbar_init(&tempty[s], 4 * NCTA);  // one lane of every epilogue warp of the tile's CTAs
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                 "r"(TMEM_COLS)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if constexpr (PAIR)
+      tmem_alloc_pair(tmem_slot, TMEM_COLS);
+    else
+      tmem_alloc(tmem_slot, TMEM_COLS);
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();  // the peer's barriers are initialised before any remote arrival
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -260,10 +277,10 @@ __global__ void __launch_bounds__(192, 1)
       float z[32];
 #pragma unroll
       for (int i = 0; i < 32; ++i) z[i] = 0.f;
-      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      for (int tile = tile0; tile < num_tiles; tile += tstep) {
         int mb, nb;
         tile_coords(tile, num_m, num_n, mb, nb);
-        const int row = mb * BM + q * 32 + lane;
+        const int row = mb * BMT + (int)rank * BM + q * 32 + lane;
         for (int c = 0; c < BN; c += 32)
           if (row < M && nb * BN + c < N) store_chunk(a, row, nb * BN + c, z);
       }
@@ -275,9 +292,11 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t phase = 0;
       long long issued = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      for (int tile = tile0; tile < num_tiles && ok; tile += tstep) {
         int mb, nb;
         tile_coords(tile, num_m, num_n, mb, nb);
+        const int arow = mb * BMT + (int)rank * BM;
+        const int brow = nb * BN + (int)rank * BN_L;
         for (int kb = 0; kb < num_kb; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.status)) {
             ok = false;
@@ -285,22 +304,44 @@ __global__ void __launch_bounds__(192, 1)
           }
           uint8_t* sa = smem + stage * STAGE_BYTES;
           uint8_t* sb = sa + A_BYTES;
-          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-          if (!A_MN) {
-            tma_load_2d(sa, &tmA, kb * BK, mb * BM, &full[stage]);
-          } else {
-            tma_load_2d(sa, &tmA, mb * BM, kb * BK, &full[stage]);
-            tma_load_2d(sa + 8192, &tmA, mb * BM + 64, kb * BK, &full[stage]);
-          }
-          if (!B_MN && a.epi == EPI_SWIGLU) {
-            // gate rows and up rows of the same hidden units side by side
-            tma_load_2d(sb, &tmB, kb * BK, nb * (BN / 2), &full[stage]);
-            tma_load_2d(sb + (BN / 2) * 128, &tmB, kb * BK, a.F + nb * (BN / 2), &full[stage]);
-          } else if (!B_MN) {
-            tma_load_2d(sb, &tmB, kb * BK, nb * BN, &full[stage]);
-          } else {
+          if constexpr (PAIR) {
+            // both CTAs' copies complete on the even CTA's full barrier,
+            // which the even CTA's MMA thread waits on
+            if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * STAGE_BYTES);
+            const uint32_t fb = cluster_addr(&full[stage], 0);
+            if (!A_MN) {
+              tma_load_2d_pair(sa, &tmA, kb * BK, arow, fb);
+            } else {
+              tma_load_2d_pair(sa, &tmA, arow, kb * BK, fb);
+              tma_load_2d_pair(sa + 8192, &tmA, arow + 64, kb * BK, fb);
+            }
+            if (!B_MN && a.epi == EPI_SWIGLU) {
+              // gate rows in the even CTA, the matching up rows in the odd one
+              tma_load_2d_pair(sb, &tmB, kb * BK, (rank ? a.F : 0) + nb * BN_L, fb);
+            } else if (!B_MN) {
+              tma_load_2d_pair(sb, &tmB, kb * BK, brow, fb);
+            } else {
 #pragma unroll
-            for (int c = 0; c < BN / 64; ++c) tma_load_2d(sb + c * 8192, &tmB, nb * BN + c * 64, kb * BK, &full[stage]);
+              for (int c = 0; c < BN_L / 64; ++c) tma_load_2d_pair(sb + c * 8192, &tmB, brow + c * 64, kb * BK, fb);
+            }
+          } else {
+            mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+            if (!A_MN) {
+              tma_load_2d(sa, &tmA, kb * BK, arow, &full[stage]);
+            } else {
+              tma_load_2d(sa, &tmA, arow, kb * BK, &full[stage]);
+              tma_load_2d(sa + 8192, &tmA, arow + 64, kb * BK, &full[stage]);
+            }
+            if (!B_MN && a.epi == EPI_SWIGLU) {
+              // gate rows and up rows of the same hidden units side by side
+              tma_load_2d(sb, &tmB, kb * BK, nb * (BN / 2), &full[stage]);
+              tma_load_2d(sb + (BN / 2) * 128, &tmB, kb * BK, a.F + nb * (BN / 2), &full[stage]);
+            } else if (!B_MN) {
+              tma_load_2d(sb, &tmB, kb * BK, brow, &full[stage]);
+            } else {
+#pragma unroll
+              for (int c = 0; c < BN / 64; ++c) tma_load_2d(sb + c * 8192, &tmB, brow + c * 64, kb * BK, &full[stage]);
+            }
           }
           ++issued;
           if (++stage == STAGES) {
@@ -309,23 +350,29 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       }
-      if (!ok) {
-        // wait (bounded) for the copies this thread still has in flight
-        for (long long i = issued > STAGES ? issued - STAGES : 0; i < issued; ++i)
-          mbar_drain(&full[i % STAGES], (uint32_t)((i / STAGES) & 1));
+      const long long first = issued > STAGES ? issued - STAGES : 0;
+      if (!ok && rank == 0) {
+        // wait (bounded) for the copies still in flight (a pair's copies all
+        // complete on the even CTA's barriers)
+        for (long long i = first; i < issued; ++i) mbar_drain(&full[i % STAGES], (uint32_t)((i / STAGES) & 1));
+      }
+      if constexpr (PAIR) {
+        // the even CTA's MMA commits arrive on these barriers of both CTAs:
+        // wait (bounded) until the last ones have landed before the CTA ends
+        for (long long i = first; i < issued; ++i) mbar_drain(&empty[i % STAGES], (uint32_t)((i / STAGES) & 1));
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && rank == 0) {
       // ------------------------------------------------ MMA issuer
-      constexpr uint32_t IDESC = idesc_bf16(BM, BN, A_MN, B_MN);
+      constexpr uint32_t IDESC = idesc_bf16(BMT, BN, A_MN, B_MN);
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
+      for (int tile = tile0; tile < num_tiles && ok; tile += tstep) {
+        if (!mbar_wait<PAIR>(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
           ok = false;
           break;
         }
@@ -346,22 +393,34 @@ __global__ void __launch_bounds__(192, 1)
             // chunks 8 KB apart (LBO), 8-row groups 1 KB apart (SBO).
             const uint64_t ad = A_MN ? sdesc(sa + k * 2048, 8192, 1024) : sdesc(sa + k * 32, 16, 1024);
             const uint64_t bd = B_MN ? sdesc(sb + k * 2048, 8192, 1024) : sdesc(sb + k * 32, 16, 1024);
-            mma_bf16(d_tmem, ad, bd, IDESC, (kb | k) != 0 ? 1u : 0u);
+            if constexpr (PAIR)
+              mma_bf16_pair(d_tmem, ad, bd, IDESC, (kb | k) != 0 ? 1u : 0u);
+            else
+              mma_bf16(d_tmem, ad, bd, IDESC, (kb | k) != 0 ? 1u : 0u);
           }
-          mma_commit(&empty[stage]);
+          if constexpr (PAIR)
+            mma_commit_pair_both(&empty[stage]);
+          else
+            mma_commit(&empty[stage]);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        mma_commit(&tfull[acc]);
+        if constexpr (PAIR)
+          mma_commit_pair_both(&tfull[acc]);
+        else
+          mma_commit(&tfull[acc]);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
       }
       if (!ok) {
         // make sure every MMA issued so far has finished before TMEM is freed
-        mma_commit(drain);
+        if constexpr (PAIR)
+          mma_commit_pair_local(drain);
+        else
+          mma_commit(drain);
         mbar_drain(drain, 0);
       }
     }
@@ -370,7 +429,7 @@ __global__ void __launch_bounds__(192, 1)
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+    for (int tile = tile0; tile < num_tiles; tile += tstep) {
       int mb, nb;
       tile_coords(tile, num_m, num_n, mb, nb);
       // one lane waits; the warp follows its verdict (tcgen05.ld below is
@@ -380,7 +439,7 @@ __global__ void __launch_bounds__(192, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
-      const int row = mb * BM + q * 32 + lane;
+      const int row = mb * BMT + (int)rank * BM + q * 32 + lane;
       const uint32_t tbase = tmem_base + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
       if (a.epi == EPI_SWIGLU) {
         // columns [0, BN/2) hold g, [BN/2, BN) hold u of hidden units j0 + c
@@ -483,7 +542,12 @@ __global__ void __launch_bounds__(192, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (lane == 0) {
+        if constexpr (PAIR)
+          mbar_arrive_cluster(cluster_addr(&tempty[acc], 0));
+        else
+          mbar_arrive(&tempty[acc]);
+      }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
@@ -491,36 +555,97 @@ __global__ void __launch_bounds__(192, 1)
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) {
+    // neither CTA ends (and frees its TMEM and shared memory) while the
+    // other may still address them
+    __syncwarp();
+    cluster_sync();
+  }
   if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
+    if constexpr (PAIR)
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else
+      tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
-template <int BN, int STAGES, bool A_MN, bool B_MN>
+template <int BN, int STAGES, bool PAIR>
+constexpr size_t smem_bytes() {
+  return (size_t)STAGES * (BM * BK * 2 + (BN / (PAIR ? 2 : 1)) * BK * 2) + 1024 + 256;
+}
+
+// Tensor cores of the pair kernels: co-resident clusters of two CTAs (0 if
+// the pair kernel cannot run).
+constexpr int PAIR_BN = 256, PAIR_STAGES = 6;
+int pair_clusters() {
+  static int n = -1;
+  if (n < 0) {
+    n = 0;
+    auto k = gemm_tc_kernel<PAIR_BN, PAIR_STAGES, false, false, true>;
+    constexpr size_t smem = smem_bytes<PAIR_BN, PAIR_STAGES, true>();
+    if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 2;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(2);
+      cfg.blockDim = dim3(192);
+      cfg.dynamicSmemBytes = smem;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      int c = 0;
+      if (cudaOccupancyMaxActiveClusters(&c, k, &cfg) == cudaSuccess && c > 0) n = c;
+    }
+    cudaGetLastError();  // a refused query leaves no sticky error behind
+  }
+  return n;
+}
+
+template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR>
 cudaError_t run(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tb, cudaStream_t st) {
-  constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + 1024 + 256;
+  constexpr size_t smem = smem_bytes<BN, STAGES, PAIR>();
+  constexpr int NCTA = PAIR ? 2 : 1;
+  auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, PAIR>;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, A_MN, B_MN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   const int mcap = a.M_cnt ? a.M_cap : a.M;
-  const long long tiles = (long long)((mcap + BM - 1) / BM) * ((a.N + BN - 1) / BN);
-  int grid = device_sm_count();
-  if (tiles < grid) grid = (int)(tiles > 0 ? tiles : 1);
-  gemm_tc_kernel<BN, STAGES, A_MN, B_MN><<<grid, 192, smem, st>>>(ta, tb, a);
+  const long long tiles = (long long)((mcap + BM * NCTA - 1) / (BM * NCTA)) * ((a.N + BN - 1) / BN);
+  int units = PAIR ? pair_clusters() : device_sm_count();
+  if (tiles < units) units = (int)(tiles > 0 ? tiles : 1);
+  if constexpr (!PAIR) {
+    kern<<<units, 192, smem, st>>>(ta, tb, a);
+  } else {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(2 * units);
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, ta, tb, a);
+    if (e != cudaSuccess) return e;
+  }
   return cudaGetLastError();
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, bool PAIR>
 cudaError_t dispatch_major(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tb, cudaStream_t st) {
-  if (!a.a_mn && !a.b_mn) return run<BN, STAGES, false, false>(a, ta, tb, st);
-  if (!a.a_mn && a.b_mn) return run<BN, STAGES, false, true>(a, ta, tb, st);
-  if (a.a_mn && !a.b_mn) return run<BN, STAGES, true, false>(a, ta, tb, st);
-  return run<BN, STAGES, true, true>(a, ta, tb, st);
+  if (!a.a_mn && !a.b_mn) return run<BN, STAGES, false, false, PAIR>(a, ta, tb, st);
+  if (!a.a_mn && a.b_mn) return run<BN, STAGES, false, true, PAIR>(a, ta, tb, st);
+  if (a.a_mn && !a.b_mn) return run<BN, STAGES, true, false, PAIR>(a, ta, tb, st);
+  return run<BN, STAGES, true, true, PAIR>(a, ta, tb, st);
 }
 
 }  // namespace
@@ -530,6 +655,8 @@ cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st) {
   const uint64_t mcap = a.M_cnt ? a.M_cap : a.M;
   const uint64_t kcap = a.K_cnt ? a.K_cap : a.K;
   if (mcap == 0 || a.N == 0) return cudaSuccess;
+  // 256-column tiles run on CTA pairs where the device can co-schedule them
+  const bool pair = BN == PAIR_BN && pair_clusters() > 0;
   CUtensorMap ta, tb;
   bool ok;
   // A(m,k): K-major = rows m of k; MN-major = rows k of m.
@@ -539,12 +666,14 @@ cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st) {
     ok = make_map(&ta, a.A, mcap, kcap ? kcap : 64, a.lda, 64, 64);
   if (!ok) return cudaErrorInvalidValue;
   if (!a.b_mn)
-    ok = make_map(&tb, a.B, kcap ? kcap : 64, a.N, a.ldb, 64, (uint32_t)(a.epi == EPI_SWIGLU ? BN / 2 : BN));
+    ok = make_map(&tb, a.B, kcap ? kcap : 64, a.N, a.ldb, 64,
+                  (uint32_t)((a.epi == EPI_SWIGLU || pair) ? BN / 2 : BN));
   else
     ok = make_map(&tb, a.B, a.N, kcap ? kcap : 64, a.ldb, 64, 64);
   if (!ok) return cudaErrorInvalidValue;
-  if (BN == 256) return dispatch_major<256, 4>(a, ta, tb, st);
-  return dispatch_major<128, 6>(a, ta, tb, st);
+  if (pair) return dispatch_major<PAIR_BN, PAIR_STAGES, true>(a, ta, tb, st);
+  if (BN == 256) return dispatch_major<256, 4, false>(a, ta, tb, st);
+  return dispatch_major<128, 6, false>(a, ta, tb, st);
 }
 
 }  // namespace ldk

@@ -29,6 +29,18 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t addr, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// As mbar_try_wait with cluster-scope acquire (phases completed by arrivals
+// from the peer CTA of a pair).
+__device__ __forceinline__ bool mbar_try_wait_cl(uint32_t addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n selp.b32 %0, 1, "
+      "0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity), "r"(2000u)
+      : "memory");
+  return ok != 0;
+}
 // As above, but the thread is suspended until the phase completes or about
 // `hint_ns` pass, so waiting warps do not take issue slots from working ones.
 __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t addr, uint32_t parity, uint32_t hint_ns) {
@@ -50,12 +62,14 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
 // Bounded wait for the phase of parity `parity`.  False if the time limit
 // passed (the block's abort flag and the status word are raised) or another
 // role of the block aborted first.
+// CL: cluster-scope acquire (the phase is completed by the peer CTA).
+template <bool CL = false>
 static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status) {
   const uint32_t addr = smem_u32(bar);
-  if (mbar_try_wait(addr, parity)) return true;
+  if (CL ? mbar_try_wait_cl(addr, parity) : mbar_try_wait(addr, parity)) return true;
   const uint64_t t0 = gtimer_ns();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait_sleep(addr, parity, 2000)) return true;
+    if (CL ? mbar_try_wait_cl(addr, parity) : mbar_try_wait_sleep(addr, parity, 2000)) return true;
     if ((it & 7) == 0) {
       if (*abort_flag) return false;
       if (gtimer_ns() - t0 > kWaitLimitNs) {
@@ -311,6 +325,72 @@ __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
 }
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
   asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// ------------------------------------------------------- CTA pairs (cluster of 2)
+// The pair kernels run as clusters of two CTAs on the two SMs of a TPC; the
+// even-rank CTA issues tcgen05.mma.cta_group::2 for both.  Every tcgen05
+// instruction of such a kernel uses .cta_group::2.
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address in the cluster shared window of the object at `p` in CTA `rank`.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t rank) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
+  return a;
+}
+// All threads of both CTAs.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\nbarrier.cluster.wait.acquire;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cl_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cl_addr) : "memory");
+}
+// TMA tile load into this CTA's shared memory whose completion is counted on
+// the mbarrier at cluster address `bar_cl` (this CTA's or the peer's).
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* tm, int c0, int c1, uint32_t bar_cl) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+      "%3}], [%4];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(bar_cl)
+      : "memory");
+}
+// D[256 x N] (+)= A B^T over the pair: rows 0..127 of A and D and columns
+// 0..N/2-1 of B in the even CTA, the rest in the odd CTA, at the same
+// shared-memory and TMEM addresses.
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                              uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+          d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+// Arrive on the mbarrier at the same offset in both CTAs of the pair when
+// the MMAs issued so far are complete.
+__device__ __forceinline__ void mma_commit_pair_both(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "h"((uint16_t)3)
+      : "memory");
+}
+// As above, on this CTA's mbarrier only.
+__device__ __forceinline__ void mma_commit_pair_local(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+// Collective over one warp of each CTA of the pair.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
 
 // Warp-uniform bounded wait: lane 0 waits, the warp follows its verdict.
