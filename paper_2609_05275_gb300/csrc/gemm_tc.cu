@@ -213,7 +213,11 @@ __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int&
 // takes 32 KB of shared memory (a deeper ring fits); the even CTA issues
 // tcgen05.mma.cta_group::2 (M = 256) for both, and each CTA's TMEM receives
 // its own BM rows of the accumulator, which its epilogue warps store.
-template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR>
+// A ring stage holds KPS consecutive 64-deep k-blocks (each laid out as A
+// then B); the MMA thread takes one barrier hand-off per stage, so KPS = 2
+// halves the hand-offs per MMA (the tensor pipe queues only a few MMAs, and
+// each hand-off costs a few hundred cycles of barrier latency).
+template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR, int KPS>
 __global__ void __launch_bounds__(192, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const GemmArgs a) {
@@ -222,7 +226,8 @@ __global__ void __launch_bounds__(192, 1)
   constexpr int BMT = BM * NCTA;   // rows of a tile
   constexpr uint32_t A_BYTES = BM * BK * 2;
   constexpr uint32_t B_BYTES = BN_L * BK * 2;
-  constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr uint32_t SUB_BYTES = A_BYTES + B_BYTES;  // one 64-deep k-block
+  constexpr uint32_t STAGE_BYTES = KPS * SUB_BYTES;
   constexpr uint32_t TMEM_COLS = 2 * BN;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -243,7 +248,8 @@ __global__ void __launch_bounds__(192, 1)
   const int N = a.N;
   const int num_m = (M + BMT - 1) / BMT, num_n = (N + BN - 1) / BN;
   const int num_tiles = num_m * num_n;
-  const int num_kb = K / BK;
+  const int num_kb = K / BK;                     // 64-deep k-blocks
+  const int num_ks = (num_kb + KPS - 1) / KPS;  // ring stages per tile
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -297,50 +303,57 @@ __global__ void __launch_bounds__(192, 1)
         tile_coords(tile, num_m, num_n, mb, nb);
         const int arow = mb * BMT + (int)rank * BM;
         const int brow = nb * BN + (int)rank * BN_L;
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int ks = 0; ks < num_ks; ++ks) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.status)) {
             ok = false;
             break;
           }
-          uint8_t* sa = smem + stage * STAGE_BYTES;
-          uint8_t* sb = sa + A_BYTES;
+          const int nk = min(KPS, num_kb - ks * KPS);  // k-blocks in this stage
           if constexpr (PAIR) {
             // both CTAs' copies complete on the even CTA's full barrier,
             // which the even CTA's MMA thread waits on
-            if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * STAGE_BYTES);
-            const uint32_t fb = cluster_addr(&full[stage], 0);
-            if (!A_MN) {
-              tma_load_2d_pair(sa, &tmA, kb * BK, arow, fb);
-            } else {
-              tma_load_2d_pair(sa, &tmA, arow, kb * BK, fb);
-              tma_load_2d_pair(sa + 8192, &tmA, arow + 64, kb * BK, fb);
-            }
-            if (!B_MN && a.epi == EPI_SWIGLU) {
-              // gate rows in the even CTA, the matching up rows in the odd one
-              tma_load_2d_pair(sb, &tmB, kb * BK, (rank ? a.F : 0) + nb * BN_L, fb);
-            } else if (!B_MN) {
-              tma_load_2d_pair(sb, &tmB, kb * BK, brow, fb);
-            } else {
-#pragma unroll
-              for (int c = 0; c < BN_L / 64; ++c) tma_load_2d_pair(sb + c * 8192, &tmB, brow + c * 64, kb * BK, fb);
-            }
+            if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2u * (uint32_t)nk * SUB_BYTES);
           } else {
-            mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-            if (!A_MN) {
-              tma_load_2d(sa, &tmA, kb * BK, arow, &full[stage]);
-            } else {
-              tma_load_2d(sa, &tmA, arow, kb * BK, &full[stage]);
-              tma_load_2d(sa + 8192, &tmA, arow + 64, kb * BK, &full[stage]);
-            }
-            if (!B_MN && a.epi == EPI_SWIGLU) {
-              // gate rows and up rows of the same hidden units side by side
-              tma_load_2d(sb, &tmB, kb * BK, nb * (BN / 2), &full[stage]);
-              tma_load_2d(sb + (BN / 2) * 128, &tmB, kb * BK, a.F + nb * (BN / 2), &full[stage]);
-            } else if (!B_MN) {
-              tma_load_2d(sb, &tmB, kb * BK, brow, &full[stage]);
-            } else {
+            mbar_arrive_expect_tx(&full[stage], (uint32_t)nk * SUB_BYTES);
+          }
+          for (int j = 0; j < nk; ++j) {
+            const int kb = ks * KPS + j;
+            uint8_t* sa = smem + stage * STAGE_BYTES + j * SUB_BYTES;
+            uint8_t* sb = sa + A_BYTES;
+            if constexpr (PAIR) {
+              const uint32_t fb = cluster_addr(&full[stage], 0);
+              if (!A_MN) {
+                tma_load_2d_pair(sa, &tmA, kb * BK, arow, fb);
+              } else {
+                tma_load_2d_pair(sa, &tmA, arow, kb * BK, fb);
+                tma_load_2d_pair(sa + 8192, &tmA, arow + 64, kb * BK, fb);
+              }
+              if (!B_MN && a.epi == EPI_SWIGLU) {
+                // gate rows in the even CTA, the matching up rows in the odd one
+                tma_load_2d_pair(sb, &tmB, kb * BK, (rank ? a.F : 0) + nb * BN_L, fb);
+              } else if (!B_MN) {
+                tma_load_2d_pair(sb, &tmB, kb * BK, brow, fb);
+              } else {
 #pragma unroll
-              for (int c = 0; c < BN / 64; ++c) tma_load_2d(sb + c * 8192, &tmB, brow + c * 64, kb * BK, &full[stage]);
+                for (int c = 0; c < BN_L / 64; ++c) tma_load_2d_pair(sb + c * 8192, &tmB, brow + c * 64, kb * BK, fb);
+              }
+            } else {
+              if (!A_MN) {
+                tma_load_2d(sa, &tmA, kb * BK, arow, &full[stage]);
+              } else {
+                tma_load_2d(sa, &tmA, arow, kb * BK, &full[stage]);
+                tma_load_2d(sa + 8192, &tmA, arow + 64, kb * BK, &full[stage]);
+              }
+              if (!B_MN && a.epi == EPI_SWIGLU) {
+                // gate rows and up rows of the same hidden units side by side
+                tma_load_2d(sb, &tmB, kb * BK, nb * (BN / 2), &full[stage]);
+                tma_load_2d(sb + (BN / 2) * 128, &tmB, kb * BK, a.F + nb * (BN / 2), &full[stage]);
+              } else if (!B_MN) {
+                tma_load_2d(sb, &tmB, kb * BK, brow, &full[stage]);
+              } else {
+#pragma unroll
+                for (int c = 0; c < BN / 64; ++c) tma_load_2d(sb + c * 8192, &tmB, brow + c * 64, kb * BK, &full[stage]);
+              }
             }
           }
           ++issued;
@@ -378,25 +391,31 @@ __global__ void __launch_bounds__(192, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int ks = 0; ks < num_ks; ++ks) {
           if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
-          const uint32_t sb = sa + A_BYTES;
+          const int nk = min(KPS, num_kb - ks * KPS);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            // K-major: +32 bytes per 16-element K step inside the 128-byte
-            // swizzle row.  MN-major: +16 rows of 128 bytes; 64-element MN
-            // chunks 8 KB apart (LBO), 8-row groups 1 KB apart (SBO).
-            const uint64_t ad = A_MN ? sdesc(sa + k * 2048, 8192, 1024) : sdesc(sa + k * 32, 16, 1024);
-            const uint64_t bd = B_MN ? sdesc(sb + k * 2048, 8192, 1024) : sdesc(sb + k * 32, 16, 1024);
-            if constexpr (PAIR)
-              mma_bf16_pair(d_tmem, ad, bd, IDESC, (kb | k) != 0 ? 1u : 0u);
-            else
-              mma_bf16(d_tmem, ad, bd, IDESC, (kb | k) != 0 ? 1u : 0u);
+          for (int j = 0; j < KPS; ++j) {
+            if (j >= nk) break;
+            const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES + j * SUB_BYTES);
+            const uint32_t sb = sa + A_BYTES;
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k) {
+              // K-major: +32 bytes per 16-element K step inside the 128-byte
+              // swizzle row.  MN-major: +16 rows of 128 bytes; 64-element MN
+              // chunks 8 KB apart (LBO), 8-row groups 1 KB apart (SBO).
+              const uint64_t ad = A_MN ? sdesc(sa + k * 2048, 8192, 1024) : sdesc(sa + k * 32, 16, 1024);
+              const uint64_t bd = B_MN ? sdesc(sb + k * 2048, 8192, 1024) : sdesc(sb + k * 32, 16, 1024);
+              const uint32_t accum = (ks | j | k) != 0 ? 1u : 0u;
+              if constexpr (PAIR)
+                mma_bf16_pair(d_tmem, ad, bd, IDESC, accum);
+              else
+                mma_bf16(d_tmem, ad, bd, IDESC, accum);
+            }
           }
           if constexpr (PAIR)
             mma_commit_pair_both(&empty[stage]);
@@ -570,20 +589,20 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
-template <int BN, int STAGES, bool PAIR>
+template <int BN, int STAGES, bool PAIR, int KPS>
 constexpr size_t smem_bytes() {
-  return (size_t)STAGES * (BM * BK * 2 + (BN / (PAIR ? 2 : 1)) * BK * 2) + 1024 + 256;
+  return (size_t)STAGES * KPS * (BM * BK * 2 + (BN / (PAIR ? 2 : 1)) * BK * 2) + 1024 + 256;
 }
 
 // Tensor cores of the pair kernels: co-resident clusters of two CTAs (0 if
 // the pair kernel cannot run).
-constexpr int PAIR_BN = 256, PAIR_STAGES = 6;
+constexpr int PAIR_BN = 256, PAIR_STAGES = 3, PAIR_KPS = 2;
 int pair_clusters() {
   static int n = -1;
   if (n < 0) {
     n = 0;
-    auto k = gemm_tc_kernel<PAIR_BN, PAIR_STAGES, false, false, true>;
-    constexpr size_t smem = smem_bytes<PAIR_BN, PAIR_STAGES, true>();
+    auto k = gemm_tc_kernel<PAIR_BN, PAIR_STAGES, false, false, true, PAIR_KPS>;
+    constexpr size_t smem = smem_bytes<PAIR_BN, PAIR_STAGES, true, PAIR_KPS>();
     if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
       cudaLaunchAttribute at[1];
@@ -604,11 +623,11 @@ int pair_clusters() {
   return n;
 }
 
-template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR>
+template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR, int KPS>
 cudaError_t run(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tb, cudaStream_t st) {
-  constexpr size_t smem = smem_bytes<BN, STAGES, PAIR>();
+  constexpr size_t smem = smem_bytes<BN, STAGES, PAIR, KPS>();
   constexpr int NCTA = PAIR ? 2 : 1;
-  auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, PAIR>;
+  auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, PAIR, KPS>;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -640,12 +659,12 @@ cudaError_t run(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tb,
   return cudaGetLastError();
 }
 
-template <int BN, int STAGES, bool PAIR>
+template <int BN, int STAGES, bool PAIR, int KPS>
 cudaError_t dispatch_major(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tb, cudaStream_t st) {
-  if (!a.a_mn && !a.b_mn) return run<BN, STAGES, false, false, PAIR>(a, ta, tb, st);
-  if (!a.a_mn && a.b_mn) return run<BN, STAGES, false, true, PAIR>(a, ta, tb, st);
-  if (a.a_mn && !a.b_mn) return run<BN, STAGES, true, false, PAIR>(a, ta, tb, st);
-  return run<BN, STAGES, true, true, PAIR>(a, ta, tb, st);
+  if (!a.a_mn && !a.b_mn) return run<BN, STAGES, false, false, PAIR, KPS>(a, ta, tb, st);
+  if (!a.a_mn && a.b_mn) return run<BN, STAGES, false, true, PAIR, KPS>(a, ta, tb, st);
+  if (a.a_mn && !a.b_mn) return run<BN, STAGES, true, false, PAIR, KPS>(a, ta, tb, st);
+  return run<BN, STAGES, true, true, PAIR, KPS>(a, ta, tb, st);
 }
 
 }  // namespace
@@ -671,9 +690,9 @@ cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st) {
   else
     ok = make_map(&tb, a.B, a.N, kcap ? kcap : 64, a.ldb, 64, 64);
   if (!ok) return cudaErrorInvalidValue;
-  if (pair) return dispatch_major<PAIR_BN, PAIR_STAGES, true>(a, ta, tb, st);
-  if (BN == 256) return dispatch_major<256, 4, false>(a, ta, tb, st);
-  return dispatch_major<128, 6, false>(a, ta, tb, st);
+  if (pair) return dispatch_major<PAIR_BN, PAIR_STAGES, true, PAIR_KPS>(a, ta, tb, st);
+  if (BN == 256) return dispatch_major<256, 4, false, 1>(a, ta, tb, st);
+  return dispatch_major<128, 3, false, 2>(a, ta, tb, st);
 }
 
 }  // namespace ldk
