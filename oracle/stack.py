@@ -31,6 +31,13 @@ projection (w_gu then holds only the F "up" rows).  Weights use the [out, in] la
 key/value head floor(h * Hkv / H).  RoPE rotates the pairs (i, i + Dh/2) by
 angle pos * theta^(-2i/Dh) at in-sequence position pos; theta = 0 disables it.
 
+With per-token masks (``per_token=True``, masks [L, B, S]; see
+``oracle/masks.py`` for this reading of the granularity the Tensor
+Granularity subsection leaves to future work) the same blocks run on the kept
+tokens of each sequence as one shorter sequence: rows in their original
+order, rotary angles and ALiBi distances from their original positions, keys
+and values of the kept tokens only; a dropped token's row is left unchanged.
+
 The backward is derived by hand from these definitions (chain rule, no
 autograd).  Everything is float64, one sequence at a time.
 """
@@ -110,12 +117,14 @@ def alibi_slopes(H):
     return np.array(geometric(n0) + geometric(2 * n0)[0::2][: H - n0])
 
 
-def attention_probs(qh, kh, slope=None):
-    """Causal softmax(q k^T / sqrt(Dh) [+ slope (j - i)]) for one head: [S, S]."""
+def attention_probs(qh, kh, slope=None, pos=None):
+    """Causal softmax(q k^T / sqrt(Dh) [+ slope (pos_j - pos_i)]) for one
+    head: [S, S].  Rows are in causal order; ``pos`` (default 0 .. S-1) are
+    their positions for the ALiBi distance."""
     S, Dh = qh.shape
     sc = (qh @ kh.T) / math.sqrt(Dh)
     if slope is not None:
-        pos = np.arange(S, dtype=np.float64)
+        pos = np.arange(S, dtype=np.float64) if pos is None else np.asarray(pos, dtype=np.float64)
         sc = sc + slope * (pos[None, :] - pos[:, None])
     causal = np.tril(np.ones((S, S), dtype=bool))
     sc = np.where(causal, sc, -np.inf)
@@ -124,20 +133,20 @@ def attention_probs(qh, kh, slope=None):
     return e / np.sum(e, axis=1, keepdims=True)
 
 
-def attention(q, k, v, slopes=None):
+def attention(q, k, v, slopes=None, pos=None):
     """Causal grouped-query attention. q [S,H,Dh], k/v [S,Hkv,Dh] -> [S,H,Dh];
-    ``slopes`` [H] adds the ALiBi bias."""
+    ``slopes`` [H] adds the ALiBi bias (at positions ``pos``)."""
     S, H, Dh = q.shape
     Hkv = k.shape[1]
     o = np.zeros_like(q)
     for h in range(H):
         j = kv_head(h, H, Hkv)
-        P = attention_probs(q[:, h, :], k[:, j, :], None if slopes is None else slopes[h])
+        P = attention_probs(q[:, h, :], k[:, j, :], None if slopes is None else slopes[h], pos)
         o[:, h, :] = P @ v[:, j, :]
     return o
 
 
-def attention_backward(do, q, k, v, slopes=None):
+def attention_backward(do, q, k, v, slopes=None, pos=None):
     """Gradients of ``attention`` w.r.t. q, k, v given d(out) = do.
 
     Per head, with P the probabilities and c = 1/sqrt(Dh):
@@ -153,7 +162,7 @@ def attention_backward(do, q, k, v, slopes=None):
     dv = np.zeros_like(v)
     for h in range(H):
         j = kv_head(h, H, Hkv)
-        P = attention_probs(q[:, h, :], k[:, j, :], None if slopes is None else slopes[h])
+        P = attention_probs(q[:, h, :], k[:, j, :], None if slopes is None else slopes[h], pos)
         doh = do[:, h, :]
         dv[:, j, :] += P.T @ doh
         dP = doh @ v[:, j, :].T
@@ -189,16 +198,23 @@ def _slopes(cfg):
     return alibi_slopes(cfg["H"]) if cfg.get("alibi") else None
 
 
-def attn_forward(x, W, cfg, s, rope_cs):
-    """Attention residual block of a kept sequence: Z = X + s f_attn(X)."""
+def _positions(S, pos):
+    return np.arange(S) if pos is None else np.asarray(pos)
+
+
+def attn_forward(x, W, cfg, s, rope_cs, pos=None):
+    """Attention residual block of a kept sequence: Z = X + s f_attn(X).
+    ``pos``: positions of the rows (default 0 .. S-1; the kept tokens'
+    original positions with per-token masks)."""
     S = x.shape[0]
+    pp = _positions(S, pos)
     xh, xn, r1 = rmsnorm(x, W["g1"], cfg["eps"])
     q, k, v = _split_qkv(xh @ W["w_qkv"].T, cfg)
     if rope_cs is not None:
         cos, sin = rope_cs
-        q = rope(q, cos[:S], sin[:S])
-        k = rope(k, cos[:S], sin[:S])
-    o = attention(q, k, v, _slopes(cfg)).reshape(S, -1)
+        q = rope(q, cos[pp], sin[pp])
+        k = rope(k, cos[pp], sin[pp])
+    o = attention(q, k, v, _slopes(cfg), pp).reshape(S, -1)
     z = x + s * (o @ W["w_o"].T)
     return z, dict(xh=xh, xn=xn, r1=r1, q=q, k=k, v=v, o=o)
 
@@ -254,20 +270,21 @@ def ffn_backward(dout, W, cfg, s, cache, G):
     return dout + dz_norm
 
 
-def attn_backward(dz, W, cfg, s, cache, G, rope_cs):
+def attn_backward(dz, W, cfg, s, cache, G, rope_cs, pos=None):
     """d Z[b] -> d X[b] through the attention block; adds into G."""
     S = dz.shape[0]
+    pp = _positions(S, pos)
     H, Dh = cfg["H"], cfg["Dh"]
     c = cache
     # z = x + s * (o w_o^T).
     da = s * dz
     G["w_o"] += da.T @ c["o"]
     do = (da @ W["w_o"]).reshape(S, H, Dh)
-    dq, dk, dv = attention_backward(do, c["q"], c["k"], c["v"], _slopes(cfg))
+    dq, dk, dv = attention_backward(do, c["q"], c["k"], c["v"], _slopes(cfg), pp)
     if rope_cs is not None:
         cos, sin = rope_cs
-        dq = rope_backward(dq, cos[:S], sin[:S])
-        dk = rope_backward(dk, cos[:S], sin[:S])
+        dq = rope_backward(dq, cos[pp], sin[pp])
+        dk = rope_backward(dk, cos[pp], sin[pp])
     dqkv = np.concatenate([dq.reshape(S, -1), dk.reshape(S, -1), dv.reshape(S, -1)], axis=1)
     G["w_qkv"] += dqkv.T @ c["xh"]
     dxh = dqkv @ W["w_qkv"]
@@ -306,9 +323,72 @@ def _branch_masks(masks):
     return masks, masks
 
 
-def stack_forward(x, layers, cfg, masks, scales):
+def _token_branch_masks(masks):
+    masks = np.asarray(masks)
+    if masks.ndim == 4:
+        return masks[0], masks[1]
+    return masks, masks
+
+
+def stack_forward_tokens(x, layers, cfg, masks, scales):
+    """Per-token masks [L, B, S] or [2, L, B, S]: each block runs on the kept
+    tokens of each sequence (original order and positions) and updates only
+    their rows."""
+    X = np.array(x, dtype=np.float64, copy=True)
+    B, S, _ = X.shape
+    ma, mf = _token_branch_masks(masks)
+    L = ma.shape[0]
+    rope_cs = _rope_cs(cfg, S)
+    caches = [[None] * B for _ in range(L)]
+    for l in range(L):
+        if not (ma[l].any() or mf[l].any()):
+            continue
+        W = _layer(layers, l)
+        for b in range(B):
+            c = {}
+            ka = np.nonzero(ma[l, b])[0]
+            if ka.size:
+                X[b, ka], ca = attn_forward(X[b, ka], W, cfg, scales[l], rope_cs, pos=ka)
+                c.update(ca)
+            kf = np.nonzero(mf[l, b])[0]
+            if kf.size:
+                X[b, kf], cf = ffn_forward(X[b, kf], W, cfg, scales[l])
+                c.update(cf)
+            c.update(ka=ka, kf=kf)
+            caches[l][b] = c
+    return X, caches
+
+
+def stack_backward_tokens(dy, layers, cfg, masks, scales, caches):
+    """Backward of ``stack_forward_tokens``: a dropped token's gradient
+    passes through the block unchanged; weight gradients sum over the kept
+    tokens only."""
+    dX = np.array(dy, dtype=np.float64, copy=True)
+    B, S, _ = dX.shape
+    ma, mf = _token_branch_masks(masks)
+    L = ma.shape[0]
+    rope_cs = _rope_cs(cfg, S)
+    grads = [None] * L
+    for l in reversed(range(L)):
+        W = _layer(layers, l) if (ma[l].any() or mf[l].any()) else None
+        G = {n: np.zeros(shape_of(cfg, n)) for n in WEIGHT_NAMES}
+        for b in range(B):
+            c = caches[l][b]
+            if c is None:
+                continue
+            if c["kf"].size:
+                dX[b, c["kf"]] = ffn_backward(dX[b, c["kf"]], W, cfg, scales[l], c, G)
+            if c["ka"].size:
+                dX[b, c["ka"]] = attn_backward(dX[b, c["ka"]], W, cfg, scales[l], c, G, rope_cs, pos=c["ka"])
+        grads[l] = G
+    return dX, grads
+
+
+def stack_forward(x, layers, cfg, masks, scales, per_token=False):
     """x [B, S, d] -> (X^L, caches).  masks [L, B] or [2, L, B] (1 = keep),
-    scales [L]."""
+    scales [L]; with ``per_token`` masks [L, B, S] or [2, L, B, S]."""
+    if per_token:
+        return stack_forward_tokens(x, layers, cfg, masks, scales)
     X = np.array(x, dtype=np.float64, copy=True)
     B, S, _ = X.shape
     ma, mf = _branch_masks(masks)
@@ -351,11 +431,13 @@ def stack_forward_eval(x, layers, cfg, execute, r_eval=None):
     return X
 
 
-def stack_backward(dy, layers, cfg, masks, scales, caches):
+def stack_backward(dy, layers, cfg, masks, scales, caches, per_token=False):
     """d X^L -> (d X^0, per-layer weight gradients).
 
     Dropped sequences pass their gradient through unchanged; a block's weight
     gradients sum over its kept sequences only (zero if none is kept)."""
+    if per_token:
+        return stack_backward_tokens(dy, layers, cfg, masks, scales, caches)
     dX = np.array(dy, dtype=np.float64, copy=True)
     B, S, _ = dX.shape
     ma, mf = _branch_masks(masks)

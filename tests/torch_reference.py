@@ -13,31 +13,34 @@ import torch
 import torch.nn.functional as F
 
 
-def _rope_complex(t, theta):
-    """t [S, heads, Dh]; pairs (i, i + Dh/2) rotated as complex numbers."""
+def _rope_complex(t, theta, pos=None):
+    """t [S, heads, Dh]; pairs (i, i + Dh/2) rotated as complex numbers by
+    angle pos * freq (pos defaults to 0 .. S-1)."""
     S, nh, Dh = t.shape
     half = Dh // 2
     freqs = 1.0 / (theta ** (torch.arange(0, Dh, 2, dtype=torch.float64) / Dh))
-    ang = torch.outer(torch.arange(S, dtype=torch.float64), freqs)
+    p = torch.arange(S, dtype=torch.float64) if pos is None else torch.as_tensor(pos, dtype=torch.float64)
+    ang = torch.outer(p, freqs)
     rot = torch.polar(torch.ones_like(ang), ang)[:, None, :]
     c = torch.complex(t[..., :half], t[..., half:]) * rot
     return torch.cat([c.real, c.imag], dim=-1)
 
 
-def dense_layer(x, W, cfg, slopes=None):
+def dense_layer(x, W, cfg, slopes=None, pos=None):
     """f for one sequence x [S, d] at rate 0 and scale 1: returns (attn, ffn)
     callables so that masks and scales can be composed outside.  With
     cfg["alibi"] the per-head ``slopes`` enter SDPA as an additive float mask
     m_h (j - i) next to -inf above the diagonal; cfg["act"] == "relu2" selects
-    the squared-ReLU feed-forward."""
+    the squared-ReLU feed-forward.  ``pos`` (increasing; default 0 .. S-1)
+    are the rows' positions for the rotary angles and ALiBi distances."""
     H, Hkv, Dh, Fh = cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"]
     eps, theta = cfg["eps"], cfg.get("rope_theta", 0.0)
     S = x.shape[0]
     alibi = cfg.get("alibi", False)
     if alibi:
         theta = 0.0
-        pos = torch.arange(S, dtype=torch.float64)
-        rel = pos[None, :] - pos[:, None]
+        pp = torch.arange(S, dtype=torch.float64) if pos is None else torch.as_tensor(pos, dtype=torch.float64)
+        rel = pp[None, :] - pp[:, None]
         bias = torch.as_tensor(slopes, dtype=torch.float64)[:, None, None] * rel[None]
         bias = bias.masked_fill(rel[None] > 0, float("-inf"))
 
@@ -48,7 +51,7 @@ def dense_layer(x, W, cfg, slopes=None):
         k = qkv[:, H * Dh : (H + Hkv) * Dh].view(S, Hkv, Dh)
         v = qkv[:, (H + Hkv) * Dh :].view(S, Hkv, Dh)
         if theta:
-            q, k = _rope_complex(q, theta), _rope_complex(k, theta)
+            q, k = _rope_complex(q, theta, pos), _rope_complex(k, theta, pos)
         rep = H // Hkv
         k = k.repeat_interleave(rep, dim=1)
         v = v.repeat_interleave(rep, dim=1)
@@ -85,6 +88,30 @@ def masked_stack(x, layers, cfg, masks, scales, slopes=None):
             s = float(scales[l])
             zb = xb + s * f_attn(xb) if ma[l, b] else xb
             xb = zb + s * f_ffn(zb) if mf[l, b] else zb
+        outs.append(xb)
+    return torch.stack(outs)
+
+
+def token_masked_stack(x, layers, cfg, masks, scales, slopes=None):
+    """Stack with per-token masks [L, B, S] (or [2, L, B, S] for separate
+    attention / FFN masks), composed from dense layers applied to each
+    sequence's kept tokens as one shorter sequence at their original
+    positions; the other rows are left as they are."""
+    masks = torch.as_tensor(masks)
+    ma, mf = (masks[0], masks[1]) if masks.ndim == 4 else (masks, masks)
+    outs = []
+    for b in range(x.shape[0]):
+        xb = x[b]
+        for l in range(ma.shape[0]):
+            s = float(scales[l])
+            ka = torch.nonzero(ma[l, b]).flatten()
+            if ka.numel():
+                f_attn, _ = dense_layer(xb[ka], layers[l], cfg, slopes, pos=ka)
+                xb = torch.index_add(xb, 0, ka, s * f_attn(xb[ka]))
+            kf = torch.nonzero(mf[l, b]).flatten()
+            if kf.numel():
+                _, f_ffn = dense_layer(xb[kf], layers[l], cfg, slopes, pos=kf)
+                xb = torch.index_add(xb, 0, kf, s * f_ffn(xb[kf]))
         outs.append(xb)
     return torch.stack(outs)
 
