@@ -63,15 +63,20 @@ typedef enum {
   LD_ERR_UNSUPPORTED = 7 /* device is not sm_103 / build lacks the kernel    */
 } ld_status;
 
-/* Tensor granularity (Tensor Granularity subsection): one Bernoulli draw per
- * sequence, or one per layer and step shared by the whole batch. */
 /* Tensor granularity of the masks (Tensor Granularity subsection):
  * per sequence, per batch (one draw per layer and step, shared by every
  * sequence), or per shard: one draw per layer and step for this batch shard
  * alone, keyed by its first global sequence b_offset, so that data-parallel
  * ranks drop different layers while each skips whole layers (the paper's
- * per-device batch dropping; on one device it is the per-batch case). */
-typedef enum { LD_PER_SEQUENCE = 0, LD_PER_BATCH = 1, LD_PER_SHARD = 2 } ld_granularity;
+ * per-device batch dropping; on one device it is the per-batch case).
+ * Per token (the finer grain that subsection leaves to future work; this
+ * library's reading): one draw per (layer, token); the kept tokens of each
+ * sequence run the layer as one shorter sequence in their original order,
+ * with rotary angles at their original positions, and a dropped token is
+ * left unchanged and contributes no key or value to that layer.  Needs
+ * rope_theta or no position scheme (no ALiBi) and, on the bf16 path,
+ * Dh = 128 and S % 128 == 0. */
+typedef enum { LD_PER_SEQUENCE = 0, LD_PER_BATCH = 1, LD_PER_SHARD = 2, LD_PER_TOKEN = 3 } ld_granularity;
 
 /* Layer distributions (Dropout Distribution section):
  *   UNIFORM  p^l = p_max
@@ -143,7 +148,8 @@ typedef struct { float *w_qkv, *w_o, *w_gu, *w_d, *g1, *g2; } ld_layer_g;
 /* Validate `cfg` and create a handle.  Allocates host memory only (no CUDA
  * call), so it can run without a GPU.  LD_ERR_SHAPE for an unsupported
  * shape, LD_ERR_ARG for null pointers, a non-finite eps/alpha, a flag out of
- * range or ALiBi together with a rotary embedding. */
+ * range, ALiBi together with a rotary embedding, or per-token granularity
+ * with ALiBi or (bf16 path) with Dh != 128 or S % 128 != 0. */
 ld_status ld_create(const ld_config* cfg, void** handle);
 
 /* Bytes of device workspace ld_forward/ld_backward need: the mask tables,
@@ -165,9 +171,12 @@ ld_status ld_get_rates(void* handle, long long step, double* p, unsigned long lo
 /* Draw the masks of step t into the workspace (the first kernel of
  * ld_forward, alone).  Philox4x32-10 (Salmon et al., SC'11): key = (seed
  * low 32 bits, seed high 32 bits), counter = (b', l, t low, t high) with
- * b' = b_offset + b per sequence and b' = 0 per batch; word 0 is u (with
- * sub-layer granularity word 0 draws the attention mask and word 1 the FFN
- * mask).  Kept lists are ascending in b (local indices). */
+ * b' = b_offset + b per sequence, b' = 0 per batch and b' = b_offset per
+ * shard; word 0 is u (with sub-layer granularity word 0 draws the attention
+ * mask and word 1 the FFN mask).  Kept lists are ascending in b (local
+ * indices).  Per token: counter (g, l, t low, t high) with g = ((b_offset +
+ * b) S + s) mod 2^32, u = word 2 (word 3 for the FFN mask with sub-layer
+ * granularity); kept lists hold the rows b S + s, ascending. */
 ld_status ld_draw_masks(void* handle, long long step, void* workspace, void* stream);
 
 /* Forward of step t, in place on x [B*S, d] (sequence b = rows b*S..b*S+S-1).
@@ -210,8 +219,11 @@ ld_status ld_backward(void* handle, const ld_layer_w* W, void* dx, ld_layer_g* G
 /* Copy the masks of the last ld_forward / ld_draw_masks to host memory:
  * mask [L*B] (1 = keep), kept_idx [L*B] (ascending, -1 padded), kept_cnt
  * [L]; with sub-layer granularity the attention tables followed by the FFN
- * tables: mask and kept_idx [2*L*B], kept_cnt [2*L].  Synchronises that
- * call's stream.  Any output may be NULL. */
+ * tables: mask and kept_idx [2*L*B], kept_cnt [2*L].  Per token: mask
+ * [L*B*S] (layer l, token b*S+s), kept_idx [L*B*S] (rows b*S+s of the kept
+ * tokens, ascending, -1 padded), kept_cnt [L] (kept tokens); [2*L*B*S] and
+ * [2*L] with sub-layer granularity.  Synchronises that call's stream.  Any
+ * output may be NULL. */
 ld_status ld_get_masks(void* handle, unsigned char* mask, int* kept_idx, int* kept_cnt);
 
 /* Synchronise the stream of the last call and return the device status word

@@ -22,13 +22,14 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "ld.h")
 
 # enums of include/ld.h
 LD_OK, LD_ERR_ARG, LD_ERR_SHAPE, LD_ERR_STATE, LD_ERR_CUDA, LD_ERR_TIMEOUT, LD_ERR_OOM, LD_ERR_UNSUPPORTED = range(8)
-LD_PER_SEQUENCE, LD_PER_BATCH, LD_PER_SHARD = 0, 1, 2
+LD_PER_SEQUENCE, LD_PER_BATCH, LD_PER_SHARD, LD_PER_TOKEN = 0, 1, 2, 3
 LD_DIST_UNIFORM, LD_DIST_ILD, LD_DIST_ALD, LD_DIST_EXPLICIT = 0, 1, 2, 3
 LD_TIME_CONST, LD_TIME_ITS, LD_TIME_DTS, LD_TIME_RAMP = 0, 1, 2, 3
 DIST = {"uniform": LD_DIST_UNIFORM, "ild": LD_DIST_ILD, "ald": LD_DIST_ALD, "explicit": LD_DIST_EXPLICIT}
 TIME = {"const": LD_TIME_CONST, "its": LD_TIME_ITS, "dts": LD_TIME_DTS, "ramp": LD_TIME_RAMP}
 ACT = {"swiglu": 0, "relu2": 1}
-GRAN = {"per_sequence": LD_PER_SEQUENCE, "per_batch": LD_PER_BATCH, "per_shard": LD_PER_SHARD}
+GRAN = {"per_sequence": LD_PER_SEQUENCE, "per_batch": LD_PER_BATCH, "per_shard": LD_PER_SHARD,
+        "per_token": LD_PER_TOKEN}
 
 
 class ld_config(ctypes.Structure):
@@ -217,18 +218,22 @@ def ld_forward_eval(h, execute, r_eval, wtab, x, workspace, stream=None):
                                  _ptr(workspace), _stream(stream)), "ld_forward_eval")
 
 
-def ld_get_masks(h, L, B, sublayer=False):
+def ld_get_masks(h, L, B, sublayer=False, S=None):
     """(mask, kept_idx, kept_cnt) as [L, B], [L, B], [L]; with sub-layer
-    granularity [2, L, B], [2, L, B], [2, L] (attention, then FFN)."""
+    granularity [2, L, B], [2, L, B], [2, L] (attention, then FFN).  Per
+    token (pass S): mask [L, B, S], kept_idx [L, B*S] (kept token rows), and
+    the kept-token counts [L] (leading axis 2 with sub-layer granularity)."""
     import numpy as np
     nm = 2 if sublayer else 1
-    mask = np.zeros(nm * L * B, dtype=np.uint8)
-    idx = np.zeros(nm * L * B, dtype=np.int32)
+    per = B * S if S else B
+    mask = np.zeros(nm * L * per, dtype=np.uint8)
+    idx = np.zeros(nm * L * per, dtype=np.int32)
     cnt = np.zeros(nm * L, dtype=np.int32)
     _check(lib().ld_get_masks(h, mask.ctypes.data, idx.ctypes.data, cnt.ctypes.data), "ld_get_masks")
+    mshape = (L, B, S) if S else (L, B)
     if sublayer:
-        return mask.reshape(2, L, B), idx.reshape(2, L, B), cnt.reshape(2, L)
-    return mask.reshape(L, B), idx.reshape(L, B), cnt
+        return mask.reshape((2,) + mshape), idx.reshape(2, L, per), cnt.reshape(2, L)
+    return mask.reshape(mshape), idx.reshape(L, per), cnt
 
 
 def ld_sync(h):
@@ -311,6 +316,7 @@ class LayerDropStack:
         import torch
         self.cfg = dict(cfg)
         self.sublayer = bool(sublayer)
+        self.per_token = granularity == "per_token" or granularity == LD_PER_TOKEN
         self.config = make_config(cfg, granularity, fp32_debug, b_offset, sublayer)
         self.h = ld_create(self.config)
         self.schedule = make_schedule(sched)
@@ -324,10 +330,11 @@ class LayerDropStack:
 
     def draw_masks(self, step, stream=None):
         ld_draw_masks(self.h, step, self.workspace, stream)
-        return ld_get_masks(self.h, self.cfg["L"], self.cfg["B"], self.sublayer)
+        return self.masks()
 
     def masks(self):
-        return ld_get_masks(self.h, self.cfg["L"], self.cfg["B"], self.sublayer)
+        return ld_get_masks(self.h, self.cfg["L"], self.cfg["B"], self.sublayer,
+                            self.cfg["S"] if self.per_token else None)
 
     def forward(self, step, wtab, x, stream=None):
         ld_forward(self.h, step, wtab, x, self.workspace, stream)

@@ -27,7 +27,7 @@ namespace {
 size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
 
 struct Layout {
-  size_t status, mask, kidx, kcnt, rcos, rsin, alibi;
+  size_t status, mask, kidx, kcnt, kseg, rcos, rsin, alibi;
   size_t layer0, per_layer;
   size_t xin, xh, qkv, o, lse, z, zh, gu, h, rstd1, rstd2;  // offsets inside a layer block
   size_t dy, dh, dgu, dzh, dz, dO, dqkv, dxh, Dvec, dqacc, part;
@@ -136,9 +136,11 @@ void make_layout(Handle* h) {
   };
   y.status = take(64);
   const size_t nm = c.sublayer ? 2 : 1;  // attention and FFN tables with sub-layer granularity
-  y.mask = take(nm * c.L * c.B);
-  y.kidx = take(nm * c.L * c.B * 4);
+  const size_t per = c.granularity == LD_PER_TOKEN ? R : (size_t)c.B;  // mask entries per (table, layer)
+  y.mask = take(nm * c.L * per);
+  y.kidx = take(nm * c.L * per * 4);
   y.kcnt = take(nm * c.L * 4);
+  y.kseg = take(nm * c.L * (c.B + 1) * 4);
   y.rcos = take((size_t)c.S * (c.Dh / 2) * 4);
   y.rsin = take((size_t)c.S * (c.Dh / 2) * 4);
   y.alibi = take((size_t)c.H * 4);
@@ -226,13 +228,50 @@ GemmArgs gemm_base() {
   return a;
 }
 
-// Forward/data-gradient product on the kept rows of layer l:
-// D[M x N] = alpha * A[M x K] B(n, k), M = kept_cnt * S (device-side).
-GemmArgs rows_gemm(const Handle* h, const int* cnt, int N, int K, const void* A, int lda, const void* B, int ldb,
+// The rows a block runs on.  Whole kept sequences: *cnt of them, `unit` =
+// S compact rows each, compact row m from sequence idx[m / S].  Per token:
+// *cnt compact rows (the kept-token count rounded up to 64), unit = 1, idx
+// the kept tokens' rows b S + s (-1 on the padding rows) and seg the
+// per-sequence segments (seg[B] = the kept-token count).
+struct Rows {
+  const int* cnt;
+  const int* idx;
+  const int* seg;
+  int unit;
+  const int* tok() const { return seg ? idx : nullptr; }
+};
+
+// Kept rows of table w (0: attention or layer mask, 1: FFN mask with
+// sub-layer granularity) of layer l.
+Rows rows_of(const Handle* h, void* ws, int w, int l) {
+  const ld_config& c = h->cfg;
+  const Layout& y = h->lay;
+  const bool tokg = c.granularity == LD_PER_TOKEN;
+  const size_t wl = (size_t)w * c.L + l;
+  Rows r;
+  r.cnt = at<int>(ws, y.kcnt) + wl;
+  r.idx = at<int>(ws, y.kidx) + wl * (tokg ? (size_t)c.B * c.S : (size_t)c.B);
+  r.seg = tokg ? at<int>(ws, y.kseg) + wl * (c.B + 1) : nullptr;
+  r.unit = tokg ? 1 : c.S;
+  return r;
+}
+
+// Per token: zero rows [kept tokens, kept tokens + 128) of a buffer the
+// attention reads (the tiles of the last sequence run past its kept tokens)
+// or a weight-gradient product contracts over (the padding rows).
+template <typename T>
+cudaError_t zero_tail(const Handle* h, const Rows& r, T* buf, int ld, int ncols, int planes, cudaStream_t st) {
+  if (!r.seg) return cudaSuccess;
+  return launch_zero_rows<T>(buf, ld, ncols, planes, (long long)h->max_rows, r.seg + h->cfg.B, 128, h->max_rows, st);
+}
+
+// Forward/data-gradient product on the kept rows:
+// D[M x N] = alpha * A[M x K] B(n, k), M = *cnt * unit (device-side).
+GemmArgs rows_gemm(const Handle* h, const Rows& r, int N, int K, const void* A, int lda, const void* B, int ldb,
                    int b_mn) {
   GemmArgs a = gemm_base();
-  a.M_cnt = cnt;
-  a.M_mul = h->cfg.S;
+  a.M_cnt = r.cnt;
+  a.M_mul = r.unit;
   a.M_cap = h->max_rows;
   a.N = N;
   a.K = K;
@@ -246,14 +285,15 @@ GemmArgs rows_gemm(const Handle* h, const int* cnt, int N, int K, const void* A,
 }
 
 // Weight-gradient product: dW[M x N] = sum over the kept rows m of
-// X1[m, i] X2[m, j]; the contraction extent is kept_cnt * S (device-side).
-GemmArgs wgrad_gemm(const Handle* h, const int* cnt, int M, int N, const void* X1, int ld1, const void* X2, int ld2,
+// X1[m, i] X2[m, j]; the contraction extent is *cnt * unit (device-side; per
+// token the padding rows hold zeros in X1 or X2).
+GemmArgs wgrad_gemm(const Handle* h, const Rows& r, int M, int N, const void* X1, int ld1, const void* X2, int ld2,
                     float* out) {
   GemmArgs a = gemm_base();
   a.M = M;
   a.N = N;
-  a.K_cnt = cnt;
-  a.K_mul = h->cfg.S;
+  a.K_cnt = r.cnt;
+  a.K_mul = r.unit;
   a.K_cap = h->max_rows;
   a.A = X1;
   a.lda = ld1;
@@ -284,22 +324,24 @@ const float* alibi_table(const Handle* h, void* ws) { return h->cfg.alibi ? at<f
 // Attention: tensor-core flash attention on the bf16 path, SIMT float32 on
 // the debug path.
 template <typename T>
-cudaError_t attn_fwd(const Handle* h, void* ws, const T* qkv, T* o, float* lse, const int* cnt, cudaStream_t st);
+cudaError_t attn_fwd(const Handle* h, void* ws, const T* qkv, T* o, float* lse, const Rows& r, cudaStream_t st);
 template <>
-cudaError_t attn_fwd<float>(const Handle* h, void* ws, const float* qkv, float* o, float* lse, const int* cnt,
+cudaError_t attn_fwd<float>(const Handle* h, void* ws, const float* qkv, float* o, float* lse, const Rows& r,
                             cudaStream_t st) {
   const ld_config& c = h->cfg;
-  return launch_attn_fwd_simt<float>(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, h->max_rows,
-                                     alibi_table(h, ws), st);
+  return launch_attn_fwd_simt<float>(qkv, h->nqkv, o, c.H * c.Dh, lse, r.cnt, c.S, c.H, c.Hkv, c.Dh, h->max_rows,
+                                     alibi_table(h, ws), r.seg, r.tok(), st);
 }
 template <>
-cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, float* lse, const int* cnt,
+cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, float* lse, const Rows& r,
                            cudaStream_t st) {
   const ld_config& c = h->cfg;
   if (attn_tc_supported(c.S, c.Dh))
-    return launch_attn_fwd_tc(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
-                              at<int>(ws, h->lay.status), st);
-  return launch_attn_fwd_mma(qkv, h->nqkv, o, c.H * c.Dh, lse, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws), st);
+    return launch_attn_fwd_tc(qkv, h->nqkv, o, c.H * c.Dh, lse, r.cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
+                              r.seg, at<int>(ws, h->lay.status), st);
+  // per-token granularity is refused at ld_create on this path
+  return launch_attn_fwd_mma(qkv, h->nqkv, o, c.H * c.Dh, lse, r.cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
+                             st);
 }
 
 // Attention backward: dq, dk, dv into dqkv with the inverse RoPE applied to
@@ -307,49 +349,52 @@ cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, 
 // the bf16 path; a separate rotation otherwise).
 template <typename T>
 cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const T* dO, const float* lse, float* Dvec,
-                     T* dqkv, const int* cnt, cudaStream_t st) {
+                     T* dqkv, const Rows& r, cudaStream_t st) {
   const ld_config& c = h->cfg;
   const bool rope = c.rope_theta != 0.0f;
   const float* rcos = rope ? at<float>(ws, h->lay.rcos) : nullptr;
   const float* rsin = rope ? at<float>(ws, h->lay.rsin) : nullptr;
-  cudaError_t e = launch_attn_rowdot<T>(dO, o, c.H * c.Dh, c.H, c.Dh, cnt, c.S, h->max_rows, Dvec, st);
+  cudaError_t e = launch_attn_rowdot<T>(dO, o, c.H * c.Dh, c.H, c.Dh, r.cnt, r.unit, h->max_rows, Dvec, st);
+  if (e == cudaSuccess) e = zero_tail<float>(h, r, Dvec, 1, 1, c.H, st);
   if (e != cudaSuccess) return e;
   if (sizeof(T) == 4) {
-    e = launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, cnt, c.S, c.H, c.Hkv, c.Dh,
-                                h->max_rows, alibi_table(h, ws), st);
+    e = launch_attn_bwd_simt<T>(qkv, h->nqkv, dO, c.H * c.Dh, lse, Dvec, dqkv, r.cnt, c.S, c.H, c.Hkv, c.Dh,
+                                h->max_rows, alibi_table(h, ws), r.seg, r.tok(), st);
     if (e != cudaSuccess || !rope) return e;
-    return launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1, st);
+    return launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, r.cnt, c.S, h->max_rows, 1, r.tok(),
+                                st);
   }
   float* dq_acc = at<float>(ws, h->lay.dqacc);
   const bf16* q16 = reinterpret_cast<const bf16*>(qkv);
   bf16* d16 = reinterpret_cast<bf16*>(dqkv);
   if (attn_bwd_tc_supported(c.S, c.Dh)) {
-    e = launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt,
-                           c.S, c.H, c.Hkv, c.B, rcos, rsin, alibi_table(h, ws), at<int>(ws, h->lay.status), st);
-  } else {
+    e = launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16, r.cnt,
+                           c.S, c.H, c.Hkv, c.B, rcos, rsin, alibi_table(h, ws), r.seg, r.tok(),
+                           at<int>(ws, h->lay.status), st);
+  } else {  // whole sequences only (per-token granularity is refused at ld_create on this path)
     e = launch_attn_bwd_mma(q16, h->nqkv, reinterpret_cast<const bf16*>(o), reinterpret_cast<const bf16*>(dO),
-                            c.H * c.Dh, lse, Dvec, dq_acc, d16, cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
+                            c.H * c.Dh, lse, Dvec, dq_acc, d16, r.cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
                             st);
     if (e == cudaSuccess && rope)  // the k heads of dqkv
-      e = launch_rope_apply<bf16>(d16 + (size_t)c.H * c.Dh, h->nqkv, c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 1,
-                                  st);
+      e = launch_rope_apply<bf16>(d16 + (size_t)c.H * c.Dh, h->nqkv, c.Hkv, c.Dh, rcos, rsin, r.cnt, c.S, h->max_rows,
+                                  1, nullptr, st);
   }
   if (e != cudaSuccess) return e;
-  return launch_dq_finish(dq_acc, d16, h->nqkv, c.H, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, st);
+  return launch_dq_finish(dq_acc, d16, h->nqkv, c.H, c.Dh, rcos, rsin, r.cnt, c.S, h->max_rows, r.tok(), st);
 }
 
 // One layer of the forward on the rows of its kept lists: the attention
-// block on (cnt, ki), the FFN block on (cntf, kif), branch scale s.  `lb` is
-// the layer's block of saved activations; x the float32 (or debug-path)
-// residual stream, updated in place.
+// block on ra, the FFN block on rf, branch scale s.  `lb` is the layer's
+// block of saved activations; x the float32 (or debug-path) residual
+// stream, updated in place.
 template <typename T>
-ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, float* x, const int* cnt, const int* ki,
-                        const int* cntf, const int* kif, float s, cudaStream_t st) {
+ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, float* x, const Rows& ra, const Rows& rf,
+                        float s, cudaStream_t st) {
   const ld_config& c = h->cfg;
   const Layout& y = h->lay;
   const bool f32 = sizeof(T) == 4;
   const bool fused_rope = !f32 && c.rope_theta != 0.0f && c.Dh >= 64;
-  const bool same_rows = cnt == cntf;  // both blocks keep the same rows
+  const bool same_rows = ra.cnt == rf.cnt;  // both blocks keep the same rows
   const int HD = c.H * c.Dh;
   float* rcos = at<float>(ws, y.rcos);
   float* rsin = at<float>(ws, y.rsin);
@@ -367,8 +412,8 @@ ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, flo
   const T* g1 = static_cast<const T*>(Wl.g1);
   const T* g2 = static_cast<const T*>(Wl.g2);
 
-  { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, ki, cnt, c.S, c.d, h->max_rows, g1, c.eps, xin, xh, rstd1, st)); }
-  GemmArgs a = rows_gemm(h, cnt, h->nqkv, c.d, xh, c.d, Wl.w_qkv, c.d, 0);
+  { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, ra.idx, ra.cnt, ra.unit, c.d, h->max_rows, g1, c.eps, xin, xh, rstd1, st)); }
+  GemmArgs a = rows_gemm(h, ra, h->nqkv, c.d, xh, c.d, Wl.w_qkv, c.d, 0);
   a.epi = EPI_STORE;
   a.D = qkv;
   a.ldd = h->nqkv;
@@ -378,30 +423,37 @@ ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, flo
     a.rope_sin = rsin;
     a.Dh = c.Dh;
     a.S = c.S;
+    a.pos_tok = ra.tok();
     a.rope_cols = (c.H + c.Hkv) * c.Dh;
   }
   { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
   if (c.rope_theta != 0.0f && !fused_rope)
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, cnt, c.S, h->max_rows, 0, st)); }
-  { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_fwd<T>(h, ws, qkv, o, lse, cnt, st)); }
-  a = rows_gemm(h, cnt, c.d, HD, o, HD, Wl.w_o, HD, 0);
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_rope_apply<T>(qkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, ra.cnt, c.S, h->max_rows, 0, ra.tok(), st)); }
+  if (ra.seg) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(zero_tail<T>(h, ra, qkv, h->nqkv, h->nqkv, 1, st)); }
+  { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_fwd<T>(h, ws, qkv, o, lse, ra, st)); }
+  if (ra.seg) {
+    Timed tm_(h, LD_KCLASS_ROWWISE, st);
+    LD_CHECK(zero_tail<T>(h, ra, o, HD, HD, 1, st));
+    LD_CHECK(zero_tail<float>(h, ra, lse, 1, 1, c.H, st));
+  }
+  a = rows_gemm(h, ra, c.d, HD, o, HD, Wl.w_o, HD, 0);
   a.epi = EPI_RESID;
   a.alpha = s;
   a.x = x;
   a.ldx = c.d;
-  a.kept_idx = ki;
-  a.S = c.S;
+  a.kept_idx = ra.idx;
+  a.S = ra.unit;
   a.save = same_rows ? z : nullptr;  // same rows feed the FFN block: keep a compact copy of Z
   a.ld_save = c.d;
   { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
   if (!same_rows) {  // the FFN block gathers its own rows of Z from the residual stream
     Timed tm_(h, LD_KCLASS_ROWWISE, st);
-    LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, kif, cntf, c.S, c.d, h->max_rows, g2, c.eps, z, zh, rstd2, st));
+    LD_CHECK(launch_rmsnorm_fwd<float, T>(x, 1, rf.idx, rf.cnt, rf.unit, c.d, h->max_rows, g2, c.eps, z, zh, rstd2, st));
   } else {
     Timed tm_(h, LD_KCLASS_ROWWISE, st);
-    LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ki, cnt, c.S, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st));
+    LD_CHECK(launch_rmsnorm_fwd<float, T>(z, 0, ra.idx, ra.cnt, ra.unit, c.d, h->max_rows, g2, c.eps, (float*)nullptr, zh, rstd2, st));
   }
-  a = rows_gemm(h, cntf, h->nf, c.d, zh, c.d, Wl.w_gu, c.d, 0);
+  a = rows_gemm(h, rf, h->nf, c.d, zh, c.d, Wl.w_gu, c.d, 0);
   a.epi = EPI_STORE;
   a.D = gu;
   a.ldd = h->nf;
@@ -413,16 +465,16 @@ ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, flo
   { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
   if (f32) {
     Timed tm_(h, LD_KCLASS_ROWWISE, st);
-    if (c.act) LD_CHECK(launch_relu2<T>(gu, (const T*)nullptr, hh, cntf, c.S, c.F, h->max_rows, st));
-    else LD_CHECK(launch_swiglu_fwd<T>(gu, hh, cntf, c.S, c.F, h->max_rows, st));
+    if (c.act) LD_CHECK(launch_relu2<T>(gu, (const T*)nullptr, hh, rf.cnt, rf.unit, c.F, h->max_rows, st));
+    else LD_CHECK(launch_swiglu_fwd<T>(gu, hh, rf.cnt, rf.unit, c.F, h->max_rows, st));
   }
-  a = rows_gemm(h, cntf, c.d, c.F, hh, c.F, Wl.w_d, c.F, 0);
+  a = rows_gemm(h, rf, c.d, c.F, hh, c.F, Wl.w_d, c.F, 0);
   a.epi = EPI_RESID;
   a.alpha = s;
   a.x = x;
   a.ldx = c.d;
-  a.kept_idx = kif;
-  a.S = c.S;
+  a.kept_idx = rf.idx;
+  a.S = rf.unit;
   a.save = nullptr;
   { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
   return LD_OK;
@@ -438,7 +490,8 @@ ld_status forward_prologue(Handle* h, const MaskParams& P, void* xv, float* x, v
   Timed tm_(h, LD_KCLASS_ROWWISE, st);
   LD_CHECK(cudaMemsetAsync(at<int>(ws, y.status), 0, sizeof(int), st));
   if (sizeof(T) == 2) LD_CHECK(launch_convert(xv, 0, x, 1, (long long)h->max_rows * c.d, st));
-  LD_CHECK(launch_mask_compact(P, at<unsigned char>(ws, y.mask), at<int>(ws, y.kidx), at<int>(ws, y.kcnt), st));
+  LD_CHECK(launch_mask_compact(P, at<unsigned char>(ws, y.mask), at<int>(ws, y.kidx), at<int>(ws, y.kcnt),
+                               at<int>(ws, y.kseg), st));
   if (c.rope_theta != 0.0f)
     LD_CHECK(launch_rope_table(at<float>(ws, y.rcos), at<float>(ws, y.rsin), c.S, c.Dh, (double)c.rope_theta, st));
   if (c.alibi) LD_CHECK(launch_alibi_table(at<float>(ws, y.alibi), c.H, st));
@@ -451,6 +504,7 @@ MaskParams mask_params(const Handle* h, long long step) {
   P.step = step;
   P.L = h->cfg.L;
   P.B = h->cfg.B;
+  P.S = h->cfg.S;
   P.granularity = h->cfg.granularity;
   P.b_offset = h->cfg.b_offset;
   P.nmask = h->cfg.sublayer ? 2 : 1;
@@ -466,22 +520,17 @@ ld_status forward_impl(Handle* h, long long step, const ld_layer_w* W, void* xv,
   // otherwise accumulate to several per cent of |X| at 32 layers.
   const bool f32 = sizeof(T) == 4;
   float* x = f32 ? static_cast<float*>(xv) : at<float>(ws, y.xres);
-  int* kidx = at<int>(ws, y.kidx);
-  int* kcnt = at<int>(ws, y.kcnt);
   MaskParams P = mask_params(h, step);
   std::vector<float> scale(c.L);
   step_rates(h, step, nullptr, P.thr, scale.data());
   ld_status r = forward_prologue<T>(h, P, xv, x, ws, st);
   if (r != LD_OK) return r;
   for (int l = 0; l < c.L; ++l) {
-    // kept lists of the attention block (cnt, ki) and of the FFN block
-    // (cntf, kif); the same list unless the masks are drawn per sub-layer
-    const int* cnt = kcnt + l;
-    const int* ki = kidx + (size_t)l * c.B;
-    const int* cntf = c.sublayer ? kcnt + c.L + l : cnt;
-    const int* kif = c.sublayer ? kidx + (size_t)(c.L + l) * c.B : ki;
-    r = forward_layer<T>(h, ws, at<char>(ws, y.layer0 + (size_t)l * y.per_layer), W[l], x, cnt, ki, cntf, kif,
-                         scale[l], st);
+    // kept rows of the attention block and of the FFN block; the same list
+    // unless the masks are drawn per sub-layer
+    const Rows ra = rows_of(h, ws, 0, l);
+    const Rows rf = c.sublayer ? rows_of(h, ws, 1, l) : ra;
+    r = forward_layer<T>(h, ws, at<char>(ws, y.layer0 + (size_t)l * y.per_layer), W[l], x, ra, rf, scale[l], st);
     if (r != LD_OK) return r;
   }
   if (!f32) {
@@ -507,14 +556,18 @@ ld_status forward_eval_impl(Handle* h, const unsigned char* execute, const float
   int* kcnt = at<int>(ws, y.kcnt);
   MaskParams P = mask_params(h, 0);
   P.nmask = 1;
+  P.granularity = LD_PER_SEQUENCE;  // every sequence runs every executed layer whole
   for (int l = 0; l < c.L; ++l) P.thr[l] = 0;  // p = 0: every sequence kept, lists 0 .. B-1
   ld_status r = forward_prologue<T>(h, P, xv, x, ws, st);
   if (r != LD_OK) return r;
   for (int l = 0; l < c.L; ++l) {
     if (!execute[l]) continue;
-    const int* cnt = kcnt + l;
-    const int* ki = kidx + (size_t)l * c.B;
-    r = forward_layer<T>(h, ws, at<char>(ws, y.layer0), W[l], x, cnt, ki, cnt, ki, r_eval ? r_eval[l] : 1.0f, st);
+    Rows ra;
+    ra.cnt = kcnt + l;
+    ra.idx = kidx + (size_t)l * c.B;
+    ra.seg = nullptr;
+    ra.unit = c.S;
+    r = forward_layer<T>(h, ws, at<char>(ws, y.layer0), W[l], x, ra, ra, r_eval ? r_eval[l] : 1.0f, st);
     if (r != LD_OK) return r;
   }
   if (!f32) {
@@ -530,8 +583,6 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
   const Layout& y = h->lay;
   const bool f32 = sizeof(T) == 4;
   float* dx = f32 ? static_cast<float*>(dxv) : at<float>(ws, y.dres);  // float32 residual gradient
-  int* kidx = at<int>(ws, y.kidx);
-  int* kcnt = at<int>(ws, y.kcnt);
   float* rcos = at<float>(ws, y.rcos);
   float* rsin = at<float>(ws, y.rsin);
   T* dy = at<T>(ws, y.dy);
@@ -551,10 +602,8 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
   }
 
   for (int l = c.L - 1; l >= 0; --l) {
-    const int* cnt = kcnt + l;  // attention block's kept list; FFN block's below
-    const int* ki = kidx + (size_t)l * c.B;
-    const int* cntf = c.sublayer ? kcnt + c.L + l : cnt;
-    const int* kif = c.sublayer ? kidx + (size_t)(c.L + l) * c.B : ki;
+    const Rows ra = rows_of(h, ws, 0, l);  // attention block's kept rows; FFN block's below
+    const Rows rf = c.sublayer ? rows_of(h, ws, 1, l) : ra;
     char* lb = at<char>(ws, y.layer0 + (size_t)l * y.per_layer);
     float* xin = reinterpret_cast<float*>(lb + y.xin);
     T* xh = reinterpret_cast<T*>(lb + y.xh);
@@ -572,8 +621,8 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     const float s = h->fwd_scale[l];
 
     // FFN branch: dy = r * dX^{l+1} on the kept rows.
-    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, kif, cntf, c.S, c.d, h->max_rows, s, dy, st)); }
-    GemmArgs a = rows_gemm(h, cntf, c.F, c.d, dy, c.d, W[l].w_d, c.F, 1);  // dh = dy W_d
+    { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, rf.idx, rf.cnt, rf.unit, c.d, h->max_rows, s, dy, st)); }
+    GemmArgs a = rows_gemm(h, rf, c.F, c.d, dy, c.d, W[l].w_d, c.F, 1);  // dh = dy W_d
     a.epi = EPI_STORE;
     a.D = dh;
     a.ldd = c.F;
@@ -586,44 +635,46 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
     if (f32) {
       Timed tm_(h, LD_KCLASS_ROWWISE, st);
-      if (c.act) LD_CHECK(launch_relu2<T>(gu, dh, dgu, cntf, c.S, c.F, h->max_rows, st));
-      else LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, cntf, c.S, c.F, h->max_rows, st));
+      if (c.act) LD_CHECK(launch_relu2<T>(gu, dh, dgu, rf.cnt, rf.unit, c.F, h->max_rows, st));
+      else LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, rf.cnt, rf.unit, c.F, h->max_rows, st));
     }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cntf, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
-    a = rows_gemm(h, cntf, c.d, h->nf, dgu, h->nf, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, rf, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
+    a = rows_gemm(h, rf, c.d, h->nf, dgu, h->nf, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
     a.epi = EPI_STORE_F32;
     a.D = dzh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cntf, h->nf, c.d, dgu, h->nf, zh, c.d, G[l].w_gu), st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, rf, h->nf, c.d, dgu, h->nf, zh, c.d, G[l].w_gu), st)); }
     // dZ = dX^{l+1} + RMSNorm_2 backward; dz = r * dZ for the attention branch
     // (written by the same kernel when both blocks keep the same rows)
     {
       Timed tm_(h, LD_KCLASS_ROWWISE, st);
-      LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, kif, cntf, c.S, c.d, h->max_rows, s,
+      LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, rf.idx, rf.cnt, rf.unit, c.d, h->max_rows, s,
                                      c.sublayer ? (T*)nullptr : dz, part, h->part_blocks, st));
     }
     { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g2, st)); }
-    if (c.sublayer) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, ki, cnt, c.S, c.d, h->max_rows, s, dz, st)); }
+    if (c.sublayer) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, ra.idx, ra.cnt, ra.unit, c.d, h->max_rows, s, dz, st)); }
     // attention branch
-    a = rows_gemm(h, cnt, HD, c.d, dz, c.d, W[l].w_o, HD, 1);  // dO = dz W_o
+    a = rows_gemm(h, ra, HD, c.d, dz, c.d, W[l].w_o, HD, 1);  // dO = dz W_o
     a.epi = EPI_STORE;
     a.D = dO;
     a.ldd = HD;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, c.d, HD, dz, c.d, o, HD, G[l].w_o), st)); }  // dW_o = dz^T o
-    { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_bwd<T>(h, ws, qkv, o, dO, lse, Dvec, dqkv, cnt, st)); }
-    a = rows_gemm(h, cnt, c.d, h->nqkv, dqkv, h->nqkv, W[l].w_qkv, c.d, 1);  // dxh = dqkv W_qkv
+    if (ra.seg) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(zero_tail<T>(h, ra, dO, HD, HD, 1, st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, ra, c.d, HD, dz, c.d, o, HD, G[l].w_o), st)); }  // dW_o = dz^T o
+    { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_bwd<T>(h, ws, qkv, o, dO, lse, Dvec, dqkv, ra, st)); }
+    if (ra.seg) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(zero_tail<T>(h, ra, dqkv, h->nqkv, h->nqkv, 1, st)); }
+    a = rows_gemm(h, ra, c.d, h->nqkv, dqkv, h->nqkv, W[l].w_qkv, c.d, 1);  // dxh = dqkv W_qkv
     a.epi = EPI_STORE_F32;
     a.D = dxh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, cnt, h->nqkv, c.d, dqkv, h->nqkv, xh, c.d, G[l].w_qkv), st)); }
+    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, ra, h->nqkv, c.d, dqkv, h->nqkv, xh, c.d, G[l].w_qkv), st)); }
     // dX^l = dZ + RMSNorm_1 backward
     {
       Timed tm_(h, LD_KCLASS_ROWWISE, st);
-      LD_CHECK(launch_rmsnorm_bwd<T>(dxh, xin, rstd1, g1, dx, ki, cnt, c.S, c.d, h->max_rows, 1.0f, (T*)nullptr,
-                                     part, h->part_blocks, st));
+      LD_CHECK(launch_rmsnorm_bwd<T>(dxh, xin, rstd1, g1, dx, ra.idx, ra.cnt, ra.unit, c.d, h->max_rows, 1.0f,
+                                     (T*)nullptr, part, h->part_blocks, st));
     }
     { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_colsum(part, h->part_blocks, c.d, G[l].g1, st)); }
   }
@@ -662,11 +713,19 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   if (c.d < 64 || c.d % 64 || c.F < 64 || c.F % 64 || c.d > 16384) return LD_ERR_SHAPE;
   if (c.Dh != 32 && c.Dh != 64 && c.Dh != 128) return LD_ERR_SHAPE;
   if (c.H < 1 || c.Hkv < 1 || c.H % c.Hkv || (c.H * c.Dh) % 64) return LD_ERR_SHAPE;
-  if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH && c.granularity != LD_PER_SHARD)
+  if (c.granularity != LD_PER_SEQUENCE && c.granularity != LD_PER_BATCH && c.granularity != LD_PER_SHARD &&
+      c.granularity != LD_PER_TOKEN)
     return LD_ERR_ARG;
   if (c.sublayer != 0 && c.sublayer != 1) return LD_ERR_ARG;
   if (c.alibi != 0 && c.alibi != 1) return LD_ERR_ARG;
   if (c.alibi && c.rope_theta != 0.0f) return LD_ERR_ARG;  // one position scheme
+  if (c.granularity == LD_PER_TOKEN) {
+    // the ALiBi distance would need the kept tokens' original positions in
+    // the attention kernels; the bf16 path runs its per-token attention on
+    // the tcgen05 kernels only
+    if (c.alibi) return LD_ERR_ARG;
+    if (!c.fp32_debug && (c.Dh != 128 || c.S % 128)) return LD_ERR_SHAPE;
+  }
   if (c.act != LD_ACT_SWIGLU && c.act != LD_ACT_RELU2) return LD_ERR_ARG;
   if (c.b_offset < 0 || (long long)c.b_offset + c.B > 0x7fffffffll) return LD_ERR_ARG;
   if ((long long)c.B * c.S > (1ll << 30)) return LD_ERR_SHAPE;
@@ -730,18 +789,12 @@ ld_status ld_draw_masks(void* handle, long long step, void* ws, void* stream) {
   Handle* h = H(handle);
   if (!h->have_sched) return LD_ERR_STATE;
   const Layout& y = h->lay;
-  MaskParams P;
-  P.seed = h->sched.seed;
-  P.step = step;
-  P.L = h->cfg.L;
-  P.B = h->cfg.B;
-  P.granularity = h->cfg.granularity;
-  P.b_offset = h->cfg.b_offset;
-  P.nmask = h->cfg.sublayer ? 2 : 1;
+  MaskParams P = mask_params(h, step);
   step_rates(h, step, nullptr, P.thr, nullptr);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   LD_CHECK(cudaMemsetAsync(at<int>(ws, y.status), 0, sizeof(int), st));
-  LD_CHECK(launch_mask_compact(P, at<unsigned char>(ws, y.mask), at<int>(ws, y.kidx), at<int>(ws, y.kcnt), st));
+  LD_CHECK(launch_mask_compact(P, at<unsigned char>(ws, y.mask), at<int>(ws, y.kidx), at<int>(ws, y.kcnt),
+                               at<int>(ws, y.kseg), st));
   h->last_ws = ws;
   h->last_stream = st;
   h->have_masks = true;
@@ -821,12 +874,20 @@ ld_status ld_get_masks(void* handle, unsigned char* mask, int* kept_idx, int* ke
   Handle* h = H(handle);
   if (!h->have_masks) return LD_ERR_STATE;
   const Layout& y = h->lay;
-  const size_t nm = h->cfg.sublayer ? 2 : 1;
-  const size_t LB = nm * h->cfg.L * h->cfg.B;
+  const ld_config& c = h->cfg;
+  const bool tokg = c.granularity == LD_PER_TOKEN;
+  const size_t nm = c.sublayer ? 2 : 1;
+  const size_t LB = nm * c.L * (tokg ? (size_t)c.B * c.S : (size_t)c.B);
   LD_CHECK(cudaStreamSynchronize(h->last_stream));
   if (mask) LD_CHECK(cudaMemcpy(mask, at<unsigned char>(h->last_ws, y.mask), LB, cudaMemcpyDeviceToHost));
   if (kept_idx) LD_CHECK(cudaMemcpy(kept_idx, at<int>(h->last_ws, y.kidx), LB * 4, cudaMemcpyDeviceToHost));
-  if (kept_cnt) LD_CHECK(cudaMemcpy(kept_cnt, at<int>(h->last_ws, y.kcnt), nm * h->cfg.L * 4, cudaMemcpyDeviceToHost));
+  if (kept_cnt && !tokg)
+    LD_CHECK(cudaMemcpy(kept_cnt, at<int>(h->last_ws, y.kcnt), nm * c.L * 4, cudaMemcpyDeviceToHost));
+  if (kept_cnt && tokg) {  // the kept-token counts: the last segment offset of each table
+    std::vector<int> seg(nm * c.L * (c.B + 1));
+    LD_CHECK(cudaMemcpy(seg.data(), at<int>(h->last_ws, y.kseg), seg.size() * 4, cudaMemcpyDeviceToHost));
+    for (size_t i = 0; i < nm * c.L; ++i) kept_cnt[i] = seg[i * (c.B + 1) + c.B];
+  }
   return LD_OK;
 }
 

@@ -383,8 +383,8 @@ __global__ void __launch_bounds__(128) attn_bwd_kernel(const bf16* __restrict__ 
 // (i, i + Dh/2) at the row's position), written as bf16 into dqkv.
 __global__ void dq_finish_kernel(const float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, int H, int Dh,
                                  float c, const float* __restrict__ rcos, const float* __restrict__ rsin,
-                                 const int* __restrict__ cnt, int S) {
-  const long long M = (long long)(*cnt) * S;
+                                 const int* __restrict__ cnt, int S, const int* __restrict__ tok) {
+  const long long M = tok ? (long long)(*cnt) : (long long)(*cnt) * S;
   const int half = Dh / 2, HD = H * Dh;
   const int per_row = H * (half / 4);
   const long long total = M * per_row;
@@ -398,7 +398,7 @@ __global__ void dq_finish_kernel(const float* __restrict__ dq_acc, bf16* __restr
     const float4 b = *reinterpret_cast<const float4*>(src + half);
     float x1[4] = {c * a.x, c * a.y, c * a.z, c * a.w}, x2[4] = {c * b.x, c * b.y, c * b.z, c * b.w};
     if (rcos) {
-      const int pos = (int)(m % S);
+      const int pos = row_pos(tok, S, m);
       const float4 cv = *reinterpret_cast<const float4*>(rcos + (size_t)pos * half + i);
       const float4 sv = *reinterpret_cast<const float4*>(rsin + (size_t)pos * half + i);
       const float cs[4] = {cv.x, cv.y, cv.z, cv.w}, sn[4] = {sv.x, sv.y, sv.z, sv.w};
@@ -473,13 +473,13 @@ cudaError_t launch_attn_bwd_mma(const bf16* qkv, int ldqkv, const bf16* o, const
 }
 
 cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const float* rcos,
-                             const float* rsin, const int* cnt, int S, int max_rows, cudaStream_t st) {
+                             const float* rsin, const int* cnt, int S, int max_rows, const int* tok, cudaStream_t st) {
   long long work = (long long)max_rows * H * (Dh / 8);
   long long grid = (work + 255) / 256;
   const long long cap = (long long)device_sm_count() * 8;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  dq_finish_kernel<<<(int)grid, 256, 0, st>>>(dq_acc, dqkv, ldqkv, H, Dh, rsqrtf((float)Dh), rcos, rsin, cnt, S);
+  dq_finish_kernel<<<(int)grid, 256, 0, st>>>(dq_acc, dqkv, ldqkv, H, Dh, rsqrtf((float)Dh), rcos, rsin, cnt, S, tok);
   return cudaGetLastError();
 }
 

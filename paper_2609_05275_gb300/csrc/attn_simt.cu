@@ -7,9 +7,31 @@
 // floor(h*Hkv/H).  Rows are compact: the
 // kept sequence s occupies rows s*S .. s*S+S-1 of qkv, whose columns are
 // [Q heads | K heads | V heads].  lse[h][m] = log sum_j exp(c q_m . k_j).
+// With per-token kept lists (seg, tok) the kept tokens of sequence b occupy
+// rows seg[b] .. seg[b+1]-1 and attend among themselves in that order; rows
+// with tok[m] < 0 (padding) belong to no sequence and are skipped.
 #include "ld_internal.cuh"
 
 namespace ldk {
+
+// Sequence of compact row m: its first row seq0, its index pos in the
+// sequence and the sequence's length; false for a padding row.
+__device__ __forceinline__ bool row_seq(long long m, int S, const int* seg, const int* tok, long long& seq0,
+                                        int& pos, int& len) {
+  if (!seg) {
+    seq0 = (m / S) * S;
+    pos = (int)(m % S);
+    len = S;
+    return true;
+  }
+  const int t = tok[m];
+  if (t < 0) return false;
+  const int b = t / S;
+  seq0 = seg[b];
+  pos = (int)(m - seq0);
+  len = seg[b + 1] - seg[b];
+  return true;
+}
 
 __device__ __forceinline__ float wsum(float v) {
 #pragma unroll
@@ -28,18 +50,20 @@ template <typename T>
 __global__ void __launch_bounds__(128) attn_fwd_simt_kernel(const T* __restrict__ qkv, int ldq, T* __restrict__ o,
                                                             int ldo, float* __restrict__ lse, int lse_ld,
                                                             const int* __restrict__ cnt, int S, int H, int Hkv,
-                                                            int Dh, const float* __restrict__ alibi) {
+                                                            int Dh, const float* __restrict__ alibi,
+                                                            const int* __restrict__ seg, const int* __restrict__ tok) {
   __shared__ float qs[kWarps][128];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long M = (long long)(*cnt) * S;
+  const long long M = seg ? (long long)(*cnt) : (long long)(*cnt) * S;
   const float c = 1.0f / sqrtf((float)Dh);
   const int ne = Dh / 32;
   const long long nwarps = (long long)gridDim.x * kWarps;
   for (long long it = (long long)blockIdx.x * kWarps + w; it < M * H; it += nwarps) {
     const long long m = it / H;
     const int h = (int)(it % H);
-    const long long seq0 = (m / S) * S;
-    const int pos = (int)(m % S);
+    long long seq0;
+    int pos, len;
+    if (!row_seq(m, S, seg, tok, seq0, pos, len)) continue;
     const int g = (h * Hkv) / H;
     for (int i = lane; i < Dh; i += 32) qs[w][i] = c * to_f(qkv[m * ldq + (long long)h * Dh + i]);
     __syncwarp();
@@ -79,19 +103,21 @@ __global__ void __launch_bounds__(128) attn_dq_simt_kernel(const T* __restrict__
                                                            const float* __restrict__ lse,
                                                            const float* __restrict__ Dvec, int lse_ld,
                                                            T* __restrict__ dqkv, const int* __restrict__ cnt, int S,
-                                                           int H, int Hkv, int Dh, const float* __restrict__ alibi) {
+                                                           int H, int Hkv, int Dh, const float* __restrict__ alibi,
+                                                           const int* __restrict__ seg, const int* __restrict__ tok) {
   __shared__ float qs[kWarps][128];
   __shared__ float ds_[kWarps][128];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long M = (long long)(*cnt) * S;
+  const long long M = seg ? (long long)(*cnt) : (long long)(*cnt) * S;
   const float c = 1.0f / sqrtf((float)Dh);
   const int ne = Dh / 32;
   const long long nwarps = (long long)gridDim.x * kWarps;
   for (long long it = (long long)blockIdx.x * kWarps + w; it < M * H; it += nwarps) {
     const long long m = it / H;
     const int h = (int)(it % H);
-    const long long seq0 = (m / S) * S;
-    const int pos = (int)(m % S);
+    long long seq0;
+    int pos, len;
+    if (!row_seq(m, S, seg, tok, seq0, pos, len)) continue;
     const int g = (h * Hkv) / H;
     for (int i = lane; i < Dh; i += 32) {
       qs[w][i] = c * to_f(qkv[m * ldq + (long long)h * Dh + i]);
@@ -135,11 +161,12 @@ __global__ void __launch_bounds__(128) attn_dkv_simt_kernel(const T* __restrict_
                                                             const float* __restrict__ Dvec, int lse_ld,
                                                             T* __restrict__ dqkv, const int* __restrict__ cnt,
                                                             int S, int H, int Hkv, int Dh,
-                                                            const float* __restrict__ alibi) {
+                                                            const float* __restrict__ alibi,
+                                                            const int* __restrict__ seg, const int* __restrict__ tok) {
   __shared__ float ks[kWarps][128];
   __shared__ float vs[kWarps][128];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long M = (long long)(*cnt) * S;
+  const long long M = seg ? (long long)(*cnt) : (long long)(*cnt) * S;
   const float c = 1.0f / sqrtf((float)Dh);
   const int ne = Dh / 32;
   const int grp = H / Hkv;
@@ -147,8 +174,9 @@ __global__ void __launch_bounds__(128) attn_dkv_simt_kernel(const T* __restrict_
   for (long long it = (long long)blockIdx.x * kWarps + w; it < M * Hkv; it += nwarps) {
     const long long mk = it / Hkv;
     const int g = (int)(it % Hkv);
-    const long long seq0 = (mk / S) * S;
-    const int pos = (int)(mk % S);
+    long long seq0;
+    int pos, len;
+    if (!row_seq(mk, S, seg, tok, seq0, pos, len)) continue;
     for (int i = lane; i < Dh; i += 32) {
       ks[w][i] = c * to_f(qkv[mk * ldq + (long long)(H + g) * Dh + i]);
       vs[w][i] = to_f(qkv[mk * ldq + (long long)(H + Hkv + g) * Dh + i]);
@@ -156,10 +184,10 @@ __global__ void __launch_bounds__(128) attn_dkv_simt_kernel(const T* __restrict_
     __syncwarp();
     float dk[4] = {0.f, 0.f, 0.f, 0.f}, dv[4] = {0.f, 0.f, 0.f, 0.f};
     for (int h = g * grp; h < (g + 1) * grp; ++h) {
-      for (int i0 = pos; i0 < S; i0 += 32) {
+      for (int i0 = pos; i0 < len; i0 += 32) {
         const int i = i0 + lane;
         float p = 0.f, dsv = 0.f;
-        if (i < S) {
+        if (i < len) {
           const long long mq = seq0 + i;
           const T* qr = qkv + mq * ldq + (long long)h * Dh;
           const T* dr = dO + mq * ldo + (long long)h * Dh;
@@ -172,7 +200,7 @@ __global__ void __launch_bounds__(128) attn_dkv_simt_kernel(const T* __restrict_
           p = expf(s - lse[(size_t)h * lse_ld + mq]);
           dsv = p * (dp - Dvec[(size_t)h * lse_ld + mq]);
         }
-        const int iend = min(32, S - i0);
+        const int iend = min(32, len - i0);
         for (int ii = 0; ii < iend; ++ii) {
           const float pi = __shfl_sync(0xffffffffu, p, ii);
           const float di = __shfl_sync(0xffffffffu, dsv, ii);
@@ -204,33 +232,35 @@ static int attn_grid(long long items) {
 
 template <typename T>
 cudaError_t launch_attn_fwd_simt(const T* qkv, int ldqkv, T* o, int ldo, float* lse, const int* cnt, int S, int H,
-                                 int Hkv, int Dh, int max_rows, const float* alibi, cudaStream_t st) {
+                                 int Hkv, int Dh, int max_rows, const float* alibi, const int* seg, const int* tok,
+                                 cudaStream_t st) {
   attn_fwd_simt_kernel<T><<<attn_grid((long long)max_rows * H), 128, 0, st>>>(qkv, ldqkv, o, ldo, lse, max_rows,
-                                                                               cnt, S, H, Hkv, Dh, alibi);
+                                                                               cnt, S, H, Hkv, Dh, alibi, seg, tok);
   return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t launch_attn_bwd_simt(const T* qkv, int ldqkv, const T* dO, int ldo, const float* lse, const float* Dvec,
                                  T* dqkv, const int* cnt, int S, int H, int Hkv, int Dh, int max_rows,
-                                 const float* alibi, cudaStream_t st) {
-  attn_dq_simt_kernel<T><<<attn_grid((long long)max_rows * H), 128, 0, st>>>(qkv, ldqkv, dO, ldo, lse, Dvec, max_rows,
-                                                                             dqkv, cnt, S, H, Hkv, Dh, alibi);
+                                 const float* alibi, const int* seg, const int* tok, cudaStream_t st) {
+  attn_dq_simt_kernel<T><<<attn_grid((long long)max_rows * H), 128, 0, st>>>(
+      qkv, ldqkv, dO, ldo, lse, Dvec, max_rows, dqkv, cnt, S, H, Hkv, Dh, alibi, seg, tok);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   attn_dkv_simt_kernel<T><<<attn_grid((long long)max_rows * Hkv), 128, 0, st>>>(
-      qkv, ldqkv, dO, ldo, lse, Dvec, max_rows, dqkv, cnt, S, H, Hkv, Dh, alibi);
+      qkv, ldqkv, dO, ldo, lse, Dvec, max_rows, dqkv, cnt, S, H, Hkv, Dh, alibi, seg, tok);
   return cudaGetLastError();
 }
 
 template cudaError_t launch_attn_fwd_simt<float>(const float*, int, float*, int, float*, const int*, int, int, int,
-                                                 int, int, const float*, cudaStream_t);
+                                                 int, int, const float*, const int*, const int*, cudaStream_t);
 template cudaError_t launch_attn_fwd_simt<bf16>(const bf16*, int, bf16*, int, float*, const int*, int, int, int, int,
-                                                int, const float*, cudaStream_t);
+                                                int, const float*, const int*, const int*, cudaStream_t);
 template cudaError_t launch_attn_bwd_simt<float>(const float*, int, const float*, int, const float*, const float*,
                                                  float*, const int*, int, int, int, int, int, const float*,
-                                                 cudaStream_t);
+                                                 const int*, const int*, cudaStream_t);
 template cudaError_t launch_attn_bwd_simt<bf16>(const bf16*, int, const bf16*, int, const float*, const float*, bf16*,
-                                                const int*, int, int, int, int, int, const float*, cudaStream_t);
+                                                const int*, int, int, int, int, int, const float*, const int*,
+                                                const int*, cudaStream_t);
 
 }  // namespace ldk

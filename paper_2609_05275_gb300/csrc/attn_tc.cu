@@ -60,7 +60,7 @@ template <int DH, bool ALIBI>
 __global__ void __launch_bounds__(320, 1)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
                        int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv,
-                       const float* __restrict__ alibi, int* status) {
+                       const float* __restrict__ alibi, const int* __restrict__ seg, int* status) {
   constexpr int NSLAB = DH / 64;
   constexpr uint32_t TILE = NSLAB * SLAB;  // one 128 x DH bf16 tile
   constexpr int NSK = 3, NSV = 2;          // K and V stages
@@ -88,12 +88,24 @@ __global__ void __launch_bounds__(320, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 4);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
+  // sequence: rows row0 .. row0+len-1 (a whole kept sequence, or with `seg`
+  // the kept tokens of sequence blockIdx.y); the rows of the last tile past
+  // len belong to other sequences: causality hides them from the valid
+  // queries, and their own results are not stored
   const int seq = blockIdx.y;
-  if (seq >= *cnt) return;
+  int row0, len;
+  if (seg) {
+    row0 = seg[seq];
+    len = seg[seq + 1] - row0;
+  } else {
+    if (seq >= *cnt) return;
+    row0 = seq * S;
+    len = S;
+  }
   const int nqt = S / 128;
   const int qt = nqt - 1 - blockIdx.z;  // slowest grid dimension: heaviest tiles are dispatched first
+  if (qt * 128 >= len) return;
   const int h = blockIdx.x, g = (h * Hkv) / H;
-  const int row0 = seq * S;
   const int nkt = qt + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -339,6 +351,7 @@ __global__ void __launch_bounds__(320, 1)
       const bool got = warp_wait(xb, nkt & 1, abort_flag, status);
       const float lt = l + (got ? xsum[half ^ 1][r] : 0.f);
       const float inv = 1.0f / lt;
+      const bool valid = qt * 128 + r < len;
       bf16* orow = o + (long long)(row0 + qt * 128 + r) * ldo + (long long)h * DH + half * (DH / 2);
 #pragma unroll 1
       for (int c = 0; c < OC; ++c) {
@@ -351,10 +364,10 @@ __global__ void __launch_bounds__(320, 1)
           __nv_bfloat162* hb = reinterpret_cast<__nv_bfloat162*>(&q);
 #pragma unroll
           for (int k = 0; k < 4; ++k) hb[k] = __floats2bfloat162_rn(t[8 * i + 2 * k] * inv, t[8 * i + 2 * k + 1] * inv);
-          dst[i] = q;
+          if (valid) dst[i] = q;
         }
       }
-      if (half == 0) lse[(size_t)h * lse_ld + row0 + qt * 128 + r] = (m_used + log2f(lt)) * kLn2;
+      if (half == 0 && valid) lse[(size_t)h * lse_ld + row0 + qt * 128 + r] = (m_used + log2f(lt)) * kLn2;
     }
   }
 
@@ -368,7 +381,7 @@ __global__ void __launch_bounds__(320, 1)
 
 template <int DH, bool ALIBI>
 cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
-                   int max_seqs, const float* alibi, int* status, cudaStream_t st) {
+                   int max_seqs, const float* alibi, const int* seg, int* status, cudaStream_t st) {
   // Q, 3 K and 2 V tiles + the row max / sum exchange + alignment + barriers
   constexpr size_t smem = (size_t)(DH / 64) * SLAB * 6 + 6 * 128 * 4 + 1024 + 256;
   static bool attr = false;
@@ -381,7 +394,8 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   dim3 grid(H, max_seqs, S / 128);
-  attn_fwd_tc_kernel<DH, ALIBI><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi, status);
+  attn_fwd_tc_kernel<DH, ALIBI><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi, seg,
+                                                         status);
   return cudaGetLastError();
 }
 
@@ -407,6 +421,13 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
+// Values 4 e4 .. 4 e4 + 3 of p (shared memory); p is 16-byte aligned when
+// off == 0 (warp-uniform), else read one by one.
+__device__ __forceinline__ float4 ld4s(const float* p, int e4, int off) {
+  if (off == 0) return reinterpret_cast<const float4*>(p)[e4];
+  return make_float4(p[4 * e4], p[4 * e4 + 1], p[4 * e4 + 2], p[4 * e4 + 3]);
+}
+
 template <bool ALIBI>
 __global__ void __launch_bounds__(448, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
@@ -414,7 +435,8 @@ __global__ void __launch_bounds__(448, 1)
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
-                       const float* __restrict__ alibi, int* status) {
+                       const float* __restrict__ alibi, const int* __restrict__ seg, const int* __restrict__ tok,
+                       int* status) {
   constexpr int DH = 128;
   constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
   constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
@@ -427,8 +449,13 @@ __global__ void __launch_bounds__(448, 1)
   uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
   uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
   float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
-  float* vecs = dqs + 64 * DH;                         // [NST][lse 64 | D 64]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * 128);
+  // [NST][lse 68 | D 68]: the 64 values of a step start at float `voff` of
+  // each half (a sequence's rows start anywhere with per-token kept lists,
+  // and a bulk copy needs a 16-byte aligned source, so 68 are copied from
+  // the aligned-down address)
+  float* vecs = dqs + 64 * DH;
+  constexpr int VS = 136;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * VS);
   uint64_t* kv_full = bars;
   uint64_t* ld_full = bars + 1;          // [NST]
   uint64_t* ld_empty = ld_full + NST;    // [NST]
@@ -442,11 +469,21 @@ __global__ void __launch_bounds__(448, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sdp_full + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
+  // rows row0 .. row0+len-1 as in the forward; queries past len (the last
+  // query tile) get P = dS = 0, keys past len are never stored
   const int seq = blockIdx.y;
-  if (seq >= *cnt) return;
+  int row0, len;
+  if (seg) {
+    row0 = seg[seq];
+    len = seg[seq + 1] - row0;
+  } else {
+    if (seq >= *cnt) return;
+    row0 = seq * S;
+    len = S;
+  }
   const int kt = blockIdx.z, g = blockIdx.x, grp = H / Hkv;  // heaviest key tiles (kt = 0) dispatched first
-  const int row0 = seq * S;
-  const int nq = S / 64, q0 = 2 * kt;          // query tiles q0 .. nq-1 overlap or follow the keys
+  if (kt * 128 >= len) return;
+  const int nq = (len + 63) / 64, q0 = 2 * kt;  // query tiles q0 .. nq-1 overlap or follow the keys
   const int n_it = grp * (nq - q0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -490,14 +527,14 @@ __global__ void __launch_bounds__(448, 1)
         const int b = i % NST;
         const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
         if (!mbar_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
-        mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 512);
+        mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 2 * 272);
         for (int c = 0; c < 2; ++c) {
           tma_load_2d(Qs + b * QT + c * HSLAB, &tmq, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
           tma_load_2d(dOs + b * QT + c * HSLAB, &tmo, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
         }
-        const size_t vo = (size_t)h * lse_ld + row0 + qt * 64;
-        bulk_load(vecs + b * 128, lse + vo, 256, &ld_full[b]);
-        bulk_load(vecs + b * 128 + 64, Dvec + vo, 256, &ld_full[b]);
+        const size_t vo = ((size_t)h * lse_ld + row0 + qt * 64) & ~(size_t)3;  // lse_ld % 4 == 0
+        bulk_load(vecs + b * VS, lse + vo, 272, &ld_full[b]);
+        bulk_load(vecs + b * VS + 68, Dvec + vo, 272, &ld_full[b]);
         ++issued;
       }
       if (*abort_flag) {
@@ -573,6 +610,7 @@ __global__ void __launch_bounds__(448, 1)
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const int voff = row0 & 3;  // first value of a step in its lse / D stage (see vecs)
     const float sl2 = kLog2e * rsqrtf((float)DH);
     bool ok = true;
     for (int i = 0; i < n_it; ++i) {
@@ -590,12 +628,14 @@ __global__ void __launch_bounds__(448, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
-      const float4* lv4 = reinterpret_cast<const float4*>(vecs + b * 128 + half * 32);       // lse of the 32 queries
-      const float4* dv4 = reinterpret_cast<const float4*>(vecs + b * 128 + 64 + half * 32);  // D of the 32 queries
+      const float* lsrc = vecs + b * VS + voff + half * 32;       // lse of the 32 queries
+      const float* dsrc = vecs + b * VS + 68 + voff + half * 32;  // D of the 32 queries
       const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
+      const int qlim = len - (qt * 64 + half * 32);  // and exists iff c < qlim (warp-uniform)
       uint32_t pk[16], dk[16];
-      // pairs of queries on the packed fp32 pipe; the causal mask only on
-      // warps whose 32 keys are not all visible to the 32 queries (warp-uniform)
+      // pairs of queries on the packed fp32 pipe; the mask only on warps
+      // whose 32 keys are not all visible to the 32 queries, or whose queries
+      // run past the sequence (warp-uniform)
       auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
         const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
@@ -604,7 +644,7 @@ __global__ void __launch_bounds__(448, 1)
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
         for (int e4 = 0; e4 < 8; ++e4) {
-          const float4 lq = lv4[e4], dq = dv4[e4];
+          const float4 lq = ld4s(lsrc, e4, voff), dq = ld4s(dsrc, e4, voff);
           uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
           if constexpr (ALIBI) {
 #pragma unroll
@@ -620,19 +660,24 @@ __global__ void __launch_bounds__(448, 1)
             float x0, x1;
             f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2, nl[h2]), x0, x1);
             float p0 = ex2(x0), p1 = ex2(x1);
+            const bool v0 = !MASK || (qbase + c >= 0 && c < qlim), v1 = !MASK || (qbase + c + 1 >= 0 && c + 1 < qlim);
             if constexpr (MASK) {
-              p0 = (qbase + c >= 0) ? p0 : 0.f;
-              p1 = (qbase + c + 1 >= 0) ? p1 : 0.f;
+              p0 = v0 ? p0 : 0.f;
+              p1 = v1 ? p1 : 0.f;
             }
             const uint64_t pp = f2_pack(p0, p1);
             float d0, d1;
             f2_unpack(f2_mul(pp, f2_sub(f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1])), dd[h2])), d0, d1);
+            if constexpr (MASK) {  // rows past the sequence may hold anything: select, do not multiply
+              d0 = v0 ? d0 : 0.f;
+              d1 = v1 ? d1 : 0.f;
+            }
             pk[c >> 1] = bf16x2_bits(p0, p1);
             dk[c >> 1] = bf16x2_bits(d0, d1);
           }
         }
       };
-      if (__shfl_sync(0xffffffffu, qbase, 31) >= 0) pass(std::false_type{});
+      if (__shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 32) pass(std::false_type{});
       else pass(std::true_type{});
       // the MMAs of step i-2 must be done with buffer i & 1 before it is rewritten
       const int pb = i & 1;
@@ -653,9 +698,11 @@ __global__ void __launch_bounds__(448, 1)
     }
     if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
       tc_fence_after();
+      const bool kvalid = key < len;
       if (half == 0) {
         // dK (times c) with the inverse rotation at the key's position
         const float c = rsqrtf((float)DH);
+        const int kpos = row_pos(tok, S, row0 + key);
         bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
 #pragma unroll 1
         for (int cc = 0; cc < 2; ++cc) {
@@ -667,14 +714,16 @@ __global__ void __launch_bounds__(448, 1)
             const float p1 = c * k1[e], p2 = c * k2[e];
             float cs = 1.f, sn = 0.f;
             if (rcos) {
-              cs = rcos[(size_t)key * 64 + cc * 32 + e];
-              sn = rsin[(size_t)key * 64 + cc * 32 + e];
+              cs = rcos[(size_t)kpos * 64 + cc * 32 + e];
+              sn = rsin[(size_t)kpos * 64 + cc * 32 + e];
             }
             k1[e] = p1 * cs + p2 * sn;
             k2[e] = p2 * cs - p1 * sn;
           }
-          st_bf16x32_(krow + cc * 32, k1);
-          st_bf16x32_(krow + 64 + cc * 32, k2);
+          if (kvalid) {
+            st_bf16x32_(krow + cc * 32, k1);
+            st_bf16x32_(krow + 64 + cc * 32, k2);
+          }
         }
       } else {
         bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
@@ -682,7 +731,7 @@ __global__ void __launch_bounds__(448, 1)
         for (int cc = 0; cc < DH / 32; ++cc) {
           float u[32];
           tmem_ld32(t_dv + cc * 32 + lane_off, u);
-          st_bf16x32_(vrow + cc * 32, u);
+          if (kvalid) st_bf16x32_(vrow + cc * 32, u);
         }
       }
     }
@@ -731,10 +780,11 @@ __global__ void __launch_bounds__(448, 1)
 template <bool ALIBI>
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
-                   const float* rsin, const float* alibi, int* status, cudaStream_t st) {
+                   const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
+                   cudaStream_t st) {
   // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
-  // vectors + dQ staging + alignment + barriers = 232,192 bytes (of 232,448)
-  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 128 * 4 + 64 * 128 * 4 + 1024 + 256;
+  // vectors + dQ staging + alignment + barriers = 232,288 bytes (of 232,448)
+  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 136 * 4 + 64 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
@@ -750,7 +800,7 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
   dim3 grid(Hkv, max_seqs, S / 128);
   attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
-                                                     H, Hkv, rcos, rsin, alibi, status);
+                                                     H, Hkv, rcos, rsin, alibi, seg, tok, status);
   return cudaGetLastError();
 }
 }  // namespace
@@ -761,25 +811,26 @@ bool attn_bwd_tc_supported(int S, int Dh) { return S % 128 == 0 && Dh == 128; }
 
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, int* status,
-                               cudaStream_t st) {
+                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, const int* seg,
+                               const int* tok, int* status, cudaStream_t st) {
   cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)max_seqs * S * H * 128 * sizeof(float), st);
   if (e != cudaSuccess) return e;
   if (alibi)
     return bwd_tc<true>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
-                        status, st);
+                        seg, tok, status, st);
   return bwd_tc<false>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
-                       status, st);
+                       seg, tok, status, st);
 }
 
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
-                               int Hkv, int Dh, int max_seqs, const float* alibi, int* status, cudaStream_t st) {
+                               int Hkv, int Dh, int max_seqs, const float* alibi, const int* seg, int* status,
+                               cudaStream_t st) {
   if (alibi) {
-    if (Dh == 64) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
-    return fwd_tc<128, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
+    if (Dh == 64) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+    return fwd_tc<128, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
   }
-  if (Dh == 64) return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
-  return fwd_tc<128, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, status, st);
+  if (Dh == 64) return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  return fwd_tc<128, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
 }
 
 }  // namespace ldk

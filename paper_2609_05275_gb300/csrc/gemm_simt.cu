@@ -63,7 +63,12 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const GemmArgs a) {
       if (n >= N) continue;
       const float v = a.alpha * acc[i][j];
       if (EPI == EPI_RESID) {
-        float* x = a.x + src_row(a.kept_idx, a.S, m) * a.ldx + n;
+        const long long r = src_row(a.kept_idx, a.S, m);
+        if (r < 0) {  // padding row of a per-token kept list: zero copy only
+          if (a.save) static_cast<float*>(a.save)[(size_t)m * a.ld_save + n] = 0.f;
+          continue;
+        }
+        float* x = a.x + r * a.ldx + n;
         const float nv = *x + v;
         *x = nv;
         if (a.save) static_cast<float*>(a.save)[(size_t)m * a.ld_save + n] = nv;

@@ -108,9 +108,14 @@ __device__ __forceinline__ void store_chunk(const GemmArgs& a, int row, int col,
     }
   } else {  // EPI_RESID: x[r] += alpha * acc on the kept row r (float32); compact float32 copy
     const long long r = src_row(a.kept_idx, a.S, row);
-    float4* px = reinterpret_cast<float4*>(a.x + r * a.ldx + col);
     float4* ps = a.save ? reinterpret_cast<float4*>(static_cast<float*>(a.save) + (size_t)row * a.ld_save + col)
                         : nullptr;
+    if (r < 0) {  // padding row of a per-token kept list: no residual row; zero copy
+      if (ps)
+        for (int i = 0; i < 8; ++i) ps[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      return;
+    }
+    float4* px = reinterpret_cast<float4*>(a.x + r * a.ldx + col);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       float4 o = px[i];
@@ -480,7 +485,7 @@ __global__ void __launch_bounds__(192, 1)
       } else if (a.epi == EPI_ROPE) {
         // rotate pairs (i, i + Dh/2) of every q / k head in the tile
         const int half = a.Dh / 2;
-        const int pos = row % a.S;
+        const int pos = row_pos(a.pos_tok, a.S, row);
 #pragma unroll 1
         for (int hb = 0; hb < BN; hb += a.Dh) {
           const int col = nb * BN + hb;
@@ -515,8 +520,10 @@ __global__ void __launch_bounds__(192, 1)
       } else if (a.epi == EPI_RESID) {
         // residual rows are read ahead (the next chunk while this one is
         // finished) so their latency overlaps the TMEM loads and the adds
-        const bool rok = row < M;
-        const long long r = rok ? src_row(a.kept_idx, a.S, row) : 0;
+        const long long rs = row < M ? src_row(a.kept_idx, a.S, row) : 0;
+        const bool pad = row < M && rs < 0;  // padding row of a per-token kept list: zero copy only
+        const bool rok = row < M && !pad;
+        const long long r = rok ? rs : 0;
         float* xrow = a.x + r * a.ldx + (size_t)nb * BN;
         float* srow = a.save ? static_cast<float*>(a.save) + (size_t)row * a.ld_save + (size_t)nb * BN : nullptr;
         float4 xv[8];
@@ -549,6 +556,9 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
               for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(srow + c)[i] = o[i];
             }
+          } else if (pad && srow && nb * BN + c < N) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(srow + c)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
           }
         }
       } else {

@@ -39,9 +39,21 @@ __device__ __forceinline__ uint64_t gtimer_ns() {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 // Row of the residual stream for compact row m of layer l: sequence
-// kept_idx[m / S], position m % S.
+// kept_idx[m / S], position m % S.  Per-token kept lists are passed with
+// S = 1 (kept_idx[m] is then the token's row b S + s); their padding rows
+// hold -1, so the result is negative for them and callers skip the row.
 __device__ __forceinline__ long long src_row(const int* kept_idx, int S, long long m) {
-  return (long long)kept_idx[m / S] * S + (m % S);
+  const long long k = kept_idx[m / S];
+  return k < 0 ? -1 : k * S + (m % S);
+}
+
+// Position of compact row m in its sequence: m % S when the compact rows
+// are whole kept sequences of S rows (tok = null), else tok[m] % S with tok
+// the per-token kept list (rows b S + s; padding rows -1 get position 0).
+__device__ __forceinline__ int row_pos(const int* tok, int S, long long m) {
+  if (!tok) return (int)(m % S);
+  const int t = tok[m];
+  return t < 0 ? 0 : t % S;
 }
 
 // ------------------------------------------------------------------------
@@ -51,12 +63,26 @@ __device__ __forceinline__ long long src_row(const int* kept_idx, int S, long lo
 struct MaskParams {
   unsigned long long seed;
   long long step;
-  int L, B, granularity, b_offset;
+  int L, B, S, granularity, b_offset;
   int nmask;  // 1: one mask per (layer, sequence); 2: attention (word 0) and FFN (word 1) masks
   unsigned long long thr[LD_MAX_L];
 };
-cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* kept_idx, int* kept_cnt,
+// Per sequence / batch / shard: mask [nmask][L][B], kept_idx [nmask][L][B]
+// (kept sequences ascending, -1 after), kept_cnt [nmask][L] (sequences).
+// Per token: mask [nmask][L][B*S], kept_idx [nmask][L][B*S] (rows b S + s of
+// the kept tokens ascending, then -1), kept_cnt [nmask][L] = the kept-token
+// count rounded up to a multiple of 64 (the row extent of the layer's
+// products; the padding rows hold -1), seg [nmask][L][B+1] (the kept tokens
+// of sequence b are compact rows seg[b] .. seg[b+1]-1; seg[B] = the count).
+cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* kept_idx, int* kept_cnt, int* seg,
                                 cudaStream_t st);
+
+// Zero rows [*start, min(*start + nrows, max_rows)) of `planes` row-major
+// matrices (plane p at buf + p * plane_ld elements, row stride ld, the first
+// ncols columns); ncols * sizeof(T) a multiple of 16 bytes when planes == 1.
+template <typename T>
+cudaError_t launch_zero_rows(T* buf, int ld, int ncols, int planes, long long plane_ld, const int* start, int nrows,
+                             int max_rows, cudaStream_t st);
 
 // Elementwise copy with conversion between float32 and bf16 (n % 8 == 0).
 cudaError_t launch_convert(const void* src, int src_f32, void* dst, int dst_f32, long long n, cudaStream_t st);
@@ -93,9 +119,11 @@ template <typename T>
 cudaError_t launch_gather_scale(const float* dx, const int* kept_idx, const int* cnt, int S, int d, int max_rows,
                                 float scale, T* out, cudaStream_t st);
 
+// Rows: (*cnt) * S compact rows at positions m % S, or, with tok (per-token
+// kept list), *cnt rows at positions tok[m] % S.
 template <typename T>
 cudaError_t launch_rope_apply(T* qkv, int ld, int nheads, int Dh, const float* cos_t, const float* sin_t,
-                              const int* cnt, int S, int max_rows, int inverse, cudaStream_t st);
+                              const int* cnt, int S, int max_rows, int inverse, const int* tok, cudaStream_t st);
 
 template <typename T>
 cudaError_t launch_swiglu_fwd(const T* gu, T* h, const int* cnt, int S, int F, int max_rows, cudaStream_t st);
@@ -115,15 +143,20 @@ cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, c
                                float* Dvec, cudaStream_t st);
 
 // Every attention launcher takes `alibi`: null, or the device table of the
-// H ALiBi slopes (scores of head h get + m_h (j - i)).
+// H ALiBi slopes (scores of head h get + m_h (j - i)), and `seg`, `tok`:
+// null for whole kept sequences (*cnt of them, S rows each), or the
+// per-token segments (sequence b = compact rows seg[b] .. seg[b+1]-1, b <
+// max_seqs) and kept list (position tok[m] % S; -1 rows belong to no
+// sequence).  Per-token attention takes no ALiBi table.
 // Reference (SIMT) attention, used by the float32 debug path.
 template <typename T>
 cudaError_t launch_attn_fwd_simt(const T* qkv, int ldqkv, T* o, int ldo, float* lse, const int* cnt, int S, int H,
-                                 int Hkv, int Dh, int max_rows, const float* alibi, cudaStream_t st);
+                                 int Hkv, int Dh, int max_rows, const float* alibi, const int* seg, const int* tok,
+                                 cudaStream_t st);
 template <typename T>
 cudaError_t launch_attn_bwd_simt(const T* qkv, int ldqkv, const T* dO, int ldo, const float* lse, const float* Dvec,
                                  T* dqkv, const int* cnt, int S, int H, int Hkv, int Dh, int max_rows,
-                                 const float* alibi, cudaStream_t st);
+                                 const float* alibi, const int* seg, const int* tok, cudaStream_t st);
 
 // Tensor-core (mma.sync) flash attention for bf16.
 cudaError_t launch_attn_fwd_mma(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S,
@@ -134,18 +167,20 @@ cudaError_t launch_attn_bwd_mma(const bf16* qkv, int ldqkv, const bf16* o, const
 // tcgen05 flash attention forward (head size 64 or 128, S % 128 == 0).
 bool attn_tc_supported(int S, int Dh);
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
-                               int Hkv, int Dh, int max_seqs, const float* alibi, int* status, cudaStream_t st);
+                               int Hkv, int Dh, int max_seqs, const float* alibi, const int* seg, int* status,
+                               cudaStream_t st);
 // tcgen05 flash attention backward (head size 128, S % 128 == 0); zeroes
 // dq_acc and accumulates dQ (unscaled) into it.
 bool attn_bwd_tc_supported(int S, int Dh);
 // dK leaves with the inverse RoPE applied (rcos = null: no rotation).
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, int* status,
-                               cudaStream_t st);
-// dqkv[:, q heads] = inverse-RoPE(dq_acc / sqrt(Dh)) as bf16 (rcos = null: no rotation)
+                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, const int* seg,
+                               const int* tok, int* status, cudaStream_t st);
+// dqkv[:, q heads] = inverse-RoPE(dq_acc / sqrt(Dh)) as bf16 (rcos = null: no rotation);
+// rows and positions as launch_rope_apply
 cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const float* rcos,
-                             const float* rsin, const int* cnt, int S, int max_rows, cudaStream_t st);
+                             const float* rsin, const int* cnt, int S, int max_rows, const int* tok, cudaStream_t st);
 
 // ------------------------------------------------------------------------
 // GEMM: D(m,n) = alpha * sum_k A(m,k) B(n,k) with a fused epilogue.
@@ -199,10 +234,11 @@ struct GemmArgs {
   int S;
   void* save;
   int ld_save;
-  // EPI_ROPE
+  // EPI_ROPE (position of row m: row_pos(pos_tok, S, m))
   const float* rope_cos;
   const float* rope_sin;
   int Dh, rope_cols;
+  const int* pos_tok;
   // EPI_SWIGLU / EPI_SWIGLU_BWD
   const void* gu;
   void* h_out;

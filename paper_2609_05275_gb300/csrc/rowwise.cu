@@ -76,6 +76,15 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const TS* __restrict__
   const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
   for (long long m = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); m < M; m += nwarps) {
     const long long r = gather ? src_row(kept_idx, S, m) : m;
+    if (r < 0) {  // padding row of a per-token kept list: zeros
+      const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      for (int i = lane * 8; i < d; i += 256) {
+        if (copy) st8(copy + m * d + i, z);
+        st8(out + m * d + i, z);
+      }
+      if (lane == 0) rstd[m] = 0.f;
+      continue;
+    }
     const TS* xr = src + r * d;
     float ss = 0.f;
     for (int i = lane * 8; i < d; i += 256) {
@@ -139,6 +148,12 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const float* __restric
       }
     }
     dot = warp_sum(dot) / (float)d;
+    if (r < 0) {  // padding row of a per-token kept list (its dyn and xs are 0)
+      const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (next)
+        for (int i = lane * 8; i < d; i += 256) st8(next + m * d + i, z);
+      continue;
+    }
     for (int i = lane * 8; i < d; i += 256) {
       float dy[8], xv[8], g[8], cur[8], nx[8];
       ld8(dyn + m * d + i, dy);
@@ -197,7 +212,7 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __re
     float pd[RPB];
     long long rr[RPB];
 #pragma unroll
-    for (int q = 0; q < RPB; ++q) rr[q] = (m0 + q < M) ? src_row(kept_idx, S, m0 + q) : 0;
+    for (int q = 0; q < RPB; ++q) rr[q] = (m0 + q < M) ? src_row(kept_idx, S, m0 + q) : -1;
 #pragma unroll
     for (int q = 0; q < RPB; ++q) {
       const long long m = m0 + q;
@@ -208,7 +223,14 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __re
         if (m < M && c8 < d8) {
           ld8(dyn + m * d + c8 * 8, dy[q][j]);
           ld8(xs + m * d + c8 * 8, xv[q][j]);
-          if constexpr (PF) ld8(dx + rr[q] * d + c8 * 8, cur[q][j]);
+          if constexpr (PF) {
+            if (rr[q] >= 0) {
+              ld8(dx + rr[q] * d + c8 * 8, cur[q][j]);
+            } else {
+#pragma unroll
+              for (int e = 0; e < 8; ++e) cur[q][j][e] = 0.f;
+            }
+          }
 #pragma unroll
           for (int e = 0; e < 8; ++e) pd[q] += dy[q][j][e] * g[j][e] * xv[q][j][e];
         }
@@ -241,8 +263,11 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __re
           if constexpr (PF) {
 #pragma unroll
             for (int e = 0; e < 8; ++e) cr[e] = cur[q][j][e];
-          } else {
+          } else if (r >= 0) {
             ld8(dx + r * d + c8 * 8, cr);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) cr[e] = 0.f;
           }
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
@@ -251,7 +276,9 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_cols_kernel(const float* __re
             nx[e] = scale * cr[e];
             gacc[j][e] += dy[q][j][e] * xn;
           }
-          st8(dx + r * d + c8 * 8, cr);
+          // a padding row of a per-token kept list (r < 0) has dyn = xs = 0:
+          // it adds nothing to the gain gradient and passes 0 on
+          if (r >= 0) st8(dx + r * d + c8 * 8, cr);
           if (next) st8(next + m * d + c8 * 8, nx);
         }
       }
@@ -327,9 +354,15 @@ __global__ void gather_scale_kernel(const float* __restrict__ dx, const int* __r
     const long long m = w / per_row;
     const int i = (int)(w % per_row) * 8;
     float v[8];
-    ld8(dx + src_row(kept_idx, S, m) * d + i, v);
+    const long long r = src_row(kept_idx, S, m);
+    if (r >= 0) {
+      ld8(dx + r * d + i, v);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) v[j] *= scale;
+      for (int j = 0; j < 8; ++j) v[j] *= scale;
+    } else {  // padding row of a per-token kept list
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = 0.f;
+    }
     st8(out + m * d + i, v);
   }
 }
@@ -390,8 +423,8 @@ cudaError_t launch_rope_table(float* cos_t, float* sin_t, int S, int Dh, double 
 template <typename T>
 __global__ void rope_apply_kernel(T* __restrict__ qkv, int ld, int nheads, int Dh, const float* __restrict__ cos_t,
                                   const float* __restrict__ sin_t, const int* __restrict__ cnt, int S,
-                                  int inverse) {
-  const long long M = (long long)(*cnt) * S;
+                                  int inverse, const int* __restrict__ tok) {
+  const long long M = tok ? (long long)(*cnt) : (long long)(*cnt) * S;
   const int half = Dh / 2, g8 = half / 8;
   const int per_row = nheads * g8;
   const long long total = M * per_row;
@@ -400,7 +433,7 @@ __global__ void rope_apply_kernel(T* __restrict__ qkv, int ld, int nheads, int D
     const long long m = w / per_row;
     const int rem = (int)(w - m * per_row);
     const int h = rem / g8, i = (rem - h * g8) * 8;
-    const int pos = (int)(m % S);
+    const int pos = row_pos(tok, S, m);
     T* p = qkv + m * ld + (long long)h * Dh;
     float a[8], b[8], c[8], sn[8];
     ld8(p + i, a);
@@ -422,9 +455,34 @@ __global__ void rope_apply_kernel(T* __restrict__ qkv, int ld, int nheads, int D
 
 template <typename T>
 cudaError_t launch_rope_apply(T* qkv, int ld, int nheads, int Dh, const float* cos_t, const float* sin_t,
-                              const int* cnt, int S, int max_rows, int inverse, cudaStream_t st) {
+                              const int* cnt, int S, int max_rows, int inverse, const int* tok, cudaStream_t st) {
   const int grid = grid_for((long long)max_rows * nheads * (Dh / 16), 256, device_sm_count() * 8);
-  rope_apply_kernel<T><<<grid, 256, 0, st>>>(qkv, ld, nheads, Dh, cos_t, sin_t, cnt, S, inverse);
+  rope_apply_kernel<T><<<grid, 256, 0, st>>>(qkv, ld, nheads, Dh, cos_t, sin_t, cnt, S, inverse, tok);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------- zero rows
+template <typename T>
+__global__ void zero_rows_kernel(T* __restrict__ buf, int ld, int ncols, int planes, long long plane_ld,
+                                 const int* __restrict__ start, int nrows, int max_rows) {
+  const long long r0 = *start;
+  const long long r1 = min((long long)max_rows, r0 + nrows);
+  if (r1 <= r0) return;
+  const long long per_plane = (r1 - r0) * ncols;
+  const long long total = per_plane * planes;
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
+       w += (long long)gridDim.x * blockDim.x) {
+    const long long p = w / per_plane, rem = w - p * per_plane;
+    const long long r = r0 + rem / ncols, c = rem % ncols;
+    buf[p * plane_ld + r * ld + c] = from_f<T>(0.f);
+  }
+}
+
+template <typename T>
+cudaError_t launch_zero_rows(T* buf, int ld, int ncols, int planes, long long plane_ld, const int* start, int nrows,
+                             int max_rows, cudaStream_t st) {
+  const int grid = grid_for((long long)nrows * ncols * planes, 256, device_sm_count() * 4);
+  zero_rows_kernel<T><<<grid, 256, 0, st>>>(buf, ld, ncols, planes, plane_ld, start, nrows, max_rows);
   return cudaGetLastError();
 }
 
@@ -579,7 +637,8 @@ cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, c
   template cudaError_t launch_gather_scale<T>(const float*, const int*, const int*, int, int, int, float, T*,    \
                                               cudaStream_t);                                                    \
   template cudaError_t launch_rope_apply<T>(T*, int, int, int, const float*, const float*, const int*, int, int, \
-                                            int, cudaStream_t);                                                 \
+                                            int, const int*, cudaStream_t);                                     \
+  template cudaError_t launch_zero_rows<T>(T*, int, int, int, long long, const int*, int, int, cudaStream_t);   \
   template cudaError_t launch_swiglu_fwd<T>(const T*, T*, const int*, int, int, int, cudaStream_t);             \
   template cudaError_t launch_swiglu_bwd<T>(const T*, const T*, T*, const int*, int, int, int, cudaStream_t);   \
   template cudaError_t launch_relu2<T>(const T*, const T*, T*, const int*, int, int, int, cudaStream_t);        \
@@ -594,7 +653,8 @@ template cudaError_t launch_rmsnorm_bwd<float>(const float*, const float*, const
 template cudaError_t launch_gather_scale<float>(const float*, const int*, const int*, int, int, int, float, float*,
                                                 cudaStream_t);
 template cudaError_t launch_rope_apply<float>(float*, int, int, int, const float*, const float*, const int*, int, int,
-                                              int, cudaStream_t);
+                                              int, const int*, cudaStream_t);
+template cudaError_t launch_zero_rows<float>(float*, int, int, int, long long, const int*, int, int, cudaStream_t);
 template cudaError_t launch_swiglu_fwd<float>(const float*, float*, const int*, int, int, int, cudaStream_t);
 template cudaError_t launch_swiglu_bwd<float>(const float*, const float*, float*, const int*, int, int, int,
                                               cudaStream_t);

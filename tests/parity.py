@@ -30,8 +30,9 @@ def oracle_masks(cfg, sched, step, granularity="per_sequence", sublayer=False):
     rates = OS.layer_rates(oracle_sched(sched), cfg["L"], step)
     thr = [OS.drop_threshold(p) for p in rates]
     scales = [OS.residual_scale(p, cfg.get("alpha", 1.0)) for p in rates]
-    gran = {"per_sequence": OM.PER_SEQUENCE, "per_batch": OM.PER_BATCH, "per_shard": OM.PER_SHARD}[granularity]
-    mask = OM.draw_masks(sched.get("seed", 0), step, thr, cfg["B"], gran, sublayer=sublayer)
+    gran = {"per_sequence": OM.PER_SEQUENCE, "per_batch": OM.PER_BATCH, "per_shard": OM.PER_SHARD,
+            "per_token": OM.PER_TOKEN}[granularity]
+    mask = OM.draw_masks(sched.get("seed", 0), step, thr, cfg["B"], gran, sublayer=sublayer, S=cfg["S"])
     return mask, thr, scales
 
 
@@ -81,14 +82,17 @@ def oracle_run(cfg, sched, step, layers_host, x_host, dy_host, granularity="per_
     x = x_host.double().numpy()
     dy = dy_host.double().numpy()
     mk = mask
+    tok = granularity == "per_token"
     if seqs is not None:
-        x, dy, mk = x[seqs], dy[seqs], mask[..., seqs]
+        x, dy, mk = x[seqs], dy[seqs], (mask[..., seqs, :] if tok else mask[..., seqs])
     if rows is not None:
         x, dy = x[:, :rows], dy[:, :rows]
+        if tok:
+            mk = mk[..., :rows]
 
     def layer(l):
         return {n: v.double().numpy() for n, v in layers_host[l].items()}
 
-    out, caches = OK.stack_forward(x, layer, cfg, mk, scales)
-    dX, grads = OK.stack_backward(dy, layer, cfg, mk, scales, caches)
+    out, caches = OK.stack_forward(x, layer, cfg, mk, scales, per_token=tok)
+    dX, grads = OK.stack_backward(dy, layer, cfg, mk, scales, caches, per_token=tok)
     return out, dX, grads, mask

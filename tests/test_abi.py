@@ -77,6 +77,32 @@ def test_position_and_activation_flags():
         P.ld_destroy(h2)
 
 
+def test_per_token_flag():
+    # per-token granularity: no ALiBi; on the bf16 path head size 128 and
+    # S % 128 == 0 (the tcgen05 attention), any supported shape on the
+    # float32 debug path; the mask tables grow to one entry per token
+    cfg = dict(synth.CONFIGS["tiny"])          # Dh = 32, S = 64
+    assert P.ld_create_status(P.make_config(cfg, "per_token")) == P.LD_ERR_SHAPE
+    assert P.ld_create_status(P.make_config(cfg, "per_token", fp32_debug=True)) == P.LD_OK
+    c128 = dict(cfg, H=2, Hkv=1, Dh=128, S=128)
+    assert P.ld_create_status(P.make_config(c128, "per_token")) == P.LD_OK
+    assert P.ld_create_status(P.make_config(dict(c128, S=192), "per_token")) == P.LD_ERR_SHAPE
+    assert P.ld_create_status(P.make_config(dict(c128, alibi=True, rope_theta=0.0), "per_token")) == P.LD_ERR_ARG
+    assert P.ld_create_status(P.make_config(dict(c128, alibi=True, rope_theta=0.0), "per_token",
+                                            fp32_debug=True)) == P.LD_ERR_ARG
+    bad = P.make_config(c128)
+    bad.granularity = 4
+    assert P.ld_create_status(bad) == P.LD_ERR_ARG
+    h1, h2 = P.ld_create(P.make_config(c128)), P.ld_create(P.make_config(c128, "per_token"))
+    try:
+        n1, n2 = P.ld_workspace_size(h1), P.ld_workspace_size(h2)
+        # at least (S - 1) more mask bytes and (S - 1) more kept-list ints per (layer, sequence)
+        assert n2 - n1 >= c128["L"] * c128["B"] * (c128["S"] - 1) * 5 - 4096
+    finally:
+        P.ld_destroy(h1)
+        P.ld_destroy(h2)
+
+
 def test_eval_entry_points():
     cfg = synth.CONFIGS["llama8b"]
     h = P.ld_create(P.make_config(cfg))
