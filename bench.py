@@ -232,7 +232,7 @@ def run_sweep(args):
             e1.record()
             torch.cuda.synchronize()
             ms.append(e0.elapsed_time(e1))
-            kept.append(int(st.masks()[2].sum()))
+            kept.append(int(st.masks()[2].sum()))  # kept (layer, sequence) pairs, or kept tokens per token
         return ms, kept
 
     dense_ms, _ = time_cell(stacks["per_sequence"], dict(dist="uniform", p_max=0.0, time="const"))
@@ -243,13 +243,16 @@ def run_sweep(args):
             for p_max in sw["p_max"]:
                 sched = dict(dist=dist, p_max=p_max, time="const")
                 ms, kept = time_cell(stacks[gran], sched)
-                p_real = 1.0 - sum(kept) / (len(kept) * L * B)
+                rows_per_unit = 1 if gran == "per_token" else S
+                p_real = 1.0 - sum(kept) * rows_per_unit / (len(kept) * L * B * S)
                 t = sum(ms) / len(ms)
                 speed = t_dense / t
                 ideal = 1.0 / (1.0 - p_real)
                 cell = {"granularity": gran, "dist": dist, "p_max": p_max, "seeds": len(seeds),
                         "ms_per_step": t, "tokens_per_s": B * S / (t / 1e3),
-                        "executed_tflops": 3.0 * f_tok * S * sum(kept) / len(kept) / (t / 1e3) / 1e12,
+                        # per token the attention term of f_tok (whole-length sequences) overstates the
+                        # work of the shortened sequences slightly
+                        "executed_tflops": 3.0 * f_tok * rows_per_unit * sum(kept) / len(kept) / (t / 1e3) / 1e12,
                         "p_bar_realized": p_real, "speedup": speed, "ideal_speedup": ideal,
                         "frac_of_ideal": speed / ideal}
                 cells.append(cell)
@@ -349,6 +352,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=1024)
     ap.add_argument("--layers", type=int, default=None, help="override L (profiling captures only)")
+    ap.add_argument("--granularity", default="per_sequence", choices=["per_sequence", "per_batch", "per_token"],
+                    help="mask granularity of the timed steps (the headline is per sequence)")
     ap.add_argument("--sweep", action="store_true",
                     help="drop-rate / distribution / granularity / seed sweep on the 1.3B shape (one JSON line "
                          "per cell, then a summary line)")
@@ -387,7 +392,8 @@ def main():
     step0 = args.step0 if args.step0 is not None else synth.STEPS[args.config][-1]
     peaks = load_peaks()
 
-    st = P.LayerDropStack(cfg, sched)
+    tok = args.granularity == "per_token"
+    st = P.LayerDropStack(cfg, sched, granularity=args.granularity)
     layers = synth.stack_weights(cfg, seed=0, device="cuda")
     wtab = P.weight_table(layers)
     grads = [{n: torch.empty(v.shape, device="cuda", dtype=torch.float32) for n, v in W.items()} for W in layers]
@@ -431,16 +437,24 @@ def main():
     P.ld_set_timing(st.h, 0)
     st.sync()
 
-    # kept counts of the timed steps (masks redrawn through the library)
-    kept = []
+    # kept counts of the timed steps (masks redrawn through the library):
+    # kept (layer, sequence) pairs, or per token the kept tokens (and the
+    # kept length of every (layer, sequence) for the attention FLOPs)
+    kept, attn_len2 = [], 0.0
     for k in range(args.steps):
-        _, _, cnt = st.draw_masks(step0 + args.warmup + k)
+        mk, _, cnt = st.draw_masks(step0 + args.warmup + k)
         kept.append([int(c) for c in cnt])
+        if tok:
+            attn_len2 += float((mk.reshape(-1, B, S).sum(axis=2).astype("float64") ** 2).sum())
     f_tok, f_proj = flops_per_token(cfg)
     kept_units = sum(sum(c) for c in kept)
-    exec_flops = 3.0 * f_tok * S * kept_units / args.steps  # per step, this rank
-    gemm_flops = 3.0 * f_proj * S * kept_units / args.steps
-    p_real = 1.0 - kept_units / (args.steps * L * B)
+    rows_per_unit = 1 if tok else S
+    if tok:  # projections per kept token; attention 2 H Dh len^2 per kept sequence of length len (forward)
+        exec_flops = 3.0 * (f_proj * kept_units + 2.0 * cfg["H"] * cfg["Dh"] * attn_len2) / args.steps
+    else:
+        exec_flops = 3.0 * f_tok * S * kept_units / args.steps  # per step, this rank
+    gemm_flops = 3.0 * f_proj * rows_per_unit * kept_units / args.steps
+    p_real = 1.0 - kept_units * rows_per_unit / (args.steps * L * B * S)
     _, thr, _ = st.rates(step0 + args.warmup)
     p_exp = sum(t / 2 ** 32 for t in thr) / L
     tflops = exec_flops / (ms / 1e3) / 1e12
@@ -480,13 +494,14 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu:
         w0 = {n: v.cpu() for n, v in layers[0].items()}
         _, _, sc = st.rates(step0 + args.warmup)
-        cpu = cpu_baseline(cfg, w0, x0[0].cpu(), dy0[0].cpu(), min(args.cpu_rows, S), kept_units / args.steps, sc[0])
+        cpu = cpu_baseline(cfg, w0, x0[0].cpu(), dy0[0].cpu(), min(args.cpu_rows, S),
+                           kept_units * rows_per_unit / S / args.steps, sc[0])
 
     gemm_achieved = gemm_flops * args.steps / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
     # 12 GEMM launches per executed layer (4 forward, 8 backward)
     traffic = None
     if args.config == "llama8b" and gemm_launches > 0:
-        rows_per_launch = kept_units * S / (gemm_launches / 12.0)
+        rows_per_launch = kept_units * rows_per_unit / (gemm_launches / 12.0)
         traffic = GEMM_DRAM_BYTES_PER_ROW * rows_per_launch
     roof = {"kernel": "gemm_tc_kernel (tcgen05 projections, fwd dgrad wgrad)", "bound": "tensor",
             "achieved": gemm_achieved, "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
@@ -499,7 +514,7 @@ def main():
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": args.config, **{k: cfg[k] for k in ("L", "d", "H", "Hkv", "Dh", "F", "B", "S")},
-                   "schedule": sched, "granularity": "per_sequence", "first_step": step0 + args.warmup,
+                   "schedule": sched, "granularity": args.granularity, "first_step": step0 + args.warmup,
                    "parallelism": f"replicas x{world}", "l2": "inputs and weights larger than L2 (no flush)"},
         "executed_tflops": tflops, "pct_bf16_peak": 100.0 * tflops / peaks["bf16"],
         "pct_bf16_peak_sustained": 100.0 * tflops / peaks["bf16_sustained"],
@@ -515,8 +530,9 @@ def main():
     # kernel and the RoPE table, then per layer 4 GEMMs + attention + 4
     # row-wise kernels forward, 8 GEMMs + 3 attention kernels + 7 row-wise
     # kernels backward (RoPE kernels drop out when theta = 0)
+    # (per token also 3 + 3 tail-zeroing launches per layer)
     rope = 1 if cfg.get("rope_theta") else 0
-    line["gpu_launches"] = args.steps * (1 + rope + L * (4 + 1 + 3 + rope + 8 + 3 + 6 + rope))
+    line["gpu_launches"] = args.steps * (1 + rope + L * (4 + 1 + 3 + rope + 8 + 3 + 6 + rope + (6 if tok else 0)))
     if rank == 0:
         print(json.dumps(line), flush=True)
     st.close()

@@ -49,7 +49,7 @@ STEPS = {"tiny": [0], "gpt2": [0], "1.3b": [0, 500, 2000], "llama8b": [0], "pape
 
 # Sweep on the 1.3B shape: p_max x distribution x granularity x seeds.
 SWEEP = dict(base="1.3b", p_max=[0.0, 0.1, 0.2, 0.3, 0.5], dist=["ild", "uniform"],
-             granularity=["per_sequence", "per_batch"], seeds=list(range(1, 21)))
+             granularity=["per_sequence", "per_batch", "per_token"], seeds=list(range(1, 21)))
 
 _TAGS = {"x": 11, "dy": 12, "w_qkv": 21, "w_o": 22, "w_gu": 23, "w_d": 24, "g1": 25, "g2": 26}
 
