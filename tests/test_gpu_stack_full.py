@@ -97,3 +97,17 @@ def test_paper_arch_3p9b_full():
     # the paper's architecture: ALiBi (16 heads) + squared-ReLU FFN, 40 layers
     mask, seqs = _run("paper-3.9b", 0, R=32)
     assert mask[0].all() and not mask.all()
+
+
+def test_1p3b_full_per_token():
+    # per-token masks at full size: the kept tokens among the first R rows of a
+    # sequence depend only on each other (causality holds for the kept
+    # subsequences), so the truncation protocol applies unchanged
+    mask, _ = _run("1.3b", 2000, R=64, granularity="per_token", seqs=[1, 6])
+    assert not mask.all() and mask.any()
+
+
+def test_llama8b_full_per_token():
+    mask, _ = _run("llama8b", 0, R=32, granularity="per_token", seqs=[0, 3])
+    kept = mask[:, [0, 3], :32]
+    assert kept[0].all() and not kept.all()  # layer 0 keeps everything (ILD), later layers drop tokens
