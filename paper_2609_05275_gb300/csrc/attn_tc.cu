@@ -39,6 +39,47 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescale = 8.0f;  // move the running max only when it grows by > 2^8
 
+__device__ __forceinline__ void st_volatile_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.volatile.shared.u64 [%0], %1;" ::"r"(smem_u32(p)), "l"(v) : "memory");
+}
+__device__ __forceinline__ uint64_t ld_volatile_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.volatile.shared.u64 %0, [%1];" : "=l"(v) : "r"(smem_u32(p)) : "memory");
+  return v;
+}
+// Warp-uniform bounded wait for a (tag << 32 | value) word written by a
+// partner thread: true with the value once every lane's word carries `tag`;
+// false (abort flag and status raised) after kWaitLimitNs or when another
+// role aborted.
+__device__ __forceinline__ bool xchg_wait(const uint64_t* p, uint32_t tag, float& v, volatile int* abort_flag,
+                                          int* status) {
+  uint64_t w = ld_volatile_u64(p);
+  if (__all_sync(0xffffffffu, (uint32_t)(w >> 32) == tag)) {
+    v = __uint_as_float((uint32_t)w);
+    return true;
+  }
+  const uint64_t t0 = gtimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    w = ld_volatile_u64(p);
+    if (__all_sync(0xffffffffu, (uint32_t)(w >> 32) == tag)) {
+      v = __uint_as_float((uint32_t)w);
+      return true;
+    }
+    if ((it & 255) == 0) {
+      int bad = 0;
+      if ((threadIdx.x & 31) == 0) {
+        bad = *abort_flag ? 1 : 0;
+        if (!bad && gtimer_ns() - t0 > kWaitLimitNs) {
+          *abort_flag = 1;
+          set_status(status, LD_ERR_TIMEOUT);
+          bad = 1;
+        }
+      }
+      if (__shfl_sync(0xffffffffu, bad, 0)) return false;
+    }
+  }
+}
+
 __device__ __forceinline__ void st_bf16x32_(bf16* dst, const float* v) {
   uint4* p = reinterpret_cast<uint4*>(dst);
 #pragma unroll
@@ -70,9 +111,10 @@ __global__ void __launch_bounds__(320, 1)
   uint8_t* Ks = Qs + TILE;
   uint8_t* Vs = Ks + NSK * TILE;
   uint8_t* xch = Vs + NSV * TILE;
-  float(*xmax)[2][128] = reinterpret_cast<float(*)[2][128]>(xch);  // [tile parity][half][row]
-  float(*xsum)[128] = reinterpret_cast<float(*)[128]>(xch + 2 * 2 * 128 * 4);  // [half][row]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(xch + 6 * 128 * 4);
+  // row-max exchange words (tile index << 32 | max bits), [tile parity][half][row]
+  uint64_t(*xmax)[2][128] = reinterpret_cast<uint64_t(*)[2][128]>(xch);
+  float(*xsum)[128] = reinterpret_cast<float(*)[128]>(xch + 2 * 2 * 128 * 8);  // [half][row]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xch + 10 * 128 * 4);
   uint64_t* q_full = bars;
   uint64_t* k_full = bars + 1;        // [NSK] K ring: a stage frees once S_j has read it
   uint64_t* k_empty = k_full + NSK;
@@ -133,6 +175,7 @@ __global__ void __launch_bounds__(320, 1)
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  for (int i = threadIdx.x; i < 2 * 2 * 128; i += blockDim.x) (&xmax[0][0][0])[i] = ~0ull;  // no tile yet
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
@@ -276,11 +319,14 @@ __global__ void __launch_bounds__(320, 1)
         for (int e = 0; e < 64; e += 2)
           mraw = fmax3(mraw, __uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1]));
       }
-      xmax[j & 1][half][r] = mraw;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(xb);
-      if (!warp_wait(xb, j & 1, abort_flag, status)) { ok = false; break; }
-      mraw = fmaxf(mraw, xmax[j & 1][half ^ 1][r]);
+      // partner's max of this row through a (tile, value) word: a shared-
+      // memory round trip instead of an mbarrier phase (whose arrival takes
+      // a few hundred cycles to be seen); parity double-buffered, so a word
+      // is rewritten only after the partner has passed the next exchange
+      st_volatile_u64(&xmax[j & 1][half][r], ((uint64_t)(uint32_t)j << 32) | __float_as_uint(mraw));
+      float pmax;
+      if (!xchg_wait(&xmax[j & 1][half ^ 1][r], (uint32_t)j, pmax, abort_flag, status)) { ok = false; break; }
+      mraw = fmaxf(mraw, pmax);
       const float mt = mraw * sl2e;
       const bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
@@ -348,7 +394,7 @@ __global__ void __launch_bounds__(320, 1)
       xsum[half][r] = l;
       __syncwarp();
       if (lane == 0) mbar_arrive(xb);
-      const bool got = warp_wait(xb, nkt & 1, abort_flag, status);
+      const bool got = warp_wait(xb, 0, abort_flag, status);  // the barrier's only phase
       const float lt = l + (got ? xsum[half ^ 1][r] : 0.f);
       const float inv = 1.0f / lt;
       const bool valid = qt * 128 + r < len;
@@ -383,7 +429,7 @@ template <int DH, bool ALIBI>
 cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
                    int max_seqs, const float* alibi, const int* seg, int* status, cudaStream_t st) {
   // Q, 3 K and 2 V tiles + the row max / sum exchange + alignment + barriers
-  constexpr size_t smem = (size_t)(DH / 64) * SLAB * 6 + 6 * 128 * 4 + 1024 + 256;
+  constexpr size_t smem = (size_t)(DH / 64) * SLAB * 6 + 10 * 128 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =

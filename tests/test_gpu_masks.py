@@ -1,6 +1,7 @@
-"""Masks and kept-sequence lists of the device kernel against the oracle,
-bit for bit: every workload schedule at its benchmark steps, and the whole
-drop-rate / distribution / granularity / seed sweep on the 1.3B shape."""
+"""Masks and kept-sequence (per token: kept-token) lists of the device kernel
+against the oracle, bit for bit: every workload schedule at its benchmark
+steps, and the whole drop-rate / distribution / granularity / seed sweep on
+the 1.3B shape."""
 
 import numpy as np
 import pytest
@@ -21,7 +22,10 @@ def _check(cfg, sched, steps, granularity, sublayer=False):
         for t in steps:
             mask, idx, cnt = st.draw_masks(t)
             ref, _, _ = oracle_masks(cfg, sched, t, granularity, sublayer)
-            ridx, rcnt = OM.kept_lists(ref)
+            if granularity == "per_token":
+                ridx, rcnt, _ = OM.kept_token_lists(ref)
+            else:
+                ridx, rcnt = OM.kept_lists(ref)
             assert (mask == ref).all(), t
             assert (cnt == rcnt).all(), t
             assert (idx == ridx).all(), t
