@@ -15,7 +15,10 @@ per-sequence masks).  Reported:
   pct_bf16_peak  executed FLOPs / time / measured bf16 peak (sustained)
   skip_speedup   t(p=0) / t(p), next to the ideal 1/(1 - p_bar)
   roofline       the tcgen05 GEMM class (the dominant kernel), timed with CUDA
-                 events around its launches inside the timed region
+                 events around each of its launches over a second pass of the
+                 same steps (the library then keeps the backward's weight-
+                 gradient products on one stream, so no launch overlaps
+                 another; in the headline pass they run on a side stream)
   cpu_baseline   the CPU oracle on a bounded sample of the same workload
 
 --impl reference times the CPU oracle alone (this workload has no runnable
@@ -426,11 +429,17 @@ def main():
     for k in range(args.warmup):
         step(step0 + k)
     st.sync()
-    P.ld_set_timing(st.h, 1)
     clocks = Clocks(local)
     clocks.start()
     ms = timed(args.steps, step0 + args.warmup, step)
     clk = clocks.stop()
+    st.sync()
+    # ---- device time by kernel class: the same steps again with the
+    # library's per-launch events on, which keep the backward's
+    # weight-gradient products on the one stream (no overlap), so each
+    # launch is timed alone
+    P.ld_set_timing(st.h, 1)
+    ms_serial = timed(args.steps, step0 + args.warmup, step)
     gemm_ms, gemm_launches = P.ld_get_timing(st.h, P.LD_KCLASS_GEMM)
     attn_ms, attn_launches = P.ld_get_timing(st.h, P.LD_KCLASS_ATTN)
     row_ms, row_launches = P.ld_get_timing(st.h, P.LD_KCLASS_ROWWISE)
@@ -522,7 +531,9 @@ def main():
         "skip_speedup": (dense_ms / ms) if dense_ms else None,
         "ideal_speedup": 1.0 / (1.0 - p_real), "dense_ms_per_step": dense_ms,
         "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "attention": attn_ms / args.steps,
-                               "rowwise": row_ms / args.steps},
+                               "rowwise": row_ms / args.steps,
+                               "serialized_ms_per_step": ms_serial,
+                               "note": "separate pass, weight-gradient products not overlapped"},
         "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
         "gpu_launches": None,
     }

@@ -35,8 +35,12 @@
  *     which case every activation, weight and gain is float32.  Weight and
  *     gain gradients are always float32.
  *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All device
- *     work is enqueued on it; no entry point synchronises the host except
- *     ld_get_masks and ld_sync.
+ *     work is ordered on it: ld_backward runs the weight-gradient products
+ *     on an internal stream of the handle that forks from `stream` and joins
+ *     back into it before the call returns (so the call's work is complete
+ *     when `stream` reaches that point, and it can be captured into a CUDA
+ *     graph).  No entry point synchronises the host except ld_get_masks and
+ *     ld_sync.
  *   - Errors: argument and shape errors are returned synchronously and
  *     enqueue nothing.  A device-side error (a bounded wait that expired) is
  *     recorded in the workspace status word and returned by ld_sync.  No
@@ -249,7 +253,9 @@ typedef enum {
  * roofline of each kernel class).  enable = 1 starts recording a CUDA event
  * pair on the call's stream around every launch of ld_forward / ld_backward
  * and resets the totals; enable = 0 stops recording.  The events add no
- * synchronisation. */
+ * synchronisation.  While recording, ld_backward keeps its weight-gradient
+ * products on the caller's stream (no side stream), so that every
+ * recorded duration belongs to one launch running alone. */
 ld_status ld_set_timing(void* handle, int enable);
 
 /* Sum of the device time (ms) and number of launch groups of class `kclass`

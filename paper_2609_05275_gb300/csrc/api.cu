@@ -54,11 +54,34 @@ struct Handle {
   bool timing = false;
   std::vector<cudaEvent_t> ev[LD_KCLASS_COUNT];
   size_t ev_used[LD_KCLASS_COUNT] = {};
+  // backward: the four weight-gradient products of a layer run on a side
+  // stream forked from (and joined back to) the caller's stream; wg_in[k]
+  // orders product k after its inputs, wg_out[k] the next write of those
+  // inputs after product k
+  cudaStream_t side = nullptr;
+  cudaEvent_t wg_in[4] = {}, wg_out[4] = {};
   ~Handle() {
     for (auto& v : ev)
       for (cudaEvent_t e : v) cudaEventDestroy(e);
+    for (int k = 0; k < 4; ++k) {
+      if (wg_in[k]) cudaEventDestroy(wg_in[k]);
+      if (wg_out[k]) cudaEventDestroy(wg_out[k]);
+    }
+    if (side) cudaStreamDestroy(side);
   }
 };
+
+// Create the side stream and its events (once per handle, at the first
+// backward).
+cudaError_t ensure_side(Handle* h) {
+  if (h->side) return cudaSuccess;
+  cudaError_t e = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking);
+  for (int k = 0; k < 4 && e == cudaSuccess; ++k) {
+    e = cudaEventCreateWithFlags(&h->wg_in[k], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->wg_out[k], cudaEventDisableTiming);
+  }
+  return e;
+}
 
 // Records an event pair around the launches of its scope when timing is on.
 struct Timed {
@@ -600,6 +623,37 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     Timed tm_(h, LD_KCLASS_ROWWISE, st);
     LD_CHECK(launch_convert(dxv, 0, dx, 1, (long long)h->max_rows * c.d, st));
   }
+  // The weight gradients of a layer (dW_d, dW_gu, dW_o, dW_qkv: products
+  // 0..3) need nothing from each other or from the data-gradient chain after
+  // them, so they run on the side stream, where they fill the last partial
+  // wave of the persistent GEMMs on the caller's stream.  Product k waits
+  // for its inputs (wg_in[k]); the caller's stream waits for product k
+  // (wg_out[k]) before the next layer rewrites its scratch input.
+  // With device-time accounting on (ld_set_timing) everything stays on the
+  // caller's stream, so that each launch's events time it alone.
+  const bool overlap = !h->timing;
+  if (overlap) {
+    LD_CHECK(ensure_side(h));
+    // start every wait of this call from a record on the caller's stream (so
+    // that a stream capture never waits on an event recorded outside it)
+    for (int k = 0; k < 4; ++k) LD_CHECK(cudaEventRecord(h->wg_out[k], st));
+  }
+  auto wgrad = [&](int k, const GemmArgs& a) -> cudaError_t {
+    if (!overlap) {
+      Timed tm_(h, LD_KCLASS_GEMM, st);
+      return gemm<T>(a, st);
+    }
+    cudaError_t e = cudaEventRecord(h->wg_in[k], st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->wg_in[k], 0);
+    if (e != cudaSuccess) return e;
+    {
+      Timed tm_(h, LD_KCLASS_GEMM, h->side);
+      e = gemm<T>(a, h->side);
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(h->wg_out[k], h->side);
+    return e;
+  };
+  auto before_rewrite = [&](int k) { return overlap ? cudaStreamWaitEvent(st, h->wg_out[k], 0) : cudaSuccess; };
 
   for (int l = c.L - 1; l >= 0; --l) {
     const Rows ra = rows_of(h, ws, 0, l);  // attention block's kept rows; FFN block's below
@@ -621,7 +675,9 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     const float s = h->fwd_scale[l];
 
     // FFN branch: dy = r * dX^{l+1} on the kept rows.
+    LD_CHECK(before_rewrite(0));  // dW_d of the layer above has read dy
     { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(launch_gather_scale<T>(dx, rf.idx, rf.cnt, rf.unit, c.d, h->max_rows, s, dy, st)); }
+    LD_CHECK(before_rewrite(1));  // dW_gu of the layer above has read dgu
     GemmArgs a = rows_gemm(h, rf, c.F, c.d, dy, c.d, W[l].w_d, c.F, 1);  // dh = dy W_d
     a.epi = EPI_STORE;
     a.D = dh;
@@ -638,15 +694,16 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
       if (c.act) LD_CHECK(launch_relu2<T>(gu, dh, dgu, rf.cnt, rf.unit, c.F, h->max_rows, st));
       else LD_CHECK(launch_swiglu_bwd<T>(dh, gu, dgu, rf.cnt, rf.unit, c.F, h->max_rows, st));
     }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, rf, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d), st)); }  // dW_d = dy^T h
+    LD_CHECK(wgrad(0, wgrad_gemm(h, rf, c.d, c.F, dy, c.d, hh, c.F, G[l].w_d)));  // dW_d = dy^T h
     a = rows_gemm(h, rf, c.d, h->nf, dgu, h->nf, W[l].w_gu, c.d, 1);  // dzh = dgu W_gu
     a.epi = EPI_STORE_F32;
     a.D = dzh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, rf, h->nf, c.d, dgu, h->nf, zh, c.d, G[l].w_gu), st)); }
+    LD_CHECK(wgrad(1, wgrad_gemm(h, rf, h->nf, c.d, dgu, h->nf, zh, c.d, G[l].w_gu)));  // dW_gu = dgu^T zh
     // dZ = dX^{l+1} + RMSNorm_2 backward; dz = r * dZ for the attention branch
     // (written by the same kernel when both blocks keep the same rows)
+    LD_CHECK(before_rewrite(2));  // dW_o of the layer above has read dz
     {
       Timed tm_(h, LD_KCLASS_ROWWISE, st);
       LD_CHECK(launch_rmsnorm_bwd<T>(dzh, z, rstd2, g2, dx, rf.idx, rf.cnt, rf.unit, c.d, h->max_rows, s,
@@ -661,7 +718,8 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     a.ldd = HD;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
     if (ra.seg) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(zero_tail<T>(h, ra, dO, HD, HD, 1, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, ra, c.d, HD, dz, c.d, o, HD, G[l].w_o), st)); }  // dW_o = dz^T o
+    LD_CHECK(wgrad(2, wgrad_gemm(h, ra, c.d, HD, dz, c.d, o, HD, G[l].w_o)));  // dW_o = dz^T o
+    LD_CHECK(before_rewrite(3));  // dW_qkv of the layer above has read dqkv
     { Timed tm_(h, LD_KCLASS_ATTN, st); LD_CHECK(attn_bwd<T>(h, ws, qkv, o, dO, lse, Dvec, dqkv, ra, st)); }
     if (ra.seg) { Timed tm_(h, LD_KCLASS_ROWWISE, st); LD_CHECK(zero_tail<T>(h, ra, dqkv, h->nqkv, h->nqkv, 1, st)); }
     a = rows_gemm(h, ra, c.d, h->nqkv, dqkv, h->nqkv, W[l].w_qkv, c.d, 1);  // dxh = dqkv W_qkv
@@ -669,7 +727,7 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     a.D = dxh;
     a.ldd = c.d;
     { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
-    { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(wgrad_gemm(h, ra, h->nqkv, c.d, dqkv, h->nqkv, xh, c.d, G[l].w_qkv), st)); }
+    LD_CHECK(wgrad(3, wgrad_gemm(h, ra, h->nqkv, c.d, dqkv, h->nqkv, xh, c.d, G[l].w_qkv)));  // dW_qkv = dqkv^T xh
     // dX^l = dZ + RMSNorm_1 backward
     {
       Timed tm_(h, LD_KCLASS_ROWWISE, st);
@@ -682,6 +740,7 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
     Timed tm_(h, LD_KCLASS_ROWWISE, st);
     LD_CHECK(launch_convert(dx, 1, dxv, 0, (long long)h->max_rows * c.d, st));
   }
+  for (int k = 0; k < 4; ++k) LD_CHECK(before_rewrite(k));  // join: every weight gradient is done
   return LD_OK;
 }
 
