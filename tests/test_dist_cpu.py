@@ -5,7 +5,9 @@ sequence index, so each shard draws exactly its slice of the full batch's
 masks, computes its sequences independently, and the only exchange is the
 all-reduce (sum) of the weight gradients.  Checked with the oracle: shard
 outputs equal the full-batch slices, the all-reduced shard gradients equal
-the full-batch gradients.  Also the benchmark's max-over-ranks step time."""
+the full-batch gradients, for per-sequence masks and for per-token masks
+(keyed by the global token index).  Also the benchmark's max-over-ranks step
+time."""
 
 import os
 import socket
@@ -51,6 +53,11 @@ def _worker(rank, world, port, q):
         # per-shard granularity: each rank draws for its whole shard, keyed by its first global sequence
         shard = OM.draw_masks(5, 3, thr, Bs, OM.PER_SHARD, b_offset=rank * Bs)
         ok_mask = ok_mask and bool((shard == full_mask[:, rank * Bs:rank * Bs + 1]).all())
+        # per-token granularity: a shard's tokens are the global tokens of its sequences
+        S = cfg["S"]
+        full_tok = OM.draw_masks(5, 3, thr, B, OM.PER_TOKEN, S=S)
+        tok = OM.draw_masks(5, 3, thr, Bs, OM.PER_TOKEN, b_offset=rank * Bs, S=S)
+        ok_mask = ok_mask and bool((tok == full_tok[:, rank * Bs:(rank + 1) * Bs]).all())
         layers = [{n: v.double().numpy() for n, v in W.items()} for W in synth.stack_weights(cfg, seed=0)]
         x = synth.activations(cfg, seed=0, B=B).double().numpy()
         dy = synth.upstream_grad(cfg, B=B).double().numpy()
@@ -63,6 +70,15 @@ def _worker(rank, world, port, q):
                 t = torch.from_numpy(g.copy())
                 dist.all_reduce(t, op=dist.ReduceOp.SUM)
                 summed[(l, n)] = t.numpy()
+        # the same with per-token masks
+        tout, tc = OK.stack_forward(x[sl], layers, cfg, tok, scales, per_token=True)
+        tdX, tgrads = OK.stack_backward(dy[sl], layers, cfg, tok, scales, tc, per_token=True)
+        tsummed = {}
+        for l in range(cfg["L"]):
+            for n, g in tgrads[l].items():
+                t = torch.from_numpy(g.copy())
+                dist.all_reduce(t, op=dist.ReduceOp.SUM)
+                tsummed[(l, n)] = t.numpy()
         ms = bench.max_over_ranks(10.0 + rank, world, device="cpu")
         res = dict(rank=rank, ok_mask=ok_mask, ms=ms)
         if rank == 0:
@@ -71,6 +87,11 @@ def _worker(rank, world, port, q):
             res["out_ok"] = bool(np.array_equal(out, fout[sl]) and np.array_equal(dX, fdX[sl]))
             res["grad_err"] = max(float(np.abs(summed[(l, n)] - fg[l][n]).max() / (np.abs(fg[l][n]).max() + 1e-30))
                                   for l in range(cfg["L"]) for n in fg[l])
+            gout, gc = OK.stack_forward(x, layers, cfg, full_tok, scales, per_token=True)
+            gdX, gg = OK.stack_backward(dy, layers, cfg, full_tok, scales, gc, per_token=True)
+            res["tok_out_ok"] = bool(np.array_equal(tout, gout[sl]) and np.array_equal(tdX, gdX[sl]))
+            res["tok_grad_err"] = max(float(np.abs(tsummed[(l, n)] - gg[l][n]).max() / (np.abs(gg[l][n]).max() + 1e-30))
+                                      for l in range(cfg["L"]) for n in gg[l])
         q.put(res)
     finally:
         dist.destroy_process_group()
@@ -93,3 +114,5 @@ def test_two_rank_shards_match_full_batch():
     assert all(r["ms"] == 11.0 for r in res.values())  # slowest rank's time
     assert res[0]["out_ok"]
     assert res[0]["grad_err"] < 1e-12
+    assert res[0]["tok_out_ok"]
+    assert res[0]["tok_grad_err"] < 1e-12
