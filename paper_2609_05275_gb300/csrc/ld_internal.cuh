@@ -79,7 +79,7 @@ cudaError_t launch_mask_compact(const MaskParams& P, unsigned char* mask, int* k
 
 // Zero rows [*start, min(*start + nrows, max_rows)) of `planes` row-major
 // matrices (plane p at buf + p * plane_ld elements, row stride ld, the first
-// ncols columns); ncols * sizeof(T) a multiple of 16 bytes when planes == 1.
+// ncols columns), one element per thread.
 template <typename T>
 cudaError_t launch_zero_rows(T* buf, int ld, int ncols, int planes, long long plane_ld, const int* start, int nrows,
                              int max_rows, cudaStream_t st);
