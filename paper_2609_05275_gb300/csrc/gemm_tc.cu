@@ -10,7 +10,8 @@
 //
 // Structure (persistent, one CTA per SM, 192 threads):
 //   warp 0      TMA producer: 128B-swizzled tiles of A (128 x 64) and
-//               B (BN x 64) into a STAGES-deep shared-memory ring;
+//               B (BN x 64) into a STAGES-deep shared-memory ring whose
+//               stages hold KPS such k-blocks (one barrier hand-off each);
 //   warp 1      allocates 2*BN TMEM columns (two accumulators) and issues
 //               tcgen05.mma (M=128, N=BN, K=16) from one thread;
 //   warps 2..5  epilogue: tcgen05.ld of the accumulator (each warp reads
@@ -26,7 +27,10 @@
 //
 // Every mbarrier wait is bounded: after kWaitLimitNs the CTA raises the
 // status word (LD_ERR_TIMEOUT), drains its own TMA copies and MMAs with a
-// further bounded wait, frees its TMEM and exits.
+// further bounded wait, frees its TMEM and exits (a CTA pair meets at a
+// cluster barrier first, so neither frees memory the other may address).
+// Per-token kept lists pass padding rows (kept index -1): the residual
+// epilogue skips them and writes zeros to its compact copy.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
