@@ -12,6 +12,10 @@
 // Dropout Scale paragraph).  Rows of dropped sequences are never touched.
 // The backward walks the layers in reverse and mirrors this; the gradient
 // of a dropped row passes through unchanged (it is the identity there).
+// Per-token kept lists run the same sequence with row unit 1 (see Rows): the
+// compact rows are kept tokens, attention works on per-sequence segments.
+// The backward's weight-gradient products run on a side stream (see
+// backward_impl).
 #include <cmath>
 #include <cstdio>
 #include <cstring>

@@ -26,6 +26,10 @@
 // m_h (j - i) to the scaled score of query i and key j: the scores are first
 // turned into biased base-2 logits x = S c log2e + m_h log2e (j - i), and the
 // max and P = exp2(x - m) work on x.
+// The two warps of a row pass their partial maxima through tagged 64-bit
+// shared-memory words (tile index, value), a bounded spin per tile.
+// With per-token kept lists a sequence is a segment of arbitrary length
+// (seg[b] .. seg[b+1]-1); rows of a tile past its end are never stored.
 #include <type_traits>
 
 #include "tc_common.cuh"
