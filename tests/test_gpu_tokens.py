@@ -135,3 +135,14 @@ def test_token_all_dropped_is_identity(fp32):
     for G in grads:
         for n, g in G.items():
             assert (g == 0).all(), n
+
+
+@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
+def test_token_tiny_and_empty_segments(fp32):
+    # p close to 1 over short sequences: segments of 0, 1, 2, ... kept tokens
+    # side by side (a sequence with none, its neighbours with a few)
+    cfg = dict(TINY, B=16, S=64) if fp32 else dict(TOK, B=16, S=128, L=2)
+    sched = dict(dist="uniform", p_max=0.985 if not fp32 else 0.97, time="const", seed=21)
+    rmask = _compare(cfg, sched, 0, fp32)
+    lens = rmask.reshape(-1, cfg["B"], cfg["S"]).sum(axis=2)
+    assert (lens == 0).any() and (lens > 0).any() and (lens <= 3).any()
