@@ -83,3 +83,28 @@ def test_eval_matches_training_forward_at_p0():
                                                for W in layers]))
     finally:
         st.close()
+
+
+@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
+def test_eval_on_per_token_handle(fp32):
+    # the evaluation forward runs whole sequences whatever the handle's
+    # granularity: a per-token handle gives the per-sequence handle's output
+    # bit for bit (its larger mask tables hold the per-sequence lists)
+    cfg = (dict(synth.CONFIGS["tiny"], L=3) if fp32 else
+           dict(L=3, d=256, H=2, Hkv=1, Dh=128, F=512, B=3, S=256, eps=1e-6, rope_theta=1e4, alpha=1.0))
+    dtype = torch.float32 if fp32 else torch.bfloat16
+    host = synth.stack_weights(cfg, seed=4, gamma_noise=0.1)
+    dev = [{n: v.to(dtype).cuda() for n, v in W.items()} for W in host]
+    x = synth.activations(cfg, seed=4).to(dtype).cuda()
+    outs = []
+    for gran in ("per_sequence", "per_token"):
+        st = P.LayerDropStack(cfg, dict(dist="uniform", p_max=0.0, seed=1), granularity=gran, fp32_debug=fp32)
+        try:
+            out = x.clone()
+            st.forward_eval([1, 0, 1], P.weight_table(dev), out)
+            torch.cuda.synchronize()
+            st.sync()
+            outs.append(out)
+        finally:
+            st.close()
+    assert torch.equal(outs[0], outs[1])
