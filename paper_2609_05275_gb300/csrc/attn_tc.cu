@@ -451,6 +451,306 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 
 
 // ---------------------------------------------------------------------------
+// Forward, head size 128 without a position bias: two 128-query tiles per CTA
+// ("ping-pong").  Each tile has its own softmax group of four warps with one
+// query row and all 128 keys of a K tile per thread, so no two warps share a
+// row; the MMA warp alternates between the groups, and one group's softmax
+// runs while the tensor pipe works for the other:
+//   warp 0      TMA: both Q tiles once, then K_j and V_j (three-stage K ring,
+//               two-stage V ring), K one tile ahead of V;
+//   warp 1      TMEM allocation and, per K tile j: P_A(j-1) V_{j-1}, S_A(j) =
+//               Q_A K_j^T, P_B(j-1) V_{j-1}, S_B(j) = Q_B K_j^T;
+//   warps 2..5  softmax of tile A (the block's first 128 queries), warps
+//               6..9 of tile B.
+// TMEM columns: S_A 0-127, S_B 128-255, O_A 256-383, O_B 384-511.  P_g is
+// written as bf16 pairs over the first 64 columns of S_g once S_g has been
+// read (the next S_g MMA is issued after the P_g V MMA that reads it).  MMAs
+// run in issue order, so S_g(j) complete implies P_g(j-1) V_{j-1} complete:
+// the group may rescale O_g as soon as S_g(j) is ready.  Tile B is skipped
+// when the sequence ends before it.
+constexpr int PP_NSK = 3, PP_NSV = 2;
+
+__global__ void __launch_bounds__(320, 1)
+    attn_fwd_pp_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
+                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv, const int* __restrict__ seg,
+                       int* status) {
+  constexpr int DH = 128;
+  constexpr uint32_t TILE = 2 * SLAB;  // one 128 x 128 bf16 tile (two 64-column slabs)
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Qs = smem;                 // [2] query tiles
+  uint8_t* Ks = Qs + 2 * TILE;        // [PP_NSK]
+  uint8_t* Vs = Ks + PP_NSK * TILE;   // [PP_NSV]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + PP_NSV * TILE);
+  uint64_t* q_full = bars;
+  uint64_t* k_full = q_full + 1;      // [PP_NSK]
+  uint64_t* k_empty = k_full + PP_NSK;
+  uint64_t* v_full = k_empty + PP_NSK;  // [PP_NSV]
+  uint64_t* v_empty = v_full + PP_NSV;
+  uint64_t* s_full = v_empty + PP_NSV;  // [2] per query tile
+  uint64_t* p_full = s_full + 2;        // [2]
+  uint64_t* o_full = p_full + 2;        // [2]
+  uint64_t* drain = o_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int seq = blockIdx.y;
+  int row0, len;
+  if (seg) {
+    row0 = seg[seq];
+    len = seg[seq + 1] - row0;
+  } else {
+    if (seq >= *cnt) return;
+    row0 = seq * S;
+    len = S;
+  }
+  const int nqb = (S + 255) / 256;
+  const int qb = nqb - 1 - blockIdx.z;  // heaviest query blocks first
+  if (qb * 256 >= len) return;
+  const bool vB = qb * 256 + 128 < len;  // tile B holds queries of the sequence
+  const int nkA = 2 * qb + 1, nkB = vB ? 2 * qb + 2 : 0;  // K tiles of tile A / B (through its diagonal)
+  const int nkt = vB ? nkB : nkA;
+  const int h = blockIdx.x, g = (h * Hkv) / H;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < PP_NSK; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < PP_NSV; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&p_full[b], 4);
+      mbar_init(&o_full[b], 1);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      const int qcol = h * DH, kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
+      const int nq = vB ? 2 : 1;
+      mbar_arrive_expect_tx(q_full, nq * TILE);
+      for (int t = 0; t < nq; ++t)
+        for (int c = 0; c < 2; ++c)
+          tma_load_2d(Qs + t * TILE + c * SLAB, &tm, qcol + 64 * c, row0 + qb * 256 + t * 128, q_full);
+      int nkl = 0, nvl = 0;
+      for (int j = 0; j <= nkt; ++j) {
+        if (j < nkt) {
+          const int s = j % PP_NSK;
+          if (!mbar_wait(&k_empty[s], ((j / PP_NSK) & 1) ^ 1u, abort_flag, status)) break;
+          mbar_arrive_expect_tx(&k_full[s], TILE);
+          for (int c = 0; c < 2; ++c)
+            tma_load_2d(Ks + s * TILE + c * SLAB, &tm, kcol + 64 * c, row0 + j * 128, &k_full[s]);
+          ++nkl;
+        }
+        if (j >= 1) {
+          const int jv = j - 1, s = jv % PP_NSV;
+          if (!mbar_wait(&v_empty[s], ((jv / PP_NSV) & 1) ^ 1u, abort_flag, status)) break;
+          mbar_arrive_expect_tx(&v_full[s], TILE);
+          for (int c = 0; c < 2; ++c)
+            tma_load_2d(Vs + s * TILE + c * SLAB, &tm, vcol + 64 * c, row0 + jv * 128, &v_full[s]);
+          ++nvl;
+        }
+      }
+      if (*abort_flag) {
+        mbar_drain(q_full, 0);
+        for (int j = nkl > PP_NSK ? nkl - PP_NSK : 0; j < nkl; ++j) mbar_drain(&k_full[j % PP_NSK], (j / PP_NSK) & 1);
+        for (int j = nvl > PP_NSV ? nvl - PP_NSV : 0; j < nvl; ++j) mbar_drain(&v_full[j % PP_NSV], (j / PP_NSV) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
+      constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
+      const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
+      bool ok = mbar_wait(q_full, 0, abort_flag, status);
+      for (int j = 0; ok && j <= nkt; ++j) {
+        if (j < nkt && !mbar_wait(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
+        if (j >= 1 && !mbar_wait(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
+          ok = false;
+          break;
+        }
+        for (int gi = 0; gi < 2; ++gi) {
+          const int nkg = gi ? nkB : nkA;
+          if (j >= 1 && j - 1 < nkg) {
+            // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
+            if (!mbar_wait(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
+            tc_fence_after();
+            const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              mma_bf16_ta(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
+                          (j > 1 || kk > 0) ? 1u : 0u);
+            if (j == nkg) mma_commit(&o_full[gi]);  // the group's last P V
+          }
+          if (j < nkg) {
+            // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
+            const uint64_t kb = DK + (uint64_t)(((j % PP_NSK) * TILE) >> 4);
+            const uint64_t qd = DQ + (uint64_t)((gi * TILE) >> 4);
+#pragma unroll
+            for (int kk = 0; kk < DH / 16; ++kk) {
+              const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+              mma_bf16(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
+            }
+            mma_commit(&s_full[gi]);
+          }
+        }
+        if (!ok) break;
+        if (j < nkt) mma_commit(&k_empty[j % PP_NSK]);
+        if (j >= 1) mma_commit(&v_empty[(j - 1) % PP_NSV]);
+      }
+      if (!ok) {
+        mma_commit(drain);
+        mbar_drain(drain, 0);
+      }
+    }
+  } else {
+    // ------------------------------------------------ softmax (warps 2..9)
+    const int gi = (warp - 2) >> 2;  // 0: tile A, 1: tile B
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;  // query row within the tile
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const uint32_t t_s = tmem + gi * 128, t_og = tmem + 256 + gi * 128;
+    const int nkg = gi ? nkB : nkA;
+    const int jdiag = 2 * qb + gi;  // the K tile on this query tile's diagonal
+    const float sl2 = kLog2e * rsqrtf((float)DH);
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkg; ++j) {
+      if (!warp_wait(&s_full[gi], j & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      const bool diag = (j == jdiag);  // keys after the query are left out (block-uniform)
+      // pass 1: row max of the raw scores (the scale is positive)
+      float mraw = -INFINITY;
+#pragma unroll 1
+      for (int c2 = 0; c2 < 2; ++c2) {
+        uint32_t sr[2][32];
+        tmem_ld32_nw(t_s + c2 * 64 + lane_off, sr[0]);
+        tmem_ld32_nw(t_s + c2 * 64 + 32 + lane_off, sr[1]);
+        tmem_wait_ld();
+        if (diag) {
+#pragma unroll
+          for (int e = 0; e < 64; ++e)
+            mraw = fmaxf(mraw, c2 * 64 + e <= r ? __uint_as_float(sr[e >> 5][e & 31]) : -INFINITY);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 64; e += 2)
+            mraw = fmax3(mraw, __uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1]));
+        }
+      }
+      const float mt = mraw * sl2;
+      const bool rescale = mt > m_used + kRescale;
+      const float m_new = rescale ? mt : m_used;
+      // O_g is rescaled in TMEM when any lane of the warp moved its max
+      // (P_g(j-1) V_{j-1} is complete: it was issued before S_g(j))
+      if (j >= 1 && __any_sync(0xffffffffu, rescale)) {
+        const float corr = rescale ? exp2f(m_used - m_new) : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < DH / 32; ++c) {
+          float t[32];
+          tmem_ld32(t_og + c * 32 + lane_off, t);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) t[e] *= corr;
+          tmem_st32(t_og + c * 32 + lane_off, t);
+        }
+      }
+      if (rescale) {
+        l *= exp2f(m_used - m_new);
+        m_used = m_new;
+      }
+      // pass 2: P = exp2(S c log2e - m) for 32 keys at a time, written as
+      // bf16 pairs over S columns that have already been read
+      const uint64_t sl2x2 = f2_pack(sl2, sl2), nm2 = f2_pack(-m_new, -m_new);
+      uint64_t ls2 = f2_pack(0.f, 0.f);
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        uint32_t sr[32];
+        tmem_ld32_nw(t_s + c * 32 + lane_off, sr);
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, nm2), x0, x1);
+          float p0 = ex2(x0), p1 = ex2(x1);
+          if (diag) {
+            p0 = (c * 32 + 2 * e <= r) ? p0 : 0.f;
+            p1 = (c * 32 + 2 * e + 1 <= r) ? p1 : 0.f;
+          }
+          ls2 = f2_add(ls2, f2_pack(p0, p1));
+          pk[e] = bf16x2_bits(p0, p1);
+        }
+        tmem_st16(t_s + c * 16 + lane_off, pk);  // keys 32c .. 32c+31 -> packed columns 16c .. 16c+15
+      }
+      tmem_wait_st();
+      float ls_a, ls_b;
+      f2_unpack(ls2, ls_a, ls_b);
+      l += ls_a + ls_b;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[gi]);
+    }
+    const bool has_tile = gi == 0 || vB;
+    if (ok && has_tile && warp_wait(&o_full[gi], 0, abort_flag, status)) {
+      tc_fence_after();
+      const float inv = 1.0f / l;
+      const int qrow = qb * 256 + gi * 128 + r;
+      const bool valid = qrow < len;
+      bf16* orow = o + (long long)(row0 + qrow) * ldo + (long long)h * DH;
+#pragma unroll 1
+      for (int c = 0; c < DH / 32; ++c) {
+        float t[32];
+        tmem_ld32(t_og + c * 32 + lane_off, t);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) t[e] *= inv;
+        if (valid) st_bf16x32_(orow + c * 32, t);
+      }
+      if (valid) lse[(size_t)h * lse_ld + row0 + qrow] = (m_used + log2f(l)) * kLn2;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
+                   int max_seqs, const int* seg, int* status, cudaStream_t st) {
+  // 2 Q, 3 K and 2 V tiles of 32 KB + alignment + barriers = 230,656 bytes (of 232,448)
+  constexpr size_t smem = (size_t)(2 + PP_NSK + PP_NSV) * 2 * SLAB + 1024 + 256;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_pp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  CUtensorMap tm;
+  if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
+  dim3 grid(H, max_seqs, (S + 255) / 256);
+  attn_fwd_pp_kernel<<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, seg, status);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // Backward, head size 128.  One CTA per (128-key tile, kv head, kept
 // sequence), looping over the query heads of the group and the 64-query
 // tiles at or after the key tile.  448 threads:
@@ -880,7 +1180,7 @@ cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, flo
     return fwd_tc<128, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
   }
   if (Dh == 64) return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
-  return fwd_tc<128, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  return fwd_pp(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, seg, status, st);
 }
 
 }  // namespace ldk
