@@ -221,51 +221,51 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
-      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
-      constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
-      // descriptors built once, advanced by (byte offset >> 4) per MMA
-      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
-      const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
-      bool ok = mbar_wait(q_full, 0, abort_flag, status);
-      for (int j = 0; ok && j <= nkt; ++j) {
-        if (j < nkt) {
-          const int s = j % NSK;
-          if (!mbar_wait(&k_full[s], (j / NSK) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t kb = DK + (uint64_t)((s * TILE) >> 4);
+    __syncwarp();
+    // ------------------------------------------------ MMA issuer
+    constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
+    constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
+    // descriptors built once, advanced by (byte offset >> 4) per MMA
+    const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
+    const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
+    bool ok = warp_wait(q_full, 0, abort_flag, status);
+    for (int j = 0; ok && j <= nkt; ++j) {
+      if (j < nkt) {
+        const int s = j % NSK;
+        if (!warp_wait(&k_full[s], (j / NSK) & 1, abort_flag, status)) { ok = false; break; }
+        if (!warp_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+        const uint64_t kb = DK + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk) {
-            const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-            mma_bf16(tmem + (j & 1) * 128, DQ + off, kb + off, ID_S, kk > 0);
-          }
-          mma_commit(&s_full[j & 1]);
-          mma_commit(&k_empty[s]);
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+          mma_bf16_w(tmem + (j & 1) * 128, DQ + off, kb + off, ID_S, kk > 0);
         }
-        if (j >= 1) {
-          const int jp = j - 1, s = jp % NSV, pb = jp & 1;
-          if (!mbar_wait(&p_full[pb], (jp >> 1) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(&v_full[s], (jp / NSV) & 1, abort_flag, status)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t vb = DV + (uint64_t)((s * TILE) >> 4);
+        mma_commit_w(&s_full[j & 1]);
+        mma_commit_w(&k_empty[s]);
+      }
+      if (j >= 1) {
+        const int jp = j - 1, s = jp % NSV, pb = jp & 1;
+        if (!warp_wait(&p_full[pb], (jp >> 1) & 1, abort_flag, status)) { ok = false; break; }
+        if (!warp_wait(&v_full[s], (jp / NSV) & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+        const uint64_t vb = DV + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            // A = P from TMEM (16 keys = 8 columns a step); B = V as MN-major
-            // (dh contiguous): 64-dh chunks one slab apart, 8-key groups 1 KB
-            mma_bf16_ta(t_o, t_p + pb * 64 + kk * 8, vb + ((kk * 2048) >> 4), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
-          }
-          mma_commit(&pv_done[pb]);
-          mma_commit(&v_empty[s]);
+        for (int kk = 0; kk < 8; ++kk) {
+          // A = P from TMEM (16 keys = 8 columns a step); B = V as MN-major
+          // (dh contiguous): 64-dh chunks one slab apart, 8-key groups 1 KB
+          mma_bf16_ta_w(t_o, t_p + pb * 64 + kk * 8, vb + ((kk * 2048) >> 4), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
         }
+        mma_commit_w(&pv_done[pb]);
+        mma_commit_w(&v_empty[s]);
       }
-      if (ok) {
-        mma_commit(o_full);
-      } else {
-        mma_commit(drain);
-        mbar_drain(drain, 0);
-      }
+    }
+    if (ok) {
+      mma_commit_w(o_full);
+    } else {
+      mma_commit_w(drain);
+      if (lane == 0) mbar_drain(drain, 0);
+      __syncwarp();
     }
   } else {
     // ------------------------------------------------ softmax (warps 2..9)
@@ -573,52 +573,52 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
-      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
-      constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
-      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
-      const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
-      bool ok = mbar_wait(q_full, 0, abort_flag, status);
-      for (int j = 0; ok && j <= nkt; ++j) {
-        if (j < nkt && !mbar_wait(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
-        if (j >= 1 && !mbar_wait(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
-          ok = false;
-          break;
-        }
-        for (int gi = 0; gi < 2; ++gi) {
-          const int nkg = gi ? nkB : nkA;
-          if (j >= 1 && j - 1 < nkg) {
-            // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
-            if (!mbar_wait(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
-            tc_fence_after();
-            const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
+    // ------------------------------------------------ MMA issuer (whole warp, converged; one elected lane issues)
+    constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
+    constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
+    const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
+    const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
+    __syncwarp();
+    bool ok = warp_wait(q_full, 0, abort_flag, status);
+    for (int j = 0; ok && j <= nkt; ++j) {
+      if (j < nkt && !warp_wait(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
+      if (j >= 1 && !warp_wait(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
+        ok = false;
+        break;
+      }
+      for (int gi = 0; gi < 2; ++gi) {
+        const int nkg = gi ? nkB : nkA;
+        if (j >= 1 && j - 1 < nkg) {
+          // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
+          if (!warp_wait(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_bf16_ta(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
+          for (int kk = 0; kk < 8; ++kk)
+            mma_bf16_ta_w(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
                           (j > 1 || kk > 0) ? 1u : 0u);
-            if (j == nkg) mma_commit(&o_full[gi]);  // the group's last P V
-          }
-          if (j < nkg) {
-            // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
-            const uint64_t kb = DK + (uint64_t)(((j % PP_NSK) * TILE) >> 4);
-            const uint64_t qd = DQ + (uint64_t)((gi * TILE) >> 4);
-#pragma unroll
-            for (int kk = 0; kk < DH / 16; ++kk) {
-              const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-              mma_bf16(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
-            }
-            mma_commit(&s_full[gi]);
-          }
+          if (j == nkg) mma_commit_w(&o_full[gi]);  // the group's last P V
         }
-        if (!ok) break;
-        if (j < nkt) mma_commit(&k_empty[j % PP_NSK]);
-        if (j >= 1) mma_commit(&v_empty[(j - 1) % PP_NSV]);
+        if (j < nkg) {
+          // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
+          const uint64_t kb = DK + (uint64_t)(((j % PP_NSK) * TILE) >> 4);
+          const uint64_t qd = DQ + (uint64_t)((gi * TILE) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+            mma_bf16_w(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
+          }
+          mma_commit_w(&s_full[gi]);
+        }
       }
-      if (!ok) {
-        mma_commit(drain);
-        mbar_drain(drain, 0);
-      }
+      if (!ok) break;
+      if (j < nkt) mma_commit_w(&k_empty[j % PP_NSK]);
+      if (j >= 1) mma_commit_w(&v_empty[(j - 1) % PP_NSV]);
+    }
+    if (!ok) {
+      mma_commit_w(drain);
+      if (lane == 0) mbar_drain(drain, 0);
+      __syncwarp();
     }
   } else {
     // ------------------------------------------------ softmax (warps 2..9)
@@ -893,63 +893,63 @@ __global__ void __launch_bounds__(448, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
-      constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
-      constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
-      constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
-      // shared-memory descriptors built once; an MMA's operand is its base
-      // plus (byte offset >> 4) in the address field (every tile lies below
-      // 256 KB, so the 14-bit field never carries)
-      const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
-      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
-      const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
-      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
-      bool ok = mbar_wait(kv_full, 0, abort_flag, status);
-      for (int i = 0; ok && i <= n_it; ++i) {
-        if (i < n_it) {
-          const int b = i % NST;
-          if (!mbar_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t st = (uint64_t)((b * QT) >> 4);
+    __syncwarp();
+    // ------------------------------------------------ MMA issuer
+    constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
+    constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
+    constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
+    // shared-memory descriptors built once; an MMA's operand is its base
+    // plus (byte offset >> 4) in the address field (every tile lies below
+    // 256 KB, so the 14-bit field never carries)
+    const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
+    const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
+    const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
+    const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
+    bool ok = warp_wait(kv_full, 0, abort_flag, status);
+    for (int i = 0; ok && i <= n_it; ++i) {
+      if (i < n_it) {
+        const int b = i % NST;
+        if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
+        if (!warp_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+        const uint64_t st = (uint64_t)((b * QT) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk) {
-            const uint32_t koff = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-            const uint32_t qoff = ((kk >> 2) * HSLAB + (kk & 3) * 32) >> 4;
-            mma_bf16(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
-            mma_bf16(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
-          }
-          mma_commit(sdp_full);
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const uint32_t koff = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+          const uint32_t qoff = ((kk >> 2) * HSLAB + (kk & 3) * 32) >> 4;
+          mma_bf16_w(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
+          mma_bf16_w(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
         }
-        if (i >= 1) {
-          const int ip = i - 1, b = ip % NST, pb = ip & 1;
-          if (!mbar_wait(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t st = (uint64_t)((b * QT) >> 4), ds = (uint64_t)((pb * SLAB) >> 4);
-          const uint32_t first = ip > 0 ? 1u : 0u;
+        mma_commit_w(sdp_full);
+      }
+      if (i >= 1) {
+        const int ip = i - 1, b = ip % NST, pb = ip & 1;
+        if (!warp_wait(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
+        if (!warp_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+        const uint64_t st = (uint64_t)((b * QT) >> 4), ds = (uint64_t)((pb * SLAB) >> 4);
+        const uint32_t first = ip > 0 ? 1u : 0u;
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
-            const uint32_t aoff = (kk * 32) >> 4;                // dS^T, K-major
-            const uint32_t boff = (kk * 2048) >> 4;              // dO / Q as MN-major
-            mma_bf16_ta(t_dv, t_p + pb * 32 + kk * 8, DOMN + st + boff, ID_KV, kk > 0 ? 1u : first);
-            mma_bf16(t_dk, DS + ds + aoff, DQMN + st + boff, ID_KV, kk > 0 ? 1u : first);
-          }
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
-            mma_bf16(t_dq, DKMN + ((kk * 2048) >> 4), DS + ds + ((kk * 2048) >> 4), ID_Q, kk > 0);
-          }
-          mma_commit(&mm_done[pb]);
-          mma_commit(&ld_empty[b]);
+        for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
+          const uint32_t aoff = (kk * 32) >> 4;                // dS^T, K-major
+          const uint32_t boff = (kk * 2048) >> 4;              // dO / Q as MN-major
+          mma_bf16_ta_w(t_dv, t_p + pb * 32 + kk * 8, DOMN + st + boff, ID_KV, kk > 0 ? 1u : first);
+          mma_bf16_w(t_dk, DS + ds + aoff, DQMN + st + boff, ID_KV, kk > 0 ? 1u : first);
         }
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
+          mma_bf16_w(t_dq, DKMN + ((kk * 2048) >> 4), DS + ds + ((kk * 2048) >> 4), ID_Q, kk > 0);
+        }
+        mma_commit_w(&mm_done[pb]);
+        mma_commit_w(&ld_empty[b]);
       }
-      if (ok) {
-        mma_commit(acc_done);
-      } else {
-        mma_commit(drain);
-        mbar_drain(drain, 0);
-      }
+    }
+    if (ok) {
+      mma_commit_w(acc_done);
+    } else {
+      mma_commit_w(drain);
+      if (lane == 0) mbar_drain(drain, 0);
+      __syncwarp();
     }
   } else if (warp < 10) {
     // ------------------------------------------------ P / dS (warps 2..9)
