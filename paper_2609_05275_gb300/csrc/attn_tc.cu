@@ -764,7 +764,9 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 //               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
 //               swizzled shared-memory tile; at the end dK (times c) and dV
 //               from TMEM to dqkv
-//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
+//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer by global
+//               reductions from registers (shared memory bandwidth is what
+//               bounds this kernel, so dQ is not staged there)
 // P^T and dS^T are double-buffered (step i uses buffer i & 1), so the
 // softmax warps write step i while the MMAs of step i-1 still read theirs.
 // TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447,
@@ -781,7 +783,7 @@ __device__ __forceinline__ float4 ld4s(const float* p, int e4, int off) {
 template <bool ALIBI>
 __global__ void __launch_bounds__(448, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
-                       const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
+                       const __grid_constant__ CUtensorMap tmo,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
@@ -798,12 +800,11 @@ __global__ void __launch_bounds__(448, 1)
   uint8_t* Qs = Vs + KT;         // [NST][QT]
   uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
   uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
-  float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
   // [NST][lse 68 | D 68]: the 64 values of a step start at float `voff` of
   // each half (a sequence's rows start anywhere with per-token kept lists,
   // and a bulk copy needs a 16-byte aligned source, so 68 are copied from
   // the aligned-down address)
-  float* vecs = dqs + 64 * DH;
+  float* vecs = reinterpret_cast<float*>(DSs + 2 * SLAB);
   constexpr int VS = 136;
   uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * VS);
   uint64_t* kv_full = bars;
@@ -1087,12 +1088,15 @@ __global__ void __launch_bounds__(448, 1)
     }
   } else {
     // ------------------------------------------------ dQ (warps 10..13)
-    // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
-    // into dq_acc by one bulk tensor reduce per step.
+    // dQ^T from TMEM (one head dimension per thread, the step's 64 queries
+    // along the columns), added into the float32 dQ buffer by global
+    // reductions straight from registers: consecutive lanes hold consecutive
+    // head dimensions, so each reduction of a warp covers 128 contiguous
+    // bytes.  Queries past the sequence are skipped.
     const int quad = warp & 3;
     const int dd = quad * 32 + lane;  // head dimension of this thread
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const bool leader = (warp == 10 && lane == 0);
+    const size_t ldd = (size_t)H * DH;
     for (int i = 0; i < n_it; ++i) {
       const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
       if (!warp_wait(&mm_done[i & 1], (i >> 1) & 1, abort_flag, status)) break;
@@ -1103,20 +1107,22 @@ __global__ void __launch_bounds__(448, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(dq_free);
-      if (leader && i > 0) bulk_wait_read();  // the previous reduce has read the tile
-      named_barrier(1, 128);
+      const int nv = min(64, len - qt * 64);  // queries of the step inside the sequence (warp-uniform)
+      float* dst = dq_acc + (size_t)(row0 + qt * 64) * ldd + (size_t)h * DH + dd;
+      if (nv == 64) {
 #pragma unroll
-      for (int e = 0; e < 32; ++e) dqs[e * DH + dd] = t0[e];
+        for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)e * ldd, t0[e]);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) dqs[(32 + e) * DH + dd] = t1[e];
-      fence_proxy_async();
-      named_barrier(1, 128);
-      if (leader) {
-        tma_reduce_add_2d(&tmdq, h * DH, row0 + qt * 64, dqs);
-        bulk_commit();
+        for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(32 + e) * ldd, t1[e]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (e < nv) atomicAdd(dst + (size_t)e * ldd, t0[e]);
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (32 + e < nv) atomicAdd(dst + (size_t)(32 + e) * ldd, t1[e]);
       }
     }
-    if (leader) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -1133,8 +1139,8 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
                    const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
                    cudaStream_t st) {
   // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
-  // vectors + dQ staging + alignment + barriers = 232,288 bytes (of 232,448)
-  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 136 * 4 + 64 * 128 * 4 + 1024 + 256;
+  // vectors + alignment + barriers = 199,520 bytes
+  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 136 * 4 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
@@ -1142,14 +1148,12 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  CUtensorMap tkv, tq, to, tdq;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows; dQ reduce boxes
-  if (!make_map_f32(&tdq, dq_acc, (uint64_t)H * 128, (uint64_t)max_seqs * S, (uint64_t)H * 128, 128, 64))
-    return cudaErrorInvalidValue;
+  CUtensorMap tkv, tq, to;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
   dim3 grid(Hkv, max_seqs, S / 128);
-  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
+  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
                                                      H, Hkv, rcos, rsin, alibi, seg, tok, status);
   return cudaGetLastError();
 }
