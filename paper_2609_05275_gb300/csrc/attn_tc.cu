@@ -221,8 +221,8 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (whole warp, converged; one elected lane issues)
     __syncwarp();
-    // ------------------------------------------------ MMA issuer
     constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
     constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
     // descriptors built once, advanced by (byte offset >> 4) per MMA
@@ -754,16 +754,19 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // Backward, head size 128.  One CTA per (128-key tile, kv head, kept
 // sequence), looping over the query heads of the group and the 64-query
 // tiles at or after the key tile.  448 threads:
-//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
+//   warp 0      TMA: K, V once; Q_i, dO_i per step (3 stages); all lanes
+//               write the bf16 terms of -lse_i sqrt(Dh) and -D_i that two extra
+//               K = 16 MMAs fold into S^T_i and dP^T_i
 //   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
 //               (M = 128 keys, N = 64 queries); then for step i-1
 //               dV += P^T dO (P^T read from TMEM), dK += dS^T Q (M = 128
 //               keys, N = 128) and dQ^T = K^T dS^T (M = 128 head dims,
 //               N = 64 queries)
 //   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e)
-//               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
-//               swizzled shared-memory tile; at the end dK (times c) and dV
-//               from TMEM to dqkv
+//               as bf16 into TMEM and dS^T = P^T (dP^T - D) as bf16 into a
+//               swizzled shared-memory tile, the lse and D terms already
+//               inside S^T and dP^T; at the end dK (times c) and dV from
+//               TMEM to dqkv
 //   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer by global
 //               reductions from registers (shared memory bandwidth is what
 //               bounds this kernel, so dQ is not staged there)
@@ -773,11 +776,17 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
-// Values 4 e4 .. 4 e4 + 3 of p (shared memory); p is 16-byte aligned when
-// off == 0 (warp-uniform), else read one by one.
-__device__ __forceinline__ float4 ld4s(const float* p, int e4, int off) {
-  if (off == 0) return reinterpret_cast<const float4*>(p)[e4];
-  return make_float4(p[4 * e4], p[4 * e4 + 1], p[4 * e4 + 2], p[4 * e4 + 3]);
+// x as three bf16 terms, t0 + t1 + t2 = x to about 2^-24 |x| (each residual
+// is exact in float32), packed as the first 16 bytes of a K-major row:
+// t0, t1, t2, 0, 0, 0, 0, 0.
+__device__ __forceinline__ uint4 split3_bf16(float x) {
+  const bf16 t0 = __float2bfloat16_rn(x);
+  const float r1 = x - __bfloat162float(t0);
+  const bf16 t1 = __float2bfloat16_rn(r1);
+  const float r2 = r1 - __bfloat162float(t1);
+  const bf16 t2 = __float2bfloat16_rn(r2);
+  return make_uint4((uint32_t)__bfloat16_as_ushort(t0) | ((uint32_t)__bfloat16_as_ushort(t1) << 16),
+                    (uint32_t)__bfloat16_as_ushort(t2), 0u, 0u);
 }
 
 template <bool ALIBI>
@@ -800,13 +809,16 @@ __global__ void __launch_bounds__(448, 1)
   uint8_t* Qs = Vs + KT;         // [NST][QT]
   uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
   uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
-  // [NST][lse 68 | D 68]: the 64 values of a step start at float `voff` of
-  // each half (a sequence's rows start anywhere with per-token kept lists,
-  // and a bulk copy needs a 16-byte aligned source, so 68 are copied from
-  // the aligned-down address)
-  float* vecs = reinterpret_cast<float*>(DSs + 2 * SLAB);
-  constexpr int VS = 136;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * VS);
+  // XT: 128 rows x 128 bytes (128-byte swizzle) of the extra K = 16 chunks
+  // that fold the softmax statistics into the MMAs.  Chunk 0 of every row is
+  // the A operand (1, 1, 1, 0, ...); chunk 1 + b of rows 0..63 holds, for
+  // the 64 queries of a step in stage b, the three bf16 terms of
+  // -lse sqrt(Dh), and of rows 64..127 those of -D.  The exponent of P is
+  // c S - lse log2(e) = c (S - lse sqrt(Dh)) with c = log2(e) / sqrt(Dh), so
+  // S^T comes out of the MMAs as S^T - lse sqrt(Dh) and dP^T as dP^T - D,
+  // and the softmax warps read no per-query vectors.
+  uint8_t* XT = DSs + 2 * SLAB;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(XT + SLAB);
   uint64_t* kv_full = bars;
   uint64_t* ld_full = bars + 1;          // [NST]
   uint64_t* ld_empty = ld_full + NST;    // [NST]
@@ -856,6 +868,16 @@ __global__ void __launch_bounds__(448, 1)
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if (threadIdx.x < 128) {
+    // row r of XT: the ones of chunk 0, zeros everywhere else (the term
+    // chunks are written per step, their upper halves stay zero)
+    const int r = threadIdx.x;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      *reinterpret_cast<uint4*>(XT + swz(r, u)) =
+          u == 0 ? make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
+    fence_proxy_async();
+  }
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
@@ -865,37 +887,66 @@ __global__ void __launch_bounds__(448, 1)
   const uint32_t t_p = tmem + 448;  // [2] x 32 columns: P^T as bf16 pairs
 
   if (warp == 0) {
+    // ------------------------------------------------ producer (warp 0)
+    // lane 0: TMA of K, V once and of Q_i, dO_i per step; all lanes: the
+    // terms of -lse sqrt(Dh) and -D of step i into XT (two queries a lane,
+    // zero past the sequence), loaded from global memory one step ahead
+    const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
     if (lane == 0) {
-      // ------------------------------------------------ TMA producer
-      const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
       mbar_arrive_expect_tx(kv_full, 2 * KT);
       for (int c = 0; c < 2; ++c) {
         tma_load_2d(Ks + c * SLAB, &tmkv, kcol + 64 * c, row0 + kt * 128, kv_full);
         tma_load_2d(Vs + c * SLAB, &tmkv, vcol + 64 * c, row0 + kt * 128, kv_full);
       }
-      int issued = 0;
-      for (int i = 0; i < n_it; ++i) {
-        const int b = i % NST;
-        const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
-        if (!mbar_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
-        mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 2 * 272);
+    }
+    const float sq_dh = 1.f / rsqrtf((float)DH);  // sqrt(Dh) as the softmax warps' scale c = log2(e) rsqrt(Dh) divides it
+    float xl[2], xd[2];
+    auto load_terms = [&](int i) {
+      const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {
+        const int q = qt * 64 + hf * 32 + lane;
+        xl[hf] = 0.f;
+        xd[hf] = 0.f;
+        if (q < len) {
+          const size_t at = (size_t)h * lse_ld + row0 + q;
+          xl[hf] = -lse[at] * sq_dh;
+          xd[hf] = -Dvec[at];
+        }
+      }
+    };
+    if (n_it > 0) load_terms(0);
+    int issued = 0;
+    for (int i = 0; i < n_it; ++i) {
+      const int b = i % NST;
+      const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
+      if (!warp_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {
+        const int r = hf * 32 + lane;
+        *reinterpret_cast<uint4*>(XT + swz(r, 2 + 2 * b)) = split3_bf16(xl[hf]);
+        *reinterpret_cast<uint4*>(XT + swz(64 + r, 2 + 2 * b)) = split3_bf16(xd[hf]);
+      }
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&ld_full[b], 2 * QT);
         for (int c = 0; c < 2; ++c) {
           tma_load_2d(Qs + b * QT + c * HSLAB, &tmq, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
           tma_load_2d(dOs + b * QT + c * HSLAB, &tmo, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
         }
-        const size_t vo = ((size_t)h * lse_ld + row0 + qt * 64) & ~(size_t)3;  // lse_ld % 4 == 0
-        bulk_load(vecs + b * VS, lse + vo, 272, &ld_full[b]);
-        bulk_load(vecs + b * VS + 68, Dvec + vo, 272, &ld_full[b]);
-        ++issued;
       }
-      if (*abort_flag) {
-        mbar_drain(kv_full, 0);
-        for (int i = issued > NST ? issued - NST : 0; i < issued; ++i) mbar_drain(&ld_full[i % NST], (i / NST) & 1);
-      }
+      ++issued;
+      if (i + 1 < n_it) load_terms(i + 1);
     }
-  } else if (warp == 1) {
+    if (lane == 0 && *abort_flag) {
+      mbar_drain(kv_full, 0);
+      for (int i = issued > NST ? issued - NST : 0; i < issued; ++i) mbar_drain(&ld_full[i % NST], (i / NST) & 1);
+    }
     __syncwarp();
-    // ------------------------------------------------ MMA issuer
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (whole warp, converged; one elected lane issues)
+    __syncwarp();
     constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
     constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
     constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
@@ -906,6 +957,7 @@ __global__ void __launch_bounds__(448, 1)
     const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
     const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
     const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
+    const uint64_t DX = sdesc(smem_u32(XT), 16, 1024);  // ones (chunk 0) and the statistics' terms
     bool ok = warp_wait(kv_full, 0, abort_flag, status);
     for (int i = 0; ok && i <= n_it; ++i) {
       if (i < n_it) {
@@ -921,6 +973,9 @@ __global__ void __launch_bounds__(448, 1)
           mma_bf16_w(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
           mma_bf16_w(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
         }
+        // S^T -= lse sqrt(Dh) and dP^T -= D: ones (128 x 16) times the step's terms (64 x 16)
+        mma_bf16_w(t_s, DX, DX + (uint64_t)(((1 + b) * 32) >> 4), ID_SP, 1u);
+        mma_bf16_w(t_dp, DX, DX + (uint64_t)((64 * 128 + (1 + b) * 32) >> 4), ID_SP, 1u);
         mma_commit_w(sdp_full);
       }
       if (i >= 1) {
@@ -961,16 +1016,14 @@ __global__ void __launch_bounds__(448, 1)
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const int voff = row0 & 3;  // first value of a step in its lse / D stage (see vecs)
     const float sl2 = kLog2e * rsqrtf((float)DH);
     bool ok = true;
     for (int i = 0; i < n_it; ++i) {
-      const int b = i % NST;
       const int qt = q0 + i % (nq - q0);
       // ALiBi: logit bias slope2 (key - query) of this step's query head
       const float slope2 = ALIBI ? alibi[g * grp + i / (nq - q0)] * kLog2e : 0.f;
+      // S^T and dP^T arrive with -lse sqrt(Dh) and -D folded in (see XT)
       if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
-      if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
       uint32_t sr[32], dr[32];
       tmem_ld32_nw(t_s + half * 32 + lane_off, sr);
@@ -979,8 +1032,6 @@ __global__ void __launch_bounds__(448, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
-      const float* lsrc = vecs + b * VS + voff + half * 32;       // lse of the 32 queries
-      const float* dsrc = vecs + b * VS + 68 + voff + half * 32;  // D of the 32 queries
       const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
       const int qlim = len - (qt * 64 + half * 32);  // and exists iff c < qlim (warp-uniform)
       uint32_t pk[16], dk[16];
@@ -989,43 +1040,30 @@ __global__ void __launch_bounds__(448, 1)
       // run past the sequence (warp-uniform)
       auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
-        const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
+        const uint64_t sl2x2 = f2_pack(sl2, sl2);
         // bias of query c: slope2 (key - qt*64 - half*32 - c) = b0 - slope2 c
         const float b0 = slope2 * (float)(-qbase);
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
-        for (int e4 = 0; e4 < 8; ++e4) {
-          const float4 lq = ld4s(lsrc, e4, voff), dq = ld4s(dsrc, e4, voff);
-          uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
-          if constexpr (ALIBI) {
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-              const float c0 = (float)(4 * e4 + 2 * h2);
-              nl[h2] = f2_add(nl[h2], f2_fma(f2_pack(c0, c0 + 1.f), nsx2, b0x2));
-            }
+        for (int c = 0; c < 32; c += 2) {
+          uint64_t x2 = f2_mul(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2);
+          if constexpr (ALIBI) x2 = f2_add(x2, f2_fma(f2_pack((float)c, (float)(c + 1)), nsx2, b0x2));
+          float x0, x1;
+          f2_unpack(x2, x0, x1);
+          float p0 = ex2(x0), p1 = ex2(x1);
+          const bool v0 = !MASK || (qbase + c >= 0 && c < qlim), v1 = !MASK || (qbase + c + 1 >= 0 && c + 1 < qlim);
+          if constexpr (MASK) {
+            p0 = v0 ? p0 : 0.f;
+            p1 = v1 ? p1 : 0.f;
           }
-          const uint64_t dd[2] = {f2_pack(dq.x, dq.y), f2_pack(dq.z, dq.w)};
-#pragma unroll
-          for (int h2 = 0; h2 < 2; ++h2) {
-            const int c = 4 * e4 + 2 * h2;
-            float x0, x1;
-            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2, nl[h2]), x0, x1);
-            float p0 = ex2(x0), p1 = ex2(x1);
-            const bool v0 = !MASK || (qbase + c >= 0 && c < qlim), v1 = !MASK || (qbase + c + 1 >= 0 && c + 1 < qlim);
-            if constexpr (MASK) {
-              p0 = v0 ? p0 : 0.f;
-              p1 = v1 ? p1 : 0.f;
-            }
-            const uint64_t pp = f2_pack(p0, p1);
-            float d0, d1;
-            f2_unpack(f2_mul(pp, f2_sub(f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1])), dd[h2])), d0, d1);
-            if constexpr (MASK) {  // rows past the sequence may hold anything: select, do not multiply
-              d0 = v0 ? d0 : 0.f;
-              d1 = v1 ? d1 : 0.f;
-            }
-            pk[c >> 1] = bf16x2_bits(p0, p1);
-            dk[c >> 1] = bf16x2_bits(d0, d1);
+          float d0, d1;
+          f2_unpack(f2_mul(f2_pack(p0, p1), f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1]))), d0, d1);
+          if constexpr (MASK) {  // rows past the sequence may hold anything: select, do not multiply
+            d0 = v0 ? d0 : 0.f;
+            d1 = v1 ? d1 : 0.f;
           }
+          pk[c >> 1] = bf16x2_bits(p0, p1);
+          dk[c >> 1] = bf16x2_bits(d0, d1);
         }
       };
       if (__shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 32) pass(std::false_type{});
@@ -1138,9 +1176,9 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
                    cudaStream_t st) {
-  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
-  // vectors + alignment + barriers = 199,520 bytes
-  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 136 * 4 + 1024 + 256;
+  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + XT (one
+  // slab) + alignment + barriers = 214,272 bytes
+  constexpr size_t smem = 7 * SLAB + 12 * HSLAB + 1024 + 256;
   static bool attr = false;
   if (!attr) {
     cudaError_t e =
