@@ -469,6 +469,31 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // the group may rescale O_g as soon as S_g(j) is ready.  Tile B is skipped
 // when the sequence ends before it.
 constexpr int PP_NSK = 3, PP_NSV = 2;
+// Pairs (of the 16 in each 32-key chunk) whose exponentials run on the FMA
+// pipe (ex2_poly2) instead of MUFU: the 128 x 128 exponentials of a tile
+// take as many cycles at 16 a clock as the tile's two MMAs.
+constexpr int PP_POLY = 0;
+
+// 2^x for two values on the FMA pipe: x = n + f with n = rint(x) and f in
+// [-1/2, 1/2]; 2^f = 1 + f (C1 + f (C2 + f C3)), the cubic fitted to 2^f on
+// that interval by minimising the largest relative error (1.0e-4 in float32,
+// below the 2^-9 half-ulp of the bf16 P is stored in); 2^n is added into the
+// exponent field.  x is clamped at -127, where the result is below 2^-126
+// instead of 0.
+__device__ __forceinline__ void ex2_poly2(float x0, float x1, float& y0, float& y1) {
+  constexpr float C1 = 0.6932829022407532f, C2 = 0.24221037328243256f, C3 = 0.05500858277082443f;
+  x0 = fmaxf(x0, -127.f);
+  x1 = fmaxf(x1, -127.f);
+  const float n0 = rintf(x0), n1 = rintf(x1);
+  const uint64_t f = f2_sub(f2_pack(x0, x1), f2_pack(n0, n1));
+  uint64_t p = f2_fma(f, f2_pack(C3, C3), f2_pack(C2, C2));
+  p = f2_fma(p, f, f2_pack(C1, C1));
+  p = f2_fma(p, f, f2_pack(1.f, 1.f));
+  float p0, p1;
+  f2_unpack(p, p0, p1);
+  y0 = __int_as_float(__float_as_int(p0) + ((int)n0 << 23));
+  y1 = __int_as_float(__float_as_int(p1) + ((int)n1 << 23));
+}
 
 __global__ void __launch_bounds__(320, 1)
     attn_fwd_pp_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
@@ -688,7 +713,13 @@ __global__ void __launch_bounds__(320, 1)
         for (int e = 0; e < 16; ++e) {
           float x0, x1;
           f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, nm2), x0, x1);
-          float p0 = ex2(x0), p1 = ex2(x1);
+          float p0, p1;
+          if (e >= 16 - PP_POLY) {
+            ex2_poly2(x0, x1, p0, p1);
+          } else {
+            p0 = ex2(x0);
+            p1 = ex2(x1);
+          }
           if (diag) {
             p0 = (c * 32 + 2 * e <= r) ? p0 : 0.f;
             p1 = (c * 32 + 2 * e + 1 <= r) ? p1 : 0.f;
