@@ -495,10 +495,11 @@ __device__ __forceinline__ void ex2_poly2(float x0, float x1, float& y0, float& 
   y1 = __int_as_float(__float_as_int(p1) + ((int)n1 << 23));
 }
 
+template <bool ALIBI>
 __global__ void __launch_bounds__(320, 1)
     attn_fwd_pp_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
-                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv, const int* __restrict__ seg,
-                       int* status) {
+                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv,
+                       const float* __restrict__ alibi, const int* __restrict__ seg, int* status) {
   constexpr int DH = 128;
   constexpr uint32_t TILE = 2 * SLAB;  // one 128 x 128 bf16 tile (two 64-column slabs)
   extern __shared__ uint8_t smem_raw[];
@@ -655,20 +656,40 @@ __global__ void __launch_bounds__(320, 1)
     const int nkg = gi ? nkB : nkA;
     const int jdiag = 2 * qb + gi;  // the K tile on this query tile's diagonal
     const float sl2 = kLog2e * rsqrtf((float)DH);
+    // ALiBi: the exponent is x = S sl2 + slope2 (key - query), and the
+    // running max m is kept on x (the max of S alone, scaled, otherwise)
+    const float slope2 = ALIBI ? alibi[h] * kLog2e : 0.f;
+    const int qrow_t = qb * 256 + gi * 128 + r;  // this thread's query within the sequence
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nkg; ++j) {
       if (!warp_wait(&s_full[gi], j & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
       const bool diag = (j == jdiag);  // keys after the query are left out (block-uniform)
-      // pass 1: row max of the raw scores (the scale is positive)
+      // pass 1: row max of the raw scores (the scale is positive), or of x
+      // with ALiBi
       float mraw = -INFINITY;
+      const float b0 = slope2 * (float)(j * 128 - qrow_t);  // bias of key 0 of the tile
 #pragma unroll 1
       for (int c2 = 0; c2 < 2; ++c2) {
         uint32_t sr[2][32];
         tmem_ld32_nw(t_s + c2 * 64 + lane_off, sr[0]);
         tmem_ld32_nw(t_s + c2 * 64 + 32 + lane_off, sr[1]);
         tmem_wait_ld();
+        if constexpr (ALIBI) {
+          const uint64_t sl2x2 = f2_pack(sl2, sl2), sx2 = f2_pack(slope2, slope2);
+          const float bc = b0 + slope2 * (float)(c2 * 64);
+          const uint64_t bx2 = f2_pack(bc, bc);
+#pragma unroll
+          for (int e = 0; e < 64; e += 2) {
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1])),
+                             sl2x2, f2_fma(f2_pack((float)e, (float)(e + 1)), sx2, bx2)),
+                      x0, x1);
+            sr[e >> 5][e & 31] = __float_as_uint(x0);
+            sr[e >> 5][(e & 31) + 1] = __float_as_uint(x1);
+          }
+        }
         if (diag) {
 #pragma unroll
           for (int e = 0; e < 64; ++e)
@@ -679,7 +700,7 @@ __global__ void __launch_bounds__(320, 1)
             mraw = fmax3(mraw, __uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1]));
         }
       }
-      const float mt = mraw * sl2;
+      const float mt = ALIBI ? mraw : mraw * sl2;
       const bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
       // O_g is rescaled in TMEM when any lane of the warp moved its max
@@ -702,6 +723,7 @@ __global__ void __launch_bounds__(320, 1)
       // pass 2: P = exp2(S c log2e - m) for 32 keys at a time, written as
       // bf16 pairs over S columns that have already been read
       const uint64_t sl2x2 = f2_pack(sl2, sl2), nm2 = f2_pack(-m_new, -m_new);
+      const uint64_t sx2 = f2_pack(slope2, slope2);
       uint64_t ls2 = f2_pack(0.f, 0.f);
 #pragma unroll 1
       for (int c = 0; c < 4; ++c) {
@@ -709,10 +731,13 @@ __global__ void __launch_bounds__(320, 1)
         tmem_ld32_nw(t_s + c * 32 + lane_off, sr);
         tmem_wait_ld();
         uint32_t pk[16];
+        const float bm = b0 + slope2 * (float)(c * 32) - m_new;  // ALiBi: bias of key 32c minus the max
+        const uint64_t bmx2 = f2_pack(bm, bm);
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           float x0, x1;
-          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, nm2), x0, x1);
+          const uint64_t add = ALIBI ? f2_fma(f2_pack((float)(2 * e), (float)(2 * e + 1)), sx2, bmx2) : nm2;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, add), x0, x1);
           float p0, p1;
           if (e >= 16 - PP_POLY) {
             ex2_poly2(x0, x1, p0, p1);
@@ -764,20 +789,22 @@ __global__ void __launch_bounds__(320, 1)
   }
 }
 
+template <bool ALIBI>
 cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
-                   int max_seqs, const int* seg, int* status, cudaStream_t st) {
+                   int max_seqs, const float* alibi, const int* seg, int* status, cudaStream_t st) {
   // 2 Q, 3 K and 2 V tiles of 32 KB + alignment + barriers = 230,656 bytes (of 232,448)
   constexpr size_t smem = (size_t)(2 + PP_NSK + PP_NSV) * 2 * SLAB + 1024 + 256;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_pp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(attn_fwd_pp_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   dim3 grid(H, max_seqs, (S + 255) / 256);
-  attn_fwd_pp_kernel<<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, seg, status);
+  attn_fwd_pp_kernel<ALIBI><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi, seg, status);
   return cudaGetLastError();
 }
 
@@ -1248,12 +1275,12 @@ cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int l
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
                                int Hkv, int Dh, int max_seqs, const float* alibi, const int* seg, int* status,
                                cudaStream_t st) {
-  if (alibi) {
-    if (Dh == 64) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
-    return fwd_tc<128, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  if (Dh == 64) {
+    if (alibi) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+    return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
   }
-  if (Dh == 64) return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
-  return fwd_pp(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, seg, status, st);
+  if (alibi) return fwd_pp<true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  return fwd_pp<false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
 }
 
 }  // namespace ldk
