@@ -622,7 +622,7 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk)
             mma_bf16_ta_w(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
-                          (j > 1 || kk > 0) ? 1u : 0u);
+                            (j > 1 || kk > 0) ? 1u : 0u);
           if (j == nkg) mma_commit_w(&o_full[gi]);  // the group's last P V
         }
         if (j < nkg) {
