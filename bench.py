@@ -129,6 +129,21 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
+SLOWDOWNS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown")
+
+
+def clocks_rejected(clk, stuck_frac=0.75):
+    """True when a clock record disqualifies its timing: a hardware or
+    thermal slowdown was active, or the median SM clock sat below
+    `stuck_frac` of the maximum with no reason given (a leftover clock
+    lock).  sw_power_cap alone is normal under a dense load and is kept."""
+    if not clk:
+        return False
+    if any(r in clk["reasons"] for r in SLOWDOWNS):
+        return True
+    return not clk["reasons"] and clk["sm_mhz"] < stuck_frac * clk["sm_max_mhz"]
+
+
 def cpu_baseline(cfg, host_w0, x_seq, dy_seq, rows, kept_units_per_step, s_l0):
     """The oracle (float64 numpy) on a bounded sample: layer 0, sequence 0,
     its first `rows` rows, forward + backward.  Extrapolated to a step by the
@@ -429,10 +444,20 @@ def main():
     for k in range(args.warmup):
         step(step0 + k)
     st.sync()
-    clocks = Clocks(local)
-    clocks.start()
-    ms = timed(args.steps, step0 + args.warmup, step)
-    clk = clocks.stop()
+    def measured():
+        clocks = Clocks(local)
+        clocks.start()
+        t = timed(args.steps, step0 + args.warmup, step)
+        return t, clocks.stop()
+
+    ms, clk = measured()
+    # a run whose clocks show a slowdown (or a clock lock) is measured once
+    # more, on every rank, and the second run is the one reported
+    if max_over_ranks(1.0 if clocks_rejected(clk) else 0.0, world) > 0.0:
+        first = clk
+        ms, clk = measured()
+        if clk is not None:
+            clk["remeasured_after"] = first
     st.sync()
     # ---- device time by kernel class: the same steps again with the
     # library's per-launch events on, which keep the backward's
