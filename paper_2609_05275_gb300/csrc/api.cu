@@ -1043,4 +1043,12 @@ ld_status ld_gemm_bf16(int M, int N, int K, const void* A, int lda, int a_mn, co
   return LD_OK;
 }
 
+ld_status ld_check_wait_timeout(int* status_ws, void* stream) {
+  if (!status_ws) return LD_ERR_ARG;
+  ld_status r = check_device();
+  if (r != LD_OK) return r;
+  LD_CHECK(launch_wait_timeout(status_ws, static_cast<cudaStream_t>(stream)));
+  return LD_OK;
+}
+
 }  // extern "C"

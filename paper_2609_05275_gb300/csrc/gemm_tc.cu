@@ -673,6 +673,25 @@ cudaError_t dispatch_major(const GemmArgs& a, const CUtensorMap& ta, const CUten
 
 }  // namespace
 
+// One block waiting on an mbarrier phase that nothing completes: the
+// bounded wait gives up after its limit and records LD_ERR_TIMEOUT.
+__global__ void wait_timeout_kernel(int* status) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) tc::mbar_wait(&bar, 0, reinterpret_cast<volatile int*>(&abort_flag), status);
+}
+
+cudaError_t launch_wait_timeout(int* status, cudaStream_t st) {
+  wait_timeout_kernel<<<1, 32, 0, st>>>(status);
+  return cudaGetLastError();
+}
+
 cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st) {
   const int BN = (a.N % 256 == 0) ? 256 : 128;
   const uint64_t mcap = a.M_cnt ? a.M_cap : a.M;
