@@ -892,7 +892,10 @@ __global__ void __launch_bounds__(448, 1)
 
   // rows row0 .. row0+len-1 as in the forward; queries past len (the last
   // query tile) get P = dS = 0, keys past len are never stored
-  const int seq = blockIdx.y;
+  // grid (kv head, key tile, sequence): the blocks of one sequence are
+  // dispatched together, heaviest key tiles (kt = 0) first, so the Q, dO and
+  // dQ rows in use at a time are one sequence's (they stay in L2)
+  const int seq = blockIdx.z;
   int row0, len;
   if (seg) {
     row0 = seg[seq];
@@ -902,7 +905,7 @@ __global__ void __launch_bounds__(448, 1)
     row0 = seq * S;
     len = S;
   }
-  const int kt = blockIdx.z, g = blockIdx.x, grp = H / Hkv;  // heaviest key tiles (kt = 0) dispatched first
+  const int kt = blockIdx.y, g = blockIdx.x, grp = H / Hkv;
   if (kt * 128 >= len) return;
   const int nq = (len + 63) / 64, q0 = 2 * kt;  // query tiles q0 .. nq-1 overlap or follow the keys
   const int n_it = grp * (nq - q0);
@@ -1248,7 +1251,7 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
-  dim3 grid(Hkv, max_seqs, S / 128);
+  dim3 grid(Hkv, S / 128, max_seqs);
   attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
                                                      H, Hkv, rcos, rsin, alibi, seg, tok, status);
   return cudaGetLastError();
