@@ -162,10 +162,12 @@ def cpu_baseline(cfg, host_w0, x_seq, dy_seq, rows, kept_units_per_step, s_l0):
     dt = time.perf_counter() - t0
     per_token = dt / rows
     step_time = per_token * kept_units_per_step * cfg["S"]
+    note = ("the whole sequence, so the per-sequence cost is measured, not extrapolated" if rows >= cfg["S"] else
+            "attention cost of later rows under-represented, so the CPU figure is optimistic")
     return {"value": cfg["B"] * cfg["S"] / step_time, "unit": "tokens/s", "cores": os.cpu_count(),
             "kind": "oracle", "sample": f"layer 0, sequence 0, rows 0..{rows - 1} of {cfg['S']}, fwd+bwd, float64 "
-            f"numpy ({dt:.1f} s); extrapolated by the step's kept tokens (attention cost of later rows "
-            f"under-represented, so the CPU figure is optimistic)", "sample_seconds": dt}
+            f"numpy ({dt:.1f} s); scaled to a step by the step's kept (layer, sequence) pairs ({note})",
+            "sample_seconds": dt}
 
 
 def run_reference(args):
@@ -177,7 +179,7 @@ def run_reference(args):
     if rank != 0:
         return 0
     cfg, sched = synth.CONFIGS[args.config], synth.SCHEDULES[args.config]
-    rows = args.cpu_rows
+    rows = min(args.cpu_rows or 1024, cfg["S"])  # per step: a bounded sample, so the run stays within minutes
     w0 = synth.layer_weights(cfg, 0, seed=0)
     x = synth.activations(cfg, seed=0, B=1)[0]
     dy = synth.upstream_grad(cfg, B=1)[0]
@@ -368,7 +370,9 @@ def main():
     ap.add_argument("--no-dense", action="store_true", help="skip the p=0 run (no skip_speedup)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--cpu-rows", type=int, default=1024)
+    ap.add_argument("--cpu-rows", type=int, default=0,
+                    help="rows of the CPU oracle sample (default: a whole sequence for the cpu_baseline leg, "
+                         "1024 per step for --impl reference)")
     ap.add_argument("--layers", type=int, default=None, help="override L (profiling captures only)")
     ap.add_argument("--granularity", default="per_sequence", choices=["per_sequence", "per_batch", "per_token"],
                     help="mask granularity of the timed steps (the headline is per sequence)")
@@ -528,7 +532,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu:
         w0 = {n: v.cpu() for n, v in layers[0].items()}
         _, _, sc = st.rates(step0 + args.warmup)
-        cpu = cpu_baseline(cfg, w0, x0[0].cpu(), dy0[0].cpu(), min(args.cpu_rows, S),
+        cpu = cpu_baseline(cfg, w0, x0[0].cpu(), dy0[0].cpu(), min(args.cpu_rows or S, S),
                            kept_units * rows_per_unit / S / args.steps, sc[0])
 
     gemm_achieved = gemm_flops * args.steps / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
