@@ -227,15 +227,15 @@ bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
   } while (0)
 
 ld_status check_device() {
-  static int ok = -1;
-  if (ok < 0) {
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const ld_status verdict = [] {
     int dev = 0, major = 0, minor = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LD_ERR_CUDA;
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-    ok = (major == 10 && minor == 3) ? 1 : 0;
-  }
-  return ok ? LD_OK : LD_ERR_UNSUPPORTED;
+    return (major == 10 && minor == 3) ? LD_OK : LD_ERR_UNSUPPORTED;
+  }();
+  return verdict;
 }
 
 ld_status check_weights(const Handle* h, const ld_layer_w* W) {

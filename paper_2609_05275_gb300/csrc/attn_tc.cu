@@ -434,13 +434,10 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
                    int max_seqs, const float* alibi, const int* seg, int* status, cudaStream_t st) {
   // Q, 3 K and 2 V tiles + the row max / sum exchange + alignment + barriers
   constexpr size_t smem = (size_t)(DH / 64) * SLAB * 6 + 10 * 128 * 4 + 1024 + 256;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e =
-        cudaFuncSetAttribute(attn_fwd_tc_kernel<DH, ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(attn_fwd_tc_kernel<DH, ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   dim3 grid(H, max_seqs, S / 128);
@@ -794,13 +791,10 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
                    int max_seqs, const float* alibi, const int* seg, int* status, cudaStream_t st) {
   // 2 Q, 3 K and 2 V tiles of 32 KB + alignment + barriers = 230,656 bytes (of 232,448)
   constexpr size_t smem = (size_t)(2 + PP_NSK + PP_NSV) * 2 * SLAB + 1024 + 256;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e =
-        cudaFuncSetAttribute(attn_fwd_pp_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(attn_fwd_pp_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   dim3 grid(H, max_seqs, (S + 255) / 256);
@@ -1240,13 +1234,10 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
   // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + XT (one
   // slab) + alignment + barriers = 214,272 bytes
   constexpr size_t smem = 7 * SLAB + 12 * HSLAB + 1024 + 256;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e =
-        cudaFuncSetAttribute(attn_bwd_tc_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(attn_bwd_tc_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   CUtensorMap tkv, tq, to;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;

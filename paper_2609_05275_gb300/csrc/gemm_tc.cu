@@ -602,9 +602,9 @@ constexpr size_t smem_bytes() {
 // the pair kernel cannot run).
 constexpr int PAIR_BN = 256, PAIR_STAGES = 3, PAIR_KPS = 2;
 int pair_clusters() {
-  static int n = -1;
-  if (n < 0) {
-    n = 0;
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const int clusters = [] {
+    int n = 0;
     auto k = gemm_tc_kernel<PAIR_BN, PAIR_STAGES, false, false, true, PAIR_KPS>;
     constexpr size_t smem = smem_bytes<PAIR_BN, PAIR_STAGES, true, PAIR_KPS>();
     if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess) {
@@ -623,8 +623,9 @@ int pair_clusters() {
       if (cudaOccupancyMaxActiveClusters(&c, k, &cfg) == cudaSuccess && c > 0) n = c;
     }
     cudaGetLastError();  // a refused query leaves no sticky error behind
-  }
-  return n;
+    return n;
+  }();
+  return clusters;
 }
 
 template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR, int KPS>
@@ -632,12 +633,10 @@ cudaError_t run(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tb,
   constexpr size_t smem = smem_bytes<BN, STAGES, PAIR, KPS>();
   constexpr int NCTA = PAIR ? 2 : 1;
   auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, PAIR, KPS>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   const int mcap = a.M_cnt ? a.M_cap : a.M;
   const long long tiles = (long long)((mcap + BM * NCTA - 1) / (BM * NCTA)) * ((a.N + BN - 1) / BN);
   int units = PAIR ? pair_clusters() : device_sm_count();
