@@ -136,8 +136,17 @@ def test_schedule_validation_and_state():
                dict(dist="ild", p_max=0.2, time="ramp", ramp=(10, 10, 0.0, 1.0))]
         for s in bad:
             assert P.ld_set_schedule_status(h, P.make_schedule(s)) == P.LD_ERR_ARG, s
-        # backward without forward: state error (argument checks pass first)
+        # backward without forward: argument errors first, then a state error
+        # (the pointers below are aligned and never dereferenced: the checks
+        # run on the host before any device work)
         assert L.ld_backward(h, None, None, None, None, None) == P.LD_ERR_ARG
+        cfg = synth.CONFIGS["tiny"]
+        fake = ctypes.c_void_p(1 << 20)
+        W = (P.ld_layer_w * cfg["L"])(*[P.ld_layer_w(*([1 << 20] * 6)) for _ in range(cfg["L"])])
+        G = (P.ld_layer_g * cfg["L"])(*[P.ld_layer_g(*([1 << 20] * 6)) for _ in range(cfg["L"])])
+        assert L.ld_backward(h, W, fake, G, fake, None) == P.LD_ERR_STATE
+        Wmis = (P.ld_layer_w * cfg["L"])(*[P.ld_layer_w(*([(1 << 20) + 4] * 6)) for _ in range(cfg["L"])])
+        assert L.ld_backward(h, Wmis, fake, G, fake, None) == P.LD_ERR_ARG  # misaligned weights
         assert L.ld_get_masks(h, None, None, None) == P.LD_ERR_STATE
         assert L.ld_create(None, None) == P.LD_ERR_ARG
     finally:
