@@ -60,14 +60,18 @@ def load_peaks():
         return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
 
 
-def flops_per_token(cfg):
+def flops_per_token(cfg, split=False):
     """Forward FLOPs per token per layer (2 x MACs; causal attention counted
-    as S/2 keys per query) and the part of it in the projections."""
+    as S/2 keys per query) and the part of it in the projections; with
+    split=True the projections of the attention block and of the FFN block
+    separately: (total, attention-block projections, FFN)."""
     d, H, Hkv, Dh, F, S = cfg["d"], cfg["H"], cfg["Hkv"], cfg["Dh"], cfg["F"], cfg["S"]
     ffn = 4 * d * F if cfg.get("act") == "relu2" else 6 * d * F  # up (+ gate) and down
-    proj = 2 * d * (H + 2 * Hkv) * Dh + 2 * d * H * Dh + ffn
+    attn_proj = 2 * d * (H + 2 * Hkv) * Dh + 2 * d * H * Dh
     attn = 2 * H * Dh * S
-    return proj + attn, proj
+    if split:
+        return attn_proj + ffn + attn, attn_proj, ffn
+    return attn_proj + ffn + attn, attn_proj + ffn
 
 
 def max_over_ranks(ms, world, device="cuda"):
@@ -376,6 +380,8 @@ def main():
     ap.add_argument("--layers", type=int, default=None, help="override L (profiling captures only)")
     ap.add_argument("--granularity", default="per_sequence", choices=["per_sequence", "per_batch", "per_token"],
                     help="mask granularity of the timed steps (the headline is per sequence)")
+    ap.add_argument("--sublayer", action="store_true",
+                    help="independent attention and FFN masks (sub-layer granularity) in the timed steps")
     ap.add_argument("--sweep", action="store_true",
                     help="drop-rate / distribution / granularity / seed sweep on the 1.3B shape (one JSON line "
                          "per cell, then a summary line)")
@@ -415,7 +421,8 @@ def main():
     peaks = load_peaks()
 
     tok = args.granularity == "per_token"
-    st = P.LayerDropStack(cfg, sched, granularity=args.granularity)
+    sub = args.sublayer
+    st = P.LayerDropStack(cfg, sched, granularity=args.granularity, sublayer=sub)
     layers = synth.stack_weights(cfg, seed=0, device="cuda")
     wtab = P.weight_table(layers)
     grads = [{n: torch.empty(v.shape, device="cuda", dtype=torch.float32) for n, v in W.items()} for W in layers]
@@ -478,20 +485,26 @@ def main():
     # kept counts of the timed steps (masks redrawn through the library):
     # kept (layer, sequence) pairs, or per token the kept tokens (and the
     # kept length of every (layer, sequence) for the attention FLOPs)
-    kept, attn_len2 = [], 0.0
+    # (with sub-layer masks the attention and FFN blocks keep their own units)
+    kept_a, kept_f, attn_len2 = 0, 0, 0.0
     for k in range(args.steps):
         mk, _, cnt = st.draw_masks(step0 + args.warmup + k)
-        kept.append([int(c) for c in cnt])
+        ka = int(cnt[0].sum()) if sub else int(cnt.sum())
+        kept_a += ka
+        kept_f += int(cnt[1].sum()) if sub else ka
         if tok:
-            attn_len2 += float((mk.reshape(-1, B, S).sum(axis=2).astype("float64") ** 2).sum())
-    f_tok, f_proj = flops_per_token(cfg)
-    kept_units = sum(sum(c) for c in kept)
+            mka = mk[0] if sub else mk
+            attn_len2 += float((mka.reshape(-1, B, S).sum(axis=2).astype("float64") ** 2).sum())
+    f_tok, f_aproj, f_ffn = flops_per_token(cfg, split=True)
+    f_attn = f_tok - f_aproj - f_ffn  # attention scores and weighted sum, per token at full length
+    kept_units = 0.5 * (kept_a + kept_f)  # per branch on average (equal without sub-layer masks)
     rows_per_unit = 1 if tok else S
+    proj_flops = f_aproj * kept_a + f_ffn * kept_f  # per kept unit row
     if tok:  # projections per kept token; attention 2 H Dh len^2 per kept sequence of length len (forward)
-        exec_flops = 3.0 * (f_proj * kept_units + 2.0 * cfg["H"] * cfg["Dh"] * attn_len2) / args.steps
+        exec_flops = 3.0 * (proj_flops + 2.0 * cfg["H"] * cfg["Dh"] * attn_len2) / args.steps
     else:
-        exec_flops = 3.0 * f_tok * S * kept_units / args.steps  # per step, this rank
-    gemm_flops = 3.0 * f_proj * rows_per_unit * kept_units / args.steps
+        exec_flops = 3.0 * S * (proj_flops + f_attn * kept_a) / args.steps  # per step, this rank
+    gemm_flops = 3.0 * rows_per_unit * proj_flops / args.steps
     p_real = 1.0 - kept_units * rows_per_unit / (args.steps * L * B * S)
     _, thr, _ = st.rates(step0 + args.warmup)
     p_exp = sum(t / 2 ** 32 for t in thr) / L
@@ -552,7 +565,8 @@ def main():
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": args.config, **{k: cfg[k] for k in ("L", "d", "H", "Hkv", "Dh", "F", "B", "S")},
-                   "schedule": sched, "granularity": args.granularity, "first_step": step0 + args.warmup,
+                   "schedule": sched, "granularity": args.granularity, "sublayer": sub,
+                   "first_step": step0 + args.warmup,
                    "parallelism": f"replicas x{world}", "l2": "inputs and weights larger than L2 (no flush)"},
         "executed_tflops": tflops, "pct_bf16_peak": 100.0 * tflops / peaks["bf16"],
         "pct_bf16_peak_sustained": 100.0 * tflops / peaks["bf16_sustained"],
@@ -570,9 +584,11 @@ def main():
     # kernel and the RoPE table, then per layer 4 GEMMs + attention + 4
     # row-wise kernels forward, 8 GEMMs + 3 attention kernels + 7 row-wise
     # kernels backward (RoPE kernels drop out when theta = 0)
-    # (per token also 3 + 3 tail-zeroing launches per layer)
+    # (per token also 3 + 3 tail-zeroing launches per layer; with sub-layer
+    # masks one more row-wise gather per layer in the backward)
     rope = 1 if cfg.get("rope_theta") else 0
-    line["gpu_launches"] = args.steps * (1 + rope + L * (4 + 1 + 3 + rope + 8 + 3 + 6 + rope + (6 if tok else 0)))
+    line["gpu_launches"] = args.steps * (1 + rope + L * (4 + 1 + 3 + rope + 8 + 3 + 6 + rope + (6 if tok else 0) +
+                                                         (1 if sub else 0)))
     if rank == 0:
         print(json.dumps(line), flush=True)
     st.close()
