@@ -318,6 +318,16 @@ ld_status ld_rmsnorm_backward_noalloc(int B, int S, int d, const float* dyn, con
                                       const void* gamma, const int* kept_idx, const int* kept_cnt, float* dx,
                                       void* next, float scale, float* dgamma, void* stream);
 
+/* Exercise the failure path of the pipelined kernels without a fault: one
+ * block waits, with the same bounded wait as every tcgen05 kernel, on an
+ * mbarrier phase that nothing completes.  After the wait limit (about 2 s of
+ * GPU time) it records LD_ERR_TIMEOUT in *status_ws (an int on the device;
+ * a nonzero value already there is kept) and exits; the context stays
+ * usable.  Async on `stream`: read *status_ws after synchronising.  The
+ * paper has no counterpart: this checks the library's own error handling.
+ * LD_ERR_ARG if status_ws is NULL. */
+ld_status ld_check_wait_timeout(int* status_ws, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -98,6 +98,7 @@ def lib():
                                                     c_void_p]),
             "ld_gemm_bf16": (c_int, [c_int, c_int, c_int, c_void_p, c_int, c_int, c_void_p, c_int, c_int, c_void_p,
                                      c_int, c_int, c_float, c_void_p, c_void_p]),
+            "ld_check_wait_timeout": (c_int, [c_void_p, c_void_p]),
         }
         for name, (res, args) in sigs.items():
             f = getattr(L, name)
@@ -263,6 +264,12 @@ def ld_gemm_bf16(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, alpha=1.0, status=
     d_f32 = 1 if D.dtype == torch.float32 else 0
     _check(lib().ld_gemm_bf16(M, N, K, _ptr(A), lda, int(a_mn), _ptr(B), ldb, int(b_mn), _ptr(D), ldd, d_f32,
                               float(alpha), _ptr(status), _stream(stream)), "ld_gemm_bf16")
+
+
+def ld_check_wait_timeout(status, stream=None):
+    """Launch the bounded-wait failure-path check (include/ld.h); `status`
+    is an int32 device tensor of one element."""
+    _check(lib().ld_check_wait_timeout(_ptr(status), _stream(stream)), "ld_check_wait_timeout")
 
 
 def rmsnorm_backward_scratch_bytes(B, S, d):

@@ -227,15 +227,15 @@ bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
   } while (0)
 
 ld_status check_device() {
-  static int ok = -1;
-  if (ok < 0) {
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const ld_status verdict = [] {
     int dev = 0, major = 0, minor = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LD_ERR_CUDA;
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-    ok = (major == 10 && minor == 3) ? 1 : 0;
-  }
-  return ok ? LD_OK : LD_ERR_UNSUPPORTED;
+    return (major == 10 && minor == 3) ? LD_OK : LD_ERR_UNSUPPORTED;
+  }();
+  return verdict;
 }
 
 ld_status check_weights(const Handle* h, const ld_layer_w* W) {
@@ -1040,6 +1040,14 @@ ld_status ld_gemm_bf16(int M, int N, int K, const void* A, int lda, int a_mn, co
   a.alpha = alpha;
   a.status = status_ws;
   LD_CHECK(gemm_tc(a, static_cast<cudaStream_t>(stream)));
+  return LD_OK;
+}
+
+ld_status ld_check_wait_timeout(int* status_ws, void* stream) {
+  if (!status_ws) return LD_ERR_ARG;
+  ld_status r = check_device();
+  if (r != LD_OK) return r;
+  LD_CHECK(launch_wait_timeout(status_ws, static_cast<cudaStream_t>(stream)));
   return LD_OK;
 }
 

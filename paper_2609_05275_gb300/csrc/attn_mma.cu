@@ -424,12 +424,10 @@ template <int DH>
 cudaError_t fwd_launch(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
                        int max_seqs, const float* alibi, cudaStream_t st) {
   constexpr size_t smem = (size_t)5 * 64 * (DH + 8) * sizeof(bf16);
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(attn_fwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   dim3 grid(S / 64, H, max_seqs);
   attn_fwd_kernel<DH><<<grid, 128, smem, st>>>(qkv, ldq, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi);
   return cudaGetLastError();
@@ -440,12 +438,10 @@ cudaError_t bwd_launch(const bf16* qkv, int ldq, const bf16* dO, int ldo, const 
                        float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs,
                        const float* alibi, cudaStream_t st) {
   constexpr size_t smem = (size_t)4 * 64 * (DH + 8) * sizeof(bf16) + 64 * 72 * sizeof(bf16) + 128 * sizeof(float);
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(attn_bwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   dim3 grid(S / 64, Hkv, max_seqs);
   attn_bwd_kernel<DH><<<grid, 128, smem, st>>>(qkv, ldq, dO, ldo, lse, Dvec, max_seqs * S, dq_acc, dqkv, cnt, S, H,
                                                Hkv, alibi);

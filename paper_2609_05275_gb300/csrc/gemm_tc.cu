@@ -66,19 +66,6 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, 
   return r == CUDA_SUCCESS;
 }
 
-bool make_map_f32(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld, uint32_t box_inner,
-                  uint32_t box_outer) {
-  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
-  if (!enc) return false;
-  cuuint64_t dims[2] = {inner, outer};
-  cuuint64_t strides[1] = {ld * 4};
-  cuuint32_t box[2] = {box_inner, box_outer};
-  cuuint32_t estr[2] = {1, 1};
-  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, estr,
-                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS;
-}
 }  // namespace tc
 
 namespace {
@@ -385,8 +372,10 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && rank == 0) {
-      // ------------------------------------------------ MMA issuer
+    if (rank == 0) {
+      // ------------------------------------------------ MMA issuer (whole warp, converged;
+      // one elected lane issues)
+      __syncwarp();
       constexpr uint32_t IDESC = idesc_bf16(BMT, BN, A_MN, B_MN);
       int stage = 0;
       uint32_t phase = 0;
@@ -394,14 +383,14 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t acc_phase = 0;
       bool ok = true;
       for (int tile = tile0; tile < num_tiles && ok; tile += tstep) {
-        if (!mbar_wait<PAIR>(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
+        if (!warp_wait<PAIR>(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         for (int ks = 0; ks < num_ks; ++ks) {
-          if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
+          if (!warp_wait(&full[stage], phase, abort_flag, a.status)) {
             ok = false;
             break;
           }
@@ -421,15 +410,15 @@ __global__ void __launch_bounds__(192, 1)
               const uint64_t bd = B_MN ? sdesc(sb + k * 2048, 8192, 1024) : sdesc(sb + k * 32, 16, 1024);
               const uint32_t accum = (ks | j | k) != 0 ? 1u : 0u;
               if constexpr (PAIR)
-                mma_bf16_pair(d_tmem, ad, bd, IDESC, accum);
+                mma_bf16_pair_w(d_tmem, ad, bd, IDESC, accum);
               else
-                mma_bf16(d_tmem, ad, bd, IDESC, accum);
+                mma_bf16_w(d_tmem, ad, bd, IDESC, accum);
             }
           }
           if constexpr (PAIR)
-            mma_commit_pair_both(&empty[stage]);
+            mma_commit_pair_both_w(&empty[stage]);
           else
-            mma_commit(&empty[stage]);
+            mma_commit_w(&empty[stage]);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -437,19 +426,20 @@ __global__ void __launch_bounds__(192, 1)
         }
         if (!ok) break;
         if constexpr (PAIR)
-          mma_commit_pair_both(&tfull[acc]);
+          mma_commit_pair_both_w(&tfull[acc]);
         else
-          mma_commit(&tfull[acc]);
+          mma_commit_w(&tfull[acc]);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
       }
       if (!ok) {
         // make sure every MMA issued so far has finished before TMEM is freed
         if constexpr (PAIR)
-          mma_commit_pair_local(drain);
+          mma_commit_pair_local_w(drain);
         else
-          mma_commit(drain);
-        mbar_drain(drain, 0);
+          mma_commit_w(drain);
+        if (lane == 0) mbar_drain(drain, 0);
+        __syncwarp();
       }
     }
   } else {
@@ -612,9 +602,9 @@ constexpr size_t smem_bytes() {
 // the pair kernel cannot run).
 constexpr int PAIR_BN = 256, PAIR_STAGES = 3, PAIR_KPS = 2;
 int pair_clusters() {
-  static int n = -1;
-  if (n < 0) {
-    n = 0;
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const int clusters = [] {
+    int n = 0;
     auto k = gemm_tc_kernel<PAIR_BN, PAIR_STAGES, false, false, true, PAIR_KPS>;
     constexpr size_t smem = smem_bytes<PAIR_BN, PAIR_STAGES, true, PAIR_KPS>();
     if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess) {
@@ -633,8 +623,9 @@ int pair_clusters() {
       if (cudaOccupancyMaxActiveClusters(&c, k, &cfg) == cudaSuccess && c > 0) n = c;
     }
     cudaGetLastError();  // a refused query leaves no sticky error behind
-  }
-  return n;
+    return n;
+  }();
+  return clusters;
 }
 
 template <int BN, int STAGES, bool A_MN, bool B_MN, bool PAIR, int KPS>
@@ -642,12 +633,10 @@ cudaError_t run(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tb,
   constexpr size_t smem = smem_bytes<BN, STAGES, PAIR, KPS>();
   constexpr int NCTA = PAIR ? 2 : 1;
   auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, PAIR, KPS>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   const int mcap = a.M_cnt ? a.M_cap : a.M;
   const long long tiles = (long long)((mcap + BM * NCTA - 1) / (BM * NCTA)) * ((a.N + BN - 1) / BN);
   int units = PAIR ? pair_clusters() : device_sm_count();
@@ -682,6 +671,25 @@ cudaError_t dispatch_major(const GemmArgs& a, const CUtensorMap& ta, const CUten
 }
 
 }  // namespace
+
+// One block waiting on an mbarrier phase that nothing completes: the
+// bounded wait gives up after its limit and records LD_ERR_TIMEOUT.
+__global__ void wait_timeout_kernel(int* status) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) tc::mbar_wait(&bar, 0, reinterpret_cast<volatile int*>(&abort_flag), status);
+}
+
+cudaError_t launch_wait_timeout(int* status, cudaStream_t st) {
+  wait_timeout_kernel<<<1, 32, 0, st>>>(status);
+  return cudaGetLastError();
+}
 
 cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st) {
   const int BN = (a.N % 256 == 0) ? 256 : 128;

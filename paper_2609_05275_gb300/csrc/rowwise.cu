@@ -52,15 +52,15 @@ static int grid_for(long long work_items, int per_block, int cap) {
   if (g > cap) g = cap;
   return (int)g;
 }
-static int g_sms = 0;
 int device_sm_count() {
-  if (!g_sms) {
-    int dev = 0;
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const int n = [] {
+    int dev = 0, v = 0;
     cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (g_sms <= 0) g_sms = 148;
-  }
-  return g_sms;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    return v > 0 ? v : 152;
+  }();
+  return n;
 }
 
 // ---------------------------------------------------------------- RMSNorm fwd
