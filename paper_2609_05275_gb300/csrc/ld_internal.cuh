@@ -246,9 +246,9 @@ struct GemmArgs {
   int* status;
 };
 
-cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st);
+cudaError_t gemm_tc(const GemmArgs& a, cudaStream_t st);    // bf16 operands, tcgen05
 // One block whose bounded wait never completes: records LD_ERR_TIMEOUT.
-cudaError_t launch_wait_timeout(int* status, cudaStream_t st);    // bf16 operands, tcgen05
+cudaError_t launch_wait_timeout(int* status, cudaStream_t st);
 cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);  // float operands, SIMT
 int device_sm_count();
 
