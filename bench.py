@@ -74,6 +74,46 @@ def flops_per_token(cfg, split=False):
     return attn_proj + ffn + attn, attn_proj + ffn
 
 
+def replica_command(n, argv, port):
+    """The command that runs this script as n replica processes, one per
+    GPU of this node (torchrun; rendezvous on 127.0.0.1): what `--gpus N`
+    does when no launcher has set WORLD_SIZE."""
+    return [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+            "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__)] + list(argv)
+
+
+def free_port():
+    import socket
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def tensor_peak_at_clock(sm_mhz, sms=152):
+    """Dense bf16 tensor rate of the whole GPU at a given SM clock: 8192
+    FLOP per clock per SM (one M = 128, N = 256, K = 16 tcgen05 MMA every 128
+    clocks, measured on this GPU), in TFLOP/s."""
+    return sms * 8192.0 * sm_mhz * 1e6 / 1e12
+
+
+def result_line(world, B, S, ms, **extra):
+    """The JSON line's job-level fields: whole-job throughput over every
+    replica (each rank processes its own batch of B x S tokens) from the
+    slowest rank's step time `ms`."""
+    return dict({"value": world * B * S / (ms / 1e3), "unit": "tokens/s", "n_gpus": world, "ms_per_step": ms,
+                 "scaling": "weak"}, **extra)
+
+
+def config_of(args, cfg, sched, first_step, world):
+    """The `config` object of the JSON line (the same for both arms)."""
+    return {"workload": args.config, **{k: cfg[k] for k in ("L", "d", "H", "Hkv", "Dh", "F", "B", "S")},
+            "schedule": sched, "granularity": args.granularity, "sublayer": args.sublayer,
+            "first_step": first_step, "parallelism": f"replicas x{world}",
+            "l2": "inputs and weights larger than L2 (no flush)"}
+
+
 def max_over_ranks(ms, world, device="cuda"):
     """Step time of the whole job: the slowest rank's."""
     if world <= 1:
@@ -183,31 +223,35 @@ def run_reference(args):
     if rank != 0:
         return 0
     cfg, sched = synth.CONFIGS[args.config], synth.SCHEDULES[args.config]
-    rows = min(args.cpu_rows or 1024, cfg["S"])  # per step: a bounded sample, so the run stays within minutes
+    rows = min(args.cpu_rows or cfg["S"], cfg["S"])  # a whole sequence unless asked otherwise
     w0 = synth.layer_weights(cfg, 0, seed=0)
     x = synth.activations(cfg, seed=0, B=1)[0]
     dy = synth.upstream_grad(cfg, B=1)[0]
     osched = dict(dist=sched["dist"], p_max=sched.get("p_max", 0.0), p_explicit=sched.get("p_explicit"),
                   time=sched.get("time", "const"), T=sched.get("T"), ramp=sched.get("ramp"))
-    times, units = [], []
-    for k in range(args.warmup + args.steps):
-        t = k
+    # the oracle's cost of one kept (layer, sequence) is measured once, on
+    # layer 0 and sequence 0 (one forward + backward of `rows` rows); each
+    # step's time is that cost times the step's kept (layer, sequence) pairs
+    # from the step's own masks, so the run stays within minutes
+    step0 = args.step0 if args.step0 is not None else synth.STEPS[args.config][-1]
+    rates0 = OS.layer_rates(osched, cfg["L"], step0)
+    r = cpu_baseline(cfg, w0, x, dy, rows, 1, OS.residual_scale(rates0[0]))
+    per_pair = cfg["B"] * cfg["S"] / r["value"]  # seconds per kept (layer, sequence)
+    times = []
+    for k in range(args.warmup, args.warmup + args.steps):
+        t = step0 + k
         rates = OS.layer_rates(osched, cfg["L"], t)
         mk = OM.draw_masks(sched["seed"], t, [OS.drop_threshold(p) for p in rates], cfg["B"])
-        r = cpu_baseline(cfg, w0, x, dy, rows, int(mk.sum()), OS.residual_scale(rates[0]))
-        if k >= args.warmup:
-            times.append(cfg["B"] * cfg["S"] / r["value"])
-            units.append(int(mk.sum()))
+        times.append(per_pair * int(mk.sum()))
     step = sum(times) / len(times)
     value = cfg["B"] * cfg["S"] / step
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": args.config, **{k: cfg[k] for k in ("L", "d", "H", "Hkv", "Dh", "F", "B", "S")},
-                       "schedule": sched},
+            "config": config_of(args, cfg, sched, step0 + args.warmup, args.gpus),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": f"per step: layer 0, sequence 0, rows 0..{rows - 1}, fwd+bwd, extrapolated "
-                                       f"by the step's kept tokens"},
+                             "sample": r["sample"].split(";")[0] + "; measured once, each step scaled by its own "
+                                       "kept (layer, sequence) pairs", "sample_seconds": r["sample_seconds"]},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
@@ -389,6 +433,10 @@ def main():
                     help="depth-elastic inference forward (full depth, early exit, layer skipping) at the "
                          "workload shape and batch-1 shapes; one JSON line per setting")
     args = ap.parse_args()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        # no outer launcher: start the N replicas here (each rank reads its
+        # RANK / LOCAL_RANK / WORLD_SIZE from the environment torchrun sets)
+        return subprocess.call(replica_command(args.gpus, sys.argv[1:], free_port()))
     if args.impl == "reference":
         return run_reference(args)
     if args.sweep:
@@ -475,7 +523,10 @@ def main():
     # weight-gradient products on the one stream (no overlap), so each
     # launch is timed alone
     P.ld_set_timing(st.h, 1)
+    clk_serial = Clocks(local)
+    clk_serial.start()
     ms_serial = timed(args.steps, step0 + args.warmup, step)
+    clk_serial = clk_serial.stop()
     gemm_ms, gemm_launches = P.ld_get_timing(st.h, P.LD_KCLASS_GEMM)
     attn_ms, attn_launches = P.ld_get_timing(st.h, P.LD_KCLASS_ATTN)
     row_ms, row_launches = P.ld_get_timing(st.h, P.LD_KCLASS_ROWWISE)
@@ -560,19 +611,34 @@ def main():
             "traffic_source": "ncu DRAM bytes of a 2-layer capture per kept row, times kept rows per launch",
             "peak_kind": f"bf16 sustained ({peaks['source']})", "launches_per_step": gemm_launches / args.steps,
             "avg_launch_ms": gemm_ms / max(gemm_launches, 1)}
+    # attention class (forward and backward kernels) on model FLOPs: 3 x the
+    # forward's 4 (len^2 / 2) Dh per head and kept sequence (the backward's
+    # recomputation of the scores gets no credit)
+    attn_flops = exec_flops - gemm_flops  # per step
+    attn_achieved = attn_flops * args.steps / (attn_ms / 1e3) / 1e12 if attn_ms > 0 else None
+    attn_roof = {"kernel": "attn_fwd_pp_kernel / attn_fwd_tc_kernel + attn_bwd_tc_kernel", "bound": "tensor",
+                 "achieved": attn_achieved, "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
+                 "frac": attn_achieved / peaks["bf16_sustained"] if attn_achieved else None,
+                 "launches_per_step": attn_launches / args.steps}
+    if clk_serial and attn_achieved:
+        attn_roof["frac_at_clock"] = attn_achieved / tensor_peak_at_clock(clk_serial["sm_mhz"])
+    if clk_serial and gemm_achieved:
+        # the same launches against the tensor rate at the SM clock sampled
+        # while they ran: separates kernel efficiency from the clock
+        pk = tensor_peak_at_clock(clk_serial["sm_mhz"])
+        roof.update({"sm_mhz_timing_pass": clk_serial["sm_mhz"], "peak_at_clock": pk,
+                     "frac_at_clock": gemm_achieved / pk})
     line = {
-        "metric": METRIC, "value": world * B * S / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": args.config, **{k: cfg[k] for k in ("L", "d", "H", "Hkv", "Dh", "F", "B", "S")},
-                   "schedule": sched, "granularity": args.granularity, "sublayer": sub,
-                   "first_step": step0 + args.warmup,
-                   "parallelism": f"replicas x{world}", "l2": "inputs and weights larger than L2 (no flush)"},
+        "metric": METRIC, **result_line(world, B, S, ms),
+        "steps": args.steps, "warmup": args.warmup, "higher_is_better": True,
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": config_of(args, cfg, sched, step0 + args.warmup, world),
         "executed_tflops": tflops, "pct_bf16_peak": 100.0 * tflops / peaks["bf16"],
         "pct_bf16_peak_sustained": 100.0 * tflops / peaks["bf16_sustained"],
         "p_bar_expected": p_exp, "p_bar_realized": p_real,
         "skip_speedup": (dense_ms / ms) if dense_ms else None,
         "ideal_speedup": 1.0 / (1.0 - p_real), "dense_ms_per_step": dense_ms,
+        "attention_roofline": attn_roof,
         "kernel_ms_per_step": {"gemm": gemm_ms / args.steps, "attention": attn_ms / args.steps,
                                "rowwise": row_ms / args.steps,
                                "serialized_ms_per_step": ms_serial,

@@ -311,7 +311,9 @@ ld_status ld_rmsnorm_backward(int B, int S, int d, const float* dyn, const void*
  * min(ceil(B*S / 8), 320) * d <= 2,621,440 (e.g. d <= 8192 once B*S >= 2560);
  * larger sizes return LD_ERR_SHAPE.  The first call on each device looks up
  * the array's address with that device current, so make it before any stream
- * capture.  All calls share the array: nothing in it needs clearing (each
+ * capture; the address is kept per device and context, and the first call
+ * after cudaDeviceReset (a new context) looks it up again, so that call too
+ * belongs before any capture.  All calls share the array: nothing in it needs clearing (each
  * call overwrites every partial sum it reads), but calls that overlap on the
  * GPU race on it and must be serialised by the caller.  Allocates nothing. */
 ld_status ld_rmsnorm_backward_noalloc(int B, int S, int d, const float* dyn, const void* xs, const float* rstd,

@@ -13,14 +13,20 @@
 // library holds it (kNoallocScratchFloats floats = 10 MiB) until the process
 // exits.  Host code cannot use the array's name as a device address: on the
 // first call on each device (with that device current) the entry point asks
-// the runtime for the address with cudaGetSymbolAddress and keeps it.  That
-// first call should therefore come before any stream capture.
+// the runtime for the address with cudaGetSymbolAddress and keeps it, keyed
+// by the device and its current context.  That first call should therefore
+// come before any stream capture.  After cudaDeviceReset the device has a new
+// primary context in which the module, and so the array, is loaded afresh:
+// the next call sees the new context and looks the address up again (that
+// call, too, should come before any capture).
 //
 // All calls share the one array.  Every call writes each partial sum it later
 // reads (block b fills row b completely before the column sum runs), so
 // nothing has to start at zero; but calls that overlap on the GPU (two
 // streams, or two host threads) race on the array and must be serialised by
 // the caller.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "ld_internal.cuh"
@@ -32,21 +38,48 @@ constexpr int kMaxDevices = 64;
 
 __device__ __align__(256) float g_noalloc_scratch[kNoallocScratchFloats];
 
-float* g_scratch_addr[kMaxDevices] = {};
+struct ScratchAddr {
+  CUcontext ctx;  // the context the address belongs to
+  float* ptr;
+};
+ScratchAddr g_scratch_addr[kMaxDevices] = {};
 std::mutex g_scratch_mu;
 
-// Device address of g_noalloc_scratch on the current device (looked up once
-// per device); null on failure.
+// The driver's cuCtxGetCurrent, reached through the runtime (the library
+// links the runtime only).
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+CtxGetCurrentFn ctx_get_current() {
+  static const CtxGetCurrentFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<CtxGetCurrentFn>(nullptr);
+    return reinterpret_cast<CtxGetCurrentFn>(p);
+  }();
+  return fn;
+}
+
+// Device address of g_noalloc_scratch on the current device, looked up once
+// per (device, context); null on failure.
 float* scratch_address() {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  CtxGetCurrentFn get = ctx_get_current();
+  CUcontext ctx = nullptr;
+  if (!get || get(&ctx) != CUDA_SUCCESS) return nullptr;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_addr[dev]) {
+  ScratchAddr& a = g_scratch_addr[dev];
+  if (!ctx || !a.ptr || a.ctx != ctx) {
+    // the lookup also makes the device's primary context current when no
+    // context is yet
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return nullptr;
-    g_scratch_addr[dev] = static_cast<float*>(p);
+    if (get(&ctx) != CUDA_SUCCESS || !ctx) return nullptr;
+    a.ctx = ctx;
+    a.ptr = static_cast<float*>(p);
   }
-  return g_scratch_addr[dev];
+  return a.ptr;
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }

@@ -62,6 +62,17 @@ def test_noalloc_matches_scratch_entry_point_twice():
         assert torch.isfinite(dg2).all()
 
 
+def test_noalloc_wide_rows_after_a_larger_call():
+    # d > 8192 runs the shared-memory row kernel (its own launch attribute);
+    # B*S = 512 gives 64 partial-sum rows of 16384, inside the fixed array.
+    # The first call fills more of the array (320 rows at d = 8192), so stale
+    # partial sums would show up in the second call's dgamma.
+    for B, S, d, kept, seed in ((2, 2048, 8192, [0, 1], 4), (2, 256, 16384, [1, 0], 5)):
+        (dx, nx, dg), (dx2, nx2, dg2) = _both(B, S, d, kept, seed)
+        assert _close(dx2, dx) and _close(nx2, nx) and _close(dg2, dg)
+        assert torch.isfinite(dg2).all()
+
+
 def test_noalloc_rejects_sizes_beyond_its_array():
     t = _inputs(1, 2560, 16384, [0], 3)
     dg = torch.empty(16384, device="cuda")
