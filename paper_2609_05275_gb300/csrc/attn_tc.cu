@@ -221,51 +221,51 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer (whole warp, converged; one elected lane issues)
-    __syncwarp();
-    constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
-    constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
-    // descriptors built once, advanced by (byte offset >> 4) per MMA
-    const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
-    const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
-    bool ok = warp_wait(q_full, 0, abort_flag, status);
-    for (int j = 0; ok && j <= nkt; ++j) {
-      if (j < nkt) {
-        const int s = j % NSK;
-        if (!warp_wait(&k_full[s], (j / NSK) & 1, abort_flag, status)) { ok = false; break; }
-        if (!warp_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
-        const uint64_t kb = DK + (uint64_t)((s * TILE) >> 4);
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
+      constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
+      // descriptors built once, advanced by (byte offset >> 4) per MMA
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
+      const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
+      bool ok = mbar_wait(q_full, 0, abort_flag, status);
+      for (int j = 0; ok && j <= nkt; ++j) {
+        if (j < nkt) {
+          const int s = j % NSK;
+          if (!mbar_wait(&k_full[s], (j / NSK) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t kb = DK + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-          mma_bf16_w(tmem + (j & 1) * 128, DQ + off, kb + off, ID_S, kk > 0);
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+            mma_bf16(tmem + (j & 1) * 128, DQ + off, kb + off, ID_S, kk > 0);
+          }
+          mma_commit(&s_full[j & 1]);
+          mma_commit(&k_empty[s]);
         }
-        mma_commit_w(&s_full[j & 1]);
-        mma_commit_w(&k_empty[s]);
-      }
-      if (j >= 1) {
-        const int jp = j - 1, s = jp % NSV, pb = jp & 1;
-        if (!warp_wait(&p_full[pb], (jp >> 1) & 1, abort_flag, status)) { ok = false; break; }
-        if (!warp_wait(&v_full[s], (jp / NSV) & 1, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
-        const uint64_t vb = DV + (uint64_t)((s * TILE) >> 4);
+        if (j >= 1) {
+          const int jp = j - 1, s = jp % NSV, pb = jp & 1;
+          if (!mbar_wait(&p_full[pb], (jp >> 1) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(&v_full[s], (jp / NSV) & 1, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t vb = DV + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          // A = P from TMEM (16 keys = 8 columns a step); B = V as MN-major
-          // (dh contiguous): 64-dh chunks one slab apart, 8-key groups 1 KB
-          mma_bf16_ta_w(t_o, t_p + pb * 64 + kk * 8, vb + ((kk * 2048) >> 4), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < 8; ++kk) {
+            // A = P from TMEM (16 keys = 8 columns a step); B = V as MN-major
+            // (dh contiguous): 64-dh chunks one slab apart, 8-key groups 1 KB
+            mma_bf16_ta(t_o, t_p + pb * 64 + kk * 8, vb + ((kk * 2048) >> 4), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
+          }
+          mma_commit(&pv_done[pb]);
+          mma_commit(&v_empty[s]);
         }
-        mma_commit_w(&pv_done[pb]);
-        mma_commit_w(&v_empty[s]);
       }
-    }
-    if (ok) {
-      mma_commit_w(o_full);
-    } else {
-      mma_commit_w(drain);
-      if (lane == 0) mbar_drain(drain, 0);
-      __syncwarp();
+      if (ok) {
+        mma_commit(o_full);
+      } else {
+        mma_commit(drain);
+        mbar_drain(drain, 0);
+      }
     }
   } else {
     // ------------------------------------------------ softmax (warps 2..9)
@@ -466,37 +466,11 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // the group may rescale O_g as soon as S_g(j) is ready.  Tile B is skipped
 // when the sequence ends before it.
 constexpr int PP_NSK = 3, PP_NSV = 2;
-// Pairs (of the 16 in each 32-key chunk) whose exponentials run on the FMA
-// pipe (ex2_poly2) instead of MUFU: the 128 x 128 exponentials of a tile
-// take as many cycles at 16 a clock as the tile's two MMAs.
-constexpr int PP_POLY = 0;
 
-// 2^x for two values on the FMA pipe: x = n + f with n = rint(x) and f in
-// [-1/2, 1/2]; 2^f = 1 + f (C1 + f (C2 + f C3)), the cubic fitted to 2^f on
-// that interval by minimising the largest relative error (1.0e-4 in float32,
-// below the 2^-9 half-ulp of the bf16 P is stored in); 2^n is added into the
-// exponent field.  x is clamped at -127, where the result is below 2^-126
-// instead of 0.
-__device__ __forceinline__ void ex2_poly2(float x0, float x1, float& y0, float& y1) {
-  constexpr float C1 = 0.6932829022407532f, C2 = 0.24221037328243256f, C3 = 0.05500858277082443f;
-  x0 = fmaxf(x0, -127.f);
-  x1 = fmaxf(x1, -127.f);
-  const float n0 = rintf(x0), n1 = rintf(x1);
-  const uint64_t f = f2_sub(f2_pack(x0, x1), f2_pack(n0, n1));
-  uint64_t p = f2_fma(f, f2_pack(C3, C3), f2_pack(C2, C2));
-  p = f2_fma(p, f, f2_pack(C1, C1));
-  p = f2_fma(p, f, f2_pack(1.f, 1.f));
-  float p0, p1;
-  f2_unpack(p, p0, p1);
-  y0 = __int_as_float(__float_as_int(p0) + ((int)n0 << 23));
-  y1 = __int_as_float(__float_as_int(p1) + ((int)n1 << 23));
-}
-
-template <bool ALIBI>
 __global__ void __launch_bounds__(320, 1)
     attn_fwd_pp_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
-                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv,
-                       const float* __restrict__ alibi, const int* __restrict__ seg, int* status) {
+                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv, const int* __restrict__ seg,
+                       int* status) {
   constexpr int DH = 128;
   constexpr uint32_t TILE = 2 * SLAB;  // one 128 x 128 bf16 tile (two 64-column slabs)
   extern __shared__ uint8_t smem_raw[];
@@ -596,52 +570,52 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer (whole warp, converged; one elected lane issues)
-    constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
-    constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
-    const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
-    const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
-    __syncwarp();
-    bool ok = warp_wait(q_full, 0, abort_flag, status);
-    for (int j = 0; ok && j <= nkt; ++j) {
-      if (j < nkt && !warp_wait(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
-      if (j >= 1 && !warp_wait(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
-        ok = false;
-        break;
-      }
-      for (int gi = 0; gi < 2; ++gi) {
-        const int nkg = gi ? nkB : nkA;
-        if (j >= 1 && j - 1 < nkg) {
-          // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
-          if (!warp_wait(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk)
-            mma_bf16_ta_w(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
-                            (j > 1 || kk > 0) ? 1u : 0u);
-          if (j == nkg) mma_commit_w(&o_full[gi]);  // the group's last P V
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
+      constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
+      const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
+      bool ok = mbar_wait(q_full, 0, abort_flag, status);
+      for (int j = 0; ok && j <= nkt; ++j) {
+        if (j < nkt && !mbar_wait(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
+        if (j >= 1 && !mbar_wait(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
+          ok = false;
+          break;
         }
-        if (j < nkg) {
-          // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
-          const uint64_t kb = DK + (uint64_t)(((j % PP_NSK) * TILE) >> 4);
-          const uint64_t qd = DQ + (uint64_t)((gi * TILE) >> 4);
+        for (int gi = 0; gi < 2; ++gi) {
+          const int nkg = gi ? nkB : nkA;
+          if (j >= 1 && j - 1 < nkg) {
+            // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
+            if (!mbar_wait(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
+            tc_fence_after();
+            const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk) {
-            const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-            mma_bf16_w(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
+            for (int kk = 0; kk < 8; ++kk)
+              mma_bf16_ta(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
+                          (j > 1 || kk > 0) ? 1u : 0u);
+            if (j == nkg) mma_commit(&o_full[gi]);  // the group's last P V
           }
-          mma_commit_w(&s_full[gi]);
+          if (j < nkg) {
+            // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
+            const uint64_t kb = DK + (uint64_t)(((j % PP_NSK) * TILE) >> 4);
+            const uint64_t qd = DQ + (uint64_t)((gi * TILE) >> 4);
+#pragma unroll
+            for (int kk = 0; kk < DH / 16; ++kk) {
+              const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+              mma_bf16(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
+            }
+            mma_commit(&s_full[gi]);
+          }
         }
+        if (!ok) break;
+        if (j < nkt) mma_commit(&k_empty[j % PP_NSK]);
+        if (j >= 1) mma_commit(&v_empty[(j - 1) % PP_NSV]);
       }
-      if (!ok) break;
-      if (j < nkt) mma_commit_w(&k_empty[j % PP_NSK]);
-      if (j >= 1) mma_commit_w(&v_empty[(j - 1) % PP_NSV]);
-    }
-    if (!ok) {
-      mma_commit_w(drain);
-      if (lane == 0) mbar_drain(drain, 0);
-      __syncwarp();
+      if (!ok) {
+        mma_commit(drain);
+        mbar_drain(drain, 0);
+      }
     }
   } else {
     // ------------------------------------------------ softmax (warps 2..9)
@@ -653,40 +627,20 @@ __global__ void __launch_bounds__(320, 1)
     const int nkg = gi ? nkB : nkA;
     const int jdiag = 2 * qb + gi;  // the K tile on this query tile's diagonal
     const float sl2 = kLog2e * rsqrtf((float)DH);
-    // ALiBi: the exponent is x = S sl2 + slope2 (key - query), and the
-    // running max m is kept on x (the max of S alone, scaled, otherwise)
-    const float slope2 = ALIBI ? alibi[h] * kLog2e : 0.f;
-    const int qrow_t = qb * 256 + gi * 128 + r;  // this thread's query within the sequence
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nkg; ++j) {
       if (!warp_wait(&s_full[gi], j & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
       const bool diag = (j == jdiag);  // keys after the query are left out (block-uniform)
-      // pass 1: row max of the raw scores (the scale is positive), or of x
-      // with ALiBi
+      // pass 1: row max of the raw scores (the scale is positive)
       float mraw = -INFINITY;
-      const float b0 = slope2 * (float)(j * 128 - qrow_t);  // bias of key 0 of the tile
 #pragma unroll 1
       for (int c2 = 0; c2 < 2; ++c2) {
         uint32_t sr[2][32];
         tmem_ld32_nw(t_s + c2 * 64 + lane_off, sr[0]);
         tmem_ld32_nw(t_s + c2 * 64 + 32 + lane_off, sr[1]);
         tmem_wait_ld();
-        if constexpr (ALIBI) {
-          const uint64_t sl2x2 = f2_pack(sl2, sl2), sx2 = f2_pack(slope2, slope2);
-          const float bc = b0 + slope2 * (float)(c2 * 64);
-          const uint64_t bx2 = f2_pack(bc, bc);
-#pragma unroll
-          for (int e = 0; e < 64; e += 2) {
-            float x0, x1;
-            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1])),
-                             sl2x2, f2_fma(f2_pack((float)e, (float)(e + 1)), sx2, bx2)),
-                      x0, x1);
-            sr[e >> 5][e & 31] = __float_as_uint(x0);
-            sr[e >> 5][(e & 31) + 1] = __float_as_uint(x1);
-          }
-        }
         if (diag) {
 #pragma unroll
           for (int e = 0; e < 64; ++e)
@@ -697,7 +651,7 @@ __global__ void __launch_bounds__(320, 1)
             mraw = fmax3(mraw, __uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1]));
         }
       }
-      const float mt = ALIBI ? mraw : mraw * sl2;
+      const float mt = mraw * sl2;
       const bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
       // O_g is rescaled in TMEM when any lane of the warp moved its max
@@ -720,7 +674,6 @@ __global__ void __launch_bounds__(320, 1)
       // pass 2: P = exp2(S c log2e - m) for 32 keys at a time, written as
       // bf16 pairs over S columns that have already been read
       const uint64_t sl2x2 = f2_pack(sl2, sl2), nm2 = f2_pack(-m_new, -m_new);
-      const uint64_t sx2 = f2_pack(slope2, slope2);
       uint64_t ls2 = f2_pack(0.f, 0.f);
 #pragma unroll 1
       for (int c = 0; c < 4; ++c) {
@@ -728,20 +681,11 @@ __global__ void __launch_bounds__(320, 1)
         tmem_ld32_nw(t_s + c * 32 + lane_off, sr);
         tmem_wait_ld();
         uint32_t pk[16];
-        const float bm = b0 + slope2 * (float)(c * 32) - m_new;  // ALiBi: bias of key 32c minus the max
-        const uint64_t bmx2 = f2_pack(bm, bm);
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           float x0, x1;
-          const uint64_t add = ALIBI ? f2_fma(f2_pack((float)(2 * e), (float)(2 * e + 1)), sx2, bmx2) : nm2;
-          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, add), x0, x1);
-          float p0, p1;
-          if (e >= 16 - PP_POLY) {
-            ex2_poly2(x0, x1, p0, p1);
-          } else {
-            p0 = ex2(x0);
-            p1 = ex2(x1);
-          }
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, nm2), x0, x1);
+          float p0 = ex2(x0), p1 = ex2(x1);
           if (diag) {
             p0 = (c * 32 + 2 * e <= r) ? p0 : 0.f;
             p1 = (c * 32 + 2 * e + 1 <= r) ? p1 : 0.f;
@@ -786,19 +730,18 @@ __global__ void __launch_bounds__(320, 1)
   }
 }
 
-template <bool ALIBI>
 cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
-                   int max_seqs, const float* alibi, const int* seg, int* status, cudaStream_t st) {
+                   int max_seqs, const int* seg, int* status, cudaStream_t st) {
   // 2 Q, 3 K and 2 V tiles of 32 KB + alignment + barriers = 230,656 bytes (of 232,448)
   constexpr size_t smem = (size_t)(2 + PP_NSK + PP_NSV) * 2 * SLAB + 1024 + 256;
   // once per process (initialisation of a function-local static is thread-safe)
   static const cudaError_t attr =
-      cudaFuncSetAttribute(attn_fwd_pp_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      cudaFuncSetAttribute(attn_fwd_pp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   dim3 grid(H, max_seqs, (S + 255) / 256);
-  attn_fwd_pp_kernel<ALIBI><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi, seg, status);
+  attn_fwd_pp_kernel<<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, seg, status);
   return cudaGetLastError();
 }
 
@@ -806,45 +749,34 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // Backward, head size 128.  One CTA per (128-key tile, kv head, kept
 // sequence), looping over the query heads of the group and the 64-query
 // tiles at or after the key tile.  448 threads:
-//   warp 0      TMA: K, V once; Q_i, dO_i per step (3 stages); all lanes
-//               write the bf16 terms of -lse_i sqrt(Dh) and -D_i that two extra
-//               K = 16 MMAs fold into S^T_i and dP^T_i
+//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
 //   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
 //               (M = 128 keys, N = 64 queries); then for step i-1
 //               dV += P^T dO (P^T read from TMEM), dK += dS^T Q (M = 128
 //               keys, N = 128) and dQ^T = K^T dS^T (M = 128 head dims,
 //               N = 64 queries)
 //   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e)
-//               as bf16 into TMEM and dS^T = P^T (dP^T - D) as bf16 into a
-//               swizzled shared-memory tile, the lse and D terms already
-//               inside S^T and dP^T; at the end dK (times c) and dV from
-//               TMEM to dqkv
-//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer by global
-//               reductions from registers (shared memory bandwidth is what
-//               bounds this kernel, so dQ is not staged there)
+//               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
+//               swizzled shared-memory tile; at the end dK (times c) and dV
+//               from TMEM to dqkv
+//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
 // P^T and dS^T are double-buffered (step i uses buffer i & 1), so the
 // softmax warps write step i while the MMAs of step i-1 still read theirs.
 // TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447,
 // P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
-// x as three bf16 terms, t0 + t1 + t2 = x to about 2^-24 |x| (each residual
-// is exact in float32), packed as the first 16 bytes of a K-major row:
-// t0, t1, t2, 0, 0, 0, 0, 0.
-__device__ __forceinline__ uint4 split3_bf16(float x) {
-  const bf16 t0 = __float2bfloat16_rn(x);
-  const float r1 = x - __bfloat162float(t0);
-  const bf16 t1 = __float2bfloat16_rn(r1);
-  const float r2 = r1 - __bfloat162float(t1);
-  const bf16 t2 = __float2bfloat16_rn(r2);
-  return make_uint4((uint32_t)__bfloat16_as_ushort(t0) | ((uint32_t)__bfloat16_as_ushort(t1) << 16),
-                    (uint32_t)__bfloat16_as_ushort(t2), 0u, 0u);
+// Values 4 e4 .. 4 e4 + 3 of p (shared memory); p is 16-byte aligned when
+// off == 0 (warp-uniform), else read one by one.
+__device__ __forceinline__ float4 ld4s(const float* p, int e4, int off) {
+  if (off == 0) return reinterpret_cast<const float4*>(p)[e4];
+  return make_float4(p[4 * e4], p[4 * e4 + 1], p[4 * e4 + 2], p[4 * e4 + 3]);
 }
 
 template <bool ALIBI>
 __global__ void __launch_bounds__(448, 1)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
-                       const __grid_constant__ CUtensorMap tmo,
+                       const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
@@ -861,16 +793,14 @@ __global__ void __launch_bounds__(448, 1)
   uint8_t* Qs = Vs + KT;         // [NST][QT]
   uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
   uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
-  // XT: 128 rows x 128 bytes (128-byte swizzle) of the extra K = 16 chunks
-  // that fold the softmax statistics into the MMAs.  Chunk 0 of every row is
-  // the A operand (1, 1, 1, 0, ...); chunk 1 + b of rows 0..63 holds, for
-  // the 64 queries of a step in stage b, the three bf16 terms of
-  // -lse sqrt(Dh), and of rows 64..127 those of -D.  The exponent of P is
-  // c S - lse log2(e) = c (S - lse sqrt(Dh)) with c = log2(e) / sqrt(Dh), so
-  // S^T comes out of the MMAs as S^T - lse sqrt(Dh) and dP^T as dP^T - D,
-  // and the softmax warps read no per-query vectors.
-  uint8_t* XT = DSs + 2 * SLAB;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(XT + SLAB);
+  float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
+  // [NST][lse 68 | D 68]: the 64 values of a step start at float `voff` of
+  // each half (a sequence's rows start anywhere with per-token kept lists,
+  // and a bulk copy needs a 16-byte aligned source, so 68 are copied from
+  // the aligned-down address)
+  float* vecs = dqs + 64 * DH;
+  constexpr int VS = 136;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * VS);
   uint64_t* kv_full = bars;
   uint64_t* ld_full = bars + 1;          // [NST]
   uint64_t* ld_empty = ld_full + NST;    // [NST]
@@ -886,10 +816,7 @@ __global__ void __launch_bounds__(448, 1)
 
   // rows row0 .. row0+len-1 as in the forward; queries past len (the last
   // query tile) get P = dS = 0, keys past len are never stored
-  // grid (kv head, key tile, sequence): the blocks of one sequence are
-  // dispatched together, heaviest key tiles (kt = 0) first, so the Q, dO and
-  // dQ rows in use at a time are one sequence's (they stay in L2)
-  const int seq = blockIdx.z;
+  const int seq = blockIdx.y;
   int row0, len;
   if (seg) {
     row0 = seg[seq];
@@ -899,7 +826,7 @@ __global__ void __launch_bounds__(448, 1)
     row0 = seq * S;
     len = S;
   }
-  const int kt = blockIdx.y, g = blockIdx.x, grp = H / Hkv;
+  const int kt = blockIdx.z, g = blockIdx.x, grp = H / Hkv;  // heaviest key tiles (kt = 0) dispatched first
   if (kt * 128 >= len) return;
   const int nq = (len + 63) / 64, q0 = 2 * kt;  // query tiles q0 .. nq-1 overlap or follow the keys
   const int n_it = grp * (nq - q0);
@@ -923,16 +850,6 @@ __global__ void __launch_bounds__(448, 1)
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (threadIdx.x < 128) {
-    // row r of XT: the ones of chunk 0, zeros everywhere else (the term
-    // chunks are written per step, their upper halves stay zero)
-    const int r = threadIdx.x;
-#pragma unroll
-    for (int u = 0; u < 8; ++u)
-      *reinterpret_cast<uint4*>(XT + swz(r, u)) =
-          u == 0 ? make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
-    fence_proxy_async();
-  }
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
@@ -942,125 +859,92 @@ __global__ void __launch_bounds__(448, 1)
   const uint32_t t_p = tmem + 448;  // [2] x 32 columns: P^T as bf16 pairs
 
   if (warp == 0) {
-    // ------------------------------------------------ producer (warp 0)
-    // lane 0: TMA of K, V once and of Q_i, dO_i per step; all lanes: the
-    // terms of -lse sqrt(Dh) and -D of step i into XT (two queries a lane,
-    // zero past the sequence), loaded from global memory one step ahead
-    const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
     if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
       mbar_arrive_expect_tx(kv_full, 2 * KT);
       for (int c = 0; c < 2; ++c) {
         tma_load_2d(Ks + c * SLAB, &tmkv, kcol + 64 * c, row0 + kt * 128, kv_full);
         tma_load_2d(Vs + c * SLAB, &tmkv, vcol + 64 * c, row0 + kt * 128, kv_full);
       }
-    }
-    const float sq_dh = 1.f / rsqrtf((float)DH);  // sqrt(Dh) as the softmax warps' scale c = log2(e) rsqrt(Dh) divides it
-    float xl[2], xd[2];
-    auto load_terms = [&](int i) {
-      const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
-#pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        const int q = qt * 64 + hf * 32 + lane;
-        xl[hf] = 0.f;
-        xd[hf] = 0.f;
-        if (q < len) {
-          const size_t at = (size_t)h * lse_ld + row0 + q;
-          xl[hf] = -lse[at] * sq_dh;
-          xd[hf] = -Dvec[at];
-        }
-      }
-    };
-    if (n_it > 0) load_terms(0);
-    int issued = 0;
-    for (int i = 0; i < n_it; ++i) {
-      const int b = i % NST;
-      const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
-      if (!warp_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
-#pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        const int r = hf * 32 + lane;
-        *reinterpret_cast<uint4*>(XT + swz(r, 2 + 2 * b)) = split3_bf16(xl[hf]);
-        *reinterpret_cast<uint4*>(XT + swz(64 + r, 2 + 2 * b)) = split3_bf16(xd[hf]);
-      }
-      fence_proxy_async();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive_expect_tx(&ld_full[b], 2 * QT);
+      int issued = 0;
+      for (int i = 0; i < n_it; ++i) {
+        const int b = i % NST;
+        const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
+        if (!mbar_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 2 * 272);
         for (int c = 0; c < 2; ++c) {
           tma_load_2d(Qs + b * QT + c * HSLAB, &tmq, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
           tma_load_2d(dOs + b * QT + c * HSLAB, &tmo, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
         }
+        const size_t vo = ((size_t)h * lse_ld + row0 + qt * 64) & ~(size_t)3;  // lse_ld % 4 == 0
+        bulk_load(vecs + b * VS, lse + vo, 272, &ld_full[b]);
+        bulk_load(vecs + b * VS + 68, Dvec + vo, 272, &ld_full[b]);
+        ++issued;
       }
-      ++issued;
-      if (i + 1 < n_it) load_terms(i + 1);
+      if (*abort_flag) {
+        mbar_drain(kv_full, 0);
+        for (int i = issued > NST ? issued - NST : 0; i < issued; ++i) mbar_drain(&ld_full[i % NST], (i / NST) & 1);
+      }
     }
-    if (lane == 0 && *abort_flag) {
-      mbar_drain(kv_full, 0);
-      for (int i = issued > NST ? issued - NST : 0; i < issued; ++i) mbar_drain(&ld_full[i % NST], (i / NST) & 1);
-    }
-    __syncwarp();
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer (whole warp, converged; one elected lane issues)
-    __syncwarp();
-    constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
-    constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
-    constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
-    // shared-memory descriptors built once; an MMA's operand is its base
-    // plus (byte offset >> 4) in the address field (every tile lies below
-    // 256 KB, so the 14-bit field never carries)
-    const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
-    const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
-    const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
-    const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
-    const uint64_t DX = sdesc(smem_u32(XT), 16, 1024);  // ones (chunk 0) and the statistics' terms
-    bool ok = warp_wait(kv_full, 0, abort_flag, status);
-    for (int i = 0; ok && i <= n_it; ++i) {
-      if (i < n_it) {
-        const int b = i % NST;
-        if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
-        if (!warp_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
-        const uint64_t st = (uint64_t)((b * QT) >> 4);
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
+      constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
+      constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
+      // shared-memory descriptors built once; an MMA's operand is its base
+      // plus (byte offset >> 4) in the address field (every tile lies below
+      // 256 KB, so the 14-bit field never carries)
+      const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
+      const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
+      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
+      bool ok = mbar_wait(kv_full, 0, abort_flag, status);
+      for (int i = 0; ok && i <= n_it; ++i) {
+        if (i < n_it) {
+          const int b = i % NST;
+          if (!mbar_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t st = (uint64_t)((b * QT) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint32_t koff = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-          const uint32_t qoff = ((kk >> 2) * HSLAB + (kk & 3) * 32) >> 4;
-          mma_bf16_w(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
-          mma_bf16_w(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const uint32_t koff = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+            const uint32_t qoff = ((kk >> 2) * HSLAB + (kk & 3) * 32) >> 4;
+            mma_bf16(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
+            mma_bf16(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
+          }
+          mma_commit(sdp_full);
         }
-        // S^T -= lse sqrt(Dh) and dP^T -= D: ones (128 x 16) times the step's terms (64 x 16)
-        mma_bf16_w(t_s, DX, DX + (uint64_t)(((1 + b) * 32) >> 4), ID_SP, 1u);
-        mma_bf16_w(t_dp, DX, DX + (uint64_t)((64 * 128 + (1 + b) * 32) >> 4), ID_SP, 1u);
-        mma_commit_w(sdp_full);
+        if (i >= 1) {
+          const int ip = i - 1, b = ip % NST, pb = ip & 1;
+          if (!mbar_wait(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t st = (uint64_t)((b * QT) >> 4), ds = (uint64_t)((pb * SLAB) >> 4);
+          const uint32_t first = ip > 0 ? 1u : 0u;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
+            const uint32_t aoff = (kk * 32) >> 4;                // dS^T, K-major
+            const uint32_t boff = (kk * 2048) >> 4;              // dO / Q as MN-major
+            mma_bf16_ta(t_dv, t_p + pb * 32 + kk * 8, DOMN + st + boff, ID_KV, kk > 0 ? 1u : first);
+            mma_bf16(t_dk, DS + ds + aoff, DQMN + st + boff, ID_KV, kk > 0 ? 1u : first);
+          }
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
+            mma_bf16(t_dq, DKMN + ((kk * 2048) >> 4), DS + ds + ((kk * 2048) >> 4), ID_Q, kk > 0);
+          }
+          mma_commit(&mm_done[pb]);
+          mma_commit(&ld_empty[b]);
+        }
       }
-      if (i >= 1) {
-        const int ip = i - 1, b = ip % NST, pb = ip & 1;
-        if (!warp_wait(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
-        if (!warp_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
-        const uint64_t st = (uint64_t)((b * QT) >> 4), ds = (uint64_t)((pb * SLAB) >> 4);
-        const uint32_t first = ip > 0 ? 1u : 0u;
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
-          const uint32_t aoff = (kk * 32) >> 4;                // dS^T, K-major
-          const uint32_t boff = (kk * 2048) >> 4;              // dO / Q as MN-major
-          mma_bf16_ta_w(t_dv, t_p + pb * 32 + kk * 8, DOMN + st + boff, ID_KV, kk > 0 ? 1u : first);
-          mma_bf16_w(t_dk, DS + ds + aoff, DQMN + st + boff, ID_KV, kk > 0 ? 1u : first);
-        }
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
-          mma_bf16_w(t_dq, DKMN + ((kk * 2048) >> 4), DS + ds + ((kk * 2048) >> 4), ID_Q, kk > 0);
-        }
-        mma_commit_w(&mm_done[pb]);
-        mma_commit_w(&ld_empty[b]);
+      if (ok) {
+        mma_commit(acc_done);
+      } else {
+        mma_commit(drain);
+        mbar_drain(drain, 0);
       }
-    }
-    if (ok) {
-      mma_commit_w(acc_done);
-    } else {
-      mma_commit_w(drain);
-      if (lane == 0) mbar_drain(drain, 0);
-      __syncwarp();
     }
   } else if (warp < 10) {
     // ------------------------------------------------ P / dS (warps 2..9)
@@ -1071,14 +955,16 @@ __global__ void __launch_bounds__(448, 1)
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const int voff = row0 & 3;  // first value of a step in its lse / D stage (see vecs)
     const float sl2 = kLog2e * rsqrtf((float)DH);
     bool ok = true;
     for (int i = 0; i < n_it; ++i) {
+      const int b = i % NST;
       const int qt = q0 + i % (nq - q0);
       // ALiBi: logit bias slope2 (key - query) of this step's query head
       const float slope2 = ALIBI ? alibi[g * grp + i / (nq - q0)] * kLog2e : 0.f;
-      // S^T and dP^T arrive with -lse sqrt(Dh) and -D folded in (see XT)
       if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
+      if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
       uint32_t sr[32], dr[32];
       tmem_ld32_nw(t_s + half * 32 + lane_off, sr);
@@ -1087,6 +973,8 @@ __global__ void __launch_bounds__(448, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sdp_free);
+      const float* lsrc = vecs + b * VS + voff + half * 32;       // lse of the 32 queries
+      const float* dsrc = vecs + b * VS + 68 + voff + half * 32;  // D of the 32 queries
       const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
       const int qlim = len - (qt * 64 + half * 32);  // and exists iff c < qlim (warp-uniform)
       uint32_t pk[16], dk[16];
@@ -1095,30 +983,43 @@ __global__ void __launch_bounds__(448, 1)
       // run past the sequence (warp-uniform)
       auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
-        const uint64_t sl2x2 = f2_pack(sl2, sl2);
+        const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
         // bias of query c: slope2 (key - qt*64 - half*32 - c) = b0 - slope2 c
         const float b0 = slope2 * (float)(-qbase);
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
-        for (int c = 0; c < 32; c += 2) {
-          uint64_t x2 = f2_mul(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2);
-          if constexpr (ALIBI) x2 = f2_add(x2, f2_fma(f2_pack((float)c, (float)(c + 1)), nsx2, b0x2));
-          float x0, x1;
-          f2_unpack(x2, x0, x1);
-          float p0 = ex2(x0), p1 = ex2(x1);
-          const bool v0 = !MASK || (qbase + c >= 0 && c < qlim), v1 = !MASK || (qbase + c + 1 >= 0 && c + 1 < qlim);
-          if constexpr (MASK) {
-            p0 = v0 ? p0 : 0.f;
-            p1 = v1 ? p1 : 0.f;
+        for (int e4 = 0; e4 < 8; ++e4) {
+          const float4 lq = ld4s(lsrc, e4, voff), dq = ld4s(dsrc, e4, voff);
+          uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
+          if constexpr (ALIBI) {
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+              const float c0 = (float)(4 * e4 + 2 * h2);
+              nl[h2] = f2_add(nl[h2], f2_fma(f2_pack(c0, c0 + 1.f), nsx2, b0x2));
+            }
           }
-          float d0, d1;
-          f2_unpack(f2_mul(f2_pack(p0, p1), f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1]))), d0, d1);
-          if constexpr (MASK) {  // rows past the sequence may hold anything: select, do not multiply
-            d0 = v0 ? d0 : 0.f;
-            d1 = v1 ? d1 : 0.f;
+          const uint64_t dd[2] = {f2_pack(dq.x, dq.y), f2_pack(dq.z, dq.w)};
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2) {
+            const int c = 4 * e4 + 2 * h2;
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2, nl[h2]), x0, x1);
+            float p0 = ex2(x0), p1 = ex2(x1);
+            const bool v0 = !MASK || (qbase + c >= 0 && c < qlim), v1 = !MASK || (qbase + c + 1 >= 0 && c + 1 < qlim);
+            if constexpr (MASK) {
+              p0 = v0 ? p0 : 0.f;
+              p1 = v1 ? p1 : 0.f;
+            }
+            const uint64_t pp = f2_pack(p0, p1);
+            float d0, d1;
+            f2_unpack(f2_mul(pp, f2_sub(f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1])), dd[h2])), d0, d1);
+            if constexpr (MASK) {  // rows past the sequence may hold anything: select, do not multiply
+              d0 = v0 ? d0 : 0.f;
+              d1 = v1 ? d1 : 0.f;
+            }
+            pk[c >> 1] = bf16x2_bits(p0, p1);
+            dk[c >> 1] = bf16x2_bits(d0, d1);
           }
-          pk[c >> 1] = bf16x2_bits(p0, p1);
-          dk[c >> 1] = bf16x2_bits(d0, d1);
         }
       };
       if (__shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 32) pass(std::false_type{});
@@ -1181,15 +1082,12 @@ __global__ void __launch_bounds__(448, 1)
     }
   } else {
     // ------------------------------------------------ dQ (warps 10..13)
-    // dQ^T from TMEM (one head dimension per thread, the step's 64 queries
-    // along the columns), added into the float32 dQ buffer by global
-    // reductions straight from registers: consecutive lanes hold consecutive
-    // head dimensions, so each reduction of a warp covers 128 contiguous
-    // bytes.  Queries past the sequence are skipped.
+    // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
+    // into dq_acc by one bulk tensor reduce per step.
     const int quad = warp & 3;
     const int dd = quad * 32 + lane;  // head dimension of this thread
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const size_t ldd = (size_t)H * DH;
+    const bool leader = (warp == 10 && lane == 0);
     for (int i = 0; i < n_it; ++i) {
       const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
       if (!warp_wait(&mm_done[i & 1], (i >> 1) & 1, abort_flag, status)) break;
@@ -1200,22 +1098,20 @@ __global__ void __launch_bounds__(448, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(dq_free);
-      const int nv = min(64, len - qt * 64);  // queries of the step inside the sequence (warp-uniform)
-      float* dst = dq_acc + (size_t)(row0 + qt * 64) * ldd + (size_t)h * DH + dd;
-      if (nv == 64) {
+      if (leader && i > 0) bulk_wait_read();  // the previous reduce has read the tile
+      named_barrier(1, 128);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)e * ldd, t0[e]);
+      for (int e = 0; e < 32; ++e) dqs[e * DH + dd] = t0[e];
 #pragma unroll
-        for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(32 + e) * ldd, t1[e]);
-      } else {
-#pragma unroll
-        for (int e = 0; e < 32; ++e)
-          if (e < nv) atomicAdd(dst + (size_t)e * ldd, t0[e]);
-#pragma unroll
-        for (int e = 0; e < 32; ++e)
-          if (32 + e < nv) atomicAdd(dst + (size_t)(32 + e) * ldd, t1[e]);
+      for (int e = 0; e < 32; ++e) dqs[(32 + e) * DH + dd] = t1[e];
+      fence_proxy_async();
+      named_barrier(1, 128);
+      if (leader) {
+        tma_reduce_add_2d(&tmdq, h * DH, row0 + qt * 64, dqs);
+        bulk_commit();
       }
     }
+    if (leader) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -1231,19 +1127,21 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
                    cudaStream_t st) {
-  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + XT (one
-  // slab) + alignment + barriers = 214,272 bytes
-  constexpr size_t smem = 7 * SLAB + 12 * HSLAB + 1024 + 256;
+  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
+  // vectors + dQ staging + alignment + barriers = 232,288 bytes (of 232,448)
+  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 136 * 4 + 64 * 128 * 4 + 1024 + 256;
   // once per process (initialisation of a function-local static is thread-safe)
   static const cudaError_t attr =
       cudaFuncSetAttribute(attn_bwd_tc_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
-  CUtensorMap tkv, tq, to;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows
+  CUtensorMap tkv, tq, to, tdq;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows; dQ reduce boxes
+  if (!make_map_f32(&tdq, dq_acc, (uint64_t)H * 128, (uint64_t)max_seqs * S, (uint64_t)H * 128, 128, 64))
+    return cudaErrorInvalidValue;
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
-  dim3 grid(Hkv, S / 128, max_seqs);
-  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
+  dim3 grid(Hkv, max_seqs, S / 128);
+  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
                                                      H, Hkv, rcos, rsin, alibi, seg, tok, status);
   return cudaGetLastError();
 }
@@ -1269,12 +1167,12 @@ cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int l
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
                                int Hkv, int Dh, int max_seqs, const float* alibi, const int* seg, int* status,
                                cudaStream_t st) {
-  if (Dh == 64) {
-    if (alibi) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
-    return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  if (alibi) {
+    if (Dh == 64) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+    return fwd_tc<128, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
   }
-  if (alibi) return fwd_pp<true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
-  return fwd_pp<false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  if (Dh == 64) return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  return fwd_pp(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, seg, status, st);
 }
 
 }  // namespace ldk

@@ -40,15 +40,16 @@ namespace ldk {
 namespace tc {
 // ---------------------------------------------------------------- host side
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
             cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+  }();
   return fn;
 }
 
@@ -66,6 +67,19 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, 
   return r == CUDA_SUCCESS;
 }
 
+bool make_map_f32(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld, uint32_t box_inner,
+                  uint32_t box_outer) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * 4};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
 }  // namespace tc
 
 namespace {
@@ -372,10 +386,8 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else if (warp == 1) {
-    if (rank == 0) {
-      // ------------------------------------------------ MMA issuer (whole warp, converged;
-      // one elected lane issues)
-      __syncwarp();
+    if (lane == 0 && rank == 0) {
+      // ------------------------------------------------ MMA issuer
       constexpr uint32_t IDESC = idesc_bf16(BMT, BN, A_MN, B_MN);
       int stage = 0;
       uint32_t phase = 0;
@@ -383,14 +395,14 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t acc_phase = 0;
       bool ok = true;
       for (int tile = tile0; tile < num_tiles && ok; tile += tstep) {
-        if (!warp_wait<PAIR>(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
+        if (!mbar_wait<PAIR>(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         for (int ks = 0; ks < num_ks; ++ks) {
-          if (!warp_wait(&full[stage], phase, abort_flag, a.status)) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
             ok = false;
             break;
           }
@@ -410,15 +422,15 @@ __global__ void __launch_bounds__(192, 1)
               const uint64_t bd = B_MN ? sdesc(sb + k * 2048, 8192, 1024) : sdesc(sb + k * 32, 16, 1024);
               const uint32_t accum = (ks | j | k) != 0 ? 1u : 0u;
               if constexpr (PAIR)
-                mma_bf16_pair_w(d_tmem, ad, bd, IDESC, accum);
+                mma_bf16_pair(d_tmem, ad, bd, IDESC, accum);
               else
-                mma_bf16_w(d_tmem, ad, bd, IDESC, accum);
+                mma_bf16(d_tmem, ad, bd, IDESC, accum);
             }
           }
           if constexpr (PAIR)
-            mma_commit_pair_both_w(&empty[stage]);
+            mma_commit_pair_both(&empty[stage]);
           else
-            mma_commit_w(&empty[stage]);
+            mma_commit(&empty[stage]);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -426,20 +438,19 @@ __global__ void __launch_bounds__(192, 1)
         }
         if (!ok) break;
         if constexpr (PAIR)
-          mma_commit_pair_both_w(&tfull[acc]);
+          mma_commit_pair_both(&tfull[acc]);
         else
-          mma_commit_w(&tfull[acc]);
+          mma_commit(&tfull[acc]);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
       }
       if (!ok) {
         // make sure every MMA issued so far has finished before TMEM is freed
         if constexpr (PAIR)
-          mma_commit_pair_local_w(drain);
+          mma_commit_pair_local(drain);
         else
-          mma_commit_w(drain);
-        if (lane == 0) mbar_drain(drain, 0);
-        __syncwarp();
+          mma_commit(drain);
+        mbar_drain(drain, 0);
       }
     }
   } else {

@@ -111,3 +111,42 @@ def test_llama8b_full_per_token():
     mask, _ = _run("llama8b", 0, R=32, granularity="per_token", seqs=[0, 3])
     kept = mask[:, [0, 3], :32]
     assert kept[0].all() and not kept.all()  # layer 0 keeps everything (ILD), later layers drop tokens
+
+
+def _full_rows(name, p1, gamma_noise=0.1):
+    """Two layers of a workload's widths at its full sequence length, B = 2,
+    compared on the full tensors (every row of out and dX, every weight
+    gradient): layer 0 keeps both sequences, layer 1 drops exactly one (the
+    first seed of an explicit [0, p1] schedule that does so)."""
+    cfg = dict(synth.CONFIGS[name], L=2, B=2)
+    sched = None
+    for seed in range(1, 100):
+        s = dict(dist="explicit", p_max=0.0, p_explicit=[0.0, p1], time="const", seed=seed)
+        if int(oracle_masks(cfg, s, 0)[0][1].sum()) == 1:
+            sched = s
+            break
+    assert sched is not None
+    dev = synth.stack_weights(cfg, seed=0, device="cuda", gamma_noise=gamma_noise)
+    x = synth.activations(cfg, seed=0, device="cuda")
+    dy = synth.upstream_grad(cfg, device="cuda")
+    out, dX, grads, (gmask, _, _) = gpu_run(cfg, sched, 0, dev, x, dy)
+    host = [{n: v.cpu() for n, v in W.items()} for W in dev]
+    rout, rdX, rgrads, mask = oracle_run(cfg, sched, 0, host, x.cpu(), dy.cpu())
+    assert (gmask == mask).all() and mask[0].all() and int(mask[1].sum()) == 1
+    check_close(f"{name} out", to_np(out), rout)
+    check_close(f"{name} dX", to_np(dX), rdX)
+    for l in range(cfg["L"]):
+        for n in grads[l]:
+            check_close(f"{name} layer{l}.{n}", to_np(grads[l][n]), rgrads[l][n])
+
+
+def test_llama8b_attention_shape_full_rows():
+    # S = 4096 with 32 query / 8 key-value heads of 128: query tiles see up to
+    # 32 key tiles, the lazy rescale runs over long rows, every row compared
+    _full_rows("llama8b", 0.5)
+
+
+def test_paper_arch_full_rows():
+    # the paper's architecture at S = 2048: ALiBi through the two-tile forward
+    # and the backward over 16 key tiles, squared-ReLU FFN, every row compared
+    _full_rows("paper-3.9b", 0.5)
