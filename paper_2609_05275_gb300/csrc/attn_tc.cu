@@ -747,76 +747,89 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 
 // ---------------------------------------------------------------------------
 // Backward, head size 128.  One CTA per (128-key tile, kv head, kept
-// sequence), looping over the query heads of the group and the 64-query
-// tiles at or after the key tile.  448 threads:
-//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
-//   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
-//               (M = 128 keys, N = 64 queries); then for step i-1
-//               dV += P^T dO (P^T read from TMEM), dK += dS^T Q (M = 128
-//               keys, N = 128) and dQ^T = K^T dS^T (M = 128 head dims,
-//               N = 64 queries)
-//   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e)
-//               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
-//               swizzled shared-memory tile; at the end dK (times c) and dV
-//               from TMEM to dqkv
-//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
-// P^T and dS^T are double-buffered (step i uses buffer i & 1), so the
-// softmax warps write step i while the MMAs of step i-1 still read theirs.
-// TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447,
-// P^T 448-479 / 480-511.
-constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
+// sequence); it loops over the query heads of the group and, for each, the
+// 128-query tiles at or after the key tile (one step per query tile).  Every
+// MMA is M = 128, N = 128 (half-rate N = 64 shapes read their operands from
+// shared memory faster than the tensor pipe consumes them).  448 threads:
+//   warp 0      TMA: K, V once; Q_i (two stages) and dO_i (one stage); all
+//               lanes write the bf16 terms of -lse_i sqrt(Dh) and -D_i that
+//               two extra K = 16 MMAs fold into S^T_i and dP^T_i
+//   warp 1      TMEM allocation and the MMAs, issued in the order
+//                 dP^T_i, dV += P^T_i dO_i, S^T_{i+1}, dQ^T_i, dK += dS^T_i Q_i
+//               (S^T_0 first): S^T_{i+1} goes ahead of dQ^T_i and dK_i, so
+//               the exponentials of step i+1 overlap those two products
+//   warps 2..9  softmax, one key and 64 queries per thread (two warps per
+//               TMEM lane quadrant).  Phase A: P^T = exp2(S^T c) written as
+//               bf16 over the thread's own S^T columns (the A operand of dV).
+//               Phase B: dS^T = P^T (dP^T - D) as bf16 into shared memory
+//               (A of dK, B of dQ^T).  At the end dK (times c, with the
+//               inverse rotation) and dV from TMEM to dqkv
+//   warps 10..13  dQ^T_i from TMEM (one head dimension per thread), added
+//               into the float32 dQ buffer by global reductions from
+//               registers (each warp instruction covers 128 contiguous bytes)
+// TMEM columns: S^T / P^T 0-127, dP^T / dQ^T 128-255, dV 256-383, dK 384-511.
+// The exponent of P is c S - lse log2(e) = c (S - lse sqrt(Dh)) with
+// c = log2(e) / sqrt(Dh), so S^T arrives as S^T - lse sqrt(Dh) and dP^T as
+// dP^T - D, and the softmax warps read no per-query vectors.
 
-// Values 4 e4 .. 4 e4 + 3 of p (shared memory); p is 16-byte aligned when
-// off == 0 (warp-uniform), else read one by one.
-__device__ __forceinline__ float4 ld4s(const float* p, int e4, int off) {
-  if (off == 0) return reinterpret_cast<const float4*>(p)[e4];
-  return make_float4(p[4 * e4], p[4 * e4 + 1], p[4 * e4 + 2], p[4 * e4 + 3]);
+// x as three bf16 terms, t0 + t1 + t2 = x to about 2^-24 |x| (each residual
+// is exact in float32).
+__device__ __forceinline__ void split3_bf16(float x, uint32_t& t0, uint32_t& t1, uint32_t& t2) {
+  const bf16 a = __float2bfloat16_rn(x);
+  const float r1 = x - __bfloat162float(a);
+  const bf16 b = __float2bfloat16_rn(r1);
+  const float r2 = r1 - __bfloat162float(b);
+  const bf16 c = __float2bfloat16_rn(r2);
+  t0 = __bfloat16_as_ushort(a);
+  t1 = __bfloat16_as_ushort(b);
+  t2 = __bfloat16_as_ushort(c);
 }
 
 template <bool ALIBI>
 __global__ void __launch_bounds__(448, 1)
-    attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
-                       const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
+    attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmo,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
                        float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
                        const float* __restrict__ alibi, const int* __restrict__ seg, const int* __restrict__ tok,
                        int* status) {
   constexpr int DH = 128;
-  constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
-  constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
-  constexpr int NST = 3;               // stages of the Q / dO / lse / D ring
+  constexpr uint32_t TILE = 2 * SLAB;  // 128 rows x 128 bf16 (two 64-column slabs)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Ks = smem;
-  uint8_t* Vs = Ks + KT;
-  uint8_t* Qs = Vs + KT;         // [NST][QT]
-  uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
-  uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
-  float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
-  // [NST][lse 68 | D 68]: the 64 values of a step start at float `voff` of
-  // each half (a sequence's rows start anywhere with per-token kept lists,
-  // and a bulk copy needs a 16-byte aligned source, so 68 are copied from
-  // the aligned-down address)
-  float* vecs = dqs + 64 * DH;
-  constexpr int VS = 136;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * VS);
+  uint8_t* Vs = Ks + TILE;
+  uint8_t* Qs = Vs + TILE;       // [2] stages
+  uint8_t* dOs = Qs + 2 * TILE;  // one stage
+  uint8_t* DSs = dOs + TILE;     // dS^T: 128 keys x 128 queries (two 64-query slabs)
+  // XT: 128 rows x 128 bytes (128-byte swizzle) of K = 16 chunk pairs for
+  // the fold MMAs: pair 0 = (1, 1, 1, 0, ...) and pair 1 = (0, 0, 0, 1, 1,
+  // 1, 0, ...) in every row (the A operands), pair 2 + s = the terms of
+  // stage s in row q = query q of the step: (l0, l1, l2, d0, d1, d2, 0, ...)
+  // with l0 + l1 + l2 = -lse sqrt(Dh) and d0 + d1 + d2 = -D.
+  uint8_t* XT = DSs + TILE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(XT + SLAB);
   uint64_t* kv_full = bars;
-  uint64_t* ld_full = bars + 1;          // [NST]
-  uint64_t* ld_empty = ld_full + NST;    // [NST]
-  uint64_t* sdp_full = ld_empty + NST;
-  uint64_t* sdp_free = sdp_full + 1;
-  uint64_t* p_ready = sdp_full + 2;  // [2] per P^T / dS^T buffer
-  uint64_t* mm_done = sdp_full + 4;  // [2] per P^T / dS^T buffer
-  uint64_t* dq_free = sdp_full + 6;
-  uint64_t* acc_done = sdp_full + 7;
-  uint64_t* drain = sdp_full + 8;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sdp_full + 9);
+  uint64_t* q_full = bars + 1;   // [2]
+  uint64_t* q_empty = bars + 3;  // [2]
+  uint64_t* o_full = bars + 5;
+  uint64_t* o_empty = bars + 6;
+  uint64_t* s_full = bars + 7;
+  uint64_t* dp_full = bars + 8;
+  uint64_t* p_ready = bars + 9;
+  uint64_t* ds_ready = bars + 10;
+  uint64_t* dq_full = bars + 11;
+  uint64_t* dq_free = bars + 12;
+  uint64_t* acc_done = bars + 13;
+  uint64_t* drain = bars + 14;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 15);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  // rows row0 .. row0+len-1 as in the forward; queries past len (the last
-  // query tile) get P = dS = 0, keys past len are never stored
-  const int seq = blockIdx.y;
+  // rows row0 .. row0+len-1 (a kept sequence, or with `seg` the kept tokens
+  // of sequence blockIdx.z); queries past len get P = dS = 0, keys past len
+  // are never stored.  Grid (kv head, key tile, sequence): one sequence's
+  // blocks are dispatched together, heaviest key tiles (kt = 0) first.
+  const int seq = blockIdx.z;
   int row0, len;
   if (seg) {
     row0 = seg[seq];
@@ -826,118 +839,173 @@ __global__ void __launch_bounds__(448, 1)
     row0 = seq * S;
     len = S;
   }
-  const int kt = blockIdx.z, g = blockIdx.x, grp = H / Hkv;  // heaviest key tiles (kt = 0) dispatched first
+  const int kt = blockIdx.y, g = blockIdx.x, grp = H / Hkv;
   if (kt * 128 >= len) return;
-  const int nq = (len + 63) / 64, q0 = 2 * kt;  // query tiles q0 .. nq-1 overlap or follow the keys
-  const int n_it = grp * (nq - q0);
+  const int nq = (len + 127) / 128;  // query tiles kt .. nq-1 overlap or follow the keys
+  const int nqs = nq - kt;
+  const int n_it = grp * nqs;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
-    for (int b = 0; b < NST; ++b) {
-      mbar_init(&ld_full[b], 1);
-      mbar_init(&ld_empty[b], 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&q_full[s], 1);
+      mbar_init(&q_empty[s], 1);
     }
-    mbar_init(sdp_full, 1);
-    mbar_init(sdp_free, 8);
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&p_ready[b], 8);
-      mbar_init(&mm_done[b], 1);
-    }
+    mbar_init(o_full, 1);
+    mbar_init(o_empty, 1);
+    mbar_init(s_full, 1);
+    mbar_init(dp_full, 1);
+    mbar_init(p_ready, 8);
+    mbar_init(ds_ready, 8);
+    mbar_init(dq_full, 1);
     mbar_init(dq_free, 4);
     mbar_init(acc_done, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if (threadIdx.x < 128) {
+    // row r of XT: the two ones patterns, zero terms
+    const int r = threadIdx.x;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (u == 0) v = make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
+      if (u == 2) v = make_uint4(0u, 0x3F800000u, 0x3F803F80u, 0u);
+      *reinterpret_cast<uint4*>(XT + swz(r, u)) = v;
+    }
+    fence_proxy_async();
+  }
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t t_s = tmem, t_dp = tmem + 64, t_dv = tmem + 128, t_dk = tmem + 256, t_dq = tmem + 384;
-  const uint32_t t_p = tmem + 448;  // [2] x 32 columns: P^T as bf16 pairs
+  const uint32_t t_s = tmem, t_dp = tmem + 128, t_dv = tmem + 256, t_dk = tmem + 384;
 
   if (warp == 0) {
+    // ------------------------------------------------ producer (warp 0)
+    const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
     if (lane == 0) {
-      // ------------------------------------------------ TMA producer
-      const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
-      mbar_arrive_expect_tx(kv_full, 2 * KT);
+      mbar_arrive_expect_tx(kv_full, 2 * TILE);
       for (int c = 0; c < 2; ++c) {
         tma_load_2d(Ks + c * SLAB, &tmkv, kcol + 64 * c, row0 + kt * 128, kv_full);
         tma_load_2d(Vs + c * SLAB, &tmkv, vcol + 64 * c, row0 + kt * 128, kv_full);
       }
-      int issued = 0;
-      for (int i = 0; i < n_it; ++i) {
-        const int b = i % NST;
-        const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
-        if (!mbar_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
-        mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 2 * 272);
-        for (int c = 0; c < 2; ++c) {
-          tma_load_2d(Qs + b * QT + c * HSLAB, &tmq, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
-          tma_load_2d(dOs + b * QT + c * HSLAB, &tmo, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
-        }
-        const size_t vo = ((size_t)h * lse_ld + row0 + qt * 64) & ~(size_t)3;  // lse_ld % 4 == 0
-        bulk_load(vecs + b * VS, lse + vo, 272, &ld_full[b]);
-        bulk_load(vecs + b * VS + 68, Dvec + vo, 272, &ld_full[b]);
-        ++issued;
-      }
-      if (*abort_flag) {
-        mbar_drain(kv_full, 0);
-        for (int i = issued > NST ? issued - NST : 0; i < issued; ++i) mbar_drain(&ld_full[i % NST], (i / NST) & 1);
-      }
     }
+    const float sq_dh = sqrtf((float)DH);
+    int nql = 0, nol = 0;
+    for (int i = 0; i < n_it; ++i) {
+      const int s = i & 1;
+      const int h = g * grp + i / nqs, qt = kt + i % nqs;
+      // Q_i and the terms of step i into stage s once step i-2 has released it
+      if (!warp_wait(&q_empty[s], ((i >> 1) & 1) ^ 1u, abort_flag, status)) break;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int q = u * 32 + lane;
+        float xl = 0.f, xd = 0.f;
+        if (qt * 128 + q < len) {
+          const size_t at = (size_t)h * lse_ld + row0 + qt * 128 + q;
+          xl = -lse[at] * sq_dh;
+          xd = -Dvec[at];
+        }
+        uint32_t l0, l1, l2, d0, d1, d2;
+        split3_bf16(xl, l0, l1, l2);
+        split3_bf16(xd, d0, d1, d2);
+        *reinterpret_cast<uint4*>(XT + swz(q, 4 + 2 * s)) =
+            make_uint4(l0 | (l1 << 16), l2 | (d0 << 16), d1 | (d2 << 16), 0u);
+      }
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&q_full[s], TILE);
+        for (int c = 0; c < 2; ++c)
+          tma_load_2d(Qs + s * TILE + c * SLAB, &tmkv, h * DH + 64 * c, row0 + qt * 128, &q_full[s]);
+      }
+      ++nql;
+      // dO_i once dV_{i-1} has read dO_{i-1}
+      if (!warp_wait(o_empty, (i & 1) ^ 1u, abort_flag, status)) break;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(o_full, TILE);
+        for (int c = 0; c < 2; ++c)
+          tma_load_2d(dOs + c * SLAB, &tmo, h * DH + 64 * c, row0 + qt * 128, o_full);
+      }
+      ++nol;
+    }
+    if (lane == 0 && *abort_flag) {
+      // let every copy in flight land before the block exits
+      mbar_drain(kv_full, 0);
+      for (int i = nql > 2 ? nql - 2 : 0; i < nql; ++i) mbar_drain(&q_full[i & 1], (i >> 1) & 1);
+      if (nol > 0) mbar_drain(o_full, (nol - 1) & 1);
+    }
+    __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------ MMA issuer
-      constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
+      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);   // S^T, dP^T and the folds
       constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
-      constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
+      constexpr uint32_t ID_Q = idesc_bf16(128, 128, true, true);     // dQ^T (A = K, B = dS^T, MN-major)
       // shared-memory descriptors built once; an MMA's operand is its base
       // plus (byte offset >> 4) in the address field (every tile lies below
       // 256 KB, so the 14-bit field never carries)
       const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
       const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
-      const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
-      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
-      bool ok = mbar_wait(kv_full, 0, abort_flag, status);
-      for (int i = 0; ok && i <= n_it; ++i) {
-        if (i < n_it) {
-          const int b = i % NST;
-          if (!mbar_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t st = (uint64_t)((b * QT) >> 4);
+      const uint64_t DQMN = sdesc(smem_u32(Qs), SLAB, 1024), DOMN = sdesc(smem_u32(dOs), SLAB, 1024);
+      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024);
+      const uint64_t DS = sdesc(smem_u32(DSs), 16, 1024), DSMN = sdesc(smem_u32(DSs), SLAB, 1024);
+      const uint64_t DX = sdesc(smem_u32(XT), 16, 1024);
+      // offset of the K = 16 chunk kk of a K-major 128 x 128 tile (two slabs)
+      auto kmaj = [](int kk) { return (uint64_t)(((kk >> 2) * SLAB + (kk & 3) * 32) >> 4); };
+      // S^T_i = K Q_i^T - lse sqrt(Dh) (ones pattern 0 times the terms)
+      auto issue_s = [&](int i) -> bool {
+        const int s = i & 1;
+        if (!mbar_wait(&q_full[s], (i >> 1) & 1, abort_flag, status)) return false;
+        tc_fence_after();
+        const uint64_t st = (uint64_t)((s * TILE) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk) {
-            const uint32_t koff = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-            const uint32_t qoff = ((kk >> 2) * HSLAB + (kk & 3) * 32) >> 4;
-            mma_bf16(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
-            mma_bf16(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
-          }
-          mma_commit(sdp_full);
-        }
-        if (i >= 1) {
-          const int ip = i - 1, b = ip % NST, pb = ip & 1;
-          if (!mbar_wait(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t st = (uint64_t)((b * QT) >> 4), ds = (uint64_t)((pb * SLAB) >> 4);
-          const uint32_t first = ip > 0 ? 1u : 0u;
+        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_s, DK + kmaj(kk), DQ + st + kmaj(kk), ID_S, kk > 0);
+        mma_bf16(t_s, DX, DX + (uint64_t)(((2 + s) * 32) >> 4), ID_S, 1u);
+        mma_commit(s_full);
+        return true;
+      };
+      bool ok = mbar_wait(kv_full, 0, abort_flag, status) && issue_s(0);
+      for (int i = 0; ok && i < n_it; ++i) {
+        const int s = i & 1;
+        // dP^T_i = V dO_i^T - D (ones pattern 1 times the terms), over the
+        // dQ^T_{i-1} columns once the dQ warps have read them
+        if (!mbar_wait(o_full, i & 1, abort_flag, status)) { ok = false; break; }
+        if (i > 0 && !mbar_wait(dq_free, (i - 1) & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
-            const uint32_t aoff = (kk * 32) >> 4;                // dS^T, K-major
-            const uint32_t boff = (kk * 2048) >> 4;              // dO / Q as MN-major
-            mma_bf16_ta(t_dv, t_p + pb * 32 + kk * 8, DOMN + st + boff, ID_KV, kk > 0 ? 1u : first);
-            mma_bf16(t_dk, DS + ds + aoff, DQMN + st + boff, ID_KV, kk > 0 ? 1u : first);
-          }
+        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_dp, DV + kmaj(kk), DO + kmaj(kk), ID_S, kk > 0);
+        mma_bf16(t_dp, DX + (uint64_t)(32 >> 4), DX + (uint64_t)(((2 + s) * 32) >> 4), ID_S, 1u);
+        mma_commit(dp_full);
+        // dV += P^T_i dO_i: A = P^T from TMEM (queries 64h..64h+63 as bf16
+        // pairs in columns 64h..64h+31), B = dO MN-major
+        if (!mbar_wait(p_ready, i & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
-            mma_bf16(t_dq, DKMN + ((kk * 2048) >> 4), DS + ds + ((kk * 2048) >> 4), ID_Q, kk > 0);
-          }
-          mma_commit(&mm_done[pb]);
-          mma_commit(&ld_empty[b]);
-        }
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_ta(t_dv, t_s + 64 * (kk >> 2) + 8 * (kk & 3), DOMN + (uint64_t)((kk * 2048) >> 4), ID_KV,
+                      (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(o_empty);
+        // S^T_{i+1} ahead of the products that wait for dS^T_i
+        if (i + 1 < n_it && !issue_s(i + 1)) { ok = false; break; }
+        if (!mbar_wait(ds_ready, i & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+        // dQ^T_i = K^T dS^T_i (contraction over the 128 keys) into the dP^T columns
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16(t_dp, DKMN + (uint64_t)((kk * 2048) >> 4), DSMN + (uint64_t)((kk * 2048) >> 4), ID_Q, kk > 0);
+        mma_commit(dq_full);
+        // dK += dS^T_i Q_i (contraction over the 128 queries)
+        const uint64_t st = (uint64_t)((s * TILE) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16(t_dk, DS + kmaj(kk), DQMN + st + (uint64_t)((kk * 2048) >> 4), ID_KV,
+                   (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&q_empty[s]);
       }
       if (ok) {
         mma_commit(acc_done);
@@ -948,98 +1016,95 @@ __global__ void __launch_bounds__(448, 1)
     }
   } else if (warp < 10) {
     // ------------------------------------------------ P / dS (warps 2..9)
-    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..31 of the
-    // step, warps 6..9 queries 32..63, one key per thread
+    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..63 of the
+    // step, warps 6..9 queries 64..127, one key per thread
     const int quad = warp & 3;
     const int half = (warp - 2) >> 2;
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const int voff = row0 & 3;  // first value of a step in its lse / D stage (see vecs)
+    const uint32_t t_sh = t_s + half * 64 + lane_off, t_dph = t_dp + half * 64 + lane_off;
     const float sl2 = kLog2e * rsqrtf((float)DH);
+    uint8_t* dsh = DSs + half * SLAB;  // this half's 64 queries
     bool ok = true;
     for (int i = 0; i < n_it; ++i) {
-      const int b = i % NST;
-      const int qt = q0 + i % (nq - q0);
+      const int qt = kt + i % nqs;
       // ALiBi: logit bias slope2 (key - query) of this step's query head
-      const float slope2 = ALIBI ? alibi[g * grp + i / (nq - q0)] * kLog2e : 0.f;
-      if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
-      if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
+      const float slope2 = ALIBI ? alibi[g * grp + i / nqs] * kLog2e : 0.f;
+      const int qbase = qt * 128 + half * 64 - key;  // query c is visible iff qbase + c >= 0
+      const int qlim = len - (qt * 128 + half * 64);  // and exists iff c < qlim (warp-uniform)
+      // mask only where some of the warp's 32 keys do not see all 64 queries,
+      // or the queries run past the sequence (warp-uniform)
+      const bool full = __shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 64;
+      // ---- phase A: P^T from S^T (lse folded in)
+      if (!warp_wait(s_full, i & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t sr[32], dr[32];
-      tmem_ld32_nw(t_s + half * 32 + lane_off, sr);
-      tmem_ld32_nw(t_dp + half * 32 + lane_off, dr);
-      tmem_wait_ld();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(sdp_free);
-      const float* lsrc = vecs + b * VS + voff + half * 32;       // lse of the 32 queries
-      const float* dsrc = vecs + b * VS + 68 + voff + half * 32;  // D of the 32 queries
-      const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
-      const int qlim = len - (qt * 64 + half * 32);  // and exists iff c < qlim (warp-uniform)
-      uint32_t pk[16], dk[16];
-      // pairs of queries on the packed fp32 pipe; the mask only on warps
-      // whose 32 keys are not all visible to the 32 queries, or whose queries
-      // run past the sequence (warp-uniform)
-      auto pass = [&](auto masked) {
+      uint32_t pk[32];
+      auto phase_a = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
-        const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
-        // bias of query c: slope2 (key - qt*64 - half*32 - c) = b0 - slope2 c
-        const float b0 = slope2 * (float)(-qbase);
+        const uint64_t sl2x2 = f2_pack(sl2, sl2);
+        const float b0 = slope2 * (float)(-qbase);  // bias of query c: b0 - slope2 c
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
-        for (int e4 = 0; e4 < 8; ++e4) {
-          const float4 lq = ld4s(lsrc, e4, voff), dq = ld4s(dsrc, e4, voff);
-          uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
-          if constexpr (ALIBI) {
+        for (int h2 = 0; h2 < 2; ++h2) {
+          uint32_t sr[32];
+          tmem_ld32_nw(t_sh + h2 * 32, sr);
+          tmem_wait_ld();
 #pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-              const float c0 = (float)(4 * e4 + 2 * h2);
-              nl[h2] = f2_add(nl[h2], f2_fma(f2_pack(c0, c0 + 1.f), nsx2, b0x2));
-            }
-          }
-          const uint64_t dd[2] = {f2_pack(dq.x, dq.y), f2_pack(dq.z, dq.w)};
-#pragma unroll
-          for (int h2 = 0; h2 < 2; ++h2) {
-            const int c = 4 * e4 + 2 * h2;
+          for (int c2 = 0; c2 < 32; c2 += 2) {
+            const int c = h2 * 32 + c2;
+            uint64_t x2 = f2_mul(f2_pack(__uint_as_float(sr[c2]), __uint_as_float(sr[c2 + 1])), sl2x2);
+            if constexpr (ALIBI) x2 = f2_add(x2, f2_fma(f2_pack((float)c, (float)(c + 1)), nsx2, b0x2));
             float x0, x1;
-            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2, nl[h2]), x0, x1);
+            f2_unpack(x2, x0, x1);
             float p0 = ex2(x0), p1 = ex2(x1);
-            const bool v0 = !MASK || (qbase + c >= 0 && c < qlim), v1 = !MASK || (qbase + c + 1 >= 0 && c + 1 < qlim);
             if constexpr (MASK) {
-              p0 = v0 ? p0 : 0.f;
-              p1 = v1 ? p1 : 0.f;
-            }
-            const uint64_t pp = f2_pack(p0, p1);
-            float d0, d1;
-            f2_unpack(f2_mul(pp, f2_sub(f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1])), dd[h2])), d0, d1);
-            if constexpr (MASK) {  // rows past the sequence may hold anything: select, do not multiply
-              d0 = v0 ? d0 : 0.f;
-              d1 = v1 ? d1 : 0.f;
+              p0 = (qbase + c >= 0 && c < qlim) ? p0 : 0.f;
+              p1 = (qbase + c + 1 >= 0 && c + 1 < qlim) ? p1 : 0.f;
             }
             pk[c >> 1] = bf16x2_bits(p0, p1);
-            dk[c >> 1] = bf16x2_bits(d0, d1);
           }
         }
       };
-      if (__shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 32) pass(std::false_type{});
-      else pass(std::true_type{});
-      // the MMAs of step i-2 must be done with buffer i & 1 before it is rewritten
-      const int pb = i & 1;
-      if (i >= 2 && !warp_wait(&mm_done[pb], ((i >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
-      tc_fence_after();
-      tmem_st16(t_p + pb * 32 + half * 16 + lane_off, pk);
-      uint8_t* ds = DSs + pb * SLAB;
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int chunk = half * 4 + c;
-        *reinterpret_cast<uint4*>(ds + swz(r, chunk)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
-      }
-      fence_proxy_async();
+      if (full) phase_a(std::false_type{});
+      else phase_a(std::true_type{});
+      // P^T (queries 64 half .. 64 half + 63) over this warp's own S^T columns
+      tmem_st32u(t_sh, pk);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_ready[pb]);
+      if (lane == 0) mbar_arrive(p_ready);
+      // ---- phase B: dS^T = P^T (dP^T - D) (D folded in)
+      if (!warp_wait(dp_full, i & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        uint32_t dr[32];
+        tmem_ld32_nw(t_dph + h2 * 32, dr);
+        tmem_wait_ld();
+        uint32_t dk[16];
+#pragma unroll
+        for (int c2 = 0; c2 < 32; c2 += 2) {
+          const uint32_t pw = pk[(h2 * 32 + c2) >> 1];
+          const uint64_t pp = f2_pack(__uint_as_float(pw << 16), __uint_as_float(pw & 0xFFFF0000u));
+          float d0, d1;
+          f2_unpack(f2_mul(pp, f2_pack(__uint_as_float(dr[c2]), __uint_as_float(dr[c2 + 1]))), d0, d1);
+          if (!full) {  // rows past the sequence may hold anything: select, do not multiply
+            const int c = h2 * 32 + c2;
+            d0 = (qbase + c >= 0 && c < qlim) ? d0 : 0.f;
+            d1 = (qbase + c + 1 >= 0 && c + 1 < qlim) ? d1 : 0.f;
+          }
+          dk[c2 >> 1] = bf16x2_bits(d0, d1);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          *reinterpret_cast<uint4*>(dsh + swz(r, h2 * 4 + u)) =
+              make_uint4(dk[4 * u], dk[4 * u + 1], dk[4 * u + 2], dk[4 * u + 3]);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ds_ready);
     }
     if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
       tc_fence_after();
@@ -1047,7 +1112,7 @@ __global__ void __launch_bounds__(448, 1)
       if (half == 0) {
         // dK (times c) with the inverse rotation at the key's position
         const float c = rsqrtf((float)DH);
-        const int kpos = row_pos(tok, S, row0 + key);
+        const int kpos = kvalid ? row_pos(tok, S, row0 + key) : 0;  // rows past the segment are not read
         bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
 #pragma unroll 1
         for (int cc = 0; cc < 2; ++cc) {
@@ -1082,36 +1147,52 @@ __global__ void __launch_bounds__(448, 1)
     }
   } else {
     // ------------------------------------------------ dQ (warps 10..13)
-    // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
-    // into dq_acc by one bulk tensor reduce per step.
+    // dQ^T_i from TMEM (head dimension dd on this thread's lane, the step's
+    // 128 queries along the columns), added into dq_acc by global
+    // reductions: consecutive lanes hold consecutive head dimensions, so a
+    // warp's reduction covers 128 contiguous bytes of one query row.
+    // Queries past the sequence are skipped.
     const int quad = warp & 3;
-    const int dd = quad * 32 + lane;  // head dimension of this thread
+    const int dd = quad * 32 + lane;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const bool leader = (warp == 10 && lane == 0);
+    const size_t ldd = (size_t)H * DH;
     for (int i = 0; i < n_it; ++i) {
-      const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
-      if (!warp_wait(&mm_done[i & 1], (i >> 1) & 1, abort_flag, status)) break;
+      const int h = g * grp + i / nqs, qt = kt + i % nqs;
+      if (!warp_wait(dq_full, i & 1, abort_flag, status)) break;
       tc_fence_after();
-      float t0[32], t1[32];
-      tmem_ld32(t_dq + lane_off, t0);
-      tmem_ld32(t_dq + 32 + lane_off, t1);
+      const int nv = min(128, len - qt * 128);  // queries of the step inside the sequence (warp-uniform)
+      float* dst = dq_acc + (size_t)(row0 + qt * 128) * ldd + (size_t)h * DH + dd;
+      float t[2][32];
+      tmem_ld32(t_dp + lane_off, t[0]);
+      tmem_ld32(t_dp + 32 + lane_off, t[1]);
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        if (nv >= 32 * (c + 1)) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(32 * c + e) * ldd, t[c][e]);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (32 * c + e < nv) atomicAdd(dst + (size_t)(32 * c + e) * ldd, t[c][e]);
+        }
+      }
+      tmem_ld32(t_dp + 64 + lane_off, t[0]);
+      tmem_ld32(t_dp + 96 + lane_off, t[1]);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(dq_free);
-      if (leader && i > 0) bulk_wait_read();  // the previous reduce has read the tile
-      named_barrier(1, 128);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) dqs[e * DH + dd] = t0[e];
+      for (int c = 0; c < 2; ++c) {
+        if (nv >= 32 * (c + 3)) {
 #pragma unroll
-      for (int e = 0; e < 32; ++e) dqs[(32 + e) * DH + dd] = t1[e];
-      fence_proxy_async();
-      named_barrier(1, 128);
-      if (leader) {
-        tma_reduce_add_2d(&tmdq, h * DH, row0 + qt * 64, dqs);
-        bulk_commit();
+          for (int e = 0; e < 32; ++e) atomicAdd(dst + (size_t)(64 + 32 * c + e) * ldd, t[c][e]);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (64 + 32 * c + e < nv) atomicAdd(dst + (size_t)(64 + 32 * c + e) * ldd, t[c][e]);
+        }
       }
     }
-    if (leader) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -1127,22 +1208,19 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
                    float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
                    cudaStream_t st) {
-  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
-  // vectors + dQ staging + alignment + barriers = 232,288 bytes (of 232,448)
-  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 136 * 4 + 64 * 128 * 4 + 1024 + 256;
+  // K, V, 2 stages of Q, dO, dS^T (six 32 KB tiles) + XT (one slab) +
+  // alignment + barriers = 214,272 bytes
+  constexpr size_t smem = 6 * 2 * SLAB + SLAB + 1024 + 256;
   // once per process (initialisation of a function-local static is thread-safe)
   static const cudaError_t attr =
       cudaFuncSetAttribute(attn_bwd_tc_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
-  CUtensorMap tkv, tq, to, tdq;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows; dQ reduce boxes
-  if (!make_map_f32(&tdq, dq_acc, (uint64_t)H * 128, (uint64_t)max_seqs * S, (uint64_t)H * 128, 128, 64))
-    return cudaErrorInvalidValue;
+  CUtensorMap tkv, to;  // tiles of 128 rows x 64 columns: Q, K, V in qkv; dO
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
-  if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
-  if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
-  dim3 grid(Hkv, max_seqs, S / 128);
-  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
-                                                     H, Hkv, rcos, rsin, alibi, seg, tok, status);
+  if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 128)) return cudaErrorInvalidValue;
+  dim3 grid(Hkv, S / 128, max_seqs);
+  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, to, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S, H,
+                                                     Hkv, rcos, rsin, alibi, seg, tok, status);
   return cudaGetLastError();
 }
 }  // namespace
