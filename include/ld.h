@@ -241,6 +241,12 @@ ld_status ld_destroy(void* handle);
 /* Static description of a status code. */
 const char* ld_status_str(ld_status status);
 
+/* The CUDA runtime's message for the error behind the last LD_ERR_CUDA that
+ * a call of this library returned on the calling thread ("no CUDA error
+ * recorded" if none).  The pointer refers to static storage.  Not from the
+ * paper: diagnostics of the library. */
+const char* ld_last_cuda_error(void);
+
 /* Kernel classes of the device-time accounting below. */
 typedef enum {
   LD_KCLASS_GEMM = 0,    /* tcgen05 (or debug SIMT) projections and their gradients */

@@ -59,7 +59,10 @@ class ld_layer_g(ctypes.Structure):
 class LdError(RuntimeError):
     def __init__(self, status, where):
         self.status = status
-        super().__init__(f"{where}: {ld_status_str(status)} (status {status})")
+        msg = f"{where}: {ld_status_str(status)} (status {status})"
+        if status == LD_ERR_CUDA:
+            msg += ": " + lib().ld_last_cuda_error().decode()
+        super().__init__(msg)
 
 
 _lib = None
@@ -88,6 +91,7 @@ def lib():
             "ld_sync": (c_int, [c_void_p]),
             "ld_destroy": (c_int, [c_void_p]),
             "ld_status_str": (c_char_p, [c_int]),
+            "ld_last_cuda_error": (c_char_p, []),
             "ld_set_timing": (c_int, [c_void_p, c_int]),
             "ld_get_timing": (c_int, [c_void_p, c_int, POINTER(c_double), POINTER(c_longlong)]),
             "ld_rmsnorm_backward": (c_int, [c_int, c_int, c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,

@@ -221,9 +221,16 @@ T* at(void* ws, size_t off) {
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15) == 0; }
 
-#define LD_CHECK(...)                              \
-  do {                                             \
-    if ((__VA_ARGS__) != cudaSuccess) return LD_ERR_CUDA; \
+// The CUDA error behind the last LD_ERR_CUDA this thread returned.
+thread_local cudaError_t g_last_cuda = cudaSuccess;
+
+#define LD_CHECK(...)                        \
+  do {                                       \
+    const cudaError_t e_ = (__VA_ARGS__);    \
+    if (e_ != cudaSuccess) {                 \
+      g_last_cuda = e_;                      \
+      return LD_ERR_CUDA;                    \
+    }                                        \
   } while (0)
 
 ld_status check_device() {
@@ -372,8 +379,8 @@ cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, 
 }
 
 // Attention backward: dq, dk, dv into dqkv with the inverse RoPE applied to
-// dq and dk (fused into dq_finish and the tcgen05 kernel's dK epilogue on
-// the bf16 path; a separate rotation otherwise).
+// dq and dk (fused into the epilogues of the tcgen05 kernels, into dq_finish
+// on the mma.sync path, a separate rotation on the debug path).
 template <typename T>
 cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const T* dO, const float* lse, float* Dvec,
                      T* dqkv, const Rows& r, cudaStream_t st) {
@@ -391,14 +398,14 @@ cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const 
     return launch_rope_apply<T>(dqkv, h->nqkv, c.H + c.Hkv, c.Dh, rcos, rsin, r.cnt, c.S, h->max_rows, 1, r.tok(),
                                 st);
   }
-  float* dq_acc = at<float>(ws, h->lay.dqacc);
   const bf16* q16 = reinterpret_cast<const bf16*>(qkv);
   bf16* d16 = reinterpret_cast<bf16*>(dqkv);
-  if (attn_bwd_tc_supported(c.S, c.Dh)) {
-    e = launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16, r.cnt,
-                           c.S, c.H, c.Hkv, c.B, rcos, rsin, alibi_table(h, ws), r.seg, r.tok(),
-                           at<int>(ws, h->lay.status), st);
-  } else {  // whole sequences only (per-token granularity is refused at ld_create on this path)
+  if (attn_bwd_tc_supported(c.S, c.Dh))  // dK, dV and dQ (scaled and rotated) straight into dqkv
+    return launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, d16, r.cnt,
+                              c.S, c.H, c.Hkv, c.B, rcos, rsin, alibi_table(h, ws), r.seg, r.tok(),
+                              at<int>(ws, h->lay.status), st);
+  float* dq_acc = at<float>(ws, h->lay.dqacc);
+  {  // whole sequences only (per-token granularity is refused at ld_create on this path)
     e = launch_attn_bwd_mma(q16, h->nqkv, reinterpret_cast<const bf16*>(o), reinterpret_cast<const bf16*>(dO),
                             c.H * c.Dh, lse, Dvec, dq_acc, d16, r.cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
                             st);
@@ -751,6 +758,10 @@ ld_status backward_impl(Handle* h, const ld_layer_w* W, void* dxv, ld_layer_g* G
 }  // namespace
 
 extern "C" {
+
+const char* ld_last_cuda_error(void) {
+  return g_last_cuda == cudaSuccess ? "no CUDA error recorded" : cudaGetErrorString(g_last_cuda);
+}
 
 const char* ld_status_str(ld_status s) {
   switch (s) {

@@ -108,10 +108,79 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const TS* __restrict__
   }
 }
 
+// As rmsnorm_fwd_kernel for d <= 256 NV, with each warp's row held in
+// registers (NV vectors of 8 per lane), so the row is read from memory once:
+// the two-pass form re-reads it after the sum of squares, and with tens of
+// thousands of rows in flight the second read misses L2 (measured at the
+// Llama-3-8B width: DRAM reads twice the row bytes).  Four warps a block and
+// few blocks per SM still keep ~16 KB a warp in flight.
+template <typename TS, typename T, int NV>
+__global__ void __launch_bounds__(128) rmsnorm_fwd_reg_kernel(const TS* __restrict__ src, int gather,
+                                                              const int* __restrict__ kept_idx,
+                                                              const int* __restrict__ cnt, int S, int d,
+                                                              const T* __restrict__ gamma, float eps,
+                                                              TS* __restrict__ copy, T* __restrict__ out,
+                                                              float* __restrict__ rstd) {
+  const long long M = (long long)(*cnt) * S;
+  const int lane = threadIdx.x & 31;
+  const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
+  for (long long m = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); m < M; m += nwarps) {
+    const long long r = gather ? src_row(kept_idx, S, m) : m;
+    if (r < 0) {  // padding row of a per-token kept list: zeros
+      const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      for (int i = lane * 8; i < d; i += 256) {
+        if (copy) st8(copy + m * d + i, z);
+        st8(out + m * d + i, z);
+      }
+      if (lane == 0) rstd[m] = 0.f;
+      continue;
+    }
+    const TS* xr = src + r * d;
+    float v[NV][8];
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+      if (lane * 8 + 256 * j < d) ld8(xr + lane * 8 + 256 * j, v[j]);
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+      if (lane * 8 + 256 * j < d) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) ss += v[j][e] * v[j][e];
+        if (copy) st8(copy + m * d + lane * 8 + 256 * j, v[j]);
+      }
+    ss = warp_sum(ss);
+    const float rs = 1.0f / sqrtf(ss / (float)d + eps);
+    if (lane == 0) rstd[m] = rs;
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+      if (lane * 8 + 256 * j < d) {
+        float g[8], o[8];
+        ld8(gamma + lane * 8 + 256 * j, g);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) o[e] = (v[j][e] * rs) * g[e];
+        st8(out + m * d + lane * 8 + 256 * j, o);
+      }
+  }
+}
+
 template <typename TS, typename T>
 cudaError_t launch_rmsnorm_fwd(const TS* src, int gather, const int* kept_idx, const int* cnt, int S, int d,
                                int max_rows, const T* gamma, float eps, TS* copy, T* out, float* rstd,
                                cudaStream_t st) {
+  if (d <= 4096) {
+    // 4 rows a block, up to 8 blocks per SM
+    const int grid = grid_for(max_rows, 4, device_sm_count() * 8);
+    if (d <= 1024)
+      rmsnorm_fwd_reg_kernel<TS, T, 4><<<grid, 128, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy, out,
+                                                              rstd);
+    else if (d <= 2048)
+      rmsnorm_fwd_reg_kernel<TS, T, 8><<<grid, 128, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy, out,
+                                                              rstd);
+    else
+      rmsnorm_fwd_reg_kernel<TS, T, 16><<<grid, 128, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy,
+                                                               out, rstd);
+    return cudaGetLastError();
+  }
   const int grid = grid_for(max_rows, 8, device_sm_count() * 16);
   rmsnorm_fwd_kernel<TS, T><<<grid, 256, 0, st>>>(src, gather, kept_idx, cnt, S, d, gamma, eps, copy, out, rstd);
   return cudaGetLastError();
