@@ -752,7 +752,7 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // sequence); it loops over the query heads of the group and, for each, the
 // 128-query tiles at or after the key tile (one step per query tile).  Every
 // MMA is M = 128, N = 128.  320 threads:
-//   warp 0      TMA: K, V once; Q_i and dO_i (two stages each); all lanes
+//   warp 0      TMA: K, V once; Q_i (three stages) and dO_i (one); all lanes
 //               write the bf16 terms of -lse_i sqrt(Dh) and -D_i that two
 //               extra K = 16 MMAs fold into S^T_i and dP^T_i
 //   warp 1      TMEM allocation and the MMAs, issued in the order
@@ -806,20 +806,21 @@ __global__ void __launch_bounds__(320, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Ks = smem;
   uint8_t* Vs = Ks + TILE;
-  uint8_t* Qs = Vs + TILE;       // [2] stages
-  uint8_t* dOs = Qs + 2 * TILE;  // [2] stages
+  uint8_t* Qs = Vs + TILE;       // [3] stages: Q_i is read by S^T_i and, a step later, by dK
+  uint8_t* dOs = Qs + 3 * TILE;  // one stage
   // XT: 128 rows x 128 bytes (128-byte swizzle) of K = 16 chunk pairs for
   // the fold MMAs: pair 0 = (1, 1, 1, 0, ...) and pair 1 = (0, 0, 0, 1, 1,
   // 1, 0, ...) in every row (the A operands), pair 2 + s = the terms of
   // stage s in row q = query q of the step: (l0, l1, l2, d0, d1, d2, 0, ...)
   // with l0 + l1 + l2 = -lse sqrt(Dh) and d0 + d1 + d2 = -D.
-  uint8_t* XT = dOs + 2 * TILE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(XT + SLAB);
+  // (stage 2's terms are pair 0 of a second such slab, XT + SLAB)
+  uint8_t* XT = dOs + TILE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(XT + 2 * SLAB);
   uint64_t* kv_full = bars;
-  uint64_t* q_full = bars + 1;   // [2]
-  uint64_t* q_empty = bars + 3;  // [2]
-  uint64_t* o_full = bars + 5;   // [2]
-  uint64_t* o_empty = bars + 7;  // [2]
+  uint64_t* q_full = bars + 1;   // [3]
+  uint64_t* q_empty = bars + 4;  // [3]
+  uint64_t* o_full = bars + 7;
+  uint64_t* o_empty = bars + 8;
   uint64_t* s_full = bars + 9;
   uint64_t* dp_full = bars + 10;
   uint64_t* p_ready = bars + 11;
@@ -852,12 +853,12 @@ __global__ void __launch_bounds__(320, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < 3; ++s) {
       mbar_init(&q_full[s], 1);
       mbar_init(&q_empty[s], 1);
-      mbar_init(&o_full[s], 1);
-      mbar_init(&o_empty[s], 1);
     }
+    mbar_init(o_full, 1);
+    mbar_init(o_empty, 1);
     mbar_init(s_full, 1);
     mbar_init(dp_full, 1);
     mbar_init(p_ready, 8);
@@ -876,6 +877,7 @@ __global__ void __launch_bounds__(320, 1)
       if (u == 0) v = make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
       if (u == 2) v = make_uint4(0u, 0x3F800000u, 0x3F803F80u, 0u);
       *reinterpret_cast<uint4*>(XT + swz(r, u)) = v;
+      *reinterpret_cast<uint4*>(XT + SLAB + swz(r, u)) = make_uint4(0u, 0u, 0u, 0u);
     }
     fence_proxy_async();
   }
@@ -897,49 +899,62 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
     const float sq_dh = sqrtf((float)DH);
-    int nql = 0, nol = 0;
-    for (int i = 0; i < n_it; ++i) {
-      const int s = i & 1;
+    // -lse sqrt(Dh) and -D of the 128 queries of step i, four a lane, loaded
+    // one step ahead so their latency stays off the Q copy's path
+    float xl[4], xd[4];
+    auto load_terms = [&](int i) {
       const int h = g * grp + i / nqs, qt = kt + i % nqs;
-      // Q_i and the terms of step i into stage s once step i-2 has released it
-      if (!warp_wait(&q_empty[s], ((i >> 1) & 1) ^ 1u, abort_flag, status)) break;
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const int q = u * 32 + lane;
-        float xl = 0.f, xd = 0.f;
+        xl[u] = 0.f;
+        xd[u] = 0.f;
         if (qt * 128 + q < len) {
           const size_t at = (size_t)h * lse_ld + row0 + qt * 128 + q;
-          xl = -lse[at] * sq_dh;
-          xd = -Dvec[at];
+          xl[u] = -lse[at] * sq_dh;
+          xd[u] = -Dvec[at];
         }
+      }
+    };
+    if (n_it > 0) load_terms(0);
+    int nql = 0, nol = 0;
+    for (int i = 0; i < n_it; ++i) {
+      const int s = i % 3;
+      const int h = g * grp + i / nqs, qt = kt + i % nqs;
+      // Q_i and the terms of step i into stage s once step i-3 has released
+      // it; the copy is issued first (the barrier's phase cannot complete
+      // before the arrival below, which follows the terms)
+      if (!warp_wait(&q_empty[s], ((i / 3) & 1) ^ 1u, abort_flag, status)) break;
+      if (lane == 0)
+        for (int c = 0; c < 2; ++c)
+          tma_load_2d(Qs + s * TILE + c * SLAB, &tmkv, h * DH + 64 * c, row0 + qt * 128, &q_full[s]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
         uint32_t l0, l1, l2, d0, d1, d2;
-        split3_bf16(xl, l0, l1, l2);
-        split3_bf16(xd, d0, d1, d2);
-        *reinterpret_cast<uint4*>(XT + swz(q, 4 + 2 * s)) =
+        split3_bf16(xl[u], l0, l1, l2);
+        split3_bf16(xd[u], d0, d1, d2);
+        *reinterpret_cast<uint4*>(s < 2 ? XT + swz(u * 32 + lane, 4 + 2 * s) : XT + SLAB + swz(u * 32 + lane, 0)) =
             make_uint4(l0 | (l1 << 16), l2 | (d0 << 16), d1 | (d2 << 16), 0u);
       }
       fence_proxy_async();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive_expect_tx(&q_full[s], TILE);
-        for (int c = 0; c < 2; ++c)
-          tma_load_2d(Qs + s * TILE + c * SLAB, &tmkv, h * DH + 64 * c, row0 + qt * 128, &q_full[s]);
-      }
+      if (lane == 0) mbar_arrive_expect_tx(&q_full[s], TILE);
+      if (i + 1 < n_it) load_terms(i + 1);
       ++nql;
-      // dO_i into stage s once dV_{i-2} has read dO_{i-2}
-      if (!warp_wait(&o_empty[s], ((i >> 1) & 1) ^ 1u, abort_flag, status)) break;
+      // dO_i once dV_{i-1} has read dO_{i-1}
+      if (!warp_wait(o_empty, (i & 1) ^ 1u, abort_flag, status)) break;
       if (lane == 0) {
-        mbar_arrive_expect_tx(&o_full[s], TILE);
+        mbar_arrive_expect_tx(o_full, TILE);
         for (int c = 0; c < 2; ++c)
-          tma_load_2d(dOs + s * TILE + c * SLAB, &tmo, h * DH + 64 * c, row0 + qt * 128, &o_full[s]);
+          tma_load_2d(dOs + c * SLAB, &tmo, h * DH + 64 * c, row0 + qt * 128, o_full);
       }
       ++nol;
     }
     if (lane == 0 && *abort_flag) {
       // let every copy in flight land before the block exits
       mbar_drain(kv_full, 0);
-      for (int i = nql > 2 ? nql - 2 : 0; i < nql; ++i) mbar_drain(&q_full[i & 1], (i >> 1) & 1);
-      for (int i = nol > 2 ? nol - 2 : 0; i < nol; ++i) mbar_drain(&o_full[i & 1], (i >> 1) & 1);
+      for (int i = nql > 3 ? nql - 3 : 0; i < nql; ++i) mbar_drain(&q_full[i % 3], (i / 3) & 1);
+      if (nol > 0) mbar_drain(o_full, (nol - 1) & 1);
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -953,32 +968,34 @@ __global__ void __launch_bounds__(320, 1)
       const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
       const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
       const uint64_t DQMN = sdesc(smem_u32(Qs), SLAB, 1024), DOMN = sdesc(smem_u32(dOs), SLAB, 1024);
-      const uint64_t DX = sdesc(smem_u32(XT), 16, 1024);
+      const uint64_t DX = sdesc(smem_u32(XT), 16, 1024), DX2 = sdesc(smem_u32(XT + SLAB), 16, 1024);
+      // B operand of the fold MMAs: the terms of Q stage s
+      auto terms = [&](int s) { return s < 2 ? DX + (uint64_t)(((2 + s) * 32) >> 4) : DX2; };
       // offset of the K = 16 chunk kk of a K-major 128 x 128 tile (two slabs)
       auto kmaj = [](int kk) { return (uint64_t)(((kk >> 2) * SLAB + (kk & 3) * 32) >> 4); };
       // S^T_i = K Q_i^T - lse sqrt(Dh) (ones pattern 0 times the terms)
       auto issue_s = [&](int i) -> bool {
-        const int s = i & 1;
-        if (!mbar_wait(&q_full[s], (i >> 1) & 1, abort_flag, status)) return false;
+        const int s = i % 3;
+        if (!mbar_wait(&q_full[s], (i / 3) & 1, abort_flag, status)) return false;
         tc_fence_after();
         const uint64_t st = (uint64_t)((s * TILE) >> 4);
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_s, DK + kmaj(kk), DQ + st + kmaj(kk), ID_S, kk > 0);
-        mma_bf16(t_s, DX, DX + (uint64_t)(((2 + s) * 32) >> 4), ID_S, 1u);
+        mma_bf16(t_s, DX, terms(s), ID_S, 1u);
         mma_commit(s_full);
         return true;
       };
       bool ok = mbar_wait(kv_full, 0, abort_flag, status) && issue_s(0);
       for (int i = 0; ok && i < n_it; ++i) {
-        const int s = i & 1;
+        const int s = i % 3;
         const uint64_t st = (uint64_t)((s * TILE) >> 4);
         // dP^T_i = V dO_i^T - D (ones pattern 1 times the terms), over the
         // dS^T_{i-1} columns (dK_{i-1}, issued before, reads them first)
-        if (!mbar_wait(&o_full[s], (i >> 1) & 1, abort_flag, status)) { ok = false; break; }
+        if (!mbar_wait(o_full, i & 1, abort_flag, status)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_dp, DV + kmaj(kk), DO + st + kmaj(kk), ID_S, kk > 0);
-        mma_bf16(t_dp, DX + (uint64_t)(32 >> 4), DX + (uint64_t)(((2 + s) * 32) >> 4), ID_S, 1u);
+        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_dp, DV + kmaj(kk), DO + kmaj(kk), ID_S, kk > 0);
+        mma_bf16(t_dp, DX + (uint64_t)(32 >> 4), terms(s), ID_S, 1u);
         mma_commit(dp_full);
         // dV += P^T_i dO_i: A = P^T from TMEM (queries 64h..64h+63 as bf16
         // pairs in columns 64h..64h+31), B = dO MN-major
@@ -986,9 +1003,9 @@ __global__ void __launch_bounds__(320, 1)
         tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ta(t_dv, t_s + 64 * (kk >> 2) + 8 * (kk & 3), DOMN + st + (uint64_t)((kk * 2048) >> 4), ID_KV,
+          mma_bf16_ta(t_dv, t_s + 64 * (kk >> 2) + 8 * (kk & 3), DOMN + (uint64_t)((kk * 2048) >> 4), ID_KV,
                       (i > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(&o_empty[s]);
+        mma_commit(o_empty);
         // S^T_{i+1} ahead of the product that waits for dS^T_i
         if (i + 1 < n_it && !issue_s(i + 1)) { ok = false; break; }
         if (!mbar_wait(ds_ready, i & 1, abort_flag, status)) { ok = false; break; }
@@ -1039,15 +1056,16 @@ __global__ void __launch_bounds__(320, 1)
         const uint64_t sl2x2 = f2_pack(sl2, sl2);
         const float b0 = slope2 * (float)(-qbase);  // bias of query c: b0 - slope2 c
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
+        uint32_t sr[2][32];
+        tmem_ld32_nw(t_sh, sr[0]);
+        tmem_ld32_nw(t_sh + 32, sr[1]);
+        tmem_wait_ld();
 #pragma unroll
         for (int h2 = 0; h2 < 2; ++h2) {
-          uint32_t sr[32];
-          tmem_ld32_nw(t_sh + h2 * 32, sr);
-          tmem_wait_ld();
 #pragma unroll
           for (int c2 = 0; c2 < 32; c2 += 2) {
             const int c = h2 * 32 + c2;
-            uint64_t x2 = f2_mul(f2_pack(__uint_as_float(sr[c2]), __uint_as_float(sr[c2 + 1])), sl2x2);
+            uint64_t x2 = f2_mul(f2_pack(__uint_as_float(sr[h2][c2]), __uint_as_float(sr[h2][c2 + 1])), sl2x2);
             if constexpr (ALIBI) x2 = f2_add(x2, f2_fma(f2_pack((float)c, (float)(c + 1)), nsx2, b0x2));
             float x0, x1;
             f2_unpack(x2, x0, x1);
@@ -1071,28 +1089,29 @@ __global__ void __launch_bounds__(320, 1)
       // ---- phase B: dS^T = P^T (dP^T - D) (D folded in)
       if (!warp_wait(dp_full, i & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t dk[32];
+      // dS^T over the packed P^T in place (pk), both halves loaded at once
+      uint32_t dr[2][32];
+      tmem_ld32_nw(t_dph, dr[0]);
+      tmem_ld32_nw(t_dph + 32, dr[1]);
+      tmem_wait_ld();
 #pragma unroll
       for (int h2 = 0; h2 < 2; ++h2) {
-        uint32_t dr[32];
-        tmem_ld32_nw(t_dph + h2 * 32, dr);
-        tmem_wait_ld();
 #pragma unroll
         for (int c2 = 0; c2 < 32; c2 += 2) {
           const uint32_t pw = pk[(h2 * 32 + c2) >> 1];
           const uint64_t pp = f2_pack(__uint_as_float(pw << 16), __uint_as_float(pw & 0xFFFF0000u));
           float d0, d1;
-          f2_unpack(f2_mul(pp, f2_pack(__uint_as_float(dr[c2]), __uint_as_float(dr[c2 + 1]))), d0, d1);
+          f2_unpack(f2_mul(pp, f2_pack(__uint_as_float(dr[h2][c2]), __uint_as_float(dr[h2][c2 + 1]))), d0, d1);
           if (!full) {  // rows past the sequence may hold anything: select, do not multiply
             const int c = h2 * 32 + c2;
             d0 = (qbase + c >= 0 && c < qlim) ? d0 : 0.f;
             d1 = (qbase + c + 1 >= 0 && c + 1 < qlim) ? d1 : 0.f;
           }
-          dk[(h2 * 32 + c2) >> 1] = bf16x2_bits(d0, d1);
+          pk[(h2 * 32 + c2) >> 1] = bf16x2_bits(d0, d1);
         }
       }
       // dS^T (queries 64 half .. 64 half + 63) over this warp's own dP^T columns
-      tmem_st32u(t_dph, dk);
+      tmem_st32u(t_dph, pk);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -1151,7 +1170,7 @@ __global__ void __launch_bounds__(320, 1)
 // j <= qt, S_j = Q K_j^T and dP_j = dO V_j^T (M = 128 queries, N = 128 keys),
 // dS_j = P_j (dP_j - D) with P_j = exp2(S_j c - lse log2 e), and
 // dQ += dS_j K_j.  320 threads:
-//   warp 0      TMA: Q and dO once, then K_j and V_j (two stages each)
+//   warp 0      TMA: Q and dO once, then K_j (three stages) and V_j (two)
 //   warp 1      TMEM allocation and the MMAs, in the order S_0, dP_0, then
 //               per step S_{j+1}, dQ += dS_j K_j, dP_{j+1}: S is double-
 //               buffered, so S_{j+1} runs while the softmax works on step j
@@ -1176,20 +1195,20 @@ __global__ void __launch_bounds__(320, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Qs = smem;
   uint8_t* dOs = Qs + TILE;
-  uint8_t* Ks = dOs + TILE;      // [2] stages
-  uint8_t* Vs = Ks + 2 * TILE;   // [2] stages
+  uint8_t* Ks = dOs + TILE;      // [3] stages: K_j is read by S_j and, a step later, by dQ
+  uint8_t* Vs = Ks + 3 * TILE;   // [2] stages
   uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + 2 * TILE);
   uint64_t* qo_full = bars;
-  uint64_t* k_full = bars + 1;   // [2]
-  uint64_t* k_empty = bars + 3;  // [2]
-  uint64_t* v_full = bars + 5;   // [2]
-  uint64_t* v_empty = bars + 7;  // [2]
-  uint64_t* s_full = bars + 9;   // [2] per S buffer
-  uint64_t* dp_full = bars + 11;
-  uint64_t* ds_ready = bars + 12;
-  uint64_t* acc_done = bars + 13;
-  uint64_t* drain = bars + 14;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 15);
+  uint64_t* k_full = bars + 1;   // [3]
+  uint64_t* k_empty = bars + 4;  // [3]
+  uint64_t* v_full = bars + 7;   // [2]
+  uint64_t* v_empty = bars + 9;  // [2]
+  uint64_t* s_full = bars + 11;  // [2] per S buffer
+  uint64_t* dp_full = bars + 13;
+  uint64_t* ds_ready = bars + 14;
+  uint64_t* acc_done = bars + 15;
+  uint64_t* drain = bars + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   // rows row0 .. row0+len-1 as in the forward; query rows past len are not
@@ -1208,14 +1227,18 @@ __global__ void __launch_bounds__(320, 1)
   const int qt = (int)gridDim.y - 1 - (int)blockIdx.y;
   if (qt * 128 >= len) return;
   const int h = blockIdx.x, g = (h * Hkv) / H;
-  const int n_k = qt + 1;  // key tiles 0 .. qt
+  // key tiles qt, qt-1, .., 0 (step j takes tile qt - j): the blocks of a
+  // head group then fetch different K / V tiles at a time
+  const int n_k = qt + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(qo_full, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < 3; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
       mbar_init(&s_full[s], 1);
@@ -1245,20 +1268,22 @@ __global__ void __launch_bounds__(320, 1)
       }
       int nkl = 0, nvl = 0;
       for (int j = 0; j < n_k; ++j) {
-        const int s = j & 1;
-        if (!mbar_wait(&k_empty[s], ((j >> 1) & 1) ^ 1u, abort_flag, status)) break;
-        mbar_arrive_expect_tx(&k_full[s], TILE);
-        for (int c = 0; c < 2; ++c) tma_load_2d(Ks + s * TILE + c * SLAB, &tmkv, kcol + 64 * c, row0 + j * 128, &k_full[s]);
+        const int s = j & 1, sk = j % 3;
+        if (!mbar_wait(&k_empty[sk], ((j / 3) & 1) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&k_full[sk], TILE);
+        for (int c = 0; c < 2; ++c)
+          tma_load_2d(Ks + sk * TILE + c * SLAB, &tmkv, kcol + 64 * c, row0 + (qt - j) * 128, &k_full[sk]);
         ++nkl;
         if (!mbar_wait(&v_empty[s], ((j >> 1) & 1) ^ 1u, abort_flag, status)) break;
         mbar_arrive_expect_tx(&v_full[s], TILE);
-        for (int c = 0; c < 2; ++c) tma_load_2d(Vs + s * TILE + c * SLAB, &tmkv, vcol + 64 * c, row0 + j * 128, &v_full[s]);
+        for (int c = 0; c < 2; ++c)
+          tma_load_2d(Vs + s * TILE + c * SLAB, &tmkv, vcol + 64 * c, row0 + (qt - j) * 128, &v_full[s]);
         ++nvl;
       }
       if (*abort_flag) {
         // let every copy in flight land before the block exits
         mbar_drain(qo_full, 0);
-        for (int j = nkl > 2 ? nkl - 2 : 0; j < nkl; ++j) mbar_drain(&k_full[j & 1], (j >> 1) & 1);
+        for (int j = nkl > 3 ? nkl - 3 : 0; j < nkl; ++j) mbar_drain(&k_full[j % 3], (j / 3) & 1);
         for (int j = nvl > 2 ? nvl - 2 : 0; j < nvl; ++j) mbar_drain(&v_full[j & 1], (j >> 1) & 1);
       }
     }
@@ -1273,10 +1298,10 @@ __global__ void __launch_bounds__(320, 1)
       auto kmaj = [](int kk) { return (uint64_t)(((kk >> 2) * SLAB + (kk & 3) * 32) >> 4); };
       // S_j = Q K_j^T into S buffer j & 1
       auto issue_s = [&](int j) -> bool {
-        const int s = j & 1;
-        if (!mbar_wait(&k_full[s], (j >> 1) & 1, abort_flag, status)) return false;
+        const int s = j & 1, sk = j % 3;
+        if (!mbar_wait(&k_full[sk], (j / 3) & 1, abort_flag, status)) return false;
         tc_fence_after();
-        const uint64_t st = (uint64_t)((s * TILE) >> 4);
+        const uint64_t st = (uint64_t)((sk * TILE) >> 4);
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(tmem + s * 128, DQ + kmaj(kk), DK + st + kmaj(kk), ID_S, kk > 0);
         mma_commit(&s_full[s]);
@@ -1303,12 +1328,12 @@ __global__ void __launch_bounds__(320, 1)
         // in columns 64h..64h+31 of S buffer s), B = K_j MN-major
         if (!mbar_wait(ds_ready, j & 1, abort_flag, status)) { ok = false; break; }
         tc_fence_after();
-        const uint64_t st = (uint64_t)((s * TILE) >> 4);
+        const uint64_t sk = (uint64_t)(((j % 3) * TILE) >> 4);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ta(t_dq, tmem + s * 128 + 64 * (kk >> 2) + 8 * (kk & 3), DKMN + st + (uint64_t)((kk * 2048) >> 4),
+          mma_bf16_ta(t_dq, tmem + s * 128 + 64 * (kk >> 2) + 8 * (kk & 3), DKMN + sk + (uint64_t)((kk * 2048) >> 4),
                       ID_Q, (j > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(&k_empty[s]);
+        mma_commit(&k_empty[j % 3]);
         // dP_{j+1} over dP_j, which the softmax warps have read (ds_ready)
         if (j + 1 < n_k && !issue_dp(j + 1)) { ok = false; break; }
       }
@@ -1344,8 +1369,8 @@ __global__ void __launch_bounds__(320, 1)
       const int s = j & 1;
       const uint32_t t_sh = tmem + s * 128 + half * 64 + lane_off, t_dph = t_dp + half * 64 + lane_off;
       // key c of this half is visible iff kbase + c <= q
-      const int kbase = j * 128 + half * 64;
-      const bool masked = (j == qt) || any_invalid;  // warp-uniform
+      const int kbase = (qt - j) * 128 + half * 64;
+      const bool masked = (j == 0) || any_invalid;  // the diagonal tile comes first (warp-uniform)
       if (!warp_wait(&s_full[s], (j >> 1) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
       // P = exp2(S c - lse log2 e (+ ALiBi bias)) for 64 keys, kept as bf16 pairs
@@ -1354,18 +1379,19 @@ __global__ void __launch_bounds__(320, 1)
         const uint64_t sl2x2 = f2_pack(sl2, sl2), nl2 = f2_pack(-lse2, -lse2);
         const float b0 = slope2 * (float)(kbase - q);  // bias of key c: b0 + slope2 c
         const uint64_t sx2 = f2_pack(slope2, slope2), b0x2 = f2_pack(b0, b0);
+        uint32_t sr[2][32];
+        tmem_ld32_nw(t_sh, sr[0]);
+        tmem_ld32_nw(t_sh + 32, sr[1]);
+        tmem_wait_ld();
 #pragma unroll
         for (int h2 = 0; h2 < 2; ++h2) {
-          uint32_t sr[32];
-          tmem_ld32_nw(t_sh + h2 * 32, sr);
-          tmem_wait_ld();
 #pragma unroll
           for (int c2 = 0; c2 < 32; c2 += 2) {
             const int c = h2 * 32 + c2;
             uint64_t add = nl2;
             if constexpr (ALIBI) add = f2_add(nl2, f2_fma(f2_pack((float)c, (float)(c + 1)), sx2, b0x2));
             float x0, x1;
-            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c2]), __uint_as_float(sr[c2 + 1])), sl2x2, add), x0, x1);
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[h2][c2]), __uint_as_float(sr[h2][c2 + 1])), sl2x2, add), x0, x1);
             float p0 = ex2(x0), p1 = ex2(x1);
             if (masked) {  // select, do not multiply: rows past the sequence may hold anything
               p0 = (qvalid && kbase + c <= q) ? p0 : 0.f;
@@ -1378,30 +1404,32 @@ __global__ void __launch_bounds__(320, 1)
       // dS = P (dP - D), written as bf16 pairs over this warp's own S columns
       if (!warp_wait(dp_full, j & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t dk[32];
       {
+        // dS over the packed P in place (pk), both halves loaded at once
         const uint64_t nd2 = f2_pack(-dq, -dq);
+        uint32_t dr[2][32];
+        tmem_ld32_nw(t_dph, dr[0]);
+        tmem_ld32_nw(t_dph + 32, dr[1]);
+        tmem_wait_ld();
 #pragma unroll
         for (int h2 = 0; h2 < 2; ++h2) {
-          uint32_t dr[32];
-          tmem_ld32_nw(t_dph + h2 * 32, dr);
-          tmem_wait_ld();
 #pragma unroll
           for (int c2 = 0; c2 < 32; c2 += 2) {
             const int c = h2 * 32 + c2;
             const uint32_t pw = pk[c >> 1];
             const uint64_t pp = f2_pack(__uint_as_float(pw << 16), __uint_as_float(pw & 0xFFFF0000u));
             float d0, d1;
-            f2_unpack(f2_mul(pp, f2_add(f2_pack(__uint_as_float(dr[c2]), __uint_as_float(dr[c2 + 1])), nd2)), d0, d1);
+            f2_unpack(f2_mul(pp, f2_add(f2_pack(__uint_as_float(dr[h2][c2]), __uint_as_float(dr[h2][c2 + 1])), nd2)),
+                      d0, d1);
             if (masked) {
               d0 = (qvalid && kbase + c <= q) ? d0 : 0.f;
               d1 = (qvalid && kbase + c + 1 <= q) ? d1 : 0.f;
             }
-            dk[c >> 1] = bf16x2_bits(d0, d1);
+            pk[c >> 1] = bf16x2_bits(d0, d1);
           }
         }
       }
-      tmem_st32u(t_sh, dk);
+      tmem_st32u(t_sh, pk);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -1448,12 +1476,12 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
                    bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
                    cudaStream_t st) {
-  // dK / dV: K, V, 2 stages of Q and of dO (six 32 KB tiles) + XT (one
-  // slab) + alignment + barriers = 214,272 bytes
-  constexpr size_t smem_kv = 6 * 2 * SLAB + SLAB + 1024 + 256;
-  // dQ: Q, dO, 2 stages of K and of V (six 32 KB tiles) + alignment +
-  // barriers = 197,888 bytes
-  constexpr size_t smem_q = 6 * 2 * SLAB + 1024 + 256;
+  // dK / dV: K, V, 3 stages of Q, dO (six 32 KB tiles) + XT (two slabs) +
+  // alignment + barriers = 230,656 bytes
+  constexpr size_t smem_kv = 6 * 2 * SLAB + 2 * SLAB + 1024 + 256;
+  // dQ: Q, dO, 3 stages of K, 2 of V (seven 32 KB tiles) + alignment +
+  // barriers = 230,656 bytes
+  constexpr size_t smem_q = 7 * 2 * SLAB + 1024 + 256;
   // once per process (initialisation of a function-local static is thread-safe)
   static const cudaError_t attr = [] {
     cudaError_t e =

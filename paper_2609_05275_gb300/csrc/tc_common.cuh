@@ -351,6 +351,60 @@ __device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols
   asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
 
+// Warp-converged forms of the MMA issue: the whole warp executes them with
+// warp-uniform operands and `elect.sync` inside the asm block picks the one
+// lane that issues (a single thread issuing from a divergent branch costs
+// about 60 clk an MMA, as much as an N = 128 MMA's tensor time).  For a
+// full, converged warp the elected lane is the same at every call, so a
+// commit tracks the MMAs that lane issued.
+__device__ __forceinline__ void mma_bf16_w(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                           uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n setp.ne.b32 p, %4, 0;\n"
+      " @e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void mma_bf16_ta_w(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                              uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n setp.ne.b32 p, %4, 0;\n"
+      " @e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit_w(uint64_t* bar) {
+  asm volatile(
+      "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(smem_u32(bar))
+      : "memory");
+}
+// Bounded wait executed by a whole converged warp: every lane polls the
+// barrier (no divergent branch), the verdict is made warp-uniform.
+__device__ __forceinline__ bool mbar_wait_conv(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                               int* status) {
+  const uint32_t addr = smem_u32(bar);
+  if (__all_sync(0xffffffffu, mbar_try_wait(addr, parity))) return true;
+  const uint64_t t0 = gtimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    // every lane acquires the phase itself (a lane that has seen it
+    // complete sees it again at once)
+    if (__all_sync(0xffffffffu, mbar_try_wait_sleep(addr, parity, 2000))) return true;
+    if ((it & 7) == 0) {
+      int bad = 0;
+      if ((threadIdx.x & 31) == 0) {
+        bad = *abort_flag ? 1 : 0;
+        if (!bad && gtimer_ns() - t0 > kWaitLimitNs) {
+          *abort_flag = 1;
+          set_status(status, LD_ERR_TIMEOUT);
+          bad = 1;
+        }
+      }
+      if (__shfl_sync(0xffffffffu, bad, 0)) return false;
+    }
+  }
+}
+
 // Warp-uniform bounded wait: lane 0 waits, the warp follows its verdict.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status) {
   int ok = 1;
