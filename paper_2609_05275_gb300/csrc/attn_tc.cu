@@ -221,50 +221,51 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    {  // the whole warp, converged; one elected lane issues
       // ------------------------------------------------ MMA issuer
       constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
       constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
       // descriptors built once, advanced by (byte offset >> 4) per MMA
       const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
       const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
-      bool ok = mbar_wait(q_full, 0, abort_flag, status);
+      bool ok = mbar_wait_conv(q_full, 0, abort_flag, status);
       for (int j = 0; ok && j <= nkt; ++j) {
         if (j < nkt) {
           const int s = j % NSK;
-          if (!mbar_wait(&k_full[s], (j / NSK) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait_conv(&k_full[s], (j / NSK) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait_conv(&s_free[j & 1], ((j >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
           const uint64_t kb = DK + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
           for (int kk = 0; kk < DH / 16; ++kk) {
             const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-            mma_bf16(tmem + (j & 1) * 128, DQ + off, kb + off, ID_S, kk > 0);
+            mma_bf16_w(tmem + (j & 1) * 128, DQ + off, kb + off, ID_S, kk > 0);
           }
-          mma_commit(&s_full[j & 1]);
-          mma_commit(&k_empty[s]);
+          mma_commit_w(&s_full[j & 1]);
+          mma_commit_w(&k_empty[s]);
         }
         if (j >= 1) {
           const int jp = j - 1, s = jp % NSV, pb = jp & 1;
-          if (!mbar_wait(&p_full[pb], (jp >> 1) & 1, abort_flag, status)) { ok = false; break; }
-          if (!mbar_wait(&v_full[s], (jp / NSV) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait_conv(&p_full[pb], (jp >> 1) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait_conv(&v_full[s], (jp / NSV) & 1, abort_flag, status)) { ok = false; break; }
           tc_fence_after();
           const uint64_t vb = DV + (uint64_t)((s * TILE) >> 4);
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
             // A = P from TMEM (16 keys = 8 columns a step); B = V as MN-major
             // (dh contiguous): 64-dh chunks one slab apart, 8-key groups 1 KB
-            mma_bf16_ta(t_o, t_p + pb * 64 + kk * 8, vb + ((kk * 2048) >> 4), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
+            mma_bf16_ta_w(t_o, t_p + pb * 64 + kk * 8, vb + ((kk * 2048) >> 4), ID_O, (jp > 0 || kk > 0) ? 1u : 0u);
           }
-          mma_commit(&pv_done[pb]);
-          mma_commit(&v_empty[s]);
+          mma_commit_w(&pv_done[pb]);
+          mma_commit_w(&v_empty[s]);
         }
       }
       if (ok) {
-        mma_commit(o_full);
+        mma_commit_w(o_full);
       } else {
-        mma_commit(drain);
-        mbar_drain(drain, 0);
+        mma_commit_w(drain);
+        if (lane == 0) mbar_drain(drain, 0);
+        __syncwarp();
       }
     }
   } else {
@@ -570,16 +571,16 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    {  // the whole warp, converged; one elected lane issues
       // ------------------------------------------------ MMA issuer
       constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
       constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
       const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
       const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
-      bool ok = mbar_wait(q_full, 0, abort_flag, status);
+      bool ok = mbar_wait_conv(q_full, 0, abort_flag, status);
       for (int j = 0; ok && j <= nkt; ++j) {
-        if (j < nkt && !mbar_wait(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
-        if (j >= 1 && !mbar_wait(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
+        if (j < nkt && !mbar_wait_conv(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
+        if (j >= 1 && !mbar_wait_conv(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
           ok = false;
           break;
         }
@@ -587,14 +588,14 @@ __global__ void __launch_bounds__(320, 1)
           const int nkg = gi ? nkB : nkA;
           if (j >= 1 && j - 1 < nkg) {
             // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
-            if (!mbar_wait(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
+            if (!mbar_wait_conv(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
             tc_fence_after();
             const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
-              mma_bf16_ta(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
+              mma_bf16_ta_w(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
                           (j > 1 || kk > 0) ? 1u : 0u);
-            if (j == nkg) mma_commit(&o_full[gi]);  // the group's last P V
+            if (j == nkg) mma_commit_w(&o_full[gi]);  // the group's last P V
           }
           if (j < nkg) {
             // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
@@ -603,18 +604,19 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
             for (int kk = 0; kk < DH / 16; ++kk) {
               const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-              mma_bf16(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
+              mma_bf16_w(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
             }
-            mma_commit(&s_full[gi]);
+            mma_commit_w(&s_full[gi]);
           }
         }
         if (!ok) break;
-        if (j < nkt) mma_commit(&k_empty[j % PP_NSK]);
-        if (j >= 1) mma_commit(&v_empty[(j - 1) % PP_NSV]);
+        if (j < nkt) mma_commit_w(&k_empty[j % PP_NSK]);
+        if (j >= 1) mma_commit_w(&v_empty[(j - 1) % PP_NSV]);
       }
       if (!ok) {
-        mma_commit(drain);
-        mbar_drain(drain, 0);
+        mma_commit_w(drain);
+        if (lane == 0) mbar_drain(drain, 0);
+        __syncwarp();
       }
     }
   } else {
@@ -746,95 +748,77 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 }
 
 // ---------------------------------------------------------------------------
-// Backward, head size 128, in two kernels without atomics.
-//
-// attn_bwd_kv_kernel: dK and dV.  One CTA per (128-key tile, kv head, kept
-// sequence); it loops over the query heads of the group and, for each, the
-// 128-query tiles at or after the key tile (one step per query tile).  Every
-// MMA is M = 128, N = 128.  320 threads:
-//   warp 0      TMA: K, V once; Q_i (three stages) and dO_i (one); all lanes
-//               write the bf16 terms of -lse_i sqrt(Dh) and -D_i that two
-//               extra K = 16 MMAs fold into S^T_i and dP^T_i
-//   warp 1      TMEM allocation and the MMAs, issued in the order
-//                 dP^T_i, dV += P^T_i dO_i, S^T_{i+1}, dK += dS^T_i Q_i
-//               (S^T_0 first): S^T_{i+1} goes ahead of dK_i, so the
-//               exponentials of step i+1 overlap dK_i and dP^T_{i+1}
-//   warps 2..9  softmax, one key and 64 queries per thread (two warps per
-//               TMEM lane quadrant).  Phase A: P^T = exp2(S^T c) written as
-//               bf16 over the thread's own S^T columns (the A operand of dV).
-//               Phase B: dS^T = P^T (dP^T - D) written as bf16 over its own
-//               dP^T columns (the A operand of dK).  At the end dK (times c,
-//               with the inverse rotation) and dV from TMEM to dqkv
-// TMEM columns: S^T / P^T 0-127, dP^T / dS^T 128-255, dV 256-383, dK 384-511.
-// The exponent of P is c S - lse log2(e) = c (S - lse sqrt(Dh)) with
-// c = log2(e) / sqrt(Dh), so S^T arrives as S^T - lse sqrt(Dh) and dP^T as
-// dP^T - D, and the softmax warps read no per-query vectors.
-//
-// attn_bwd_q_kernel: dQ.  One CTA per (128-query tile, query head, kept
-// sequence), looping over the key tiles at or before the query tile; dQ
-// accumulates in TMEM over the loop and is written once, scaled and with the
-// inverse rotation, as bf16 (no float32 buffer, no reductions).
-// A single kernel adding each key tile's dQ^T into a float32 buffer was
-// measured bound by those reductions: 64 KB a 128 x 128 step, about 2.5 TB/s
-// of L2 reductions over the GPU, three times the MMA time of the step; the
-// second kernel recomputes S and dP instead (7 MMAs per tile pair, not 5).
+// Backward, head size 128.  One CTA per (128-key tile, kv head, kept
+// sequence), looping over the query heads of the group and the 64-query
+// tiles at or after the key tile.  448 threads:
+//   warp 0      TMA: K, V once; Q_i, dO_i, lse_i, D_i per step (3 stages)
+//   warp 1      MMAs, one step ahead: S^T_i = K Q_i^T, dP^T_i = V dO_i^T
+//               (M = 128 keys, N = 64 queries); then for step i-1
+//               dV += P^T dO (P^T read from TMEM), dK += dS^T Q (M = 128
+//               keys, N = 128) and dQ^T = K^T dS^T (M = 128 head dims,
+//               N = 64 queries)
+//   warps 2..9  one key and 32 queries per thread: P^T = exp2(S^T c log2e - lse log2e)
+//               as bf16 into TMEM, dS^T = P^T (dP^T - D) as bf16 into a
+//               swizzled shared-memory tile; at the end dK (times c) and dV
+//               from TMEM to dqkv
+//   warps 10..13  dQ^T from TMEM, added into the float32 dQ buffer
+// P^T and dS^T are double-buffered (step i uses buffer i & 1), so the
+// softmax warps write step i while the MMAs of step i-1 still read theirs.
+// TMEM columns: S^T 0-63, dP^T 64-127, dV 128-255, dK 256-383, dQ^T 384-447,
+// P^T 448-479 / 480-511.
+constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
-// x as three bf16 terms, t0 + t1 + t2 = x to about 2^-24 |x| (each residual
-// is exact in float32).
-__device__ __forceinline__ void split3_bf16(float x, uint32_t& t0, uint32_t& t1, uint32_t& t2) {
-  const bf16 a = __float2bfloat16_rn(x);
-  const float r1 = x - __bfloat162float(a);
-  const bf16 b = __float2bfloat16_rn(r1);
-  const float r2 = r1 - __bfloat162float(b);
-  const bf16 c = __float2bfloat16_rn(r2);
-  t0 = __bfloat16_as_ushort(a);
-  t1 = __bfloat16_as_ushort(b);
-  t2 = __bfloat16_as_ushort(c);
+// Values 4 e4 .. 4 e4 + 3 of p (shared memory); p is 16-byte aligned when
+// off == 0 (warp-uniform), else read one by one.
+__device__ __forceinline__ float4 ld4s(const float* p, int e4, int off) {
+  if (off == 0) return reinterpret_cast<const float4*>(p)[e4];
+  return make_float4(p[4 * e4], p[4 * e4 + 1], p[4 * e4 + 2], p[4 * e4 + 3]);
 }
 
 template <bool ALIBI>
-__global__ void __launch_bounds__(320, 1)
-    attn_bwd_kv_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmo,
+__global__ void __launch_bounds__(448, 1)
+    attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmq,
+                       const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmdq,
                        const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
-                       bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
+                       float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
                        int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
                        const float* __restrict__ alibi, const int* __restrict__ seg, const int* __restrict__ tok,
                        int* status) {
   constexpr int DH = 128;
-  constexpr uint32_t TILE = 2 * SLAB;  // 128 rows x 128 bf16 (two 64-column slabs)
+  constexpr uint32_t KT = 2 * SLAB;    // 128 keys x 128 dims
+  constexpr uint32_t QT = 2 * HSLAB;   // 64 queries x 128 dims
+  constexpr int NST = 3;               // stages of the Q / dO / lse / D ring
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Ks = smem;
-  uint8_t* Vs = Ks + TILE;
-  uint8_t* Qs = Vs + TILE;       // [3] stages: Q_i is read by S^T_i and, a step later, by dK
-  uint8_t* dOs = Qs + 3 * TILE;  // one stage
-  // XT: 128 rows x 128 bytes (128-byte swizzle) of K = 16 chunk pairs for
-  // the fold MMAs: pair 0 = (1, 1, 1, 0, ...) and pair 1 = (0, 0, 0, 1, 1,
-  // 1, 0, ...) in every row (the A operands), pair 2 + s = the terms of
-  // stage s in row q = query q of the step: (l0, l1, l2, d0, d1, d2, 0, ...)
-  // with l0 + l1 + l2 = -lse sqrt(Dh) and d0 + d1 + d2 = -D.
-  // (stage 2's terms are pair 0 of a second such slab, XT + SLAB)
-  uint8_t* XT = dOs + TILE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(XT + 2 * SLAB);
+  uint8_t* Vs = Ks + KT;
+  uint8_t* Qs = Vs + KT;         // [NST][QT]
+  uint8_t* dOs = Qs + NST * QT;  // [NST][QT]
+  uint8_t* DSs = dOs + NST * QT; // [2] 128 keys x 64 queries, one slab of 128-byte rows each
+  float* dqs = reinterpret_cast<float*>(DSs + 2 * SLAB);  // [64 queries][128 dims] float32 staging (1 KB aligned)
+  // [NST][lse 68 | D 68]: the 64 values of a step start at float `voff` of
+  // each half (a sequence's rows start anywhere with per-token kept lists,
+  // and a bulk copy needs a 16-byte aligned source, so 68 are copied from
+  // the aligned-down address)
+  float* vecs = dqs + 64 * DH;
+  constexpr int VS = 136;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + NST * VS);
   uint64_t* kv_full = bars;
-  uint64_t* q_full = bars + 1;   // [3]
-  uint64_t* q_empty = bars + 4;  // [3]
-  uint64_t* o_full = bars + 7;
-  uint64_t* o_empty = bars + 8;
-  uint64_t* s_full = bars + 9;
-  uint64_t* dp_full = bars + 10;
-  uint64_t* p_ready = bars + 11;
-  uint64_t* ds_ready = bars + 12;
-  uint64_t* acc_done = bars + 13;
-  uint64_t* drain = bars + 14;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 15);
+  uint64_t* ld_full = bars + 1;          // [NST]
+  uint64_t* ld_empty = ld_full + NST;    // [NST]
+  uint64_t* sdp_full = ld_empty + NST;
+  uint64_t* sdp_free = sdp_full + 1;
+  uint64_t* p_ready = sdp_full + 2;  // [2] per P^T / dS^T buffer
+  uint64_t* mm_done = sdp_full + 4;  // [2] per P^T / dS^T buffer
+  uint64_t* dq_free = sdp_full + 6;
+  uint64_t* acc_done = sdp_full + 7;
+  uint64_t* drain = sdp_full + 8;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sdp_full + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  // rows row0 .. row0+len-1 (a kept sequence, or with `seg` the kept tokens
-  // of sequence blockIdx.z); queries past len get P = dS = 0, keys past len
-  // are never stored.  Grid (kv head, key tile, sequence): one sequence's
-  // blocks are dispatched together, heaviest key tiles (kt = 0) first.
-  const int seq = blockIdx.z;
+  // rows row0 .. row0+len-1 as in the forward; queries past len (the last
+  // query tile) get P = dS = 0, keys past len are never stored
+  const int seq = blockIdx.y;
   int row0, len;
   if (seg) {
     row0 = seg[seq];
@@ -844,278 +828,221 @@ __global__ void __launch_bounds__(320, 1)
     row0 = seq * S;
     len = S;
   }
-  const int kt = blockIdx.y, g = blockIdx.x, grp = H / Hkv;
+  const int kt = blockIdx.z, g = blockIdx.x, grp = H / Hkv;  // heaviest key tiles (kt = 0) dispatched first
   if (kt * 128 >= len) return;
-  const int nq = (len + 127) / 128;  // query tiles kt .. nq-1 overlap or follow the keys
-  const int nqs = nq - kt;
-  const int n_it = grp * nqs;
+  const int nq = (len + 63) / 64, q0 = 2 * kt;  // query tiles q0 .. nq-1 overlap or follow the keys
+  const int n_it = grp * (nq - q0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
-    for (int s = 0; s < 3; ++s) {
-      mbar_init(&q_full[s], 1);
-      mbar_init(&q_empty[s], 1);
+    for (int b = 0; b < NST; ++b) {
+      mbar_init(&ld_full[b], 1);
+      mbar_init(&ld_empty[b], 1);
     }
-    mbar_init(o_full, 1);
-    mbar_init(o_empty, 1);
-    mbar_init(s_full, 1);
-    mbar_init(dp_full, 1);
-    mbar_init(p_ready, 8);
-    mbar_init(ds_ready, 8);
+    mbar_init(sdp_full, 1);
+    mbar_init(sdp_free, 8);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&p_ready[b], 8);
+      mbar_init(&mm_done[b], 1);
+    }
+    mbar_init(dq_free, 4);
     mbar_init(acc_done, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  if (threadIdx.x < 128) {
-    // row r of XT: the two ones patterns, zero terms
-    const int r = threadIdx.x;
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (u == 0) v = make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
-      if (u == 2) v = make_uint4(0u, 0x3F800000u, 0x3F803F80u, 0u);
-      *reinterpret_cast<uint4*>(XT + swz(r, u)) = v;
-      *reinterpret_cast<uint4*>(XT + SLAB + swz(r, u)) = make_uint4(0u, 0u, 0u, 0u);
-    }
-    fence_proxy_async();
   }
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t t_s = tmem, t_dp = tmem + 128, t_dv = tmem + 256, t_dk = tmem + 384;
+  const uint32_t t_s = tmem, t_dp = tmem + 64, t_dv = tmem + 128, t_dk = tmem + 256, t_dq = tmem + 384;
+  const uint32_t t_p = tmem + 448;  // [2] x 32 columns: P^T as bf16 pairs
 
   if (warp == 0) {
-    // ------------------------------------------------ producer (warp 0)
-    const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
     if (lane == 0) {
-      mbar_arrive_expect_tx(kv_full, 2 * TILE);
+      // ------------------------------------------------ TMA producer
+      const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
+      mbar_arrive_expect_tx(kv_full, 2 * KT);
       for (int c = 0; c < 2; ++c) {
         tma_load_2d(Ks + c * SLAB, &tmkv, kcol + 64 * c, row0 + kt * 128, kv_full);
         tma_load_2d(Vs + c * SLAB, &tmkv, vcol + 64 * c, row0 + kt * 128, kv_full);
       }
-    }
-    const float sq_dh = sqrtf((float)DH);
-    // -lse sqrt(Dh) and -D of the 128 queries of step i, four a lane, loaded
-    // one step ahead so their latency stays off the Q copy's path
-    float xl[4], xd[4];
-    auto load_terms = [&](int i) {
-      const int h = g * grp + i / nqs, qt = kt + i % nqs;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int q = u * 32 + lane;
-        xl[u] = 0.f;
-        xd[u] = 0.f;
-        if (qt * 128 + q < len) {
-          const size_t at = (size_t)h * lse_ld + row0 + qt * 128 + q;
-          xl[u] = -lse[at] * sq_dh;
-          xd[u] = -Dvec[at];
+      int issued = 0;
+      for (int i = 0; i < n_it; ++i) {
+        const int b = i % NST;
+        const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
+        if (!mbar_wait(&ld_empty[b], ((i / NST) & 1) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&ld_full[b], 2 * QT + 2 * 272);
+        for (int c = 0; c < 2; ++c) {
+          tma_load_2d(Qs + b * QT + c * HSLAB, &tmq, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
+          tma_load_2d(dOs + b * QT + c * HSLAB, &tmo, h * DH + 64 * c, row0 + qt * 64, &ld_full[b]);
         }
+        const size_t vo = ((size_t)h * lse_ld + row0 + qt * 64) & ~(size_t)3;  // lse_ld % 4 == 0
+        bulk_load(vecs + b * VS, lse + vo, 272, &ld_full[b]);
+        bulk_load(vecs + b * VS + 68, Dvec + vo, 272, &ld_full[b]);
+        ++issued;
       }
-    };
-    if (n_it > 0) load_terms(0);
-    int nql = 0, nol = 0;
-    for (int i = 0; i < n_it; ++i) {
-      const int s = i % 3;
-      const int h = g * grp + i / nqs, qt = kt + i % nqs;
-      // Q_i and the terms of step i into stage s once step i-3 has released
-      // it; the copy is issued first (the barrier's phase cannot complete
-      // before the arrival below, which follows the terms)
-      if (!warp_wait(&q_empty[s], ((i / 3) & 1) ^ 1u, abort_flag, status)) break;
-      if (lane == 0)
-        for (int c = 0; c < 2; ++c)
-          tma_load_2d(Qs + s * TILE + c * SLAB, &tmkv, h * DH + 64 * c, row0 + qt * 128, &q_full[s]);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        uint32_t l0, l1, l2, d0, d1, d2;
-        split3_bf16(xl[u], l0, l1, l2);
-        split3_bf16(xd[u], d0, d1, d2);
-        *reinterpret_cast<uint4*>(s < 2 ? XT + swz(u * 32 + lane, 4 + 2 * s) : XT + SLAB + swz(u * 32 + lane, 0)) =
-            make_uint4(l0 | (l1 << 16), l2 | (d0 << 16), d1 | (d2 << 16), 0u);
+      if (*abort_flag) {
+        mbar_drain(kv_full, 0);
+        for (int i = issued > NST ? issued - NST : 0; i < issued; ++i) mbar_drain(&ld_full[i % NST], (i / NST) & 1);
       }
-      fence_proxy_async();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_expect_tx(&q_full[s], TILE);
-      if (i + 1 < n_it) load_terms(i + 1);
-      ++nql;
-      // dO_i once dV_{i-1} has read dO_{i-1}
-      if (!warp_wait(o_empty, (i & 1) ^ 1u, abort_flag, status)) break;
-      if (lane == 0) {
-        mbar_arrive_expect_tx(o_full, TILE);
-        for (int c = 0; c < 2; ++c)
-          tma_load_2d(dOs + c * SLAB, &tmo, h * DH + 64 * c, row0 + qt * 128, o_full);
-      }
-      ++nol;
     }
-    if (lane == 0 && *abort_flag) {
-      // let every copy in flight land before the block exits
-      mbar_drain(kv_full, 0);
-      for (int i = nql > 3 ? nql - 3 : 0; i < nql; ++i) mbar_drain(&q_full[i % 3], (i / 3) & 1);
-      if (nol > 0) mbar_drain(o_full, (nol - 1) & 1);
-    }
-    __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0) {
+    {  // the whole warp, converged; one elected lane issues
       // ------------------------------------------------ MMA issuer
-      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);   // S^T, dP^T and the folds
+      constexpr uint32_t ID_SP = idesc_bf16(128, 64, false, false);   // S^T, dP^T
       constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
+      constexpr uint32_t ID_Q = idesc_bf16(128, 64, true, true);      // dQ^T (A = K, B = dS^T, MN-major)
       // shared-memory descriptors built once; an MMA's operand is its base
       // plus (byte offset >> 4) in the address field (every tile lies below
       // 256 KB, so the 14-bit field never carries)
       const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
       const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
-      const uint64_t DQMN = sdesc(smem_u32(Qs), SLAB, 1024), DOMN = sdesc(smem_u32(dOs), SLAB, 1024);
-      const uint64_t DX = sdesc(smem_u32(XT), 16, 1024), DX2 = sdesc(smem_u32(XT + SLAB), 16, 1024);
-      // B operand of the fold MMAs: the terms of Q stage s
-      auto terms = [&](int s) { return s < 2 ? DX + (uint64_t)(((2 + s) * 32) >> 4) : DX2; };
-      // offset of the K = 16 chunk kk of a K-major 128 x 128 tile (two slabs)
-      auto kmaj = [](int kk) { return (uint64_t)(((kk >> 2) * SLAB + (kk & 3) * 32) >> 4); };
-      // S^T_i = K Q_i^T - lse sqrt(Dh) (ones pattern 0 times the terms)
-      auto issue_s = [&](int i) -> bool {
-        const int s = i % 3;
-        if (!mbar_wait(&q_full[s], (i / 3) & 1, abort_flag, status)) return false;
-        tc_fence_after();
-        const uint64_t st = (uint64_t)((s * TILE) >> 4);
+      const uint64_t DQMN = sdesc(smem_u32(Qs), HSLAB, 1024), DOMN = sdesc(smem_u32(dOs), HSLAB, 1024);
+      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024), DS = sdesc(smem_u32(DSs), 16, 1024);
+      bool ok = mbar_wait_conv(kv_full, 0, abort_flag, status);
+      for (int i = 0; ok && i <= n_it; ++i) {
+        if (i < n_it) {
+          const int b = i % NST;
+          if (!mbar_wait_conv(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait_conv(sdp_free, (i & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t st = (uint64_t)((b * QT) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_s, DK + kmaj(kk), DQ + st + kmaj(kk), ID_S, kk > 0);
-        mma_bf16(t_s, DX, terms(s), ID_S, 1u);
-        mma_commit(s_full);
-        return true;
-      };
-      bool ok = mbar_wait(kv_full, 0, abort_flag, status) && issue_s(0);
-      for (int i = 0; ok && i < n_it; ++i) {
-        const int s = i % 3;
-        const uint64_t st = (uint64_t)((s * TILE) >> 4);
-        // dP^T_i = V dO_i^T - D (ones pattern 1 times the terms), over the
-        // dS^T_{i-1} columns (dK_{i-1}, issued before, reads them first)
-        if (!mbar_wait(o_full, i & 1, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const uint32_t koff = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+            const uint32_t qoff = ((kk >> 2) * HSLAB + (kk & 3) * 32) >> 4;
+            mma_bf16_w(t_s, DK + koff, DQ + st + qoff, ID_SP, kk > 0);
+            mma_bf16_w(t_dp, DV + koff, DO + st + qoff, ID_SP, kk > 0);
+          }
+          mma_commit_w(sdp_full);
+        }
+        if (i >= 1) {
+          const int ip = i - 1, b = ip % NST, pb = ip & 1;
+          if (!mbar_wait_conv(&p_ready[pb], (ip >> 1) & 1, abort_flag, status)) { ok = false; break; }
+          if (!mbar_wait_conv(dq_free, (ip & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t st = (uint64_t)((b * QT) >> 4), ds = (uint64_t)((pb * SLAB) >> 4);
+          const uint32_t first = ip > 0 ? 1u : 0u;
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_dp, DV + kmaj(kk), DO + kmaj(kk), ID_S, kk > 0);
-        mma_bf16(t_dp, DX + (uint64_t)(32 >> 4), terms(s), ID_S, 1u);
-        mma_commit(dp_full);
-        // dV += P^T_i dO_i: A = P^T from TMEM (queries 64h..64h+63 as bf16
-        // pairs in columns 64h..64h+31), B = dO MN-major
-        if (!mbar_wait(p_ready, i & 1, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
+          for (int kk = 0; kk < 4; ++kk) {  // contraction over the 64 queries
+            const uint32_t aoff = (kk * 32) >> 4;                // dS^T, K-major
+            const uint32_t boff = (kk * 2048) >> 4;              // dO / Q as MN-major
+            mma_bf16_ta_w(t_dv, t_p + pb * 32 + kk * 8, DOMN + st + boff, ID_KV, kk > 0 ? 1u : first);
+            mma_bf16_w(t_dk, DS + ds + aoff, DQMN + st + boff, ID_KV, kk > 0 ? 1u : first);
+          }
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ta(t_dv, t_s + 64 * (kk >> 2) + 8 * (kk & 3), DOMN + (uint64_t)((kk * 2048) >> 4), ID_KV,
-                      (i > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(o_empty);
-        // S^T_{i+1} ahead of the product that waits for dS^T_i
-        if (i + 1 < n_it && !issue_s(i + 1)) { ok = false; break; }
-        if (!mbar_wait(ds_ready, i & 1, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
-        // dK += dS^T_i Q_i (contraction over the 128 queries): A = dS^T from
-        // TMEM (queries 64h..64h+63 as bf16 pairs in dP^T columns
-        // 64h..64h+31), B = Q MN-major
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ta(t_dk, t_dp + 64 * (kk >> 2) + 8 * (kk & 3), DQMN + st + (uint64_t)((kk * 2048) >> 4), ID_KV,
-                      (i > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(&q_empty[s]);
+          for (int kk = 0; kk < 8; ++kk) {  // contraction over the 128 keys
+            mma_bf16_w(t_dq, DKMN + ((kk * 2048) >> 4), DS + ds + ((kk * 2048) >> 4), ID_Q, kk > 0);
+          }
+          mma_commit_w(&mm_done[pb]);
+          mma_commit_w(&ld_empty[b]);
+        }
       }
       if (ok) {
-        mma_commit(acc_done);
+        mma_commit_w(acc_done);
       } else {
-        mma_commit(drain);
-        mbar_drain(drain, 0);
+        mma_commit_w(drain);
+        if (lane == 0) mbar_drain(drain, 0);
+        __syncwarp();
       }
     }
-  } else {
+  } else if (warp < 10) {
     // ------------------------------------------------ P / dS (warps 2..9)
-    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..63 of the
-    // step, warps 6..9 queries 64..127, one key per thread
+    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..31 of the
+    // step, warps 6..9 queries 32..63, one key per thread
     const int quad = warp & 3;
     const int half = (warp - 2) >> 2;
     const int r = quad * 32 + lane;  // key within the tile
     const int key = kt * 128 + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const uint32_t t_sh = t_s + half * 64 + lane_off, t_dph = t_dp + half * 64 + lane_off;
+    const int voff = row0 & 3;  // first value of a step in its lse / D stage (see vecs)
     const float sl2 = kLog2e * rsqrtf((float)DH);
     bool ok = true;
     for (int i = 0; i < n_it; ++i) {
-      const int qt = kt + i % nqs;
+      const int b = i % NST;
+      const int qt = q0 + i % (nq - q0);
       // ALiBi: logit bias slope2 (key - query) of this step's query head
-      const float slope2 = ALIBI ? alibi[g * grp + i / nqs] * kLog2e : 0.f;
-      const int qbase = qt * 128 + half * 64 - key;  // query c is visible iff qbase + c >= 0
-      const int qlim = len - (qt * 128 + half * 64);  // and exists iff c < qlim (warp-uniform)
-      // mask only where some of the warp's 32 keys do not see all 64 queries,
-      // or the queries run past the sequence (warp-uniform)
-      const bool full = __shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 64;
-      // ---- phase A: P^T from S^T (lse folded in)
-      if (!warp_wait(s_full, i & 1, abort_flag, status)) { ok = false; break; }
+      const float slope2 = ALIBI ? alibi[g * grp + i / (nq - q0)] * kLog2e : 0.f;
+      if (!warp_wait(sdp_full, i & 1, abort_flag, status)) { ok = false; break; }
+      if (!warp_wait(&ld_full[b], (i / NST) & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      uint32_t pk[32];
-      auto phase_a = [&](auto masked) {
+      uint32_t sr[32], dr[32];
+      tmem_ld32_nw(t_s + half * 32 + lane_off, sr);
+      tmem_ld32_nw(t_dp + half * 32 + lane_off, dr);
+      tmem_wait_ld();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sdp_free);
+      const float* lsrc = vecs + b * VS + voff + half * 32;       // lse of the 32 queries
+      const float* dsrc = vecs + b * VS + 68 + voff + half * 32;  // D of the 32 queries
+      const int qbase = qt * 64 + half * 32 - key;  // query c is visible iff qbase + c >= 0
+      const int qlim = len - (qt * 64 + half * 32);  // and exists iff c < qlim (warp-uniform)
+      uint32_t pk[16], dk[16];
+      // pairs of queries on the packed fp32 pipe; the mask only on warps
+      // whose 32 keys are not all visible to the 32 queries, or whose queries
+      // run past the sequence (warp-uniform)
+      auto pass = [&](auto masked) {
         constexpr bool MASK = decltype(masked)::value;
-        const uint64_t sl2x2 = f2_pack(sl2, sl2);
-        const float b0 = slope2 * (float)(-qbase);  // bias of query c: b0 - slope2 c
+        const uint64_t sl2x2 = f2_pack(sl2, sl2), nlog2 = f2_pack(-kLog2e, -kLog2e);
+        // bias of query c: slope2 (key - qt*64 - half*32 - c) = b0 - slope2 c
+        const float b0 = slope2 * (float)(-qbase);
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
-        uint32_t sr[2][32];
-        tmem_ld32_nw(t_sh, sr[0]);
-        tmem_ld32_nw(t_sh + 32, sr[1]);
-        tmem_wait_ld();
 #pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
+        for (int e4 = 0; e4 < 8; ++e4) {
+          const float4 lq = ld4s(lsrc, e4, voff), dq = ld4s(dsrc, e4, voff);
+          uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
+          if constexpr (ALIBI) {
 #pragma unroll
-          for (int c2 = 0; c2 < 32; c2 += 2) {
-            const int c = h2 * 32 + c2;
-            uint64_t x2 = f2_mul(f2_pack(__uint_as_float(sr[h2][c2]), __uint_as_float(sr[h2][c2 + 1])), sl2x2);
-            if constexpr (ALIBI) x2 = f2_add(x2, f2_fma(f2_pack((float)c, (float)(c + 1)), nsx2, b0x2));
+            for (int h2 = 0; h2 < 2; ++h2) {
+              const float c0 = (float)(4 * e4 + 2 * h2);
+              nl[h2] = f2_add(nl[h2], f2_fma(f2_pack(c0, c0 + 1.f), nsx2, b0x2));
+            }
+          }
+          const uint64_t dd[2] = {f2_pack(dq.x, dq.y), f2_pack(dq.z, dq.w)};
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2) {
+            const int c = 4 * e4 + 2 * h2;
             float x0, x1;
-            f2_unpack(x2, x0, x1);
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sl2x2, nl[h2]), x0, x1);
             float p0 = ex2(x0), p1 = ex2(x1);
+            const bool v0 = !MASK || (qbase + c >= 0 && c < qlim), v1 = !MASK || (qbase + c + 1 >= 0 && c + 1 < qlim);
             if constexpr (MASK) {
-              p0 = (qbase + c >= 0 && c < qlim) ? p0 : 0.f;
-              p1 = (qbase + c + 1 >= 0 && c + 1 < qlim) ? p1 : 0.f;
+              p0 = v0 ? p0 : 0.f;
+              p1 = v1 ? p1 : 0.f;
+            }
+            const uint64_t pp = f2_pack(p0, p1);
+            float d0, d1;
+            f2_unpack(f2_mul(pp, f2_sub(f2_pack(__uint_as_float(dr[c]), __uint_as_float(dr[c + 1])), dd[h2])), d0, d1);
+            if constexpr (MASK) {  // rows past the sequence may hold anything: select, do not multiply
+              d0 = v0 ? d0 : 0.f;
+              d1 = v1 ? d1 : 0.f;
             }
             pk[c >> 1] = bf16x2_bits(p0, p1);
+            dk[c >> 1] = bf16x2_bits(d0, d1);
           }
         }
       };
-      if (full) phase_a(std::false_type{});
-      else phase_a(std::true_type{});
-      // P^T (queries 64 half .. 64 half + 63) over this warp's own S^T columns
-      tmem_st32u(t_sh, pk);
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(p_ready);
-      // ---- phase B: dS^T = P^T (dP^T - D) (D folded in)
-      if (!warp_wait(dp_full, i & 1, abort_flag, status)) { ok = false; break; }
+      if (__shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 32) pass(std::false_type{});
+      else pass(std::true_type{});
+      // the MMAs of step i-2 must be done with buffer i & 1 before it is rewritten
+      const int pb = i & 1;
+      if (i >= 2 && !warp_wait(&mm_done[pb], ((i >> 1) & 1) ^ 1u, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
-      // dS^T over the packed P^T in place (pk), both halves loaded at once
-      uint32_t dr[2][32];
-      tmem_ld32_nw(t_dph, dr[0]);
-      tmem_ld32_nw(t_dph + 32, dr[1]);
-      tmem_wait_ld();
+      tmem_st16(t_p + pb * 32 + half * 16 + lane_off, pk);
+      uint8_t* ds = DSs + pb * SLAB;
 #pragma unroll
-      for (int h2 = 0; h2 < 2; ++h2) {
-#pragma unroll
-        for (int c2 = 0; c2 < 32; c2 += 2) {
-          const uint32_t pw = pk[(h2 * 32 + c2) >> 1];
-          const uint64_t pp = f2_pack(__uint_as_float(pw << 16), __uint_as_float(pw & 0xFFFF0000u));
-          float d0, d1;
-          f2_unpack(f2_mul(pp, f2_pack(__uint_as_float(dr[h2][c2]), __uint_as_float(dr[h2][c2 + 1]))), d0, d1);
-          if (!full) {  // rows past the sequence may hold anything: select, do not multiply
-            const int c = h2 * 32 + c2;
-            d0 = (qbase + c >= 0 && c < qlim) ? d0 : 0.f;
-            d1 = (qbase + c + 1 >= 0 && c + 1 < qlim) ? d1 : 0.f;
-          }
-          pk[(h2 * 32 + c2) >> 1] = bf16x2_bits(d0, d1);
-        }
+      for (int c = 0; c < 4; ++c) {
+        const int chunk = half * 4 + c;
+        *reinterpret_cast<uint4*>(ds + swz(r, chunk)) = make_uint4(dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
       }
-      // dS^T (queries 64 half .. 64 half + 63) over this warp's own dP^T columns
-      tmem_st32u(t_dph, pk);
+      fence_proxy_async();
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(ds_ready);
+      if (lane == 0) mbar_arrive(&p_ready[pb]);
     }
     if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
       tc_fence_after();
@@ -1123,7 +1050,7 @@ __global__ void __launch_bounds__(320, 1)
       if (half == 0) {
         // dK (times c) with the inverse rotation at the key's position
         const float c = rsqrtf((float)DH);
-        const int kpos = kvalid ? row_pos(tok, S, row0 + key) : 0;  // rows past the segment are not read
+        const int kpos = row_pos(tok, S, row0 + key);
         bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
 #pragma unroll 1
         for (int cc = 0; cc < 2; ++cc) {
@@ -1156,311 +1083,38 @@ __global__ void __launch_bounds__(320, 1)
         }
       }
     }
-  }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, 512);
-  }
-}
-
-// dQ of one (128-query tile, query head h, kept sequence): for each key tile
-// j <= qt, S_j = Q K_j^T and dP_j = dO V_j^T (M = 128 queries, N = 128 keys),
-// dS_j = P_j (dP_j - D) with P_j = exp2(S_j c - lse log2 e), and
-// dQ += dS_j K_j.  320 threads:
-//   warp 0      TMA: Q and dO once, then K_j (three stages) and V_j (two)
-//   warp 1      TMEM allocation and the MMAs, in the order S_0, dP_0, then
-//               per step S_{j+1}, dQ += dS_j K_j, dP_{j+1}: S is double-
-//               buffered, so S_{j+1} runs while the softmax works on step j
-//   warps 2..9  softmax, one query row and 64 keys per thread (two warps per
-//               TMEM lane quadrant), lse and D of the row held in registers:
-//               P_j from S_j, then dS_j from dP_j, written as bf16 over the
-//               thread's own S_j columns (the A operand of dQ += dS_j K_j);
-//               at the end dQ (times c, with the inverse rotation at the
-//               query's position) from TMEM to dqkv
-// TMEM columns: S_0 0-127, S_1 128-255, dP 256-383, dQ 384-511.
-template <bool ALIBI>
-__global__ void __launch_bounds__(320, 1)
-    attn_bwd_q_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmo,
-                      const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
-                      bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt, int S, int H, int Hkv,
-                      const float* __restrict__ rcos, const float* __restrict__ rsin,
-                      const float* __restrict__ alibi, const int* __restrict__ seg, const int* __restrict__ tok,
-                      int* status) {
-  constexpr int DH = 128;
-  constexpr uint32_t TILE = 2 * SLAB;  // 128 rows x 128 bf16 (two 64-column slabs)
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* Qs = smem;
-  uint8_t* dOs = Qs + TILE;
-  uint8_t* Ks = dOs + TILE;      // [3] stages: K_j is read by S_j and, a step later, by dQ
-  uint8_t* Vs = Ks + 3 * TILE;   // [2] stages
-  uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + 2 * TILE);
-  uint64_t* qo_full = bars;
-  uint64_t* k_full = bars + 1;   // [3]
-  uint64_t* k_empty = bars + 4;  // [3]
-  uint64_t* v_full = bars + 7;   // [2]
-  uint64_t* v_empty = bars + 9;  // [2]
-  uint64_t* s_full = bars + 11;  // [2] per S buffer
-  uint64_t* dp_full = bars + 13;
-  uint64_t* ds_ready = bars + 14;
-  uint64_t* acc_done = bars + 15;
-  uint64_t* drain = bars + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-
-  // rows row0 .. row0+len-1 as in the forward; query rows past len are not
-  // stored (P = dS = 0 for them), keys past len are hidden by causality.
-  // Grid (query head, query tile, sequence), heaviest query tiles first.
-  const int seq = blockIdx.z;
-  int row0, len;
-  if (seg) {
-    row0 = seg[seq];
-    len = seg[seq + 1] - row0;
   } else {
-    if (seq >= *cnt) return;
-    row0 = seq * S;
-    len = S;
-  }
-  const int qt = (int)gridDim.y - 1 - (int)blockIdx.y;
-  if (qt * 128 >= len) return;
-  const int h = blockIdx.x, g = (h * Hkv) / H;
-  // key tiles qt, qt-1, .., 0 (step j takes tile qt - j): the blocks of a
-  // head group then fetch different K / V tiles at a time
-  const int n_k = qt + 1;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  if (threadIdx.x == 0) {
-    mbar_init(qo_full, 1);
-    for (int s = 0; s < 3; ++s) {
-      mbar_init(&k_full[s], 1);
-      mbar_init(&k_empty[s], 1);
-    }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&v_full[s], 1);
-      mbar_init(&v_empty[s], 1);
-      mbar_init(&s_full[s], 1);
-    }
-    mbar_init(dp_full, 1);
-    mbar_init(ds_ready, 8);
-    mbar_init(acc_done, 1);
-    mbar_init(drain, 1);
-    *abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  if (warp == 1) tmem_alloc(tmem_slot, 512);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  const uint32_t t_dp = tmem + 256, t_dq = tmem + 384;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      // ------------------------------------------------ TMA producer
-      const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
-      mbar_arrive_expect_tx(qo_full, 2 * TILE);
-      for (int c = 0; c < 2; ++c) {
-        tma_load_2d(Qs + c * SLAB, &tmkv, h * DH + 64 * c, row0 + qt * 128, qo_full);
-        tma_load_2d(dOs + c * SLAB, &tmo, h * DH + 64 * c, row0 + qt * 128, qo_full);
-      }
-      int nkl = 0, nvl = 0;
-      for (int j = 0; j < n_k; ++j) {
-        const int s = j & 1, sk = j % 3;
-        if (!mbar_wait(&k_empty[sk], ((j / 3) & 1) ^ 1u, abort_flag, status)) break;
-        mbar_arrive_expect_tx(&k_full[sk], TILE);
-        for (int c = 0; c < 2; ++c)
-          tma_load_2d(Ks + sk * TILE + c * SLAB, &tmkv, kcol + 64 * c, row0 + (qt - j) * 128, &k_full[sk]);
-        ++nkl;
-        if (!mbar_wait(&v_empty[s], ((j >> 1) & 1) ^ 1u, abort_flag, status)) break;
-        mbar_arrive_expect_tx(&v_full[s], TILE);
-        for (int c = 0; c < 2; ++c)
-          tma_load_2d(Vs + s * TILE + c * SLAB, &tmkv, vcol + 64 * c, row0 + (qt - j) * 128, &v_full[s]);
-        ++nvl;
-      }
-      if (*abort_flag) {
-        // let every copy in flight land before the block exits
-        mbar_drain(qo_full, 0);
-        for (int j = nkl > 3 ? nkl - 3 : 0; j < nkl; ++j) mbar_drain(&k_full[j % 3], (j / 3) & 1);
-        for (int j = nvl > 2 ? nvl - 2 : 0; j < nvl; ++j) mbar_drain(&v_full[j & 1], (j >> 1) & 1);
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
-      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S, dP (both operands K-major)
-      constexpr uint32_t ID_Q = idesc_bf16(128, DH, false, true);    // dQ (A = dS from TMEM, B = K MN-major)
-      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
-      const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
-      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024);
-      auto kmaj = [](int kk) { return (uint64_t)(((kk >> 2) * SLAB + (kk & 3) * 32) >> 4); };
-      // S_j = Q K_j^T into S buffer j & 1
-      auto issue_s = [&](int j) -> bool {
-        const int s = j & 1, sk = j % 3;
-        if (!mbar_wait(&k_full[sk], (j / 3) & 1, abort_flag, status)) return false;
-        tc_fence_after();
-        const uint64_t st = (uint64_t)((sk * TILE) >> 4);
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(tmem + s * 128, DQ + kmaj(kk), DK + st + kmaj(kk), ID_S, kk > 0);
-        mma_commit(&s_full[s]);
-        return true;
-      };
-      // dP_j = dO V_j^T
-      auto issue_dp = [&](int j) -> bool {
-        const int s = j & 1;
-        if (!mbar_wait(&v_full[s], (j >> 1) & 1, abort_flag, status)) return false;
-        tc_fence_after();
-        const uint64_t st = (uint64_t)((s * TILE) >> 4);
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16(t_dp, DO + kmaj(kk), DV + st + kmaj(kk), ID_S, kk > 0);
-        mma_commit(dp_full);
-        mma_commit(&v_empty[s]);
-        return true;
-      };
-      bool ok = mbar_wait(qo_full, 0, abort_flag, status) && issue_s(0) && issue_dp(0);
-      for (int j = 0; ok && j < n_k; ++j) {
-        const int s = j & 1;
-        // S_{j+1} into the other buffer (its dS_{j-1} was read by dQ, issued before)
-        if (j + 1 < n_k && !issue_s(j + 1)) { ok = false; break; }
-        // dQ += dS_j K_j: A = dS_j from TMEM (keys 64h..64h+63 as bf16 pairs
-        // in columns 64h..64h+31 of S buffer s), B = K_j MN-major
-        if (!mbar_wait(ds_ready, j & 1, abort_flag, status)) { ok = false; break; }
-        tc_fence_after();
-        const uint64_t sk = (uint64_t)(((j % 3) * TILE) >> 4);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_ta(t_dq, tmem + s * 128 + 64 * (kk >> 2) + 8 * (kk & 3), DKMN + sk + (uint64_t)((kk * 2048) >> 4),
-                      ID_Q, (j > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(&k_empty[j % 3]);
-        // dP_{j+1} over dP_j, which the softmax warps have read (ds_ready)
-        if (j + 1 < n_k && !issue_dp(j + 1)) { ok = false; break; }
-      }
-      if (ok) {
-        mma_commit(acc_done);
-      } else {
-        mma_commit(drain);
-        mbar_drain(drain, 0);
-      }
-    }
-  } else {
-    // ------------------------------------------------ softmax (warps 2..9)
-    // two warps per TMEM lane quadrant: warps 2..5 take keys 0..63 of each
-    // key tile, warps 6..9 keys 64..127, one query row per thread
+    // ------------------------------------------------ dQ (warps 10..13)
+    // dQ^T from TMEM -> a [64 x 128] float32 tile in shared memory, added
+    // into dq_acc by one bulk tensor reduce per step.
     const int quad = warp & 3;
-    const int half = (warp - 2) >> 2;
-    const int r = quad * 32 + lane;  // query row within the tile
-    const int q = qt * 128 + r;      // query within the sequence
-    const bool qvalid = q < len;
+    const int dd = quad * 32 + lane;  // head dimension of this thread
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const float sl2 = kLog2e * rsqrtf((float)DH);
-    const float slope2 = ALIBI ? alibi[h] * kLog2e : 0.f;
-    float lse2 = 0.f, dq = 0.f;  // lse log2(e) and D of this row
-    if (qvalid) {
-      const size_t at = (size_t)h * lse_ld + row0 + q;
-      lse2 = lse[at] * kLog2e;
-      dq = Dvec[at];
-    }
-    // rows past the sequence: P = dS = 0 (warp-uniform test below)
-    const bool any_invalid = __any_sync(0xffffffffu, !qvalid);
-    bool ok = true;
-    for (int j = 0; j < n_k; ++j) {
-      const int s = j & 1;
-      const uint32_t t_sh = tmem + s * 128 + half * 64 + lane_off, t_dph = t_dp + half * 64 + lane_off;
-      // key c of this half is visible iff kbase + c <= q
-      const int kbase = (qt - j) * 128 + half * 64;
-      const bool masked = (j == 0) || any_invalid;  // the diagonal tile comes first (warp-uniform)
-      if (!warp_wait(&s_full[s], (j >> 1) & 1, abort_flag, status)) { ok = false; break; }
+    const bool leader = (warp == 10 && lane == 0);
+    for (int i = 0; i < n_it; ++i) {
+      const int h = g * grp + i / (nq - q0), qt = q0 + i % (nq - q0);
+      if (!warp_wait(&mm_done[i & 1], (i >> 1) & 1, abort_flag, status)) break;
       tc_fence_after();
-      // P = exp2(S c - lse log2 e (+ ALiBi bias)) for 64 keys, kept as bf16 pairs
-      uint32_t pk[32];
-      {
-        const uint64_t sl2x2 = f2_pack(sl2, sl2), nl2 = f2_pack(-lse2, -lse2);
-        const float b0 = slope2 * (float)(kbase - q);  // bias of key c: b0 + slope2 c
-        const uint64_t sx2 = f2_pack(slope2, slope2), b0x2 = f2_pack(b0, b0);
-        uint32_t sr[2][32];
-        tmem_ld32_nw(t_sh, sr[0]);
-        tmem_ld32_nw(t_sh + 32, sr[1]);
-        tmem_wait_ld();
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
-#pragma unroll
-          for (int c2 = 0; c2 < 32; c2 += 2) {
-            const int c = h2 * 32 + c2;
-            uint64_t add = nl2;
-            if constexpr (ALIBI) add = f2_add(nl2, f2_fma(f2_pack((float)c, (float)(c + 1)), sx2, b0x2));
-            float x0, x1;
-            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[h2][c2]), __uint_as_float(sr[h2][c2 + 1])), sl2x2, add), x0, x1);
-            float p0 = ex2(x0), p1 = ex2(x1);
-            if (masked) {  // select, do not multiply: rows past the sequence may hold anything
-              p0 = (qvalid && kbase + c <= q) ? p0 : 0.f;
-              p1 = (qvalid && kbase + c + 1 <= q) ? p1 : 0.f;
-            }
-            pk[c >> 1] = bf16x2_bits(p0, p1);
-          }
-        }
-      }
-      // dS = P (dP - D), written as bf16 pairs over this warp's own S columns
-      if (!warp_wait(dp_full, j & 1, abort_flag, status)) { ok = false; break; }
-      tc_fence_after();
-      {
-        // dS over the packed P in place (pk), both halves loaded at once
-        const uint64_t nd2 = f2_pack(-dq, -dq);
-        uint32_t dr[2][32];
-        tmem_ld32_nw(t_dph, dr[0]);
-        tmem_ld32_nw(t_dph + 32, dr[1]);
-        tmem_wait_ld();
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
-#pragma unroll
-          for (int c2 = 0; c2 < 32; c2 += 2) {
-            const int c = h2 * 32 + c2;
-            const uint32_t pw = pk[c >> 1];
-            const uint64_t pp = f2_pack(__uint_as_float(pw << 16), __uint_as_float(pw & 0xFFFF0000u));
-            float d0, d1;
-            f2_unpack(f2_mul(pp, f2_add(f2_pack(__uint_as_float(dr[h2][c2]), __uint_as_float(dr[h2][c2 + 1])), nd2)),
-                      d0, d1);
-            if (masked) {
-              d0 = (qvalid && kbase + c <= q) ? d0 : 0.f;
-              d1 = (qvalid && kbase + c + 1 <= q) ? d1 : 0.f;
-            }
-            pk[c >> 1] = bf16x2_bits(d0, d1);
-          }
-        }
-      }
-      tmem_st32u(t_sh, pk);
-      tmem_wait_st();
+      float t0[32], t1[32];
+      tmem_ld32(t_dq + lane_off, t0);
+      tmem_ld32(t_dq + 32 + lane_off, t1);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(ds_ready);
-    }
-    if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
-      tc_fence_after();
-      // dQ times c with the inverse rotation at the query's position: this
-      // thread takes the pairs (i, i + 64), i = 32 half .. 32 half + 31
-      const float c = rsqrtf((float)DH);
-      const int pos = qvalid ? row_pos(tok, S, row0 + q) : 0;
-      float a1[32], a2[32];
-      tmem_ld32(t_dq + half * 32 + lane_off, a1);
-      tmem_ld32(t_dq + 64 + half * 32 + lane_off, a2);
+      if (lane == 0) mbar_arrive(dq_free);
+      if (leader && i > 0) bulk_wait_read();  // the previous reduce has read the tile
+      named_barrier(1, 128);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        const float p1 = c * a1[e], p2 = c * a2[e];
-        float cs = 1.f, sn = 0.f;
-        if (rcos) {
-          cs = rcos[(size_t)pos * 64 + half * 32 + e];
-          sn = rsin[(size_t)pos * 64 + half * 32 + e];
-        }
-        a1[e] = p1 * cs + p2 * sn;
-        a2[e] = p2 * cs - p1 * sn;
-      }
-      if (qvalid) {
-        bf16* qrow = dqkv + (long long)(row0 + q) * ldq + (long long)h * DH;
-        st_bf16x32_(qrow + half * 32, a1);
-        st_bf16x32_(qrow + 64 + half * 32, a2);
+      for (int e = 0; e < 32; ++e) dqs[e * DH + dd] = t0[e];
+#pragma unroll
+      for (int e = 0; e < 32; ++e) dqs[(32 + e) * DH + dd] = t1[e];
+      fence_proxy_async();
+      named_barrier(1, 128);
+      if (leader) {
+        tma_reduce_add_2d(&tmdq, h * DH, row0 + qt * 64, dqs);
+        bulk_commit();
       }
     }
+    if (leader) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -1473,33 +1127,25 @@ __global__ void __launch_bounds__(320, 1)
 
 template <bool ALIBI>
 cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
-                   bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
+                   float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
                    const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
                    cudaStream_t st) {
-  // dK / dV: K, V, 3 stages of Q, dO (six 32 KB tiles) + XT (two slabs) +
-  // alignment + barriers = 230,656 bytes
-  constexpr size_t smem_kv = 6 * 2 * SLAB + 2 * SLAB + 1024 + 256;
-  // dQ: Q, dO, 3 stages of K, 2 of V (seven 32 KB tiles) + alignment +
-  // barriers = 230,656 bytes
-  constexpr size_t smem_q = 7 * 2 * SLAB + 1024 + 256;
+  // K, V, 2 x dS^T (6 slabs) + 3 stages of Q, dO (12 half slabs) + lse/D
+  // vectors + dQ staging + alignment + barriers = 232,288 bytes (of 232,448)
+  constexpr size_t smem = 6 * SLAB + 12 * HSLAB + 3 * 136 * 4 + 64 * 128 * 4 + 1024 + 256;
   // once per process (initialisation of a function-local static is thread-safe)
-  static const cudaError_t attr = [] {
-    cudaError_t e =
-        cudaFuncSetAttribute(attn_bwd_kv_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_kv);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(attn_bwd_q_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_q);
-    return e;
-  }();
+  static const cudaError_t attr =
+      cudaFuncSetAttribute(attn_bwd_tc_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
-  CUtensorMap tkv, to;  // tiles of 128 rows x 64 columns: Q, K, V in qkv; dO
+  CUtensorMap tkv, tq, to, tdq;  // K/V tiles of 128 rows; Q / dO tiles of 64 rows; dQ reduce boxes
+  if (!make_map_f32(&tdq, dq_acc, (uint64_t)H * 128, (uint64_t)max_seqs * S, (uint64_t)H * 128, 128, 64))
+    return cudaErrorInvalidValue;
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
-  if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 128)) return cudaErrorInvalidValue;
-  attn_bwd_kv_kernel<ALIBI><<<dim3(Hkv, S / 128, max_seqs), 320, smem_kv, st>>>(
-      tkv, to, lse, Dvec, max_seqs * S, dqkv, ldq, cnt, S, H, Hkv, rcos, rsin, alibi, seg, tok, status);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  attn_bwd_q_kernel<ALIBI><<<dim3(H, S / 128, max_seqs), 320, smem_q, st>>>(
-      tkv, to, lse, Dvec, max_seqs * S, dqkv, ldq, cnt, S, H, Hkv, rcos, rsin, alibi, seg, tok, status);
+  if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
+  if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
+  dim3 grid(Hkv, max_seqs, S / 128);
+  attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
+                                                     H, Hkv, rcos, rsin, alibi, seg, tok, status);
   return cudaGetLastError();
 }
 }  // namespace
@@ -1509,14 +1155,16 @@ bool attn_tc_supported(int S, int Dh) { return S % 128 == 0 && (Dh == 64 || Dh =
 bool attn_bwd_tc_supported(int S, int Dh) { return S % 128 == 0 && Dh == 128; }
 
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
-                               const float* Dvec, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs,
-                               const float* rcos, const float* rsin, const float* alibi, const int* seg,
+                               const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
+                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, const int* seg,
                                const int* tok, int* status, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)max_seqs * S * H * 128 * sizeof(float), st);
+  if (e != cudaSuccess) return e;
   if (alibi)
-    return bwd_tc<true>(qkv, ldqkv, dO, ldo, lse, Dvec, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi, seg, tok,
-                        status, st);
-  return bwd_tc<false>(qkv, ldqkv, dO, ldo, lse, Dvec, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi, seg, tok,
-                       status, st);
+    return bwd_tc<true>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                        seg, tok, status, st);
+  return bwd_tc<false>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                       seg, tok, status, st);
 }
 
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,

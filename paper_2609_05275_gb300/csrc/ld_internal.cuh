@@ -169,13 +169,13 @@ bool attn_tc_supported(int S, int Dh);
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
                                int Hkv, int Dh, int max_seqs, const float* alibi, const int* seg, int* status,
                                cudaStream_t st);
-// tcgen05 flash attention backward (head size 128, S % 128 == 0): dK, dV
-// and dQ straight into dqkv, dQ scaled by 1/sqrt(Dh), dQ and dK with the
-// inverse RoPE applied (rcos = null: no rotation).
+// tcgen05 flash attention backward (head size 128, S % 128 == 0); zeroes
+// dq_acc and accumulates dQ (unscaled) into it.
 bool attn_bwd_tc_supported(int S, int Dh);
+// dK leaves with the inverse RoPE applied (rcos = null: no rotation).
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
-                               const float* Dvec, bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs,
-                               const float* rcos, const float* rsin, const float* alibi, const int* seg,
+                               const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
+                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, const int* seg,
                                const int* tok, int* status, cudaStream_t st);
 // dqkv[:, q heads] = inverse-RoPE(dq_acc / sqrt(Dh)) as bf16 (rcos = null: no rotation);
 // rows and positions as launch_rope_apply
