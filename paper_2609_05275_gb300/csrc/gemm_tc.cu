@@ -386,8 +386,9 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && rank == 0) {
-      // ------------------------------------------------ MMA issuer
+    if (rank == 0) {
+      // ------------------------------------------------ MMA issuer (whole warp, converged;
+      // one elected lane issues)
       constexpr uint32_t IDESC = idesc_bf16(BMT, BN, A_MN, B_MN);
       int stage = 0;
       uint32_t phase = 0;
@@ -395,14 +396,14 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t acc_phase = 0;
       bool ok = true;
       for (int tile = tile0; tile < num_tiles && ok; tile += tstep) {
-        if (!mbar_wait<PAIR>(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
+        if (!mbar_wait_conv<PAIR>(&tempty[acc], acc_phase ^ 1u, abort_flag, a.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         for (int ks = 0; ks < num_ks; ++ks) {
-          if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
+          if (!mbar_wait_conv(&full[stage], phase, abort_flag, a.status)) {
             ok = false;
             break;
           }
@@ -422,15 +423,15 @@ __global__ void __launch_bounds__(192, 1)
               const uint64_t bd = B_MN ? sdesc(sb + k * 2048, 8192, 1024) : sdesc(sb + k * 32, 16, 1024);
               const uint32_t accum = (ks | j | k) != 0 ? 1u : 0u;
               if constexpr (PAIR)
-                mma_bf16_pair(d_tmem, ad, bd, IDESC, accum);
+                mma_bf16_pair_w(d_tmem, ad, bd, IDESC, accum);
               else
-                mma_bf16(d_tmem, ad, bd, IDESC, accum);
+                mma_bf16_w(d_tmem, ad, bd, IDESC, accum);
             }
           }
           if constexpr (PAIR)
-            mma_commit_pair_both(&empty[stage]);
+            mma_commit_pair_both_w(&empty[stage]);
           else
-            mma_commit(&empty[stage]);
+            mma_commit_w(&empty[stage]);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -438,19 +439,20 @@ __global__ void __launch_bounds__(192, 1)
         }
         if (!ok) break;
         if constexpr (PAIR)
-          mma_commit_pair_both(&tfull[acc]);
+          mma_commit_pair_both_w(&tfull[acc]);
         else
-          mma_commit(&tfull[acc]);
+          mma_commit_w(&tfull[acc]);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
       }
       if (!ok) {
         // make sure every MMA issued so far has finished before TMEM is freed
         if constexpr (PAIR)
-          mma_commit_pair_local(drain);
+          mma_commit_pair_local_w(drain);
         else
-          mma_commit(drain);
-        mbar_drain(drain, 0);
+          mma_commit_w(drain);
+        if (lane == 0) mbar_drain(drain, 0);
+        __syncwarp();
       }
     }
   } else {

@@ -359,6 +359,29 @@ __device__ __forceinline__ void mma_commit_pair_local(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
+// Warp-converged forms of the three above (see mma_bf16_w).
+__device__ __forceinline__ void mma_bf16_pair_w(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                                uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n setp.ne.b32 p, %4, 0;\n"
+      " @e tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit_pair_both_w(uint64_t* bar) {
+  asm volatile(
+      "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n}\n" ::"r"(
+          smem_u32(bar)),
+      "h"((uint16_t)3)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit_pair_local_w(uint64_t* bar) {
+  asm volatile(
+      "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(smem_u32(bar))
+      : "memory");
+}
 // Collective over one warp of each CTA of the pair.
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t* slot, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
@@ -399,15 +422,18 @@ __device__ __forceinline__ void mma_commit_w(uint64_t* bar) {
 }
 // Bounded wait executed by a whole converged warp: every lane polls the
 // barrier (no divergent branch), the verdict is made warp-uniform.
+// CL: cluster-scope acquire (the phase is completed by the peer CTA).
+template <bool CL = false>
 __device__ __forceinline__ bool mbar_wait_conv(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                                int* status) {
   const uint32_t addr = smem_u32(bar);
-  if (__all_sync(0xffffffffu, mbar_try_wait(addr, parity))) return true;
+  if (__all_sync(0xffffffffu, CL ? mbar_try_wait_cl(addr, parity) : mbar_try_wait(addr, parity))) return true;
   const uint64_t t0 = gtimer_ns();
   for (uint32_t it = 1;; ++it) {
     // every lane acquires the phase itself (a lane that has seen it
     // complete sees it again at once)
-    if (__all_sync(0xffffffffu, mbar_try_wait_sleep(addr, parity, 2000))) return true;
+    if (__all_sync(0xffffffffu, CL ? mbar_try_wait_cl(addr, parity) : mbar_try_wait_sleep(addr, parity, 2000)))
+      return true;
     if ((it & 7) == 0) {
       int bad = 0;
       if ((threadIdx.x & 31) == 0) {
