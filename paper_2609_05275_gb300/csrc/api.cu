@@ -379,8 +379,9 @@ cudaError_t attn_fwd<bf16>(const Handle* h, void* ws, const bf16* qkv, bf16* o, 
 }
 
 // Attention backward: dq, dk, dv into dqkv with the inverse RoPE applied to
-// dq and dk (fused into dq_finish and the tcgen05 kernel's dK epilogue on
-// the bf16 path; a separate rotation otherwise).
+// dq and dk (in the tcgen05 kernels' epilogues and dq_finish on the bf16
+// tcgen05 path, dq_finish and a rotation of the k heads on the mma.sync path,
+// a separate rotation on the debug path).
 template <typename T>
 cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const T* dO, const float* lse, float* Dvec,
                      T* dqkv, const Rows& r, cudaStream_t st) {
@@ -401,11 +402,11 @@ cudaError_t attn_bwd(const Handle* h, void* ws, const T* qkv, const T* o, const 
   float* dq_acc = at<float>(ws, h->lay.dqacc);
   const bf16* q16 = reinterpret_cast<const bf16*>(qkv);
   bf16* d16 = reinterpret_cast<bf16*>(dqkv);
-  if (attn_bwd_tc_supported(c.S, c.Dh)) {
-    e = launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16, r.cnt,
-                           c.S, c.H, c.Hkv, c.B, rcos, rsin, alibi_table(h, ws), r.seg, r.tok(),
-                           at<int>(ws, h->lay.status), st);
-  } else {  // whole sequences only (per-token granularity is refused at ld_create on this path)
+  if (attn_bwd_tc_supported(c.S, c.Dh))  // dQ finished inside
+    return launch_attn_bwd_tc(q16, h->nqkv, reinterpret_cast<const bf16*>(dO), c.H * c.Dh, lse, Dvec, dq_acc, d16,
+                              r.cnt, c.S, c.H, c.Hkv, c.Dh, c.B, rcos, rsin, alibi_table(h, ws), r.seg, r.tok(),
+                              at<int>(ws, h->lay.status), st);
+  {  // whole sequences only (per-token granularity is refused at ld_create on this path)
     e = launch_attn_bwd_mma(q16, h->nqkv, reinterpret_cast<const bf16*>(o), reinterpret_cast<const bf16*>(dO),
                             c.H * c.Dh, lse, Dvec, dq_acc, d16, r.cnt, c.S, c.H, c.Hkv, c.Dh, c.B, alibi_table(h, ws),
                             st);

@@ -818,7 +818,7 @@ __global__ void __launch_bounds__(448, 1)
 
   // rows row0 .. row0+len-1 as in the forward; queries past len (the last
   // query tile) get P = dS = 0, keys past len are never stored
-  const int seq = blockIdx.y;
+  const int seq = blockIdx.z;
   int row0, len;
   if (seg) {
     row0 = seg[seq];
@@ -828,7 +828,7 @@ __global__ void __launch_bounds__(448, 1)
     row0 = seq * S;
     len = S;
   }
-  const int kt = blockIdx.z, g = blockIdx.x, grp = H / Hkv;  // heaviest key tiles (kt = 0) dispatched first
+  const int kt = blockIdx.y, g = blockIdx.x, grp = H / Hkv;
   if (kt * 128 >= len) return;
   const int nq = (len + 63) / 64, q0 = 2 * kt;  // query tiles q0 .. nq-1 overlap or follow the keys
   const int n_it = grp * (nq - q0);
@@ -1143,28 +1143,803 @@ cudaError_t bwd_tc(const bf16* qkv, int ldq, const bf16* dO, int ldo, const floa
   if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   if (!make_map(&tq, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 64)) return cudaErrorInvalidValue;
   if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 64)) return cudaErrorInvalidValue;
-  dim3 grid(Hkv, max_seqs, S / 128);
+  // grid (kv head, key tile, sequence): one sequence's blocks are dispatched
+  // together, heaviest key tiles (kt = 0) first, so the dQ rows being
+  // reduced into at a time are one sequence's (64 MB at the Llama-3-8B
+  // shape, inside L2) rather than every kept sequence's
+  dim3 grid(Hkv, S / 128, max_seqs);
   attn_bwd_tc_kernel<ALIBI><<<grid, 448, smem, st>>>(tkv, tq, to, tdq, lse, Dvec, max_seqs * S, dq_acc, dqkv, ldq, cnt, S,
                                                      H, Hkv, rcos, rsin, alibi, seg, tok, status);
+  return cudaGetLastError();
+}
+// Backward, head size 64, in two kernels without atomics.
+//
+// attn_bwd_kv_kernel: dK and dV.  One CTA per (128-key tile, kv head, kept
+// sequence); it loops over the query heads of the group and, for each, the
+// 128-query tiles at or after the key tile (one step per query tile).  Every
+// MMA is M = 128, N = 128.  320 threads:
+//   warp 0      TMA: K, V once; Q_i (three stages) and dO_i (one); all lanes
+//               write the bf16 terms of -lse_i sqrt(Dh) and -D_i that two
+//               extra K = 16 MMAs fold into S^T_i and dP^T_i
+//   warp 1      TMEM allocation and the MMAs, issued in the order
+//                 dP^T_i, dV += P^T_i dO_i, S^T_{i+1}, dK += dS^T_i Q_i
+//               (S^T_0 first): S^T_{i+1} goes ahead of dK_i, so the
+//               exponentials of step i+1 overlap dK_i and dP^T_{i+1}
+//   warps 2..9  softmax, one key and 64 queries per thread (two warps per
+//               TMEM lane quadrant).  Phase A: P^T = exp2(S^T c) written as
+//               bf16 over the thread's own S^T columns (the A operand of dV).
+//               Phase B: dS^T = P^T (dP^T - D) written as bf16 over its own
+//               dP^T columns (the A operand of dK).  At the end dK (times c,
+//               with the inverse rotation) and dV from TMEM to dqkv
+// TMEM columns: S^T / P^T 0-127, dP^T / dS^T 128-255, dV 256-383, dK 384-511.
+// The exponent of P is c S - lse log2(e) = c (S - lse sqrt(Dh)) with
+// c = log2(e) / sqrt(Dh), so S^T arrives as S^T - lse sqrt(Dh) and dP^T as
+// dP^T - D, and the softmax warps read no per-query vectors.
+//
+// attn_bwd_q_kernel: dQ.  One CTA per (128-query tile, query head, kept
+// sequence), looping over the key tiles at or before the query tile; dQ
+// accumulates in TMEM over the loop and is written once, scaled and with the
+// inverse rotation, as bf16 (no float32 buffer, no reductions).
+// Every MMA has M = 128 (at head size 64 the transposed dQ of the single
+// kernel above would be an M = 64 product); the second kernel recomputes S
+// and dP (7 MMAs per tile pair, not 5).  At head size 128 the same pair of
+// kernels measured slower than the single kernel (95 against 80 ms of
+// attention in the Llama-3-8B step), so they serve head size 64 only.
+
+// x as three bf16 terms, t0 + t1 + t2 = x to about 2^-24 |x| (each residual
+// is exact in float32).
+__device__ __forceinline__ void split3_bf16(float x, uint32_t& t0, uint32_t& t1, uint32_t& t2) {
+  const bf16 a = __float2bfloat16_rn(x);
+  const float r1 = x - __bfloat162float(a);
+  const bf16 b = __float2bfloat16_rn(r1);
+  const float r2 = r1 - __bfloat162float(b);
+  const bf16 c = __float2bfloat16_rn(r2);
+  t0 = __bfloat16_as_ushort(a);
+  t1 = __bfloat16_as_ushort(b);
+  t2 = __bfloat16_as_ushort(c);
+}
+
+template <int DH, bool ALIBI>
+__global__ void __launch_bounds__(320, 1)
+    attn_bwd_kv_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmo,
+                       const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
+                       bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt,
+                       int S, int H, int Hkv, const float* __restrict__ rcos, const float* __restrict__ rsin,
+                       const float* __restrict__ alibi, const int* __restrict__ seg, const int* __restrict__ tok,
+                       int* status) {
+  constexpr int NSL = DH / 64;           // 64-column slabs of a row
+  constexpr uint32_t TILE = NSL * SLAB;  // 128 rows x DH bf16
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Ks = smem;
+  uint8_t* Vs = Ks + TILE;
+  uint8_t* Qs = Vs + TILE;       // [3] stages: Q_i is read by S^T_i and, a step later, by dK
+  uint8_t* dOs = Qs + 3 * TILE;  // one stage
+  // XT: 128 rows x 128 bytes (128-byte swizzle) of K = 16 chunk pairs for
+  // the fold MMAs: pair 0 = (1, 1, 1, 0, ...) and pair 1 = (0, 0, 0, 1, 1,
+  // 1, 0, ...) in every row (the A operands), pair 2 + s = the terms of
+  // stage s in row q = query q of the step: (l0, l1, l2, d0, d1, d2, 0, ...)
+  // with l0 + l1 + l2 = -lse sqrt(Dh) and d0 + d1 + d2 = -D.
+  // (stage 2's terms are pair 0 of a second such slab, XT + SLAB)
+  uint8_t* XT = dOs + TILE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(XT + 2 * SLAB);
+  uint64_t* kv_full = bars;
+  uint64_t* q_full = bars + 1;   // [3]
+  uint64_t* q_empty = bars + 4;  // [3]
+  uint64_t* o_full = bars + 7;
+  uint64_t* o_empty = bars + 8;
+  uint64_t* s_full = bars + 9;
+  uint64_t* dp_full = bars + 10;
+  uint64_t* p_ready = bars + 11;
+  uint64_t* ds_ready = bars + 12;
+  uint64_t* acc_done = bars + 13;
+  uint64_t* drain = bars + 14;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 15);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  // rows row0 .. row0+len-1 (a kept sequence, or with `seg` the kept tokens
+  // of sequence blockIdx.z); queries past len get P = dS = 0, keys past len
+  // are never stored.  Grid (kv head, key tile, sequence): one sequence's
+  // blocks are dispatched together, heaviest key tiles (kt = 0) first.
+  const int seq = blockIdx.z;
+  int row0, len;
+  if (seg) {
+    row0 = seg[seq];
+    len = seg[seq + 1] - row0;
+  } else {
+    if (seq >= *cnt) return;
+    row0 = seq * S;
+    len = S;
+  }
+  const int kt = blockIdx.y, g = blockIdx.x, grp = H / Hkv;
+  if (kt * 128 >= len) return;
+  const int nq = (len + 127) / 128;  // query tiles kt .. nq-1 overlap or follow the keys
+  const int nqs = nq - kt;
+  const int n_it = grp * nqs;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(kv_full, 1);
+    for (int s = 0; s < 3; ++s) {
+      mbar_init(&q_full[s], 1);
+      mbar_init(&q_empty[s], 1);
+    }
+    mbar_init(o_full, 1);
+    mbar_init(o_empty, 1);
+    mbar_init(s_full, 1);
+    mbar_init(dp_full, 1);
+    mbar_init(p_ready, 8);
+    mbar_init(ds_ready, 8);
+    mbar_init(acc_done, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (threadIdx.x < 128) {
+    // row r of XT: the two ones patterns, zero terms
+    const int r = threadIdx.x;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (u == 0) v = make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
+      if (u == 2) v = make_uint4(0u, 0x3F800000u, 0x3F803F80u, 0u);
+      *reinterpret_cast<uint4*>(XT + swz(r, u)) = v;
+      *reinterpret_cast<uint4*>(XT + SLAB + swz(r, u)) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    fence_proxy_async();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_s = tmem, t_dp = tmem + 128, t_dv = tmem + 256, t_dk = tmem + 384;
+
+  if (warp == 0) {
+    // ------------------------------------------------ producer (warp 0)
+    const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
+    if (lane == 0) {
+      mbar_arrive_expect_tx(kv_full, 2 * TILE);
+      for (int c = 0; c < NSL; ++c) {
+        tma_load_2d(Ks + c * SLAB, &tmkv, kcol + 64 * c, row0 + kt * 128, kv_full);
+        tma_load_2d(Vs + c * SLAB, &tmkv, vcol + 64 * c, row0 + kt * 128, kv_full);
+      }
+    }
+    const float sq_dh = sqrtf((float)DH);
+    // -lse sqrt(Dh) and -D of the 128 queries of step i, four a lane, loaded
+    // one step ahead so their latency stays off the Q copy's path
+    float xl[4], xd[4];
+    auto load_terms = [&](int i) {
+      const int h = g * grp + i / nqs, qt = kt + i % nqs;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int q = u * 32 + lane;
+        xl[u] = 0.f;
+        xd[u] = 0.f;
+        if (qt * 128 + q < len) {
+          const size_t at = (size_t)h * lse_ld + row0 + qt * 128 + q;
+          xl[u] = -lse[at] * sq_dh;
+          xd[u] = -Dvec[at];
+        }
+      }
+    };
+    if (n_it > 0) load_terms(0);
+    int nql = 0, nol = 0;
+    for (int i = 0; i < n_it; ++i) {
+      const int s = i % 3;
+      const int h = g * grp + i / nqs, qt = kt + i % nqs;
+      // Q_i and the terms of step i into stage s once step i-3 has released
+      // it; the copy is issued first (the barrier's phase cannot complete
+      // before the arrival below, which follows the terms)
+      if (!warp_wait(&q_empty[s], ((i / 3) & 1) ^ 1u, abort_flag, status)) break;
+      if (lane == 0)
+        for (int c = 0; c < NSL; ++c)
+          tma_load_2d(Qs + s * TILE + c * SLAB, &tmkv, h * DH + 64 * c, row0 + qt * 128, &q_full[s]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        uint32_t l0, l1, l2, d0, d1, d2;
+        split3_bf16(xl[u], l0, l1, l2);
+        split3_bf16(xd[u], d0, d1, d2);
+        *reinterpret_cast<uint4*>(s < 2 ? XT + swz(u * 32 + lane, 4 + 2 * s) : XT + SLAB + swz(u * 32 + lane, 0)) =
+            make_uint4(l0 | (l1 << 16), l2 | (d0 << 16), d1 | (d2 << 16), 0u);
+      }
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_expect_tx(&q_full[s], TILE);
+      if (i + 1 < n_it) load_terms(i + 1);
+      ++nql;
+      // dO_i once dV_{i-1} has read dO_{i-1}
+      if (!warp_wait(o_empty, (i & 1) ^ 1u, abort_flag, status)) break;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(o_full, TILE);
+        for (int c = 0; c < NSL; ++c)
+          tma_load_2d(dOs + c * SLAB, &tmo, h * DH + 64 * c, row0 + qt * 128, o_full);
+      }
+      ++nol;
+    }
+    if (lane == 0 && *abort_flag) {
+      // let every copy in flight land before the block exits
+      mbar_drain(kv_full, 0);
+      for (int i = nql > 3 ? nql - 3 : 0; i < nql; ++i) mbar_drain(&q_full[i % 3], (i / 3) & 1);
+      if (nol > 0) mbar_drain(o_full, (nol - 1) & 1);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    {  // the whole warp, converged; one elected lane issues
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);   // S^T, dP^T and the folds
+      constexpr uint32_t ID_KV = idesc_bf16(128, DH, false, true);    // dV, dK (B = dO / Q, MN-major)
+      // shared-memory descriptors built once; an MMA's operand is its base
+      // plus (byte offset >> 4) in the address field (every tile lies below
+      // 256 KB, so the 14-bit field never carries)
+      const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
+      const uint64_t DQMN = sdesc(smem_u32(Qs), SLAB, 1024), DOMN = sdesc(smem_u32(dOs), SLAB, 1024);
+      const uint64_t DX = sdesc(smem_u32(XT), 16, 1024), DX2 = sdesc(smem_u32(XT + SLAB), 16, 1024);
+      // B operand of the fold MMAs: the terms of Q stage s
+      auto terms = [&](int s) { return s < 2 ? DX + (uint64_t)(((2 + s) * 32) >> 4) : DX2; };
+      // offset of the K = 16 chunk kk of a K-major 128 x 128 tile (two slabs)
+      auto kmaj = [](int kk) { return (uint64_t)(((kk >> 2) * SLAB + (kk & 3) * 32) >> 4); };
+      // S^T_i = K Q_i^T - lse sqrt(Dh) (ones pattern 0 times the terms)
+      auto issue_s = [&](int i) -> bool {
+        const int s = i % 3;
+        if (!mbar_wait_conv(&q_full[s], (i / 3) & 1, abort_flag, status)) return false;
+        tc_fence_after();
+        const uint64_t st = (uint64_t)((s * TILE) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16_w(t_s, DK + kmaj(kk), DQ + st + kmaj(kk), ID_S, kk > 0);
+        mma_bf16_w(t_s, DX, terms(s), ID_S, 1u);
+        mma_commit_w(s_full);
+        return true;
+      };
+      bool ok = mbar_wait_conv(kv_full, 0, abort_flag, status) && issue_s(0);
+      for (int i = 0; ok && i < n_it; ++i) {
+        const int s = i % 3;
+        const uint64_t st = (uint64_t)((s * TILE) >> 4);
+        // dP^T_i = V dO_i^T - D (ones pattern 1 times the terms), over the
+        // dS^T_{i-1} columns (dK_{i-1}, issued before, reads them first)
+        if (!mbar_wait_conv(o_full, i & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16_w(t_dp, DV + kmaj(kk), DO + kmaj(kk), ID_S, kk > 0);
+        mma_bf16_w(t_dp, DX + (uint64_t)(32 >> 4), terms(s), ID_S, 1u);
+        mma_commit_w(dp_full);
+        // dV += P^T_i dO_i: A = P^T from TMEM (queries 64h..64h+63 as bf16
+        // pairs in columns 64h..64h+31), B = dO MN-major
+        if (!mbar_wait_conv(p_ready, i & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_ta_w(t_dv, t_s + 64 * (kk >> 2) + 8 * (kk & 3), DOMN + (uint64_t)((kk * 2048) >> 4), ID_KV,
+                      (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit_w(o_empty);
+        // S^T_{i+1} ahead of the product that waits for dS^T_i
+        if (i + 1 < n_it && !issue_s(i + 1)) { ok = false; break; }
+        if (!mbar_wait_conv(ds_ready, i & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+        // dK += dS^T_i Q_i (contraction over the 128 queries): A = dS^T from
+        // TMEM (queries 64h..64h+63 as bf16 pairs in dP^T columns
+        // 64h..64h+31), B = Q MN-major
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_ta_w(t_dk, t_dp + 64 * (kk >> 2) + 8 * (kk & 3), DQMN + st + (uint64_t)((kk * 2048) >> 4), ID_KV,
+                      (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit_w(&q_empty[s]);
+      }
+      if (ok) {
+        mma_commit_w(acc_done);
+      } else {
+        mma_commit_w(drain);
+        if (lane == 0) mbar_drain(drain, 0);
+        __syncwarp();
+      }
+    }
+  } else {
+    // ------------------------------------------------ P / dS (warps 2..9)
+    // two warps per TMEM lane quadrant: warps 2..5 take queries 0..63 of the
+    // step, warps 6..9 queries 64..127, one key per thread
+    const int quad = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const int r = quad * 32 + lane;  // key within the tile
+    const int key = kt * 128 + r;
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const uint32_t t_sh = t_s + half * 64 + lane_off, t_dph = t_dp + half * 64 + lane_off;
+    const float sl2 = kLog2e * rsqrtf((float)DH);
+    bool ok = true;
+    for (int i = 0; i < n_it; ++i) {
+      const int qt = kt + i % nqs;
+      // ALiBi: logit bias slope2 (key - query) of this step's query head
+      const float slope2 = ALIBI ? alibi[g * grp + i / nqs] * kLog2e : 0.f;
+      const int qbase = qt * 128 + half * 64 - key;  // query c is visible iff qbase + c >= 0
+      const int qlim = len - (qt * 128 + half * 64);  // and exists iff c < qlim (warp-uniform)
+      // mask only where some of the warp's 32 keys do not see all 64 queries,
+      // or the queries run past the sequence (warp-uniform)
+      const bool full = __shfl_sync(0xffffffffu, qbase, 31) >= 0 && qlim >= 64;
+      // ---- phase A: P^T from S^T (lse folded in)
+      if (!warp_wait(s_full, i & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      uint32_t pk[32];
+      auto phase_a = [&](auto masked) {
+        constexpr bool MASK = decltype(masked)::value;
+        const uint64_t sl2x2 = f2_pack(sl2, sl2);
+        const float b0 = slope2 * (float)(-qbase);  // bias of query c: b0 - slope2 c
+        const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
+        uint32_t sr[2][32];
+        tmem_ld32_nw(t_sh, sr[0]);
+        tmem_ld32_nw(t_sh + 32, sr[1]);
+        tmem_wait_ld();
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+#pragma unroll
+          for (int c2 = 0; c2 < 32; c2 += 2) {
+            const int c = h2 * 32 + c2;
+            uint64_t x2 = f2_mul(f2_pack(__uint_as_float(sr[h2][c2]), __uint_as_float(sr[h2][c2 + 1])), sl2x2);
+            if constexpr (ALIBI) x2 = f2_add(x2, f2_fma(f2_pack((float)c, (float)(c + 1)), nsx2, b0x2));
+            float x0, x1;
+            f2_unpack(x2, x0, x1);
+            float p0 = ex2(x0), p1 = ex2(x1);
+            if constexpr (MASK) {
+              p0 = (qbase + c >= 0 && c < qlim) ? p0 : 0.f;
+              p1 = (qbase + c + 1 >= 0 && c + 1 < qlim) ? p1 : 0.f;
+            }
+            pk[c >> 1] = bf16x2_bits(p0, p1);
+          }
+        }
+      };
+      if (full) phase_a(std::false_type{});
+      else phase_a(std::true_type{});
+      // P^T (queries 64 half .. 64 half + 63) over this warp's own S^T columns
+      tmem_st32u(t_sh, pk);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_ready);
+      // ---- phase B: dS^T = P^T (dP^T - D) (D folded in)
+      if (!warp_wait(dp_full, i & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      // dS^T over the packed P^T in place (pk), both halves loaded at once
+      uint32_t dr[2][32];
+      tmem_ld32_nw(t_dph, dr[0]);
+      tmem_ld32_nw(t_dph + 32, dr[1]);
+      tmem_wait_ld();
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+#pragma unroll
+        for (int c2 = 0; c2 < 32; c2 += 2) {
+          const uint32_t pw = pk[(h2 * 32 + c2) >> 1];
+          const uint64_t pp = f2_pack(__uint_as_float(pw << 16), __uint_as_float(pw & 0xFFFF0000u));
+          float d0, d1;
+          f2_unpack(f2_mul(pp, f2_pack(__uint_as_float(dr[h2][c2]), __uint_as_float(dr[h2][c2 + 1]))), d0, d1);
+          if (!full) {  // rows past the sequence may hold anything: select, do not multiply
+            const int c = h2 * 32 + c2;
+            d0 = (qbase + c >= 0 && c < qlim) ? d0 : 0.f;
+            d1 = (qbase + c + 1 >= 0 && c + 1 < qlim) ? d1 : 0.f;
+          }
+          pk[(h2 * 32 + c2) >> 1] = bf16x2_bits(d0, d1);
+        }
+      }
+      // dS^T (queries 64 half .. 64 half + 63) over this warp's own dP^T columns
+      tmem_st32u(t_dph, pk);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ds_ready);
+    }
+    if (ok && warp_wait(acc_done, 0, abort_flag, status)) {
+      tc_fence_after();
+      const bool kvalid = key < len;
+      if (half == 0) {
+        // dK (times c) with the inverse rotation at the key's position
+        const float c = rsqrtf((float)DH);
+        const int kpos = kvalid ? row_pos(tok, S, row0 + key) : 0;  // rows past the segment are not read
+        bf16* krow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + g) * DH;
+#pragma unroll 1
+        for (int cc = 0; cc < DH / 64; ++cc) {
+          float k1[32], k2[32];
+          tmem_ld32(t_dk + cc * 32 + lane_off, k1);
+          tmem_ld32(t_dk + DH / 2 + cc * 32 + lane_off, k2);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const float p1 = c * k1[e], p2 = c * k2[e];
+            float cs = 1.f, sn = 0.f;
+            if (rcos) {
+              cs = rcos[(size_t)kpos * (DH / 2) + cc * 32 + e];
+              sn = rsin[(size_t)kpos * (DH / 2) + cc * 32 + e];
+            }
+            k1[e] = p1 * cs + p2 * sn;
+            k2[e] = p2 * cs - p1 * sn;
+          }
+          if (kvalid) {
+            st_bf16x32_(krow + cc * 32, k1);
+            st_bf16x32_(krow + DH / 2 + cc * 32, k2);
+          }
+        }
+      } else {
+        bf16* vrow = dqkv + (long long)(row0 + key) * ldq + (long long)(H + Hkv + g) * DH;
+#pragma unroll 1
+        for (int cc = 0; cc < DH / 32; ++cc) {
+          float u[32];
+          tmem_ld32(t_dv + cc * 32 + lane_off, u);
+          if (kvalid) st_bf16x32_(vrow + cc * 32, u);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// dQ of one (128-query tile, query head h, kept sequence): for each key tile
+// j <= qt, S_j = Q K_j^T and dP_j = dO V_j^T (M = 128 queries, N = 128 keys),
+// dS_j = P_j (dP_j - D) with P_j = exp2(S_j c - lse log2 e), and
+// dQ += dS_j K_j.  320 threads:
+//   warp 0      TMA: Q and dO once, then K_j (three stages) and V_j (two)
+//   warp 1      TMEM allocation and the MMAs, in the order S_0, dP_0, then
+//               per step S_{j+1}, dQ += dS_j K_j, dP_{j+1}: S is double-
+//               buffered, so S_{j+1} runs while the softmax works on step j
+//   warps 2..9  softmax, one query row and 64 keys per thread (two warps per
+//               TMEM lane quadrant), lse and D of the row held in registers:
+//               P_j from S_j, then dS_j from dP_j, written as bf16 over the
+//               thread's own S_j columns (the A operand of dQ += dS_j K_j);
+//               at the end dQ (times c, with the inverse rotation at the
+//               query's position) from TMEM to dqkv
+// TMEM columns: S_0 0-127, S_1 128-255, dP 256-383, dQ 384-511.
+template <int DH, bool ALIBI>
+__global__ void __launch_bounds__(320, 1)
+    attn_bwd_q_kernel(const __grid_constant__ CUtensorMap tmkv, const __grid_constant__ CUtensorMap tmo,
+                      const float* __restrict__ lse, const float* __restrict__ Dvec, int lse_ld,
+                      bf16* __restrict__ dqkv, int ldq, const int* __restrict__ cnt, int S, int H, int Hkv,
+                      const float* __restrict__ rcos, const float* __restrict__ rsin,
+                      const float* __restrict__ alibi, const int* __restrict__ seg, const int* __restrict__ tok,
+                      int* status) {
+  constexpr int NSL = DH / 64;           // 64-column slabs of a row
+  constexpr uint32_t TILE = NSL * SLAB;  // 128 rows x DH bf16
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Qs = smem;
+  uint8_t* dOs = Qs + TILE;
+  uint8_t* Ks = dOs + TILE;      // [3] stages: K_j is read by S_j and, a step later, by dQ
+  uint8_t* Vs = Ks + 3 * TILE;   // [2] stages
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + 2 * TILE);
+  uint64_t* qo_full = bars;
+  uint64_t* k_full = bars + 1;   // [3]
+  uint64_t* k_empty = bars + 4;  // [3]
+  uint64_t* v_full = bars + 7;   // [2]
+  uint64_t* v_empty = bars + 9;  // [2]
+  uint64_t* s_full = bars + 11;  // [2] per S buffer
+  uint64_t* dp_full = bars + 13;
+  uint64_t* ds_ready = bars + 14;
+  uint64_t* acc_done = bars + 15;
+  uint64_t* drain = bars + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  // rows row0 .. row0+len-1 as in the forward; query rows past len are not
+  // stored (P = dS = 0 for them), keys past len are hidden by causality.
+  // Grid (query head, query tile, sequence), heaviest query tiles first.
+  const int seq = blockIdx.z;
+  int row0, len;
+  if (seg) {
+    row0 = seg[seq];
+    len = seg[seq + 1] - row0;
+  } else {
+    if (seq >= *cnt) return;
+    row0 = seq * S;
+    len = S;
+  }
+  const int qt = (int)gridDim.y - 1 - (int)blockIdx.y;
+  if (qt * 128 >= len) return;
+  const int h = blockIdx.x, g = (h * Hkv) / H;
+  // key tiles qt, qt-1, .., 0 (step j takes tile qt - j): the blocks of a
+  // head group then fetch different K / V tiles at a time
+  const int n_k = qt + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(qo_full, 1);
+    for (int s = 0; s < 3; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+      mbar_init(&s_full[s], 1);
+    }
+    mbar_init(dp_full, 1);
+    mbar_init(ds_ready, 8);
+    mbar_init(acc_done, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_dp = tmem + 256, t_dq = tmem + 384;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      const int kcol = (H + g) * DH, vcol = (H + Hkv + g) * DH;
+      mbar_arrive_expect_tx(qo_full, 2 * TILE);
+      for (int c = 0; c < NSL; ++c) {
+        tma_load_2d(Qs + c * SLAB, &tmkv, h * DH + 64 * c, row0 + qt * 128, qo_full);
+        tma_load_2d(dOs + c * SLAB, &tmo, h * DH + 64 * c, row0 + qt * 128, qo_full);
+      }
+      int nkl = 0, nvl = 0;
+      for (int j = 0; j < n_k; ++j) {
+        const int s = j & 1, sk = j % 3;
+        if (!mbar_wait(&k_empty[sk], ((j / 3) & 1) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&k_full[sk], TILE);
+        for (int c = 0; c < NSL; ++c)
+          tma_load_2d(Ks + sk * TILE + c * SLAB, &tmkv, kcol + 64 * c, row0 + (qt - j) * 128, &k_full[sk]);
+        ++nkl;
+        if (!mbar_wait(&v_empty[s], ((j >> 1) & 1) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&v_full[s], TILE);
+        for (int c = 0; c < NSL; ++c)
+          tma_load_2d(Vs + s * TILE + c * SLAB, &tmkv, vcol + 64 * c, row0 + (qt - j) * 128, &v_full[s]);
+        ++nvl;
+      }
+      if (*abort_flag) {
+        // let every copy in flight land before the block exits
+        mbar_drain(qo_full, 0);
+        for (int j = nkl > 3 ? nkl - 3 : 0; j < nkl; ++j) mbar_drain(&k_full[j % 3], (j / 3) & 1);
+        for (int j = nvl > 2 ? nvl - 2 : 0; j < nvl; ++j) mbar_drain(&v_full[j & 1], (j >> 1) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    {  // the whole warp, converged; one elected lane issues
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S, dP (both operands K-major)
+      constexpr uint32_t ID_Q = idesc_bf16(128, DH, false, true);    // dQ (A = dS from TMEM, B = K MN-major)
+      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DO = sdesc(smem_u32(dOs), 16, 1024);
+      const uint64_t DK = sdesc(smem_u32(Ks), 16, 1024), DV = sdesc(smem_u32(Vs), 16, 1024);
+      const uint64_t DKMN = sdesc(smem_u32(Ks), SLAB, 1024);
+      auto kmaj = [](int kk) { return (uint64_t)(((kk >> 2) * SLAB + (kk & 3) * 32) >> 4); };
+      // S_j = Q K_j^T into S buffer j & 1
+      auto issue_s = [&](int j) -> bool {
+        const int s = j & 1, sk = j % 3;
+        if (!mbar_wait_conv(&k_full[sk], (j / 3) & 1, abort_flag, status)) return false;
+        tc_fence_after();
+        const uint64_t st = (uint64_t)((sk * TILE) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16_w(tmem + s * 128, DQ + kmaj(kk), DK + st + kmaj(kk), ID_S, kk > 0);
+        mma_commit_w(&s_full[s]);
+        return true;
+      };
+      // dP_j = dO V_j^T
+      auto issue_dp = [&](int j) -> bool {
+        const int s = j & 1;
+        if (!mbar_wait_conv(&v_full[s], (j >> 1) & 1, abort_flag, status)) return false;
+        tc_fence_after();
+        const uint64_t st = (uint64_t)((s * TILE) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) mma_bf16_w(t_dp, DO + kmaj(kk), DV + st + kmaj(kk), ID_S, kk > 0);
+        mma_commit_w(dp_full);
+        mma_commit_w(&v_empty[s]);
+        return true;
+      };
+      bool ok = mbar_wait_conv(qo_full, 0, abort_flag, status) && issue_s(0) && issue_dp(0);
+      for (int j = 0; ok && j < n_k; ++j) {
+        const int s = j & 1;
+        // S_{j+1} into the other buffer (its dS_{j-1} was read by dQ, issued before)
+        if (j + 1 < n_k && !issue_s(j + 1)) { ok = false; break; }
+        // dQ += dS_j K_j: A = dS_j from TMEM (keys 64h..64h+63 as bf16 pairs
+        // in columns 64h..64h+31 of S buffer s), B = K_j MN-major
+        if (!mbar_wait_conv(ds_ready, j & 1, abort_flag, status)) { ok = false; break; }
+        tc_fence_after();
+        const uint64_t sk = (uint64_t)(((j % 3) * TILE) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_ta_w(t_dq, tmem + s * 128 + 64 * (kk >> 2) + 8 * (kk & 3), DKMN + sk + (uint64_t)((kk * 2048) >> 4),
+                      ID_Q, (j > 0 || kk > 0) ? 1u : 0u);
+        mma_commit_w(&k_empty[j % 3]);
+        // dP_{j+1} over dP_j, which the softmax warps have read (ds_ready)
+        if (j + 1 < n_k && !issue_dp(j + 1)) { ok = false; break; }
+      }
+      if (ok) {
+        mma_commit_w(acc_done);
+      } else {
+        mma_commit_w(drain);
+        if (lane == 0) mbar_drain(drain, 0);
+        __syncwarp();
+      }
+    }
+  } else {
+    // ------------------------------------------------ softmax (warps 2..9)
+    // two warps per TMEM lane quadrant: warps 2..5 take keys 0..63 of each
+    // key tile, warps 6..9 keys 64..127, one query row per thread
+    const int quad = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const int r = quad * 32 + lane;  // query row within the tile
+    const int q = qt * 128 + r;      // query within the sequence
+    const bool qvalid = q < len;
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const float sl2 = kLog2e * rsqrtf((float)DH);
+    const float slope2 = ALIBI ? alibi[h] * kLog2e : 0.f;
+    float lse2 = 0.f, dq = 0.f;  // lse log2(e) and D of this row
+    if (qvalid) {
+      const size_t at = (size_t)h * lse_ld + row0 + q;
+      lse2 = lse[at] * kLog2e;
+      dq = Dvec[at];
+    }
+    // rows past the sequence: P = dS = 0 (warp-uniform test below)
+    const bool any_invalid = __any_sync(0xffffffffu, !qvalid);
+    bool ok = true;
+    for (int j = 0; j < n_k; ++j) {
+      const int s = j & 1;
+      const uint32_t t_sh = tmem + s * 128 + half * 64 + lane_off, t_dph = t_dp + half * 64 + lane_off;
+      // key c of this half is visible iff kbase + c <= q
+      const int kbase = (qt - j) * 128 + half * 64;
+      const bool masked = (j == 0) || any_invalid;  // the diagonal tile comes first (warp-uniform)
+      if (!warp_wait(&s_full[s], (j >> 1) & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      // P = exp2(S c - lse log2 e (+ ALiBi bias)) for 64 keys, kept as bf16 pairs
+      uint32_t pk[32];
+      {
+        const uint64_t sl2x2 = f2_pack(sl2, sl2), nl2 = f2_pack(-lse2, -lse2);
+        const float b0 = slope2 * (float)(kbase - q);  // bias of key c: b0 + slope2 c
+        const uint64_t sx2 = f2_pack(slope2, slope2), b0x2 = f2_pack(b0, b0);
+        uint32_t sr[2][32];
+        tmem_ld32_nw(t_sh, sr[0]);
+        tmem_ld32_nw(t_sh + 32, sr[1]);
+        tmem_wait_ld();
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+#pragma unroll
+          for (int c2 = 0; c2 < 32; c2 += 2) {
+            const int c = h2 * 32 + c2;
+            uint64_t add = nl2;
+            if constexpr (ALIBI) add = f2_add(nl2, f2_fma(f2_pack((float)c, (float)(c + 1)), sx2, b0x2));
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[h2][c2]), __uint_as_float(sr[h2][c2 + 1])), sl2x2, add), x0, x1);
+            float p0 = ex2(x0), p1 = ex2(x1);
+            if (masked) {  // select, do not multiply: rows past the sequence may hold anything
+              p0 = (qvalid && kbase + c <= q) ? p0 : 0.f;
+              p1 = (qvalid && kbase + c + 1 <= q) ? p1 : 0.f;
+            }
+            pk[c >> 1] = bf16x2_bits(p0, p1);
+          }
+        }
+      }
+      // dS = P (dP - D), written as bf16 pairs over this warp's own S columns
+      if (!warp_wait(dp_full, j & 1, abort_flag, status)) { ok = false; break; }
+      tc_fence_after();
+      {
+        // dS over the packed P in place (pk), both halves loaded at once
+        const uint64_t nd2 = f2_pack(-dq, -dq);
+        uint32_t dr[2][32];
+        tmem_ld32_nw(t_dph, dr[0]);
+        tmem_ld32_nw(t_dph + 32, dr[1]);
+        tmem_wait_ld();
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+#pragma unroll
+          for (int c2 = 0; c2 < 32; c2 += 2) {
+            const int c = h2 * 32 + c2;
+            const uint32_t pw = pk[c >> 1];
+            const uint64_t pp = f2_pack(__uint_as_float(pw << 16), __uint_as_float(pw & 0xFFFF0000u));
+            float d0, d1;
+            f2_unpack(f2_mul(pp, f2_add(f2_pack(__uint_as_float(dr[h2][c2]), __uint_as_float(dr[h2][c2 + 1])), nd2)),
+                      d0, d1);
+            if (masked) {
+              d0 = (qvalid && kbase + c <= q) ? d0 : 0.f;
+              d1 = (qvalid && kbase + c + 1 <= q) ? d1 : 0.f;
+            }
+            pk[c >> 1] = bf16x2_bits(d0, d1);
+          }
+        }
+      }
+      tmem_st32u(t_sh, pk);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ds_ready);
+    }
+    // dQ times c with the inverse rotation at the query's position: this
+    // thread takes the pairs (i, i + DH/2), i = off .. off + 31 (head size
+    // 64: the first warp of each quadrant alone)
+    const int off = DH == 128 ? half * 32 : 0;
+    if (ok && warp_wait(acc_done, 0, abort_flag, status) && (DH == 128 || half == 0)) {
+      tc_fence_after();
+      const float c = rsqrtf((float)DH);
+      const int pos = qvalid ? row_pos(tok, S, row0 + q) : 0;
+      float a1[32], a2[32];
+      tmem_ld32(t_dq + off + lane_off, a1);
+      tmem_ld32(t_dq + DH / 2 + off + lane_off, a2);
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        const float p1 = c * a1[e], p2 = c * a2[e];
+        float cs = 1.f, sn = 0.f;
+        if (rcos) {
+          cs = rcos[(size_t)pos * (DH / 2) + off + e];
+          sn = rsin[(size_t)pos * (DH / 2) + off + e];
+        }
+        a1[e] = p1 * cs + p2 * sn;
+        a2[e] = p2 * cs - p1 * sn;
+      }
+      if (qvalid) {
+        bf16* qrow = dqkv + (long long)(row0 + q) * ldq + (long long)h * DH;
+        st_bf16x32_(qrow + off, a1);
+        st_bf16x32_(qrow + DH / 2 + off, a2);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+template <int DH, bool ALIBI>
+cudaError_t bwd_split(const bf16* qkv, int ldq, const bf16* dO, int ldo, const float* lse, const float* Dvec,
+                      bf16* dqkv, const int* cnt, int S, int H, int Hkv, int max_seqs, const float* rcos,
+                      const float* rsin, const float* alibi, const int* seg, const int* tok, int* status,
+                      cudaStream_t st) {
+  constexpr size_t TILE = (size_t)(DH / 64) * SLAB;
+  // dK / dV: K, V, 3 stages of Q, dO (six tiles) + XT (two slabs) +
+  // alignment + barriers
+  constexpr size_t smem_kv = 6 * TILE + 2 * SLAB + 1024 + 256;
+  // dQ: Q, dO, 3 stages of K, 2 of V (seven tiles) + alignment + barriers
+  constexpr size_t smem_q = 7 * TILE + 1024 + 256;
+  // once per process (initialisation of a function-local static is thread-safe)
+  static const cudaError_t attr = [] {
+    cudaError_t e = cudaFuncSetAttribute(attn_bwd_kv_kernel<DH, ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem_kv);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(attn_bwd_q_kernel<DH, ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)smem_q);
+    return e;
+  }();
+  if (attr != cudaSuccess) return attr;
+  CUtensorMap tkv, to;  // tiles of 128 rows x 64 columns: Q, K, V in qkv; dO
+  if (!make_map(&tkv, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
+  if (!make_map(&to, dO, (uint64_t)ldo, (uint64_t)max_seqs * S, (uint64_t)ldo, 64, 128)) return cudaErrorInvalidValue;
+  attn_bwd_kv_kernel<DH, ALIBI><<<dim3(Hkv, S / 128, max_seqs), 320, smem_kv, st>>>(
+      tkv, to, lse, Dvec, max_seqs * S, dqkv, ldq, cnt, S, H, Hkv, rcos, rsin, alibi, seg, tok, status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  attn_bwd_q_kernel<DH, ALIBI><<<dim3(H, S / 128, max_seqs), 320, smem_q, st>>>(
+      tkv, to, lse, Dvec, max_seqs * S, dqkv, ldq, cnt, S, H, Hkv, rcos, rsin, alibi, seg, tok, status);
   return cudaGetLastError();
 }
 }  // namespace
 
 bool attn_tc_supported(int S, int Dh) { return S % 128 == 0 && (Dh == 64 || Dh == 128); }
 
-bool attn_bwd_tc_supported(int S, int Dh) { return S % 128 == 0 && Dh == 128; }
+bool attn_bwd_tc_supported(int S, int Dh) { return S % 128 == 0 && (Dh == 64 || Dh == 128); }
 
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, const int* seg,
-                               const int* tok, int* status, cudaStream_t st) {
+                               int Dh, int max_seqs, const float* rcos, const float* rsin, const float* alibi,
+                               const int* seg, const int* tok, int* status, cudaStream_t st) {
+  if (Dh == 64) {  // dQ, dK, dV straight into dqkv (two kernels, no float32 dQ)
+    if (alibi)
+      return bwd_split<64, true>(qkv, ldqkv, dO, ldo, lse, Dvec, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                                 seg, tok, status, st);
+    return bwd_split<64, false>(qkv, ldqkv, dO, ldo, lse, Dvec, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                                seg, tok, status, st);
+  }
   cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)max_seqs * S * H * 128 * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  if (alibi)
-    return bwd_tc<true>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
-                        seg, tok, status, st);
-  return bwd_tc<false>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
-                       seg, tok, status, st);
+  e = alibi ? bwd_tc<true>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                           seg, tok, status, st)
+            : bwd_tc<false>(qkv, ldqkv, dO, ldo, lse, Dvec, dq_acc, dqkv, cnt, S, H, Hkv, max_seqs, rcos, rsin, alibi,
+                            seg, tok, status, st);
+  if (e != cudaSuccess) return e;
+  // dQ from the float32 buffer: scaled and rotated into dqkv
+  return launch_dq_finish(dq_acc, dqkv, ldqkv, H, 128, rcos, rsin, cnt, S, max_seqs * S, tok, st);
 }
 
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,

@@ -169,14 +169,16 @@ bool attn_tc_supported(int S, int Dh);
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
                                int Hkv, int Dh, int max_seqs, const float* alibi, const int* seg, int* status,
                                cudaStream_t st);
-// tcgen05 flash attention backward (head size 128, S % 128 == 0); zeroes
-// dq_acc and accumulates dQ (unscaled) into it.
+// tcgen05 flash attention backward (head sizes 64 and 128, S % 128 == 0):
+// dQ (scaled by 1/sqrt(Dh)), dK and dV into dqkv, dQ and dK with the inverse
+// RoPE applied (rcos = null: no rotation).  Head size 128 accumulates dQ in
+// dq_acc (zeroed here) and finishes it with launch_dq_finish; head size 64
+// does not touch dq_acc.
 bool attn_bwd_tc_supported(int S, int Dh);
-// dK leaves with the inverse RoPE applied (rcos = null: no rotation).
 cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int ldo, const float* lse,
                                const float* Dvec, float* dq_acc, bf16* dqkv, const int* cnt, int S, int H, int Hkv,
-                               int max_seqs, const float* rcos, const float* rsin, const float* alibi, const int* seg,
-                               const int* tok, int* status, cudaStream_t st);
+                               int Dh, int max_seqs, const float* rcos, const float* rsin, const float* alibi,
+                               const int* seg, const int* tok, int* status, cudaStream_t st);
 // dqkv[:, q heads] = inverse-RoPE(dq_acc / sqrt(Dh)) as bf16 (rcos = null: no rotation);
 // rows and positions as launch_rope_apply
 cudaError_t launch_dq_finish(const float* dq_acc, bf16* dqkv, int ldqkv, int H, int Dh, const float* rcos,
