@@ -449,8 +449,8 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 
 
 // ---------------------------------------------------------------------------
-// Forward, head size 128 without a position bias: two 128-query tiles per CTA
-// ("ping-pong").  Each tile has its own softmax group of four warps with one
+// Forward, head size 128 (with or without the ALiBi bias): two 128-query
+// tiles per CTA ("ping-pong").  Each tile has its own softmax group of four warps with one
 // query row and all 128 keys of a K tile per thread, so no two warps share a
 // row; the MMA warp alternates between the groups, and one group's softmax
 // runs while the tensor pipe works for the other:
@@ -467,11 +467,37 @@ cudaError_t fwd_tc(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // the group may rescale O_g as soon as S_g(j) is ready.  Tile B is skipped
 // when the sequence ends before it.
 constexpr int PP_NSK = 3, PP_NSV = 2;
+// Pairs (of the 16 in each 32-key chunk) whose exponentials run on the FMA
+// pipe (ex2_poly2) instead of MUFU: the 128 x 128 exponentials of a tile
+// take as many cycles at 16 a clock as the tile's two MMAs.
+constexpr int PP_POLY = 0;
 
+// 2^x for two values on the FMA pipe: x = n + f with n = rint(x) and f in
+// [-1/2, 1/2]; 2^f = 1 + f (C1 + f (C2 + f C3)), the cubic fitted to 2^f on
+// that interval by minimising the largest relative error (1.0e-4 in float32,
+// below the 2^-9 half-ulp of the bf16 P is stored in); 2^n is added into the
+// exponent field.  x is clamped at -127, where the result is below 2^-126
+// instead of 0.
+__device__ __forceinline__ void ex2_poly2(float x0, float x1, float& y0, float& y1) {
+  constexpr float C1 = 0.6932829022407532f, C2 = 0.24221037328243256f, C3 = 0.05500858277082443f;
+  x0 = fmaxf(x0, -127.f);
+  x1 = fmaxf(x1, -127.f);
+  const float n0 = rintf(x0), n1 = rintf(x1);
+  const uint64_t f = f2_sub(f2_pack(x0, x1), f2_pack(n0, n1));
+  uint64_t p = f2_fma(f, f2_pack(C3, C3), f2_pack(C2, C2));
+  p = f2_fma(p, f, f2_pack(C1, C1));
+  p = f2_fma(p, f, f2_pack(1.f, 1.f));
+  float p0, p1;
+  f2_unpack(p, p0, p1);
+  y0 = __int_as_float(__float_as_int(p0) + ((int)n0 << 23));
+  y1 = __int_as_float(__float_as_int(p1) + ((int)n1 << 23));
+}
+
+template <bool ALIBI>
 __global__ void __launch_bounds__(320, 1)
     attn_fwd_pp_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o, int ldo, float* __restrict__ lse,
-                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv, const int* __restrict__ seg,
-                       int* status) {
+                       int lse_ld, const int* __restrict__ cnt, int S, int H, int Hkv,
+                       const float* __restrict__ alibi, const int* __restrict__ seg, int* status) {
   constexpr int DH = 128;
   constexpr uint32_t TILE = 2 * SLAB;  // one 128 x 128 bf16 tile (two 64-column slabs)
   extern __shared__ uint8_t smem_raw[];
@@ -571,53 +597,52 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else if (warp == 1) {
-    {  // the whole warp, converged; one elected lane issues
-      // ------------------------------------------------ MMA issuer
-      constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
-      constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
-      const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
-      const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
-      bool ok = mbar_wait_conv(q_full, 0, abort_flag, status);
-      for (int j = 0; ok && j <= nkt; ++j) {
-        if (j < nkt && !mbar_wait_conv(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
-        if (j >= 1 && !mbar_wait_conv(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
-          ok = false;
-          break;
-        }
-        for (int gi = 0; gi < 2; ++gi) {
-          const int nkg = gi ? nkB : nkA;
-          if (j >= 1 && j - 1 < nkg) {
-            // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
-            if (!mbar_wait_conv(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
-            tc_fence_after();
-            const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_bf16_ta_w(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
-                          (j > 1 || kk > 0) ? 1u : 0u);
-            if (j == nkg) mma_commit_w(&o_full[gi]);  // the group's last P V
-          }
-          if (j < nkg) {
-            // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
-            const uint64_t kb = DK + (uint64_t)(((j % PP_NSK) * TILE) >> 4);
-            const uint64_t qd = DQ + (uint64_t)((gi * TILE) >> 4);
-#pragma unroll
-            for (int kk = 0; kk < DH / 16; ++kk) {
-              const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
-              mma_bf16_w(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
-            }
-            mma_commit_w(&s_full[gi]);
-          }
-        }
-        if (!ok) break;
-        if (j < nkt) mma_commit_w(&k_empty[j % PP_NSK]);
-        if (j >= 1) mma_commit_w(&v_empty[(j - 1) % PP_NSV]);
+    // ------------------------------------------------ MMA issuer (whole warp, converged; one elected lane issues)
+    constexpr uint32_t ID_S = idesc_bf16(128, 128, false, false);  // S = Q K^T
+    constexpr uint32_t ID_O = idesc_bf16(128, DH, false, true);    // O += P V (V MN-major)
+    const uint64_t DQ = sdesc(smem_u32(Qs), 16, 1024), DK = sdesc(smem_u32(Ks), 16, 1024);
+    const uint64_t DV = sdesc(smem_u32(Vs), SLAB, 1024);
+    __syncwarp();
+    bool ok = mbar_wait_conv(q_full, 0, abort_flag, status);
+    for (int j = 0; ok && j <= nkt; ++j) {
+      if (j < nkt && !mbar_wait_conv(&k_full[j % PP_NSK], (j / PP_NSK) & 1, abort_flag, status)) { ok = false; break; }
+      if (j >= 1 && !mbar_wait_conv(&v_full[(j - 1) % PP_NSV], ((j - 1) / PP_NSV) & 1, abort_flag, status)) {
+        ok = false;
+        break;
       }
-      if (!ok) {
-        mma_commit_w(drain);
-        if (lane == 0) mbar_drain(drain, 0);
-        __syncwarp();
+      for (int gi = 0; gi < 2; ++gi) {
+        const int nkg = gi ? nkB : nkA;
+        if (j >= 1 && j - 1 < nkg) {
+          // O_g += P_g(j-1) V_{j-1}: A = P from the S_g columns, B = V MN-major
+          if (!mbar_wait_conv(&p_full[gi], (j - 1) & 1, abort_flag, status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t vb = DV + (uint64_t)((((j - 1) % PP_NSV) * TILE) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            mma_bf16_ta_w(tmem + 256 + gi * 128, tmem + gi * 128 + kk * 8, vb + ((kk * 2048) >> 4), ID_O,
+                            (j > 1 || kk > 0) ? 1u : 0u);
+          if (j == nkg) mma_commit_w(&o_full[gi]);  // the group's last P V
+        }
+        if (j < nkg) {
+          // S_g(j) = Q_g K_j^T, over the P_g the MMAs above have read
+          const uint64_t kb = DK + (uint64_t)(((j % PP_NSK) * TILE) >> 4);
+          const uint64_t qd = DQ + (uint64_t)((gi * TILE) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            const uint32_t off = ((kk >> 2) * SLAB + (kk & 3) * 32) >> 4;
+            mma_bf16_w(tmem + gi * 128, qd + off, kb + off, ID_S, kk > 0 ? 1u : 0u);
+          }
+          mma_commit_w(&s_full[gi]);
+        }
       }
+      if (!ok) break;
+      if (j < nkt) mma_commit_w(&k_empty[j % PP_NSK]);
+      if (j >= 1) mma_commit_w(&v_empty[(j - 1) % PP_NSV]);
+    }
+    if (!ok) {
+      mma_commit_w(drain);
+      if (lane == 0) mbar_drain(drain, 0);
+      __syncwarp();
     }
   } else {
     // ------------------------------------------------ softmax (warps 2..9)
@@ -629,20 +654,40 @@ __global__ void __launch_bounds__(320, 1)
     const int nkg = gi ? nkB : nkA;
     const int jdiag = 2 * qb + gi;  // the K tile on this query tile's diagonal
     const float sl2 = kLog2e * rsqrtf((float)DH);
+    // ALiBi: the exponent is x = S sl2 + slope2 (key - query), and the
+    // running max m is kept on x (the max of S alone, scaled, otherwise)
+    const float slope2 = ALIBI ? alibi[h] * kLog2e : 0.f;
+    const int qrow_t = qb * 256 + gi * 128 + r;  // this thread's query within the sequence
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nkg; ++j) {
       if (!warp_wait(&s_full[gi], j & 1, abort_flag, status)) { ok = false; break; }
       tc_fence_after();
       const bool diag = (j == jdiag);  // keys after the query are left out (block-uniform)
-      // pass 1: row max of the raw scores (the scale is positive)
+      // pass 1: row max of the raw scores (the scale is positive), or of x
+      // with ALiBi
       float mraw = -INFINITY;
+      const float b0 = slope2 * (float)(j * 128 - qrow_t);  // bias of key 0 of the tile
 #pragma unroll 1
       for (int c2 = 0; c2 < 2; ++c2) {
         uint32_t sr[2][32];
         tmem_ld32_nw(t_s + c2 * 64 + lane_off, sr[0]);
         tmem_ld32_nw(t_s + c2 * 64 + 32 + lane_off, sr[1]);
         tmem_wait_ld();
+        if constexpr (ALIBI) {
+          const uint64_t sl2x2 = f2_pack(sl2, sl2), sx2 = f2_pack(slope2, slope2);
+          const float bc = b0 + slope2 * (float)(c2 * 64);
+          const uint64_t bx2 = f2_pack(bc, bc);
+#pragma unroll
+          for (int e = 0; e < 64; e += 2) {
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1])),
+                             sl2x2, f2_fma(f2_pack((float)e, (float)(e + 1)), sx2, bx2)),
+                      x0, x1);
+            sr[e >> 5][e & 31] = __float_as_uint(x0);
+            sr[e >> 5][(e & 31) + 1] = __float_as_uint(x1);
+          }
+        }
         if (diag) {
 #pragma unroll
           for (int e = 0; e < 64; ++e)
@@ -653,7 +698,7 @@ __global__ void __launch_bounds__(320, 1)
             mraw = fmax3(mraw, __uint_as_float(sr[e >> 5][e & 31]), __uint_as_float(sr[e >> 5][(e & 31) + 1]));
         }
       }
-      const float mt = mraw * sl2;
+      const float mt = ALIBI ? mraw : mraw * sl2;
       const bool rescale = mt > m_used + kRescale;
       const float m_new = rescale ? mt : m_used;
       // O_g is rescaled in TMEM when any lane of the warp moved its max
@@ -676,6 +721,7 @@ __global__ void __launch_bounds__(320, 1)
       // pass 2: P = exp2(S c log2e - m) for 32 keys at a time, written as
       // bf16 pairs over S columns that have already been read
       const uint64_t sl2x2 = f2_pack(sl2, sl2), nm2 = f2_pack(-m_new, -m_new);
+      const uint64_t sx2 = f2_pack(slope2, slope2);
       uint64_t ls2 = f2_pack(0.f, 0.f);
 #pragma unroll 1
       for (int c = 0; c < 4; ++c) {
@@ -683,11 +729,20 @@ __global__ void __launch_bounds__(320, 1)
         tmem_ld32_nw(t_s + c * 32 + lane_off, sr);
         tmem_wait_ld();
         uint32_t pk[16];
+        const float bm = b0 + slope2 * (float)(c * 32) - m_new;  // ALiBi: bias of key 32c minus the max
+        const uint64_t bmx2 = f2_pack(bm, bm);
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           float x0, x1;
-          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, nm2), x0, x1);
-          float p0 = ex2(x0), p1 = ex2(x1);
+          const uint64_t add = ALIBI ? f2_fma(f2_pack((float)(2 * e), (float)(2 * e + 1)), sx2, bmx2) : nm2;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * e]), __uint_as_float(sr[2 * e + 1])), sl2x2, add), x0, x1);
+          float p0, p1;
+          if (e >= 16 - PP_POLY) {
+            ex2_poly2(x0, x1, p0, p1);
+          } else {
+            p0 = ex2(x0);
+            p1 = ex2(x1);
+          }
           if (diag) {
             p0 = (c * 32 + 2 * e <= r) ? p0 : 0.f;
             p1 = (c * 32 + 2 * e + 1 <= r) ? p1 : 0.f;
@@ -732,18 +787,19 @@ __global__ void __launch_bounds__(320, 1)
   }
 }
 
+template <bool ALIBI>
 cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const int* cnt, int S, int H, int Hkv,
-                   int max_seqs, const int* seg, int* status, cudaStream_t st) {
+                   int max_seqs, const float* alibi, const int* seg, int* status, cudaStream_t st) {
   // 2 Q, 3 K and 2 V tiles of 32 KB + alignment + barriers = 230,656 bytes (of 232,448)
   constexpr size_t smem = (size_t)(2 + PP_NSK + PP_NSV) * 2 * SLAB + 1024 + 256;
   // once per process (initialisation of a function-local static is thread-safe)
   static const cudaError_t attr =
-      cudaFuncSetAttribute(attn_fwd_pp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      cudaFuncSetAttribute(attn_fwd_pp_kernel<ALIBI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (attr != cudaSuccess) return attr;
   CUtensorMap tm;
   if (!make_map(&tm, qkv, (uint64_t)ldq, (uint64_t)max_seqs * S, (uint64_t)ldq, 64, 128)) return cudaErrorInvalidValue;
   dim3 grid(H, max_seqs, (S + 255) / 256);
-  attn_fwd_pp_kernel<<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, seg, status);
+  attn_fwd_pp_kernel<ALIBI><<<grid, 320, smem, st>>>(tm, o, ldo, lse, max_seqs * S, cnt, S, H, Hkv, alibi, seg, status);
   return cudaGetLastError();
 }
 
@@ -1945,12 +2001,12 @@ cudaError_t launch_attn_bwd_tc(const bf16* qkv, int ldqkv, const bf16* dO, int l
 cudaError_t launch_attn_fwd_tc(const bf16* qkv, int ldqkv, bf16* o, int ldo, float* lse, const int* cnt, int S, int H,
                                int Hkv, int Dh, int max_seqs, const float* alibi, const int* seg, int* status,
                                cudaStream_t st) {
-  if (alibi) {
-    if (Dh == 64) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
-    return fwd_tc<128, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  if (Dh == 64) {
+    if (alibi) return fwd_tc<64, true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+    return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
   }
-  if (Dh == 64) return fwd_tc<64, false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
-  return fwd_pp(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, seg, status, st);
+  if (alibi) return fwd_pp<true>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
+  return fwd_pp<false>(qkv, ldqkv, o, ldo, lse, cnt, S, H, Hkv, max_seqs, alibi, seg, status, st);
 }
 
 }  // namespace ldk
