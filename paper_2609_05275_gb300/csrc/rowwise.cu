@@ -676,23 +676,37 @@ cudaError_t launch_relu2(const T* u, const T* dh, T* out, const int* cnt, int S,
 template <typename T>
 __global__ void attn_rowdot_kernel(const T* __restrict__ dO, const T* __restrict__ O, int ld, int H, int Dh,
                                    const int* __restrict__ cnt, int S, int max_rows, float* __restrict__ Dvec) {
+  // one warp per row, all heads: lane l takes elements 8l + 256k of the row
+  // (16-byte loads), the Dh / 8 lanes of a head sum their dot products with
+  // shuffles, and the head's first lane stores it
   const long long M = (long long)(*cnt) * S;
   const int lane = threadIdx.x & 31;
+  const int HD = H * Dh, G = Dh / 8;  // lanes per head within a 256-element block
   const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
-  for (long long it = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); it < M * H; it += nwarps) {
-    const long long m = it / H;
-    const int h = (int)(it % H);
-    float s = 0.f;
-    for (int i = lane; i < Dh; i += 32) s += to_f(dO[m * ld + h * Dh + i]) * to_f(O[m * ld + h * Dh + i]);
-    s = warp_sum(s);
-    if (lane == 0) Dvec[(size_t)h * max_rows + m] = s;
+  for (long long m = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); m < M; m += nwarps) {
+    const T* a = dO + m * ld;
+    const T* b = O + m * ld;
+    for (int i0 = 0; i0 < HD; i0 += 256) {
+      const int i = i0 + lane * 8;
+      float s = 0.f;
+      if (i < HD) {
+        float x[8], y[8];
+        ld8(a + i, x);
+        ld8(b + i, y);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) s += x[e] * y[e];
+      }
+      for (int off = G >> 1; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      if (i < HD && (lane % G) == 0) Dvec[(size_t)(i / Dh) * max_rows + m] = s;
+    }
   }
 }
 
 template <typename T>
 cudaError_t launch_attn_rowdot(const T* dO, const T* O, int ld, int H, int Dh, const int* cnt, int S, int max_rows,
                                float* Dvec, cudaStream_t st) {
-  const int grid = grid_for((long long)max_rows * H, 8, device_sm_count() * 16);
+  if (Dh < 8 || Dh > 256 || (Dh & (Dh - 1))) return cudaErrorInvalidValue;  // head groups of Dh / 8 lanes
+  const int grid = grid_for((long long)max_rows, 8, device_sm_count() * 16);
   attn_rowdot_kernel<T><<<grid, 256, 0, st>>>(dO, O, ld, H, Dh, cnt, S, max_rows, Dvec);
   return cudaGetLastError();
 }
