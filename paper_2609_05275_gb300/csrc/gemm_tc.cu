@@ -568,6 +568,59 @@ __global__ void __launch_bounds__(192, 1)
             for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(srow + c)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
           }
         }
+      } else if (a.epi == EPI_SWIGLU_BWD) {
+        // the saved g and u of the next chunk are read while this one is
+        // finished (as the residual epilogue does), so their latency overlaps
+        // the TMEM load and the arithmetic
+        const bool rowok = row < M;
+        const bf16* gp = static_cast<const bf16*>(a.gu) + (size_t)(rowok ? row : 0) * 2 * a.F + (size_t)nb * BN;
+        uint4 gq[4], uq[4];
+        if (rowok && nb * BN < N) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            gq[i] = reinterpret_cast<const uint4*>(gp)[i];
+            uq[i] = reinterpret_cast<const uint4*>(gp + a.F)[i];
+          }
+        }
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float dh[32];
+          tmem_ld32(tbase + (uint32_t)c, dh);
+          const bool ok = rowok && nb * BN + c < N;
+          float g[32], u[32];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&gq[i]);
+            const __nv_bfloat162* u2 = reinterpret_cast<const __nv_bfloat162*>(&uq[i]);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float2 gf = __bfloat1622float2(g2[k]), uf = __bfloat1622float2(u2[k]);
+              g[8 * i + 2 * k] = gf.x;
+              g[8 * i + 2 * k + 1] = gf.y;
+              u[8 * i + 2 * k] = uf.x;
+              u[8 * i + 2 * k + 1] = uf.y;
+            }
+          }
+          if (rowok && c + 32 < BN && nb * BN + c + 32 < N) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              gq[i] = reinterpret_cast<const uint4*>(gp + c + 32)[i];
+              uq[i] = reinterpret_cast<const uint4*>(gp + a.F + c + 32)[i];
+            }
+          }
+          if (ok) {
+            float du[32];  // dg is written over dh
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const float sg = 1.0f / (1.0f + expf(-g[e]));
+              du[e] = dh[e] * g[e] * sg;
+              dh[e] = dh[e] * u[e] * sg * (1.0f + g[e] * (1.0f - sg));
+            }
+            bf16* dp = static_cast<bf16*>(a.D) + (size_t)row * 2 * a.F + nb * BN + c;
+            st_bf16x32(dp, dh);
+            st_bf16x32(dp + a.F, du);
+          }
+        }
       } else {
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
