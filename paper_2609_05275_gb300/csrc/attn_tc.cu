@@ -824,11 +824,19 @@ cudaError_t fwd_pp(const bf16* qkv, int ldq, bf16* o, int ldo, float* lse, const
 // P^T 448-479 / 480-511.
 constexpr uint32_t HSLAB = 64 * 128;  // bytes of a 64-row x 64-column bf16 slab
 
-// Values 4 e4 .. 4 e4 + 3 of p (shared memory); p is 16-byte aligned when
-// off == 0 (warp-uniform), else read one by one.
-__device__ __forceinline__ float4 ld4s(const float* p, int e4, int off) {
-  if (off == 0) return reinterpret_cast<const float4*>(p)[e4];
-  return make_float4(p[4 * e4], p[4 * e4 + 1], p[4 * e4 + 2], p[4 * e4 + 3]);
+// Values 4 e4 .. 4 e4 + 3 of p (shared memory), read by every lane of the
+// warp at the same address.  Four 32-bit shared-space loads: a generic
+// 128-bit read of such a broadcast cost about ten shared-memory wavefronts
+// (1,300 a step of the backward), an ld.shared.v4 about five, a 32-bit
+// ld.shared one.
+__device__ __forceinline__ float lds_f32(uint32_t a) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ float4 ld4s(const float* p, int e4) {
+  const uint32_t a = smem_u32(p + 4 * e4);
+  return make_float4(lds_f32(a), lds_f32(a + 4), lds_f32(a + 8), lds_f32(a + 12));
 }
 
 template <bool ALIBI>
@@ -1048,7 +1056,7 @@ __global__ void __launch_bounds__(448, 1)
         const uint64_t nsx2 = f2_pack(-slope2, -slope2), b0x2 = f2_pack(b0, b0);
 #pragma unroll
         for (int e4 = 0; e4 < 8; ++e4) {
-          const float4 lq = ld4s(lsrc, e4, voff), dq = ld4s(dsrc, e4, voff);
+          const float4 lq = ld4s(lsrc, e4), dq = ld4s(dsrc, e4);
           uint64_t nl[2] = {f2_mul(f2_pack(lq.x, lq.y), nlog2), f2_mul(f2_pack(lq.z, lq.w), nlog2)};
           if constexpr (ALIBI) {
 #pragma unroll
