@@ -487,13 +487,15 @@ def main():
         st.forward(t, wtab, x)
         st.backward(wtab, dx, gtab)
 
-    def timed(nsteps, first, fn):
+    def timed(nsteps, first, fn, tail=None):
         barrier()
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for k in range(nsteps):
             fn(first + k)
+        if tail is not None:
+            tail()  # work of the last step on other streams joins before the end event
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
@@ -570,22 +572,35 @@ def main():
         dense_ms = timed(args.steps, 0, step)
         P.ld_set_schedule(st.h, P.make_schedule(sched))
 
-    # ---- end to end: host inputs in pinned memory, dX read back every step
+    # ---- end to end: host inputs in pinned memory, dX read back every step.
+    # X is copied in on the compute stream (the forward starts from it); dY
+    # on a copy stream while the forward runs; dX is read back on the copy
+    # stream while the next step's forward runs, so dX alternates between two
+    # device buffers.  Every step's copies are inside the timed region (the
+    # last read-back joins the compute stream before the end event).
     e2e = None
     if not args.no_e2e:
         xh = x0.cpu().pin_memory()
         dyh = dy0.cpu().pin_memory()
         dxh = torch.empty(dx.shape, dtype=dx.dtype).pin_memory()
+        copy = torch.cuda.Stream()
+        dxs = [dx, torch.empty_like(dx)]
 
         def step_e2e(t):
+            d = dxs[t % 2]
             x.copy_(xh, non_blocking=True)
-            dx.copy_(dyh, non_blocking=True)
+            copy.wait_stream(stream)  # d's read-back two steps ago was on this stream too
+            with torch.cuda.stream(copy):
+                d.copy_(dyh, non_blocking=True)
             st.forward(t, wtab, x)
-            st.backward(wtab, dx, gtab)
-            dxh.copy_(dx, non_blocking=True)
+            stream.wait_stream(copy)
+            st.backward(wtab, d, gtab)
+            copy.wait_stream(stream)
+            with torch.cuda.stream(copy):
+                dxh.copy_(d, non_blocking=True)
 
         step_e2e(step0)
-        e2e_ms = timed(args.steps, step0 + args.warmup, step_e2e)
+        e2e_ms = timed(args.steps, step0 + args.warmup, step_e2e, tail=lambda: stream.wait_stream(copy))
         nb = x.numel() * x.element_size()
         e2e = {"value": world * B * S / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": 2 * nb,
                "d2h_bytes_per_step": nb, "ms_per_step": e2e_ms}
