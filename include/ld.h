@@ -79,7 +79,7 @@ typedef enum {
  * with rotary angles at their original positions, and a dropped token is
  * left unchanged and contributes no key or value to that layer.  Needs
  * rope_theta or no position scheme (no ALiBi) and, on the bf16 path,
- * Dh = 128 and S % 128 == 0. */
+ * Dh = 64 or 128 and S % 128 == 0. */
 typedef enum { LD_PER_SEQUENCE = 0, LD_PER_BATCH = 1, LD_PER_SHARD = 2, LD_PER_TOKEN = 3 } ld_granularity;
 
 /* Layer distributions (Dropout Distribution section):
@@ -153,7 +153,7 @@ typedef struct { float *w_qkv, *w_o, *w_gu, *w_d, *g1, *g2; } ld_layer_g;
  * call), so it can run without a GPU.  LD_ERR_SHAPE for an unsupported
  * shape, LD_ERR_ARG for null pointers, a non-finite eps/alpha, a flag out of
  * range, ALiBi together with a rotary embedding, or per-token granularity
- * with ALiBi or (bf16 path) with Dh != 128 or S % 128 != 0. */
+ * with ALiBi or (bf16 path) with Dh = 32 or S % 128 != 0. */
 ld_status ld_create(const ld_config* cfg, void** handle);
 
 /* Bytes of device workspace ld_forward/ld_backward need: the mask tables,

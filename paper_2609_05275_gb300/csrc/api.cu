@@ -797,9 +797,9 @@ ld_status ld_create(const ld_config* cfg, void** handle) {
   if (c.granularity == LD_PER_TOKEN) {
     // the ALiBi distance would need the kept tokens' original positions in
     // the attention kernels; the bf16 path runs its per-token attention on
-    // the tcgen05 kernels only
+    // the tcgen05 kernels only (head size 64 or 128, S % 128 == 0)
     if (c.alibi) return LD_ERR_ARG;
-    if (!c.fp32_debug && (c.Dh != 128 || c.S % 128)) return LD_ERR_SHAPE;
+    if (!c.fp32_debug && (c.Dh < 64 || c.S % 128)) return LD_ERR_SHAPE;
   }
   if (c.act != LD_ACT_SWIGLU && c.act != LD_ACT_RELU2) return LD_ERR_ARG;
   if (c.b_offset < 0 || (long long)c.b_offset + c.B > 0x7fffffffll) return LD_ERR_ARG;

@@ -78,8 +78,8 @@ def test_position_and_activation_flags():
 
 
 def test_per_token_flag():
-    # per-token granularity: no ALiBi; on the bf16 path head size 128 and
-    # S % 128 == 0 (the tcgen05 attention), any supported shape on the
+    # per-token granularity: no ALiBi; on the bf16 path head size 64 or 128
+    # and S % 128 == 0 (the tcgen05 attention), any supported shape on the
     # float32 debug path; the mask tables grow to one entry per token
     cfg = dict(synth.CONFIGS["tiny"])          # Dh = 32, S = 64
     assert P.ld_create_status(P.make_config(cfg, "per_token")) == P.LD_ERR_SHAPE
@@ -87,6 +87,8 @@ def test_per_token_flag():
     c128 = dict(cfg, H=2, Hkv=1, Dh=128, S=128)
     assert P.ld_create_status(P.make_config(c128, "per_token")) == P.LD_OK
     assert P.ld_create_status(P.make_config(dict(c128, S=192), "per_token")) == P.LD_ERR_SHAPE
+    assert P.ld_create_status(P.make_config(dict(c128, H=4, Hkv=2, Dh=64), "per_token")) == P.LD_OK
+    assert P.ld_create_status(P.make_config(dict(c128, H=4, Hkv=2, Dh=64, S=192), "per_token")) == P.LD_ERR_SHAPE
     assert P.ld_create_status(P.make_config(dict(c128, alibi=True, rope_theta=0.0), "per_token")) == P.LD_ERR_ARG
     assert P.ld_create_status(P.make_config(dict(c128, alibi=True, rope_theta=0.0), "per_token",
                                             fp32_debug=True)) == P.LD_ERR_ARG

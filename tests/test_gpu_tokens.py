@@ -20,6 +20,8 @@ pytestmark = pytest.mark.gpu
 # Dh = 128 and S % 128 == 0: the bf16 path's tcgen05 attention; S = 384 with
 # p ~ 0.5 gives segments of every length mod 128
 TOK = dict(L=2, d=256, H=2, Hkv=1, Dh=128, F=512, B=3, S=384, eps=1e-6, rope_theta=1e4, alpha=1.0)
+# head size 64: the tcgen05 forward and the two-kernel backward at Dh = 64
+TOK64 = dict(TOK, H=4, Hkv=2, Dh=64)
 TINY = synth.CONFIGS["tiny"]
 
 
@@ -92,11 +94,13 @@ def test_token_stack_fp32(sublayer):
     _compare(TINY, sched, 1, True, sublayer)
 
 
+@pytest.mark.parametrize("dh", [128, 64], ids=["dh128", "dh64"])
 @pytest.mark.parametrize("sublayer", [False, True], ids=["layer", "sublayer"])
-def test_token_stack_bf16(sublayer):
+def test_token_stack_bf16(sublayer, dh):
+    cfg = TOK if dh == 128 else TOK64
     sched = dict(dist="explicit", p_max=0.0, p_explicit=[0.45, 0.55], time="const", seed=5)
-    rmask = _compare(TOK, sched, 2, False, sublayer)
-    lens = rmask.reshape(-1, TOK["B"], TOK["S"]).sum(axis=2)
+    rmask = _compare(cfg, sched, 2, False, sublayer)
+    lens = rmask.reshape(-1, cfg["B"], cfg["S"]).sum(axis=2)
     assert (lens % 128 != 0).any()  # ragged segments: tiles straddle sequence ends
 
 
@@ -107,9 +111,9 @@ def test_token_stack_bf16_fp32_agree_on_gqa():
     _compare(cfg, sched, 0, False)
 
 
-@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
-def test_token_all_kept_equals_per_sequence(fp32):
-    cfg = TINY if fp32 else TOK
+@pytest.mark.parametrize("fp32,dh", [(True, 32), (False, 128), (False, 64)], ids=["fp32", "bf16", "bf16-dh64"])
+def test_token_all_kept_equals_per_sequence(fp32, dh):
+    cfg = TINY if fp32 else (TOK if dh == 128 else TOK64)
     dtype = torch.float32 if fp32 else torch.bfloat16
     host, x, dy, dev, xd, dyd = _inputs(cfg, dtype)
     sched = dict(dist="uniform", p_max=0.0, time="const", seed=1)
@@ -137,11 +141,11 @@ def test_token_all_dropped_is_identity(fp32):
             assert (g == 0).all(), n
 
 
-@pytest.mark.parametrize("fp32", [True, False], ids=["fp32", "bf16"])
-def test_token_tiny_and_empty_segments(fp32):
+@pytest.mark.parametrize("fp32,dh", [(True, 32), (False, 128), (False, 64)], ids=["fp32", "bf16", "bf16-dh64"])
+def test_token_tiny_and_empty_segments(fp32, dh):
     # p close to 1 over short sequences: segments of 0, 1, 2, ... kept tokens
     # side by side (a sequence with none, its neighbours with a few)
-    cfg = dict(TINY, B=16, S=64) if fp32 else dict(TOK, B=16, S=128, L=2)
+    cfg = dict(TINY, B=16, S=64) if fp32 else dict(TOK if dh == 128 else TOK64, B=16, S=128, L=2)
     sched = dict(dist="uniform", p_max=0.985 if not fp32 else 0.97, time="const", seed=21)
     rmask = _compare(cfg, sched, 0, fp32)
     lens = rmask.reshape(-1, cfg["B"], cfg["S"]).sum(axis=2)
