@@ -480,6 +480,9 @@ ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, flo
   a.S = ra.unit;
   a.save = same_rows ? z : nullptr;  // same rows feed the FFN block: keep a compact copy of Z
   a.ld_save = c.d;
+  // with the same rows in both blocks nothing reads x between here and the
+  // down projection, which adds into Z's compact copy and writes x itself
+  a.x_skip = same_rows ? 1 : 0;
   { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
   if (!same_rows) {  // the FFN block gathers its own rows of Z from the residual stream
     Timed tm_(h, LD_KCLASS_ROWWISE, st);
@@ -511,6 +514,10 @@ ld_status forward_layer(Handle* h, void* ws, char* lb, const ld_layer_w& Wl, flo
   a.kept_idx = rf.idx;
   a.S = rf.unit;
   a.save = nullptr;
+  if (same_rows) {  // x = Z + s FFN on the kept rows (the O projection left x as it was)
+    a.resid_src = z;
+    a.ld_src = c.d;
+  }
   { Timed tm_(h, LD_KCLASS_GEMM, st); LD_CHECK(gemm<T>(a, st)); }
   return LD_OK;
 }

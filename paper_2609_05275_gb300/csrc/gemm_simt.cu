@@ -69,8 +69,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const GemmArgs a) {
           continue;
         }
         float* x = a.x + r * a.ldx + n;
-        const float nv = *x + v;
-        *x = nv;
+        const float nv = (a.resid_src ? a.resid_src[(size_t)m * a.ld_src + n] : *x) + v;
+        if (!a.x_skip) *x = nv;
         if (a.save) static_cast<float*>(a.save)[(size_t)m * a.ld_save + n] = nv;
       } else {
         static_cast<float*>(a.D)[(size_t)m * a.ldd + n] = v;

@@ -121,14 +121,15 @@ __device__ __forceinline__ void store_chunk(const GemmArgs& a, int row, int col,
       return;
     }
     float4* px = reinterpret_cast<float4*>(a.x + r * a.ldx + col);
+    const float4* pl = a.resid_src ? reinterpret_cast<const float4*>(a.resid_src + (size_t)row * a.ld_src + col) : px;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      float4 o = px[i];
+      float4 o = pl[i];
       o.x += a.alpha * v[4 * i + 0];
       o.y += a.alpha * v[4 * i + 1];
       o.z += a.alpha * v[4 * i + 2];
       o.w += a.alpha * v[4 * i + 3];
-      px[i] = o;
+      if (!a.x_skip) px[i] = o;
       if (ps) ps[i] = o;
     }
   }
@@ -531,12 +532,15 @@ __global__ void __launch_bounds__(192, 1)
         const bool pad = row < M && rs < 0;  // padding row of a per-token kept list: zero copy only
         const bool rok = row < M && !pad;
         const long long r = rok ? rs : 0;
-        float* xrow = a.x + r * a.ldx + (size_t)nb * BN;
+        // the old value comes from x[r], or from the compact copy resid_src
+        float* xrow = a.x_skip ? nullptr : a.x + r * a.ldx + (size_t)nb * BN;
+        const float* lrow = a.resid_src ? a.resid_src + (size_t)(row < M ? row : 0) * a.ld_src + (size_t)nb * BN
+                                        : a.x + r * a.ldx + (size_t)nb * BN;
         float* srow = a.save ? static_cast<float*>(a.save) + (size_t)row * a.ld_save + (size_t)nb * BN : nullptr;
         float4 xv[8];
         if (rok && nb * BN < N) {
 #pragma unroll
-          for (int i = 0; i < 8; ++i) xv[i] = reinterpret_cast<const float4*>(xrow)[i];
+          for (int i = 0; i < 8; ++i) xv[i] = reinterpret_cast<const float4*>(lrow)[i];
         }
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
@@ -554,11 +558,13 @@ __global__ void __launch_bounds__(192, 1)
           }
           if (rok && c + 32 < BN && nb * BN + c + 32 < N) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) xv[i] = reinterpret_cast<const float4*>(xrow + c + 32)[i];
+            for (int i = 0; i < 8; ++i) xv[i] = reinterpret_cast<const float4*>(lrow + c + 32)[i];
           }
           if (ok) {
+            if (xrow) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(xrow + c)[i] = o[i];
+              for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(xrow + c)[i] = o[i];
+            }
             if (srow) {
 #pragma unroll
               for (int i = 0; i < 8; ++i) reinterpret_cast<float4*>(srow + c)[i] = o[i];

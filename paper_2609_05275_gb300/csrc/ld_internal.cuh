@@ -229,13 +229,19 @@ struct GemmArgs {
   int ldd;
   float alpha;
   // EPI_RESID: x[r] = x[r] + alpha*acc for r = src_row(kept_idx, S, m) on the
-  // float32 residual stream x; save[m] = new x[r] (float32, compact)
+  // float32 residual stream x; save[m] = new x[r] (float32, compact).
+  // Variants: with resid_src the old value is read from the compact copy
+  // resid_src[m*ld_src] instead of x[r]; with x_skip the new value goes to
+  // save only and x is left as it was.
   float* x;
   int ldx;
   const int* kept_idx;
   int S;
   void* save;
   int ld_save;
+  const float* resid_src;
+  int ld_src;
+  int x_skip;
   // EPI_ROPE (position of row m: row_pos(pos_tok, S, m))
   const float* rope_cos;
   const float* rope_sin;
