@@ -46,7 +46,7 @@ METRIC = "effective tokens/s (fwd+bwd) under layer dropout; % bf16 peak; skip-sp
 # launches of a 2-layer stack with the Llama-3-8B shapes and 12288 kept rows
 # per launch; command and per-launch table in
 # profiles/gemm_tc_llama8b_traffic.md.  Scaled by the kept rows per launch.
-GEMM_DRAM_BYTES_PER_ROW = 168232.0
+GEMM_DRAM_BYTES_PER_ROW = 166811.0
 PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 
 
